@@ -1,0 +1,199 @@
+/*
+ * sd2.h — C ABI of the SD^2 (steered speculative decoding) hot path on one GB300 (sm_103a).
+ *
+ * One draft-and-verify iteration (Sec. 3 of "Steering Pretrained Drafters during Speculative
+ * Decoding", arXiv 2511.09844):
+ *   a1  steering vector g_t = LN(W_hml [h_t, m_t, l_t]) from the verifier's hidden states at the
+ *       last returned token (Sec. 3.1; layer norm and layers 3, L/2, L-2 from App. A.2), and the
+ *       per-layer biases W_s g_t, computed once per drafting stage (Sec. 3.2);
+ *   a2  k autoregressive drafter steps whose SwiGLU MLPs are steered as in Eq. 2;
+ *   a3  the verifier's parallel forward over the k+1 block positions (Sec. 3.1), which also
+ *       writes the hidden states that a1 reads next;
+ *   a4  speculative acceptance (greedy, or min(1, p/q) with residual resampling and a bonus
+ *       token; Sec. 3.1 and Sec. 4 "Metrics"), then KV-cache rollback of rejected positions.
+ *
+ * Conventions for every call:
+ *   - All pointers prefixed d_ are DEVICE pointers owned by the caller; h_ pointers are host
+ *     memory. Weight pointers are borrowed for the lifetime of the context and never written.
+ *   - The context owns its own device memory (KV pools, activations, scratch), allocated in
+ *     sd2_init and released in sd2_free.
+ *   - Work is enqueued on the stream given to sd2_init (a cudaStream_t passed as void*); calls
+ *     return without waiting for the GPU, except where stated.
+ *   - A call returns SD2_OK or an error code; sd2_last_error(ctx) gives a message. Errors the
+ *     GPU detects (non-finite probabilities, a timed-out wait) are latched in a device error word
+ *     that sd2_check() reads. No kernel traps or asserts.
+ *   - Tensors are row-major. bf16 is IEEE bfloat16 (uint16 bit pattern); f32 is IEEE float.
+ */
+#ifndef SD2_H
+#define SD2_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  SD2_OK = 0,
+  SD2_EINVAL = 1,     /* bad argument or configuration */
+  SD2_ENOMEM = 2,     /* device allocation failed */
+  SD2_ECUDA = 3,      /* a CUDA runtime call failed */
+  SD2_ECAPACITY = 4,  /* batch, context or prompt exceeds what sd2_init sized */
+  SD2_ESTATE = 5,     /* call out of order: init -> prefill -> (step -> accept)* -> free */
+  SD2_ENUMERIC = 6,   /* the GPU saw a non-finite logit/probability (latched, see sd2_check) */
+  SD2_ETIMEOUT = 7    /* a bounded device-side wait gave up (latched, see sd2_check) */
+} sd2_status;
+
+enum { SD2_DTYPE_F32 = 0, SD2_DTYPE_BF16 = 1 };
+
+/* Tensor slots of one decoder layer, in this order, each a bf16 device pointer:
+ *   ATTN_NORM [d]            RMSNorm gain before attention
+ *   Q [H*hd, d], K [Hkv*hd, d], V [Hkv*hd, d], O [d, H*hd]   (nn.Linear layout: [out, in])
+ *   MLP_NORM [d]             RMSNorm gain before the MLP
+ *   GATE [F, d], UP [F, d], DOWN [d, F]                        (SwiGLU, Eq. 1 / Eq. 2)     */
+enum {
+  SD2_W_ATTN_NORM = 0, SD2_W_Q, SD2_W_K, SD2_W_V, SD2_W_O,
+  SD2_W_MLP_NORM, SD2_W_GATE, SD2_W_UP, SD2_W_DOWN, SD2_LAYER_SLOTS
+};
+
+/* One Llama-style pre-norm decoder (no projection biases, untied lm_head, rotate-half rotary
+ * embedding with frequencies rope_theta^(-2i/head_dim)). head_dim must be 64 or 128. */
+typedef struct {
+  int32_t n_layers, d_model, n_heads, n_kv_heads, head_dim, d_ffn, vocab;
+  float rope_theta, norm_eps;
+} sd2_lm_config;
+
+typedef struct {
+  sd2_lm_config verifier, drafter;   /* same vocab (the paper's pairs share a tokenizer) */
+  int32_t d_steer;                   /* width d_g of the steering vector */
+  int32_t tap_layers[3];             /* 1-based verifier layers (h, m, l); App. A.2: L-2, L/2, 3 */
+  float steer_ln_eps;                /* epsilon of the steering layer norm (App. A.2) */
+  int32_t k;                         /* draft length (1..16) */
+  int32_t max_batch;                 /* sequences per batch (1..256) */
+  int32_t max_ctx;                   /* per-sequence token capacity (prompt + generated + k + 2) */
+  int32_t max_prefill_tokens;        /* most prompt tokens one sd2_prefill may carry in total */
+  int32_t kv_block;                  /* paged KV-cache block size in tokens; must be 16 */
+} sd2_config;
+
+typedef struct {
+  const void* embed;                 /* [vocab, d] bf16 */
+  const void* final_norm;            /* [d] bf16 */
+  const void* lm_head;               /* [vocab, d] bf16 */
+  const void* const* layers;         /* HOST array of n_layers*SD2_LAYER_SLOTS device pointers,
+                                        layer-major, slot order above; copied by sd2_init */
+} sd2_lm_weights;
+
+typedef struct {
+  sd2_lm_weights verifier, drafter;
+  const void* w_hml;                 /* [d_g, 3*d_v] bf16, columns ordered [h | m | l] (Sec. 3.1) */
+  const void* steer_ln_gamma;        /* [d_g] bf16 layer-norm gain (App. A.2) */
+  const void* steer_ln_beta;         /* [d_g] bf16 layer-norm shift */
+  const void* w_s;                   /* [L_D*F_D, d_g] bf16: rows l*F_D.. give W_s^(l) of Eq. 2 */
+} sd2_weights;
+
+typedef struct sd2_ctx sd2_ctx;
+
+/* Validate cfg, borrow the weights, allocate the context's device memory and enqueue its
+ * initialisation on `stream` (a cudaStream_t). *out receives the context.
+ * Errors: SD2_EINVAL (shape unsupported, null pointer), SD2_ENOMEM, SD2_ECUDA. */
+sd2_status sd2_init(const sd2_config* cfg, const sd2_weights* w, void* stream, sd2_ctx** out);
+
+/* Start `batch` sequences from their prompts (Sec. 3.1 prefill). d_tokens holds the prompts
+ * back to back (int32 ids); h_cu_lens[batch+1] are host prefix offsets into it. h_temperature
+ * [batch] per sequence: 0 = greedy (T=0), else sampling at T (applied to both models).
+ * The verifier reads each prompt and its last row gives the first new token, written to
+ * d_first_token[batch]; the steering vector is read at that row; the drafter reads the prompt
+ * under its biases. seed keys the Philox stream of every later random draw.
+ * Errors: SD2_EINVAL, SD2_ECAPACITY (batch, prompt length or total tokens too large). */
+sd2_status sd2_prefill(sd2_ctx* ctx, int32_t batch, const int32_t* d_tokens, const int32_t* h_cu_lens,
+                       const float* h_temperature, uint64_t seed, int32_t* d_first_token);
+
+/* a1 + a2 + a3 of one iteration for every live sequence: compute the steering biases, draft k
+ * tokens, and run the verifier over the k+1 block positions. Asynchronous on the ctx stream.
+ * Errors: SD2_ESTATE (no prefill, or the previous step was not accepted). */
+sd2_status sd2_step(sd2_ctx* ctx);
+
+/* a4: acceptance and rollback for the block of the last sd2_step. Writes, per sequence b,
+ * d_tokens[b*(k+1) + t] for t < d_n_emitted[b] (the j kept drafts then one verifier token) and
+ * d_n_emitted[b] = j+1 (0 once a sequence has stopped because its capacity is reached).
+ * Errors: SD2_ESTATE (no step to accept). */
+sd2_status sd2_accept(sd2_ctx* ctx, int32_t* d_tokens, int32_t* d_n_emitted);
+
+/* Wait for the context's stream and report the device error word (SD2_OK, SD2_ENUMERIC or
+ * SD2_ETIMEOUT), clearing it. */
+sd2_status sd2_check(sd2_ctx* ctx);
+
+/* Release everything the context owns (waits for its stream first). Null is allowed. */
+sd2_status sd2_free(sd2_ctx* ctx);
+
+/* Message of the last error on this context (or of the last failed context-free call if ctx
+ * is null). Valid until the next call on the same context. */
+const char* sd2_last_error(const sd2_ctx* ctx);
+
+/* Use CUDA graphs for sd2_step/sd2_accept (default on). Graphs are captured on first use after
+ * each prefill; 0 launches every kernel directly. */
+sd2_status sd2_set_graphs(sd2_ctx* ctx, int32_t enable);
+
+/* Read-only views of the context's device buffers, for tests and measurement. `which`:
+ *   0 target logits  [B, k+1, V] f32     1 draft logits [B, k, V] f32     2 drafts x^ [B, k] i32
+ *   3 verifier taps  [B, k+1, 3, d_v] f32 (order h, m, l)   4 steering vector g [B, d_g] f32
+ *   5 steering biases [B, L_D*F_D] f32   6 committed tokens [B, max_ctx] i32
+ *   7 per-sequence state [B, 4] i32: committed length n, drafter cached length, j, stopped
+ *   8 iteration counter [1] i32 (the `step` of the Philox counters; 0 = prefill)
+ * *d_ptr, *n_elems and *dtype (SD2_DTYPE_*) describe the buffer; B is the prefilled batch. */
+sd2_status sd2_debug_buffer(const sd2_ctx* ctx, int32_t which, void** d_ptr, int64_t* n_elems,
+                            int32_t* dtype);
+
+/* Per-kernel-class timing of the iterations that follow, measured with CUDA events on the ctx
+ * stream (graphs are not used while profiling is on). sd2_profile_read returns, per class,
+ * launches, total milliseconds and algorithmic bytes. Classes: 0 GEMM (weight streaming),
+ * 1 attention, 2 acceptance, 3 sampling, 4 other, 5 verify stage (a3), 6 draft stage (a2),
+ * 7 steering stage (a1). */
+sd2_status sd2_profile(sd2_ctx* ctx, int32_t enable);
+sd2_status sd2_profile_read(sd2_ctx* ctx, int64_t* launches, double* ms, double* bytes, int32_t n_classes);
+
+/* ---------------------------------------------------------------------------------------------
+ * Standalone kernels (no context): the acceptance and steering steps on caller buffers.
+ * ------------------------------------------------------------------------------------------- */
+
+/* Scratch bytes sd2_accept_logits needs for batch B and draft length k. */
+size_t sd2_accept_workspace_bytes(int32_t B, int32_t k);
+
+/* Speculative acceptance of B independent blocks (a4 without rollback), Sec. 3.1:
+ *   d_target [B, k+1, V], d_draft [B, k, V] logits of `dtype` (SD2_DTYPE_F32 or _BF16);
+ *   row i of d_target is the verifier's distribution after block input i, row i-1 of d_draft
+ *   is the distribution q_i draft i was drawn from; d_xhat [B, k] int32 drafts;
+ *   d_temperature [B] f32 (0 = greedy). Random draws use Philox4x32-10 (Salmon et al. SC'11)
+ *   with key (seed mod 2^32, seed >> 32) and counter (c0, purpose<<16 | i, b, step):
+ *   the uniform of draft i's test is word 0 of (0, 1<<16 | i, b, step); the replacement or
+ *   bonus token drawn from block row i uses, for vocabulary entry v, word v&3 of
+ *   (v>>2, 2<<16 | i, b, step); u = (2*(word>>9)+1) * 2^-24. Outputs d_tokens [B, k+1] int32
+ *   (first d_n[b] entries valid) and d_n [B] = accepted + 1.
+ *   d_workspace: caller device scratch of sd2_accept_workspace_bytes(B, k) bytes, 256-byte
+ *   aligned; contents need not be initialised. Errors: SD2_EINVAL (sizes, null, alignment). */
+sd2_status sd2_accept_logits(const void* d_target, const void* d_draft, int32_t dtype,
+                             const int32_t* d_xhat, const float* d_temperature, int32_t B, int32_t k,
+                             int32_t V, uint64_t seed, uint32_t step, int32_t* d_tokens, int32_t* d_n,
+                             void* d_workspace, size_t workspace_bytes, void* stream);
+
+/* Steering step a1 on caller buffers: g = LN(W_hml [h; m; l]) * gamma + beta and biases
+ * W_s g for B sequences (Sec. 3.1, Eq. 2, App. A.2).
+ *   d_taps [B, 3, d_v] f32 in the order (h, m, l); weights bf16 as in sd2_weights;
+ *   outputs d_g [B, d_g] f32 and d_bias [B, n_bias] f32, n_bias = L_D * F_D.
+ *   d_workspace: scratch of sd2_steer_workspace_bytes(B, d_v, d_g) bytes. */
+size_t sd2_steer_workspace_bytes(int32_t B, int32_t d_v, int32_t d_g);
+sd2_status sd2_steer(const float* d_taps, int32_t B, int32_t d_v, const void* w_hml, const void* ln_gamma,
+                     const void* ln_beta, float ln_eps, int32_t d_g, const void* w_s, int32_t n_bias,
+                     float* d_g_out, float* d_bias, void* d_workspace, size_t workspace_bytes, void* stream);
+
+/* Steered SwiGLU activation of Eq. 2 on caller buffers (the injection step of a2):
+ *   h[m, f] = (up[m, f] + bias[seq[m], f]) * SiLU(gate[m, f]) as bf16, with gate/up [M, F] f32,
+ *   bias [*, F] f32 (row seq[m]; d_seq may be null for bias row 0), h [M, F] bf16. */
+sd2_status sd2_swiglu_steered(const float* d_gate, const float* d_up, const float* d_bias,
+                              const int32_t* d_seq, int32_t M, int32_t F, void* d_h, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* SD2_H */

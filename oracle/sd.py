@@ -60,6 +60,7 @@ class OracleSD:
         self.seed = int(seed)
         self.exact_rows = exact_rows
         self.biases: List[torch.Tensor] = []              # [L_D, F_D] per stage
+        self.gs: List[torch.Tensor] = []                  # the steering vector g of each stage
         self.seqs: List[SeqState] = []
 
     # -- model evaluations --------------------------------------------------------------------
@@ -85,16 +86,25 @@ class OracleSD:
 
     def _new_bias(self, taps_hml: torch.Tensor) -> int:
         g = steering.steering_vector(taps_hml, self.st, self.work.steer_ln_eps)
+        self.gs.append(g)
         self.biases.append(steering.steering_bias(g, self.st, self.ds.n_layers, self.ds.d_ffn))
         return len(self.biases) - 1
 
     # -- the loop -------------------------------------------------------------------------------
-    def prefill(self, prompts: Sequence[Sequence[int]], temps: Sequence[float]) -> List[int]:
+    def prefill(self, prompts: Sequence[Sequence[int]], temps: Sequence[float],
+                forced_first: Optional[Sequence[int]] = None) -> List[int]:
+        """Start every sequence; forced_first replaces the sampled first tokens (teacher forcing)."""
         firsts = []
+        self.prefill_logits, self.prefill_taps = [], []
         for b, (prompt, temp) in enumerate(zip(prompts, temps)):
             n0 = len(prompt)
             z, tp = self.verifier_rows(list(prompt), n0 - 1, n0 - 1)
-            y = sampling.sample_from_target(z[0].numpy(), temp, self.seed, b, 0, 0)
+            self.prefill_logits.append(z[0])
+            self.prefill_taps.append(tp[0])
+            if forced_first is not None:
+                y = int(forced_first[b])
+            else:
+                y = sampling.sample_from_target(z[0].numpy(), temp, self.seed, b, 0, 0)
             s = SeqState(tokens=list(prompt) + [y], prompt_len=n0, temp=float(temp))
             s.cur_bias = self._new_bias(tp[0])
             s.bias_ids = [s.cur_bias] * n0          # drafter prefill under the first g

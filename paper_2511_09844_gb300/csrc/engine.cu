@@ -1,0 +1,823 @@
+// SD^2 engine: host orchestration of one draft-and-verify iteration behind the C ABI of sd2.h.
+//
+//   sd2_prefill  verifier over the prompts -> first token (bonus-style sample at step 0) ->
+//                steering from the last prompt row -> drafter over the prompts under its biases
+//   sd2_step     a1 steering (Sec. 3.1, App. A.2) -> a2 k drafter steps with Eq. 2 biases ->
+//                a3 verifier over the k+1 block rows, writing taps and logits
+//   sd2_accept   a4 acceptance (Sec. 3.1) -> commit and rollback of both caches
+//
+// All per-sequence lengths live on the device (state.cu), so step and accept are each captured
+// once into a CUDA graph and replayed. The decoder forward is a fixed chain per layer:
+// RMSNorm(+taps) -> QKV GEMM -> rotary + paged KV append -> attention -> O GEMM (+residual) ->
+// RMSNorm -> gate/up GEMM with the steered SwiGLU epilogue -> down GEMM (+residual).
+#include <math.h>
+#include <string.h>
+
+#include <algorithm>
+#include <string>
+#include <vector>
+
+#include "../../include/sd2.h"
+#include "common.cuh"
+#include "kernels.h"
+#include "state.h"
+
+using namespace sd2;
+
+namespace {
+
+thread_local std::string g_last_error;
+
+struct Model {
+  sd2_lm_config c{};
+  const void* embed = nullptr;
+  const void* final_norm = nullptr;
+  const void* lm_head = nullptr;
+  std::vector<const void*> w;
+  void* kv_pool = nullptr;
+  int* table = nullptr;
+  int bt_stride = 0, n_blocks = 0;
+  float* rope_cs = nullptr;
+  const void* W(int l, int s) const { return w[static_cast<size_t>(l) * SD2_LAYER_SLOTS + s]; }
+  int qkv_width() const { return (c.n_heads + 2 * c.n_kv_heads) * c.head_dim; }
+  int group_rows() const { return std::max(1, 64 / (c.n_heads / c.n_kv_heads)); }
+  KVCache cache() const {
+    KVCache k;
+    k.pool = kv_pool; k.table = table; k.bt_stride = bt_stride; k.n_blocks = n_blocks;
+    k.Hkv = c.n_kv_heads; k.hd = c.head_dim;
+    return k;
+  }
+};
+
+struct Plan {
+  int M = 0;
+  const int* tok = nullptr;
+  const int* pos = nullptr;
+  const int* seq = nullptr;
+  const int* valid = nullptr;
+  int n_groups = 0;
+  const int* g_row0 = nullptr;
+  const int* g_nrows = nullptr;
+  const int* g_seq = nullptr;
+  int n_splits = 1, chunk = 64;
+};
+
+struct ProfRec {
+  int cls;
+  double bytes;
+  cudaEvent_t e0, e1;
+};
+
+}  // namespace
+
+struct sd2_ctx {
+  sd2_config cfg{};
+  Model V, D;
+  const void *w_hml = nullptr, *ln_g = nullptr, *ln_b = nullptr, *w_s = nullptr;
+  cudaStream_t st = nullptr, cap_st = nullptr;
+  int B = 0, phase = 0, maxB = 0, max_rows = 0;
+  unsigned long long seed = 0;
+  std::string err;
+  std::vector<void*> allocs;
+  // device state
+  int *state = nullptr, *committed = nullptr, *iter = nullptr, *xhat = nullptr;
+  float* temp = nullptr;
+  unsigned* errw = nullptr;
+  int *row_tok = nullptr, *row_pos = nullptr, *row_seq = nullptr, *row_valid = nullptr;
+  int* statics = nullptr;  // group tables and row lists of the step shapes, then prefill's
+  int statics_cap = 0;
+  // activations
+  float *x = nullptr, *qkv = nullptr, *q = nullptr, *part = nullptr, *logits_t = nullptr, *logits_d = nullptr;
+  float *taps = nullptr, *g_pre = nullptr, *g = nullptr, *bias = nullptr;
+  void *a = nullptr, *attn = nullptr, *h = nullptr, *g_bf = nullptr, *hml_in = nullptr;
+  size_t part_elems = 0;
+  unsigned long long* samp_slot = nullptr;
+  int* samp_counter = nullptr;
+  AcceptScratch as{};
+  int *tok_out = nullptr, *n_out = nullptr, *first = nullptr, *cu = nullptr;
+  // step-shape plans
+  Plan p_d1, p_dn, p_v;
+  const int* logit_rows_d1 = nullptr;
+  // graphs
+  bool use_graphs = true;
+  cudaGraphExec_t g_step = nullptr, g_accept = nullptr;
+  // profiling
+  bool prof = false;
+  std::vector<ProfRec> recs;
+  std::vector<cudaEvent_t> ev_pool;
+  std::vector<int> h_n;  // host copy of committed lengths while profiling
+};
+
+// ------------------------------------------------------------------------------------------------
+// helpers
+// ------------------------------------------------------------------------------------------------
+namespace {
+
+sd2_status fail(sd2_ctx* c, sd2_status s, const std::string& m) {
+  if (c) c->err = m;
+  g_last_error = m;
+  return s;
+}
+
+#define CK(call)                                                                                   \
+  do {                                                                                             \
+    cudaError_t e_ = (call);                                                                       \
+    if (e_ != cudaSuccess) return fail(c, SD2_ECUDA, std::string(#call) + ": " + cudaGetErrorString(e_)); \
+  } while (0)
+
+template <typename T>
+sd2_status dalloc(sd2_ctx* c, T** p, size_t n) {
+  void* v = nullptr;
+  const size_t bytes = std::max<size_t>(n * sizeof(T), 256);
+  if (cudaMalloc(&v, bytes) != cudaSuccess) {
+    cudaGetLastError();
+    return fail(c, SD2_ENOMEM, "cudaMalloc of " + std::to_string(bytes) + " bytes failed");
+  }
+  c->allocs.push_back(v);
+  *p = static_cast<T*>(v);
+  return SD2_OK;
+}
+#define ALLOC(p, n)                                  \
+  do {                                               \
+    sd2_status s_ = dalloc(c, &(p), (size_t)(n));    \
+    if (s_ != SD2_OK) return s_;                     \
+  } while (0)
+
+cudaEvent_t take_event(sd2_ctx* c) {
+  cudaEvent_t e;
+  if (!c->ev_pool.empty()) {
+    e = c->ev_pool.back();
+    c->ev_pool.pop_back();
+  } else {
+    cudaEventCreate(&e);
+  }
+  return e;
+}
+
+// Run `fn` (which enqueues on c->st) and, when profiling, bracket it with events.
+template <typename F>
+cudaError_t timed(sd2_ctx* c, int cls, double bytes, F fn) {
+  if (!c->prof) return fn();
+  ProfRec r{cls, bytes, take_event(c), take_event(c)};
+  cudaEventRecord(r.e0, c->st);
+  cudaError_t e = fn();
+  cudaEventRecord(r.e1, c->st);
+  c->recs.push_back(r);
+  return e;
+}
+enum { PC_GEMM = 0, PC_ATTN = 1, PC_ACCEPT = 2, PC_SAMPLE = 3, PC_OTHER = 4, PC_VERIFY = 5, PC_DRAFT = 6, PC_STEER = 7,
+       PC_N = 8 };
+
+bool valid_lm(const sd2_lm_config& m) {
+  return m.n_layers > 0 && m.d_model > 0 && m.d_model % 8 == 0 && (m.head_dim == 64 || m.head_dim == 128) &&
+         m.n_heads > 0 && m.n_kv_heads > 0 && m.n_heads % m.n_kv_heads == 0 && m.n_heads / m.n_kv_heads <= 64 &&
+         m.d_ffn > 0 && m.d_ffn % 8 == 0 && m.vocab > 0 && m.vocab % 4 == 0 && m.rope_theta > 0 && m.norm_eps > 0;
+}
+bool aligned16(const void* p) { return p && (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
+
+sd2_status load_model(sd2_ctx* c, Model& m, const sd2_lm_config& cfg, const sd2_lm_weights& w, const char* name) {
+  m.c = cfg;
+  if (!aligned16(w.embed) || !aligned16(w.final_norm) || !aligned16(w.lm_head) || !w.layers)
+    return fail(c, SD2_EINVAL, std::string(name) + ": null or unaligned embed/final_norm/lm_head/layers");
+  m.embed = w.embed; m.final_norm = w.final_norm; m.lm_head = w.lm_head;
+  m.w.assign(w.layers, w.layers + static_cast<size_t>(cfg.n_layers) * SD2_LAYER_SLOTS);
+  for (size_t i = 0; i < m.w.size(); ++i)
+    if (!aligned16(m.w[i]))
+      return fail(c, SD2_EINVAL, std::string(name) + ": layer weight " + std::to_string(i) + " null or not 16-byte aligned");
+  const int maxB = c->cfg.max_batch;
+  m.bt_stride = (c->cfg.max_ctx + 15) / 16;
+  m.n_blocks = maxB * m.bt_stride;
+  const size_t kv_elems = static_cast<size_t>(cfg.n_layers) * m.n_blocks * 2 * cfg.n_kv_heads * 16 * cfg.head_dim;
+  void* pool;
+  ALLOC(pool, kv_elems * 2);
+  m.kv_pool = pool;
+  int* table;
+  ALLOC(table, static_cast<size_t>(maxB) * m.bt_stride);
+  m.table = table;
+  std::vector<int> ht(static_cast<size_t>(maxB) * m.bt_stride);
+  for (int b = 0; b < maxB; ++b)       // block i of sequence b: interleaved across sequences
+    for (int i = 0; i < m.bt_stride; ++i) ht[static_cast<size_t>(b) * m.bt_stride + i] = i * maxB + b;
+  CK(cudaMemcpy(table, ht.data(), ht.size() * sizeof(int), cudaMemcpyHostToDevice));
+  CK(cudaMemset(pool, 0, kv_elems * 2));
+  const int half = cfg.head_dim / 2;
+  std::vector<float> cs(static_cast<size_t>(c->cfg.max_ctx) * half * 2);
+  for (int p = 0; p < c->cfg.max_ctx; ++p)
+    for (int i = 0; i < half; ++i) {
+      const double ang = p * pow(static_cast<double>(cfg.rope_theta), -2.0 * i / cfg.head_dim);
+      cs[(static_cast<size_t>(p) * half + i) * 2] = static_cast<float>(cos(ang));
+      cs[(static_cast<size_t>(p) * half + i) * 2 + 1] = static_cast<float>(sin(ang));
+    }
+  float* rcs;
+  ALLOC(rcs, cs.size());
+  m.rope_cs = rcs;
+  CK(cudaMemcpy(rcs, cs.data(), cs.size() * sizeof(float), cudaMemcpyHostToDevice));
+  return SD2_OK;
+}
+
+// ------------------------------------------------------------------------------------------------
+// forward of one decoder over a row plan
+// ------------------------------------------------------------------------------------------------
+struct FwdOut {
+  const float* bias = nullptr;    // [*, L*F] steering biases (drafter) or null
+  float* taps = nullptr;          // [rows, 3, d] (verifier) or null
+  const int* tap_row = nullptr;
+  int tap_layers[3] = {0, 0, 0};
+  const int* logit_rows = nullptr;
+  int n_logit_rows = 0;
+  float* logits = nullptr;
+  long long ld_logits = 0;
+};
+
+double gemm_bytes(int M, int N, int K, int out_bytes) {
+  return 2.0 * N * K + 2.0 * M * K + static_cast<double>(out_bytes) * M * N;
+}
+
+sd2_status forward(sd2_ctx* c, const Model& m, const Plan& p, const FwdOut& o) {
+  const sd2_lm_config& mc = m.c;
+  const int M = p.M, d = mc.d_model, H = mc.n_heads, Hkv = mc.n_kv_heads, hd = mc.head_dim, F = mc.d_ffn;
+  const int L = mc.n_layers;
+  auto tap_mask = [&](int layer_out) {
+    int mask = 0;
+    if (!o.taps) return 0;
+    for (int s = 0; s < 3; ++s)
+      if (o.tap_layers[s] == layer_out) mask |= 1 << s;
+    return mask;
+  };
+  CK(timed(c, PC_OTHER, 0, [&] {
+    return embed_rmsnorm(p.tok, m.embed, m.W(0, SD2_W_ATTN_NORM), mc.norm_eps, M, d, mc.vocab, c->x, c->a, c->st);
+  }));
+  for (int l = 0; l < L; ++l) {
+    if (l > 0)
+      CK(timed(c, PC_OTHER, 0, [&] {
+        return rmsnorm(c->x, nullptr, m.W(l, SD2_W_ATTN_NORM), mc.norm_eps, M, d, c->a, o.taps, o.tap_row, tap_mask(l),
+                       c->st);
+      }));
+    GemmArgs g{};
+    g.x = c->a; g.ldx = d; g.M = M; g.K = d;
+    g.seg[0] = {m.W(l, SD2_W_Q), H * hd};
+    g.seg[1] = {m.W(l, SD2_W_K), Hkv * hd};
+    g.seg[2] = {m.W(l, SD2_W_V), Hkv * hd};
+    g.nseg = 3; g.epi = EPI_STORE; g.out = c->qkv; g.ldo = m.qkv_width();
+    CK(timed(c, PC_GEMM, gemm_bytes(M, m.qkv_width(), d, 4), [&] { return gemm(g, c->st); }));
+    CK(timed(c, PC_OTHER, 0, [&] {
+      return rope_append(c->qkv, m.rope_cs, M, H, Hkv, hd, p.seq, p.pos, p.valid, m.cache(), l, c->q, c->st);
+    }));
+    AttnArgs at{};
+    at.q = c->q; at.kv = m.cache(); at.layer = l; at.row_pos = p.pos;
+    at.grp_row0 = p.g_row0; at.grp_nrows = p.g_nrows; at.grp_seq = p.g_seq; at.n_groups = p.n_groups;
+    at.M = M; at.H = H; at.hd = hd; at.n_splits = p.n_splits; at.chunk = p.chunk; at.part = c->part; at.out = c->attn;
+    double kvb = 0;
+    if (c->prof && !c->h_n.empty()) {
+      for (int b = 0; b < c->B; ++b) kvb += 2.0 * 2.0 * Hkv * hd * (c->h_n[b] + 16);
+    }
+    CK(timed(c, PC_ATTN, kvb, [&] { return attention(at, c->st); }));
+    GemmArgs go{};
+    go.x = c->attn; go.ldx = H * hd; go.M = M; go.K = H * hd;
+    go.seg[0] = {m.W(l, SD2_W_O), d}; go.nseg = 1; go.epi = EPI_ADD; go.out = c->x; go.ldo = d;
+    CK(timed(c, PC_GEMM, gemm_bytes(M, d, H * hd, 8), [&] { return gemm(go, c->st); }));
+    CK(timed(c, PC_OTHER, 0, [&] {
+      return rmsnorm(c->x, nullptr, m.W(l, SD2_W_MLP_NORM), mc.norm_eps, M, d, c->a, nullptr, nullptr, 0, c->st);
+    }));
+    GemmArgs gu{};
+    gu.x = c->a; gu.ldx = d; gu.M = M; gu.K = d;
+    gu.seg[0] = {m.W(l, SD2_W_GATE), F}; gu.seg[1] = {m.W(l, SD2_W_UP), F}; gu.nseg = 2;
+    gu.epi = EPI_SWIGLU; gu.out_bf = c->h; gu.ldh = F;
+    gu.bias = o.bias ? o.bias + static_cast<size_t>(l) * F : nullptr;
+    gu.ld_bias = L * F; gu.row_seq = p.seq;
+    CK(timed(c, PC_GEMM, gemm_bytes(M, 2 * F, d, 1), [&] { return gemm(gu, c->st); }));
+    GemmArgs gd{};
+    gd.x = c->h; gd.ldx = F; gd.M = M; gd.K = F;
+    gd.seg[0] = {m.W(l, SD2_W_DOWN), d}; gd.nseg = 1; gd.epi = EPI_ADD; gd.out = c->x; gd.ldo = d;
+    CK(timed(c, PC_GEMM, gemm_bytes(M, d, F, 8), [&] { return gemm(gd, c->st); }));
+  }
+  if (o.n_logit_rows > 0 || tap_mask(L)) {
+    const int nr = o.n_logit_rows > 0 ? o.n_logit_rows : M;
+    CK(timed(c, PC_OTHER, 0, [&] {
+      return rmsnorm(c->x, o.logit_rows, m.final_norm, mc.norm_eps, nr, d, c->a, o.taps, o.tap_row, tap_mask(L), c->st);
+    }));
+  }
+  if (o.n_logit_rows > 0) {
+    GemmArgs gl{};
+    gl.x = c->a; gl.ldx = d; gl.M = o.n_logit_rows; gl.K = d;
+    gl.seg[0] = {m.lm_head, mc.vocab}; gl.nseg = 1; gl.epi = EPI_STORE; gl.out = o.logits;
+    gl.ldo = static_cast<int>(o.ld_logits);
+    CK(timed(c, PC_GEMM, gemm_bytes(o.n_logit_rows, mc.vocab, d, 4), [&] { return gemm(gl, c->st); }));
+  }
+  return SD2_OK;
+}
+
+// a1: g = LN(W_hml [h; m; l]) at each sequence's steering row, biases = W_s g.
+sd2_status steer(sd2_ctx* c, const int* row_idx) {
+  const int B = c->B, dv = c->V.c.d_model, dg = c->cfg.d_steer, k = c->cfg.k;
+  const int nb = c->D.c.n_layers * c->D.c.d_ffn;
+  CK(timed(c, PC_OTHER, 0, [&] {
+    return gather_rows_bf16(c->taps, (k + 1) * 3 * dv, row_idx, 3 * dv, B, c->hml_in, c->st);
+  }));
+  GemmArgs g{};
+  g.x = c->hml_in; g.ldx = 3 * dv; g.M = B; g.K = 3 * dv;
+  g.seg[0] = {c->w_hml, dg}; g.nseg = 1; g.epi = EPI_STORE; g.out = c->g_pre; g.ldo = dg;
+  CK(timed(c, PC_GEMM, gemm_bytes(B, dg, 3 * dv, 4), [&] { return gemm(g, c->st); }));
+  CK(timed(c, PC_OTHER, 0, [&] {
+    return layernorm(c->g_pre, c->ln_g, c->ln_b, c->cfg.steer_ln_eps, B, dg, c->g, c->g_bf, c->st);
+  }));
+  GemmArgs gs{};
+  gs.x = c->g_bf; gs.ldx = dg; gs.M = B; gs.K = dg;
+  gs.seg[0] = {c->w_s, nb}; gs.nseg = 1; gs.epi = EPI_STORE; gs.out = c->bias; gs.ldo = nb;
+  CK(timed(c, PC_GEMM, gemm_bytes(B, nb, dg, 4), [&] { return gemm(gs, c->st); }));
+  return SD2_OK;
+}
+
+sd2_status run_step(sd2_ctx* c) {
+  const int B = c->B, k = c->cfg.k, V = c->V.c.vocab;
+  cudaEvent_t s0 = nullptr, s1 = nullptr;
+  auto stage_begin = [&]() {
+    if (c->prof) { s0 = take_event(c); cudaEventRecord(s0, c->st); }
+  };
+  auto stage_end = [&](int cls, double bytes) {
+    if (c->prof) { s1 = take_event(c); cudaEventRecord(s1, c->st); c->recs.push_back({cls, bytes, s0, s1}); }
+  };
+  stage_begin();
+  sd2_status s = steer(c, c->state + 2 * c->maxB);
+  if (s != SD2_OK) return s;
+  stage_end(PC_STEER, 2.0 * c->cfg.d_steer * 3 * c->V.c.d_model +
+                          2.0 * c->cfg.d_steer * c->D.c.n_layers * static_cast<double>(c->D.c.d_ffn));
+  for (int i = 1; i <= k; ++i) {
+    stage_begin();
+    const Plan& p = (i == 1) ? c->p_d1 : c->p_dn;
+    CK(timed(c, PC_OTHER, 0, [&] {
+      return plan_rows(i == 1 ? PLAN_DRAFT_FIRST : PLAN_DRAFT_NEXT, i, B, k, c->cfg.max_ctx, c->state, c->maxB,
+                       c->committed, c->xhat, c->row_tok, c->row_pos, c->row_seq, c->row_valid, c->st);
+    }));
+    FwdOut o;
+    o.bias = c->bias;
+    o.logit_rows = (i == 1) ? c->logit_rows_d1 : nullptr;
+    o.n_logit_rows = B;
+    o.logits = c->logits_d + static_cast<size_t>(i - 1) * V;
+    o.ld_logits = static_cast<long long>(k) * V;
+    s = forward(c, c->D, p, o);
+    if (s != SD2_OK) return s;
+    CK(timed(c, PC_SAMPLE, 4.0 * B * V, [&] {
+      return sample_rows(o.logits, o.ld_logits, B, V, c->temp, c->seed, RNG_DRAFT, i, c->iter, 0, c->xhat + (i - 1), k,
+                         nullptr, 0, c->samp_slot, c->samp_counter, c->errw, c->st);
+    }));
+    stage_end(PC_DRAFT, 2.0 * c->D.c.n_layers * (static_cast<double>(c->D.c.d_model) * c->D.qkv_width() +
+                                                  static_cast<double>(c->D.c.n_heads) * c->D.c.head_dim * c->D.c.d_model +
+                                                  3.0 * c->D.c.d_model * c->D.c.d_ffn) +
+                            2.0 * V * c->D.c.d_model);
+  }
+  stage_begin();
+  CK(timed(c, PC_OTHER, 0, [&] {
+    return plan_rows(PLAN_VERIFY, 0, B, k, c->cfg.max_ctx, c->state, c->maxB, c->committed, c->xhat, c->row_tok,
+                     c->row_pos, c->row_seq, c->row_valid, c->st);
+  }));
+  FwdOut o;
+  o.taps = c->taps;
+  o.tap_row = nullptr;
+  for (int t = 0; t < 3; ++t) o.tap_layers[t] = c->cfg.tap_layers[t];
+  o.n_logit_rows = B * (k + 1);
+  o.logit_rows = nullptr;
+  o.logits = c->logits_t;
+  o.ld_logits = V;
+  s = forward(c, c->V, c->p_v, o);
+  if (s != SD2_OK) return s;
+  stage_end(PC_VERIFY, 2.0 * c->V.c.n_layers * (static_cast<double>(c->V.c.d_model) * c->V.qkv_width() +
+                                                 static_cast<double>(c->V.c.n_heads) * c->V.c.head_dim * c->V.c.d_model +
+                                                 3.0 * c->V.c.d_model * c->V.c.d_ffn) +
+                          2.0 * V * c->V.c.d_model);
+  return SD2_OK;
+}
+
+sd2_status run_accept(sd2_ctx* c) {
+  const int B = c->B, k = c->cfg.k, V = c->V.c.vocab;
+  CK(timed(c, PC_ACCEPT, 4.0 * B * (2 * k + 1) * V, [&] {
+    return accept_blocks(c->logits_t, c->logits_d, SD2_DTYPE_F32, c->xhat, c->temp, B, k, V, c->seed, 0, c->iter,
+                         c->state + 3 * c->maxB, c->tok_out, c->n_out, c->as, c->errw, c->st);
+  }));
+  CK(timed(c, PC_OTHER, 0, [&] {
+    return commit(B, k, c->cfg.max_ctx, c->state, c->maxB, c->committed, c->tok_out, c->n_out, c->iter, c->st);
+  }));
+  return SD2_OK;
+}
+
+template <typename F>
+sd2_status capture(sd2_ctx* c, cudaGraphExec_t* exec, F body) {
+  cudaStream_t user = c->st;
+  c->st = c->cap_st;
+  cudaError_t e = cudaStreamBeginCapture(c->st, cudaStreamCaptureModeThreadLocal);
+  if (e != cudaSuccess) { c->st = user; return fail(c, SD2_ECUDA, std::string("begin capture: ") + cudaGetErrorString(e)); }
+  sd2_status s = body();
+  cudaGraph_t graph = nullptr;
+  e = cudaStreamEndCapture(c->st, &graph);
+  c->st = user;
+  if (s != SD2_OK) { if (graph) cudaGraphDestroy(graph); return s; }
+  if (e != cudaSuccess) return fail(c, SD2_ECUDA, std::string("end capture: ") + cudaGetErrorString(e));
+  e = cudaGraphInstantiate(exec, graph, 0);
+  cudaGraphDestroy(graph);
+  if (e != cudaSuccess) return fail(c, SD2_ECUDA, std::string("graph instantiate: ") + cudaGetErrorString(e));
+  return SD2_OK;
+}
+
+void drop_graphs(sd2_ctx* c) {
+  if (c->g_step) cudaGraphExecDestroy(c->g_step);
+  if (c->g_accept) cudaGraphExecDestroy(c->g_accept);
+  c->g_step = c->g_accept = nullptr;
+}
+
+// Attention row groups: consecutive rows of one sequence, at most `cap` rows per group.
+void add_groups(std::vector<int>& r0, std::vector<int>& nr, std::vector<int>& sq, int row0, int rows, int seq, int cap) {
+  for (int t = 0; t < rows; t += cap) {
+    r0.push_back(row0 + t);
+    nr.push_back(std::min(cap, rows - t));
+    sq.push_back(seq);
+  }
+}
+
+}  // namespace
+
+// ------------------------------------------------------------------------------------------------
+// C ABI
+// ------------------------------------------------------------------------------------------------
+extern "C" {
+
+const char* sd2_last_error(const sd2_ctx* c) { return c ? c->err.c_str() : g_last_error.c_str(); }
+
+sd2_status sd2_init(const sd2_config* cfg, const sd2_weights* w, void* stream, sd2_ctx** out) {
+  sd2_ctx* c = nullptr;
+  if (!cfg || !w || !out) return fail(nullptr, SD2_EINVAL, "null argument");
+  *out = nullptr;
+  if (!valid_lm(cfg->verifier) || !valid_lm(cfg->drafter))
+    return fail(nullptr, SD2_EINVAL, "unsupported model shape (head_dim 64/128, dims multiple of 8, vocab of 4)");
+  if (cfg->verifier.vocab != cfg->drafter.vocab) return fail(nullptr, SD2_EINVAL, "verifier and drafter vocab differ");
+  if (cfg->k < 1 || cfg->k > 16) return fail(nullptr, SD2_EINVAL, "k must be in [1, 16]");
+  if (cfg->max_batch < 1 || cfg->max_batch > 256) return fail(nullptr, SD2_EINVAL, "max_batch must be in [1, 256]");
+  if (cfg->kv_block != 16) return fail(nullptr, SD2_EINVAL, "kv_block must be 16");
+  if (cfg->max_ctx < cfg->k + 3) return fail(nullptr, SD2_EINVAL, "max_ctx too small for one block");
+  if (cfg->d_steer <= 0 || cfg->d_steer % 8) return fail(nullptr, SD2_EINVAL, "d_steer must be a positive multiple of 8");
+  if (cfg->max_prefill_tokens < 1) return fail(nullptr, SD2_EINVAL, "max_prefill_tokens must be positive");
+  for (int t = 0; t < 3; ++t)
+    if (cfg->tap_layers[t] < 1 || cfg->tap_layers[t] > cfg->verifier.n_layers)
+      return fail(nullptr, SD2_EINVAL, "tap_layers must be 1-based verifier layers");
+  if (!aligned16(w->w_hml) || !aligned16(w->w_s) || !w->steer_ln_gamma || !w->steer_ln_beta)
+    return fail(nullptr, SD2_EINVAL, "steering weights null or not 16-byte aligned");
+
+  c = new sd2_ctx();
+  c->cfg = *cfg;
+  c->st = static_cast<cudaStream_t>(stream);
+  c->maxB = cfg->max_batch;
+  c->w_hml = w->w_hml; c->ln_g = w->steer_ln_gamma; c->ln_b = w->steer_ln_beta; c->w_s = w->w_s;
+  sd2_status s;
+  if ((s = load_model(c, c->V, cfg->verifier, w->verifier, "verifier")) != SD2_OK ||
+      (s = load_model(c, c->D, cfg->drafter, w->drafter, "drafter")) != SD2_OK) {
+    g_last_error = c->err;
+    sd2_free(c);
+    return s;
+  }
+  const int k = cfg->k, maxB = c->maxB, Vv = cfg->verifier.vocab;
+  const int step_rows = std::max(maxB * (k + 1), 2 * maxB);
+  c->max_rows = std::max(cfg->max_prefill_tokens, step_rows);
+  const int R = c->max_rows;
+  const int dmax = std::max(cfg->verifier.d_model, cfg->drafter.d_model);
+  const int fmax = std::max(cfg->verifier.d_ffn, cfg->drafter.d_ffn);
+  const int qkvmax = std::max(c->V.qkv_width(), c->D.qkv_width());
+  const int hmax = std::max(cfg->verifier.n_heads * cfg->verifier.head_dim, cfg->drafter.n_heads * cfg->drafter.head_dim);
+  const int splits = (cfg->max_ctx + 63) / 64;
+  const int hdmax = std::max(cfg->verifier.head_dim, cfg->drafter.head_dim);
+  const int headsmax = std::max(cfg->verifier.n_heads, cfg->drafter.n_heads);
+  auto go = [&]() -> sd2_status {
+    ALLOC(c->state, 4 * maxB);
+    ALLOC(c->committed, static_cast<size_t>(maxB) * cfg->max_ctx);
+    ALLOC(c->iter, 1);
+    ALLOC(c->xhat, static_cast<size_t>(maxB) * k);
+    ALLOC(c->temp, maxB);
+    ALLOC(c->errw, 1);
+    ALLOC(c->row_tok, R); ALLOC(c->row_pos, R); ALLOC(c->row_seq, R); ALLOC(c->row_valid, R);
+    c->statics_cap = 8 * R + 64;
+    ALLOC(c->statics, c->statics_cap);
+    ALLOC(c->x, static_cast<size_t>(R) * dmax);
+    ALLOC(c->a, static_cast<size_t>(R) * dmax * 2);
+    ALLOC(c->qkv, static_cast<size_t>(R) * qkvmax);
+    ALLOC(c->q, static_cast<size_t>(R) * hmax);
+    ALLOC(c->attn, static_cast<size_t>(R) * hmax * 2);
+    c->part_elems = static_cast<size_t>(step_rows) * headsmax * splits * (hdmax + 2);
+    ALLOC(c->part, c->part_elems);
+    ALLOC(c->h, static_cast<size_t>(R) * fmax * 2);
+    ALLOC(c->logits_t, static_cast<size_t>(maxB) * (k + 1) * Vv);
+    ALLOC(c->logits_d, static_cast<size_t>(maxB) * k * Vv);
+    ALLOC(c->taps, static_cast<size_t>(maxB) * (k + 1) * 3 * cfg->verifier.d_model);
+    ALLOC(c->hml_in, static_cast<size_t>(maxB) * 3 * cfg->verifier.d_model * 2);
+    ALLOC(c->g_pre, static_cast<size_t>(maxB) * cfg->d_steer);
+    ALLOC(c->g, static_cast<size_t>(maxB) * cfg->d_steer);
+    ALLOC(c->g_bf, static_cast<size_t>(maxB) * cfg->d_steer * 2);
+    ALLOC(c->bias, static_cast<size_t>(maxB) * cfg->drafter.n_layers * cfg->drafter.d_ffn);
+    ALLOC(c->samp_slot, maxB);
+    ALLOC(c->samp_counter, maxB);
+    void* acc;
+    ALLOC(acc, accept_scratch_bytes(maxB, k));
+    c->as = accept_scratch_carve(acc, maxB, k);
+    ALLOC(c->tok_out, static_cast<size_t>(maxB) * (k + 1));
+    ALLOC(c->n_out, maxB);
+    ALLOC(c->first, maxB);
+    ALLOC(c->cu, maxB + 1);
+    CK(cudaMemset(c->samp_slot, 0, sizeof(unsigned long long) * maxB));
+    CK(cudaMemset(c->samp_counter, 0, sizeof(int) * maxB));
+    CK(cudaMemset(c->errw, 0, sizeof(unsigned)));
+    CK(cudaMemset(c->state, 0, sizeof(int) * 4 * maxB));
+    CK(cudaMemset(c->taps, 0, sizeof(float) * static_cast<size_t>(maxB) * (k + 1) * 3 * cfg->verifier.d_model));
+    CK(cudaStreamCreateWithFlags(&c->cap_st, cudaStreamNonBlocking));
+    return SD2_OK;
+  };
+  if ((s = go()) != SD2_OK) {
+    g_last_error = c->err;
+    sd2_free(c);
+    return s;
+  }
+  *out = c;
+  return SD2_OK;
+}
+
+sd2_status sd2_prefill(sd2_ctx* c, int32_t batch, const int32_t* d_tokens, const int32_t* h_cu_lens,
+                       const float* h_temperature, uint64_t seed, int32_t* d_first_token) {
+  if (!c) return fail(nullptr, SD2_EINVAL, "null context");
+  if (!d_tokens || !h_cu_lens || !h_temperature) return fail(c, SD2_EINVAL, "null argument");
+  if (batch < 1 || batch > c->maxB) return fail(c, SD2_ECAPACITY, "batch exceeds max_batch");
+  const int k = c->cfg.k, V = c->V.c.vocab;
+  if (h_cu_lens[0] != 0) return fail(c, SD2_EINVAL, "h_cu_lens[0] must be 0");
+  int total = 0, maxlen = 0;
+  for (int b = 0; b < batch; ++b) {
+    const int len = h_cu_lens[b + 1] - h_cu_lens[b];
+    if (len < 1) return fail(c, SD2_EINVAL, "empty prompt");
+    if (len + k + 2 > c->cfg.max_ctx) return fail(c, SD2_ECAPACITY, "prompt too long for max_ctx");
+    if (!(h_temperature[b] >= 0.f) || !isfinite(h_temperature[b])) return fail(c, SD2_EINVAL, "bad temperature");
+    total += len;
+    maxlen = std::max(maxlen, len);
+  }
+  if (total > c->cfg.max_prefill_tokens) return fail(c, SD2_ECAPACITY, "prompt tokens exceed max_prefill_tokens");
+  drop_graphs(c);
+  c->B = batch;
+  c->seed = seed;
+  c->phase = 0;
+
+  // host-built plans: prefill rows, then the static groups of the step shapes
+  std::vector<int> pos(total), seq(total), valid(total, 1), logit_rows(batch), tap_row(total, -1);
+  for (int b = 0; b < batch; ++b) {
+    for (int t = h_cu_lens[b]; t < h_cu_lens[b + 1]; ++t) { pos[t] = t - h_cu_lens[b]; seq[t] = b; }
+    logit_rows[b] = h_cu_lens[b + 1] - 1;
+    tap_row[h_cu_lens[b + 1] - 1] = b * (k + 1);
+  }
+  std::vector<int> st;  // the statics buffer, assembled in order
+  auto push = [&](const std::vector<int>& v) { int off = (int)st.size(); st.insert(st.end(), v.begin(), v.end()); return off; };
+  auto groups_of = [&](const Model& m, std::vector<int>& r0, std::vector<int>& nr, std::vector<int>& sq, bool prefill) {
+    const int cap = m.group_rows();
+    for (int b = 0; b < batch; ++b) {
+      if (prefill) add_groups(r0, nr, sq, h_cu_lens[b], h_cu_lens[b + 1] - h_cu_lens[b], b, cap);
+    }
+  };
+  std::vector<int> vr0, vnr, vsq, dr0, dnr, dsq, d1r0, d1nr, d1sq, dnr0, dnnr, dnsq, sr0, snr, ssq, lr1;
+  groups_of(c->V, vr0, vnr, vsq, true);
+  groups_of(c->D, dr0, dnr, dsq, true);
+  for (int b = 0; b < batch; ++b) {
+    add_groups(d1r0, d1nr, d1sq, 2 * b, 2, b, c->D.group_rows());
+    add_groups(dnr0, dnnr, dnsq, b, 1, b, c->D.group_rows());
+    add_groups(sr0, snr, ssq, b * (k + 1), k + 1, b, c->V.group_rows());
+    lr1.push_back(2 * b + 1);
+  }
+  const int o_pos = push(pos), o_seq = push(seq), o_valid = push(valid), o_lr = push(logit_rows), o_tr = push(tap_row);
+  const int o_vr0 = push(vr0), o_vnr = push(vnr), o_vsq = push(vsq);
+  const int o_dr0 = push(dr0), o_dnr = push(dnr), o_dsq = push(dsq);
+  const int o_d1r0 = push(d1r0), o_d1nr = push(d1nr), o_d1sq = push(d1sq);
+  const int o_dnr0 = push(dnr0), o_dnnr = push(dnnr), o_dnsq = push(dnsq);
+  const int o_sr0 = push(sr0), o_snr = push(snr), o_ssq = push(ssq), o_lr1 = push(lr1);
+  std::vector<int> cu(h_cu_lens, h_cu_lens + batch + 1);
+  const int o_cu = push(cu);
+  if ((int)st.size() > c->statics_cap) return fail(c, SD2_ECAPACITY, "plan tables exceed their buffer");
+  CK(cudaMemcpyAsync(c->statics, st.data(), st.size() * sizeof(int), cudaMemcpyHostToDevice, c->st));
+  std::vector<float> temps(h_temperature, h_temperature + batch);
+  CK(cudaMemcpyAsync(c->temp, temps.data(), batch * sizeof(float), cudaMemcpyHostToDevice, c->st));
+  CK(cudaMemsetAsync(c->iter, 0, sizeof(int), c->st));
+  const int* S = c->statics;
+  Plan pv;
+  pv.M = total; pv.tok = d_tokens; pv.pos = S + o_pos; pv.seq = S + o_seq; pv.valid = S + o_valid;
+  pv.n_groups = (int)vr0.size(); pv.g_row0 = S + o_vr0; pv.g_nrows = S + o_vnr; pv.g_seq = S + o_vsq;
+  pv.n_splits = 1; pv.chunk = ((maxlen + 63) / 64) * 64;
+  Plan pd = pv;
+  pd.n_groups = (int)dr0.size(); pd.g_row0 = S + o_dr0; pd.g_nrows = S + o_dnr; pd.g_seq = S + o_dsq;
+  // step-shape plans (rows filled on the device each step)
+  const int splits = (c->cfg.max_ctx + 63) / 64;
+  auto step_plan = [&](int M, int ng, int o0, int o1, int o2) {
+    Plan p;
+    p.M = M; p.tok = c->row_tok; p.pos = c->row_pos; p.seq = c->row_seq; p.valid = c->row_valid;
+    p.n_groups = ng; p.g_row0 = S + o0; p.g_nrows = S + o1; p.g_seq = S + o2; p.n_splits = splits; p.chunk = 64;
+    return p;
+  };
+  c->p_d1 = step_plan(2 * batch, (int)d1r0.size(), o_d1r0, o_d1nr, o_d1sq);
+  c->p_dn = step_plan(batch, (int)dnr0.size(), o_dnr0, o_dnnr, o_dnsq);
+  c->p_v = step_plan(batch * (k + 1), (int)sr0.size(), o_sr0, o_snr, o_ssq);
+  c->logit_rows_d1 = S + o_lr1;
+
+  // verifier over the prompts: logits of each last row -> row b*(k+1) of the target buffer
+  FwdOut o;
+  o.taps = c->taps; o.tap_row = S + o_tr;
+  for (int t = 0; t < 3; ++t) o.tap_layers[t] = c->cfg.tap_layers[t];
+  o.logit_rows = S + o_lr; o.n_logit_rows = batch; o.logits = c->logits_t; o.ld_logits = static_cast<long long>(k + 1) * V;
+  sd2_status s = forward(c, c->V, pv, o);
+  if (s != SD2_OK) return s;
+  CK(sample_rows(c->logits_t, static_cast<long long>(k + 1) * V, batch, V, c->temp, seed, RNG_RESAMPLE, 0, nullptr, 0,
+                 c->first, 1, nullptr, 0, c->samp_slot, c->samp_counter, c->errw, c->st));
+  CK(prefill_init(batch, c->cfg.max_ctx, d_tokens, S + o_cu, c->first, c->state, c->maxB, c->committed, d_first_token,
+                  c->st));
+  // steering from the last prompt row (j = 0 -> tap row b*(k+1)), then the drafter prefill
+  s = steer(c, c->state + 2 * c->maxB);
+  if (s != SD2_OK) return s;
+  FwdOut od;
+  od.bias = c->bias;
+  s = forward(c, c->D, pd, od);
+  if (s != SD2_OK) return s;
+  const int one = 1;
+  CK(cudaMemcpyAsync(c->iter, &one, sizeof(int), cudaMemcpyHostToDevice, c->st));
+  CK(cudaStreamSynchronize(c->st));  // host staging buffers above go out of scope
+  c->phase = 1;
+  return SD2_OK;
+}
+
+sd2_status sd2_step(sd2_ctx* c) {
+  if (!c) return fail(nullptr, SD2_EINVAL, "null context");
+  if (c->phase != 1) return fail(c, SD2_ESTATE, "sd2_step needs a prefill or an accepted previous step");
+  if (c->prof) {
+    c->h_n.assign(c->B, 0);
+    CK(cudaMemcpyAsync(c->h_n.data(), c->state, sizeof(int) * c->B, cudaMemcpyDeviceToHost, c->st));
+    CK(cudaStreamSynchronize(c->st));
+  }
+  sd2_status s;
+  if (c->use_graphs && !c->prof) {
+    if (!c->g_step && (s = capture(c, &c->g_step, [&] { return run_step(c); })) != SD2_OK) return s;
+    CK(cudaGraphLaunch(c->g_step, c->st));
+  } else if ((s = run_step(c)) != SD2_OK) {
+    return s;
+  }
+  c->phase = 2;
+  return SD2_OK;
+}
+
+sd2_status sd2_accept(sd2_ctx* c, int32_t* d_tokens, int32_t* d_n) {
+  if (!c) return fail(nullptr, SD2_EINVAL, "null context");
+  if (c->phase != 2) return fail(c, SD2_ESTATE, "sd2_accept needs a preceding sd2_step");
+  if (!d_tokens || !d_n) return fail(c, SD2_EINVAL, "null output");
+  sd2_status s;
+  if (c->use_graphs && !c->prof) {
+    if (!c->g_accept && (s = capture(c, &c->g_accept, [&] { return run_accept(c); })) != SD2_OK) return s;
+    CK(cudaGraphLaunch(c->g_accept, c->st));
+  } else if ((s = run_accept(c)) != SD2_OK) {
+    return s;
+  }
+  CK(cudaMemcpyAsync(d_tokens, c->tok_out, sizeof(int) * c->B * (c->cfg.k + 1), cudaMemcpyDeviceToDevice, c->st));
+  CK(cudaMemcpyAsync(d_n, c->n_out, sizeof(int) * c->B, cudaMemcpyDeviceToDevice, c->st));
+  c->phase = 1;
+  return SD2_OK;
+}
+
+sd2_status sd2_check(sd2_ctx* c) {
+  if (!c) return fail(nullptr, SD2_EINVAL, "null context");
+  unsigned w = 0;
+  CK(cudaStreamSynchronize(c->st));
+  CK(cudaMemcpy(&w, c->errw, sizeof(unsigned), cudaMemcpyDeviceToHost));
+  CK(cudaMemset(c->errw, 0, sizeof(unsigned)));
+  if (w & ERR_NONFINITE) return fail(c, SD2_ENUMERIC, "non-finite logits seen on the device");
+  if (w & ERR_TIMEOUT) return fail(c, SD2_ETIMEOUT, "a device-side wait timed out");
+  return SD2_OK;
+}
+
+sd2_status sd2_set_graphs(sd2_ctx* c, int32_t enable) {
+  if (!c) return fail(nullptr, SD2_EINVAL, "null context");
+  c->use_graphs = enable != 0;
+  if (!c->use_graphs) drop_graphs(c);
+  return SD2_OK;
+}
+
+sd2_status sd2_free(sd2_ctx* c) {
+  if (!c) return SD2_OK;
+  if (c->st) cudaStreamSynchronize(c->st);
+  drop_graphs(c);
+  for (void* p : c->allocs) cudaFree(p);
+  for (auto& r : c->recs) { cudaEventDestroy(r.e0); cudaEventDestroy(r.e1); }
+  for (auto e : c->ev_pool) cudaEventDestroy(e);
+  if (c->cap_st) cudaStreamDestroy(c->cap_st);
+  delete c;
+  return SD2_OK;
+}
+
+sd2_status sd2_debug_buffer(const sd2_ctx* c, int32_t which, void** d_ptr, int64_t* n_elems, int32_t* dtype) {
+  if (!c || !d_ptr || !n_elems || !dtype) return fail(nullptr, SD2_EINVAL, "null argument");
+  const int64_t B = c->B, k = c->cfg.k, V = c->V.c.vocab;
+  switch (which) {
+    case 0: *d_ptr = c->logits_t; *n_elems = B * (k + 1) * V; *dtype = SD2_DTYPE_F32; break;
+    case 1: *d_ptr = c->logits_d; *n_elems = B * k * V; *dtype = SD2_DTYPE_F32; break;
+    case 2: *d_ptr = c->xhat; *n_elems = B * k; *dtype = -1; break;
+    case 3: *d_ptr = c->taps; *n_elems = B * (k + 1) * 3 * c->V.c.d_model; *dtype = SD2_DTYPE_F32; break;
+    case 4: *d_ptr = c->g; *n_elems = B * c->cfg.d_steer; *dtype = SD2_DTYPE_F32; break;
+    case 5: *d_ptr = c->bias; *n_elems = B * c->D.c.n_layers * c->D.c.d_ffn; *dtype = SD2_DTYPE_F32; break;
+    case 6: *d_ptr = c->committed; *n_elems = B * c->cfg.max_ctx; *dtype = -1; break;
+    case 7: *d_ptr = c->state; *n_elems = 4 * static_cast<int64_t>(c->maxB); *dtype = -1; break;
+    case 8: *d_ptr = c->iter; *n_elems = 1; *dtype = -1; break;
+    default: return fail(const_cast<sd2_ctx*>(c), SD2_EINVAL, "unknown buffer");
+  }
+  return SD2_OK;
+}
+
+sd2_status sd2_profile(sd2_ctx* c, int32_t enable) {
+  if (!c) return fail(nullptr, SD2_EINVAL, "null context");
+  c->prof = enable != 0;
+  for (auto& r : c->recs) { c->ev_pool.push_back(r.e0); c->ev_pool.push_back(r.e1); }
+  c->recs.clear();
+  return SD2_OK;
+}
+
+sd2_status sd2_profile_read(sd2_ctx* c, int64_t* launches, double* ms, double* bytes, int32_t n_classes) {
+  if (!c || !launches || !ms || !bytes) return fail(nullptr, SD2_EINVAL, "null argument");
+  CK(cudaStreamSynchronize(c->st));
+  for (int i = 0; i < n_classes; ++i) { launches[i] = 0; ms[i] = 0; bytes[i] = 0; }
+  for (auto& r : c->recs) {
+    if (r.cls >= n_classes) continue;
+    float t = 0;
+    CK(cudaEventElapsedTime(&t, r.e0, r.e1));
+    launches[r.cls] += 1;
+    ms[r.cls] += t;
+    bytes[r.cls] += r.bytes;
+  }
+  return SD2_OK;
+}
+
+// ------------------------------------------------------------------------------------------------
+// standalone kernels
+// ------------------------------------------------------------------------------------------------
+size_t sd2_accept_workspace_bytes(int32_t B, int32_t k) {
+  if (B < 1 || k < 1) return 0;
+  return (accept_scratch_bytes(B, k) + 255) / 256 * 256;
+}
+
+sd2_status sd2_accept_logits(const void* d_target, const void* d_draft, int32_t dtype, const int32_t* d_xhat,
+                             const float* d_temperature, int32_t B, int32_t k, int32_t V, uint64_t seed, uint32_t step,
+                             int32_t* d_tokens, int32_t* d_n, void* d_workspace, size_t workspace_bytes, void* stream) {
+  sd2_ctx* c = nullptr;
+  if (!d_target || !d_draft || !d_xhat || !d_temperature || !d_tokens || !d_n || !d_workspace)
+    return fail(nullptr, SD2_EINVAL, "null argument");
+  if (dtype != SD2_DTYPE_F32 && dtype != SD2_DTYPE_BF16) return fail(nullptr, SD2_EINVAL, "dtype must be F32 or BF16");
+  if (B < 1 || k < 1 || k > 64 || V < 4 || V % 4) return fail(nullptr, SD2_EINVAL, "need B >= 1, 1 <= k <= 64, V % 4 == 0");
+  if (workspace_bytes < sd2_accept_workspace_bytes(B, k)) return fail(nullptr, SD2_EINVAL, "workspace too small");
+  if (reinterpret_cast<uintptr_t>(d_workspace) & 255) return fail(nullptr, SD2_EINVAL, "workspace not 256-byte aligned");
+  const size_t align = dtype == SD2_DTYPE_F32 ? 16 : 8;
+  if ((reinterpret_cast<uintptr_t>(d_target) | reinterpret_cast<uintptr_t>(d_draft)) & (align - 1))
+    return fail(nullptr, SD2_EINVAL, "logits not aligned for vector loads");
+  unsigned* err = nullptr;
+  AcceptScratch s = accept_scratch_carve(d_workspace, B, k);
+  err = reinterpret_cast<unsigned*>(s.jmode + 2 * B);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  CK(cudaMemsetAsync(err, 0, sizeof(unsigned), st));
+  CK(accept_blocks(d_target, d_draft, dtype, d_xhat, d_temperature, B, k, V, seed, step, nullptr, nullptr, d_tokens, d_n,
+                   s, err, st));
+  return SD2_OK;
+}
+
+size_t sd2_steer_workspace_bytes(int32_t B, int32_t d_v, int32_t d_g) {
+  if (B < 1 || d_v < 1 || d_g < 1) return 0;
+  const size_t b = static_cast<size_t>(B);
+  return ((b * 3 * d_v * 2 + 255) / 256 + (b * d_g * 4 + 255) / 256 + (b * d_g * 2 + 255) / 256) * 256;
+}
+
+sd2_status sd2_steer(const float* d_taps, int32_t B, int32_t d_v, const void* w_hml, const void* ln_gamma,
+                     const void* ln_beta, float ln_eps, int32_t d_g, const void* w_s, int32_t n_bias, float* d_g_out,
+                     float* d_bias, void* d_workspace, size_t workspace_bytes, void* stream) {
+  sd2_ctx* c = nullptr;
+  if (!d_taps || !aligned16(w_hml) || !ln_gamma || !ln_beta || !aligned16(w_s) || !d_g_out || !d_bias || !d_workspace)
+    return fail(nullptr, SD2_EINVAL, "null or unaligned argument");
+  if (B < 1 || d_v < 1 || d_v % 8 || d_g < 1 || d_g % 8 || n_bias < 1)
+    return fail(nullptr, SD2_EINVAL, "need B >= 1 and d_v, d_g multiples of 8");
+  if (workspace_bytes < sd2_steer_workspace_bytes(B, d_v, d_g)) return fail(nullptr, SD2_EINVAL, "workspace too small");
+  if (reinterpret_cast<uintptr_t>(d_workspace) & 255) return fail(nullptr, SD2_EINVAL, "workspace not 256-byte aligned");
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  char* ws = static_cast<char*>(d_workspace);
+  const size_t b = static_cast<size_t>(B);
+  void* x_bf = ws;
+  float* g_pre = reinterpret_cast<float*>(ws + (b * 3 * d_v * 2 + 255) / 256 * 256);
+  void* g_bf = ws + (b * 3 * d_v * 2 + 255) / 256 * 256 + (b * d_g * 4 + 255) / 256 * 256;
+  CK(gather_rows_bf16(d_taps, 3 * d_v, nullptr, 3 * d_v, B, x_bf, st));
+  GemmArgs g{};
+  g.x = x_bf; g.ldx = 3 * d_v; g.M = B; g.K = 3 * d_v;
+  g.seg[0] = {w_hml, d_g}; g.nseg = 1; g.epi = EPI_STORE; g.out = g_pre; g.ldo = d_g;
+  CK(gemm(g, st));
+  CK(layernorm(g_pre, ln_gamma, ln_beta, ln_eps, B, d_g, d_g_out, g_bf, st));
+  GemmArgs gs{};
+  gs.x = g_bf; gs.ldx = d_g; gs.M = B; gs.K = d_g;
+  gs.seg[0] = {w_s, n_bias}; gs.nseg = 1; gs.epi = EPI_STORE; gs.out = d_bias; gs.ldo = n_bias;
+  CK(gemm(gs, st));
+  return SD2_OK;
+}
+
+sd2_status sd2_swiglu_steered(const float* d_gate, const float* d_up, const float* d_bias, const int32_t* d_seq,
+                              int32_t M, int32_t F, void* d_h, void* stream) {
+  sd2_ctx* c = nullptr;
+  if (!d_gate || !d_up || !d_h || M < 0 || F < 1) return fail(nullptr, SD2_EINVAL, "bad argument");
+  CK(swiglu(d_gate, d_up, d_bias, d_seq, M, F, d_h, static_cast<cudaStream_t>(stream)));
+  return SD2_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,116 @@
+// Host-side launchers of the SD^2 kernels (one declaration per kernel family). Every
+// launcher enqueues on `st` and returns the launch's cudaError_t.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+namespace sd2 {
+
+// ---------------------------------------------------------------- weight-streaming GEMM
+// Y[m, n] = sum_k X[m, k] W[n, k] for m < M, with W the row concatenation of up to three
+// bf16 segments (e.g. W_q | W_k | W_v). X is bf16 with row stride ldx; K % 8 == 0.
+enum GemmEpilogue {
+  EPI_STORE = 0,    // out[m*ldo + n] = y (f32)
+  EPI_ADD = 1,      // out[m*ldo + n] += y (f32 residual stream)
+  EPI_SWIGLU = 2,   // Eq. 2: h[m*ldh + f] = bf16((up + bias[seq[m]*ld_bias + f]) * SiLU(gate));
+                    //   segments: seg0 = W_gate [F, K], seg1 = W_up [F, K]
+};
+struct GemmSeg {
+  const void* w;
+  int rows;
+};
+struct GemmArgs {
+  const void* x;
+  int ldx, M, K;
+  GemmSeg seg[3];
+  int nseg;
+  int epi;
+  float* out;
+  int ldo;
+  void* out_bf;
+  int ldh;
+  const float* bias;
+  int ld_bias;
+  const int* row_seq;
+};
+cudaError_t gemm(const GemmArgs& a, cudaStream_t st);
+
+// ---------------------------------------------------------------- decoder elementwise
+// x[m] = embed[tok[m]] (f32), a[m] = bf16(RMSNorm(x[m]) * gamma); ids are clamped to [0, vocab).
+cudaError_t embed_rmsnorm(const int* tok, const void* embed, const void* gamma, float eps, int M, int d, int vocab,
+                          float* x, void* a, cudaStream_t st);
+// a[i] = bf16(RMSNorm(x[src(i)]) * gamma) for i < M, src(i) = rows ? rows[i] : i.
+// Taps: for each of up to 3 slots s with tap_mask bit s, tap[(tap_row[src] * 3 + s) * d] = x[src]
+// for source rows whose tap_row >= 0 (tap_row may be null = identity).
+cudaError_t rmsnorm(const float* x, const int* rows, const void* gamma, float eps, int M, int d, void* a,
+                    float* tap, const int* tap_row, int tap_mask, cudaStream_t st);
+// Rotary embedding + paged KV append. qkv [M, (H + 2 Hkv) hd] f32 -> q [M, H, hd] f32 (rotated);
+// rotated k and v go to the cache of `layer` at each valid row's (seq, pos).
+struct KVCache {
+  void* pool;          // bf16 [L][n_blocks][2][Hkv][16][hd]
+  const int* table;    // [max_batch, bt_stride] block ids
+  int bt_stride, n_blocks, Hkv, hd;
+};
+cudaError_t rope_append(const float* qkv, const float* rope_cs, int M, int H, int Hkv, int hd, const int* row_seq,
+                        const int* row_pos, const int* row_valid, const KVCache& kv, int layer, float* q,
+                        cudaStream_t st);
+// Steering layer norm: g = LN(x) * gamma + beta (f32 and bf16 copies), rows of width d.
+cudaError_t layernorm(const float* x, const void* gamma, const void* beta, float eps, int B, int d, float* g,
+                      void* g_bf, cudaStream_t st);
+// Steered SwiGLU on precomputed projections (standalone form of EPI_SWIGLU).
+cudaError_t swiglu(const float* gate, const float* up, const float* bias, const int* seq, int M, int F, void* h,
+                   cudaStream_t st);
+// f32 -> bf16 rows: out[b, :] = src[b*ld_src + off(b)*width .. +width], off(b) = idx ? idx[b] : 0.
+cudaError_t gather_rows_bf16(const float* src, int ld_src, const int* idx, int width, int B, void* out,
+                             cudaStream_t st);
+
+// ---------------------------------------------------------------- attention
+// Causal paged attention for query rows grouped by sequence: group g covers rows
+// grp_row0[g] .. +grp_nrows[g] of sequence grp_seq[g]; row r attends to cache positions
+// 0..row_pos[r]. The context is cut into splits of `chunk` positions (a multiple of 64);
+// with n_splits == 1 the result goes straight to out, otherwise partials are merged.
+struct AttnArgs {
+  const float* q;        // [M, H, hd] rotated queries
+  KVCache kv;
+  int layer;
+  const int* row_pos;
+  const int* grp_row0;
+  const int* grp_nrows;
+  const int* grp_seq;
+  int n_groups, M, H, hd;
+  int n_splits, chunk;
+  float* part;           // [M, H, n_splits, hd + 2] scratch (n_splits > 1)
+  void* out;             // [M, H * hd] bf16
+};
+cudaError_t attention(const AttnArgs& a, cudaStream_t st);
+
+// ---------------------------------------------------------------- sampling / acceptance
+// Scratch layout used by the acceptance kernels for R = B(2k+1) rows and B sequences.
+struct AcceptScratch {
+  unsigned long long* rowkey;   // [R] packed (max of z/T or z, argmax)
+  unsigned long long* rowsum;   // [R] fixed-point normaliser
+  unsigned long long* slot;     // [B, 2] race maxima (residual, log-form)
+  int* counter;                 // [B] CTAs finished in the race
+  int* jmode;                   // [B, 2] j and mode
+};
+size_t accept_scratch_bytes(int B, int k);
+AcceptScratch accept_scratch_carve(void* base, int B, int k);
+// Acceptance of B blocks. logits are f32 (dtype 0) or bf16 (1); target row stride ld_t
+// between consecutive rows of one sequence is V and sequence stride (k+1)V, likewise the draft
+// with kV. Writes tokens [B, k+1] and n [B]; n_live (optional) masks stopped sequences
+// (n_live[b] == 0 -> n[b] = 0). step_ptr (optional) overrides `step` from device memory.
+cudaError_t accept_blocks(const void* target, const void* draft, int dtype, const int* xhat, const float* temp,
+                          int B, int k, int V, unsigned long long seed, unsigned step, const int* step_ptr,
+                          const int* live, int* tokens, int* n, const AcceptScratch& s, unsigned* err,
+                          cudaStream_t st);
+// Token from one row per sequence (draft sample or bonus/first token): T = 0 -> argmax,
+// else the exponential race argmax_v (z_v/T - ln(-ln u_v)) with u from counter
+// (v>>2, purpose<<16 | i, b, step). Row of sequence b at logits + b*ld. The result goes to
+// out[b*ld_out] and, if out2, out2[b*ld_out2].
+cudaError_t sample_rows(const float* logits, long long ld, int B, int V, const float* temp, unsigned long long seed,
+                        int purpose, int i, const int* step_ptr, unsigned step, int* out, int ld_out, int* out2,
+                        int ld_out2, unsigned long long* slot, int* counter, unsigned* err, cudaStream_t st);
+
+}  // namespace sd2

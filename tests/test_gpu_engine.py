@@ -1,0 +1,116 @@
+"""End-to-end GPU parity of the SD^2 engine against the oracle (teacher-forced, see parity.py)."""
+import dataclasses
+
+import pytest
+import torch
+
+import parity
+from oracle import steering
+from oracle import model as omodel
+from paper_2511_09844_gb300 import sd2
+from paper_2511_09844_gb300 import workloads as W
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.mark.parametrize("temp", [0.0, 1.0])
+def test_tiny_single_sequence(temp):
+    work = parity.tiny_work()
+    vw, dw, st = parity.tiny_weights(work)
+    prompts = W.make_prompts(work.verifier.vocab, 1, (32, 32), seed=7)
+    rep = parity.run(work, vw, dw, st, prompts, [temp], seed=1234, n_steps=8)
+    assert rep.blocks == 8 and rep.decisions > 8 * work.k
+
+
+def test_tiny_ragged_batch_mixed_temperatures_gqa():
+    """Ragged prompts, per-sequence temperatures, grouped KV heads, block-crossing lengths."""
+    base = parity.tiny_work()
+    vs = W.shrink(base.verifier, n_kv_heads=2)
+    ds = W.shrink(base.drafter, n_kv_heads=1)
+    work = dataclasses.replace(base, verifier=vs, drafter=ds, k=5, batch=3)
+    vw, dw, st = parity.tiny_weights(work, seed=3)
+    prompts = W.make_prompts(vs.vocab, 3, (15, 49), seed=8)
+    rep = parity.run(work, vw, dw, st, prompts, [0.0, 0.7, 1.0], seed=77, n_steps=6)
+    assert rep.blocks == 18
+
+
+def test_high_acceptance_with_self_drafting():
+    """Drafter = verifier with W_s = 0 at T = 0: every block is fully accepted (tau = k + 1)."""
+    base = parity.tiny_work()
+    work = dataclasses.replace(base, drafter=base.verifier)
+    vw = W.make_lm_weights(work.verifier, 11, norm_jitter=0.1)
+    st = W.make_steering_weights(work, 12, zero_ws=True)
+    prompts = W.make_prompts(work.verifier.vocab, 2, (20, 33), seed=9)
+    rep = parity.run(work, vw, vw, st, prompts, [0.0, 0.0], seed=5, n_steps=5)
+    assert rep.accepted >= 0.8 * rep.blocks * work.k     # bf16 near-ties may cut a block short
+
+
+def test_graphs_and_direct_launches_agree():
+    work = parity.tiny_work()
+    vw, dw, st = parity.tiny_weights(work, seed=4)
+    prompts = W.make_prompts(work.verifier.vocab, 2, (30, 40), seed=10)
+    outs = []
+    for graphs in (True, False):
+        dev = [parity.to_device(x) for x in (vw, dw, st)]
+        eng = sd2.SD2Engine(work, *dev, max_batch=2, max_ctx=120, max_prefill_tokens=80)
+        eng.set_graphs(graphs)
+        eng.prefill(prompts, [1.0, 0.0], seed=42)
+        toks = []
+        for _ in range(6):
+            eng.step()
+            t, n = eng.accept()
+            toks.append((t.cpu().clone(), n.cpu().clone()))
+        outs.append(toks)
+        eng.close()
+    for (ta, na), (tb, nb) in zip(*outs):
+        assert torch.equal(na, nb)
+        for b in range(2):
+            assert torch.equal(ta[b, :na[b]], tb[b, :nb[b]])
+
+
+def test_capacity_stop_and_call_order():
+    work = parity.tiny_work()
+    vw, dw, st = parity.tiny_weights(work)
+    dev = [parity.to_device(x) for x in (vw, dw, st)]
+    eng = sd2.SD2Engine(work, *dev, max_batch=1, max_ctx=48, max_prefill_tokens=64)
+    with pytest.raises(sd2.SD2Error, match="ESTATE"):
+        eng.step()
+    with pytest.raises(sd2.SD2Error, match="ECAPACITY"):
+        eng.prefill([list(range(60))], [1.0], seed=1)
+    eng.prefill([list(range(30))], [1.0], seed=1)
+    with pytest.raises(sd2.SD2Error, match="ESTATE"):
+        eng.accept()
+    total = 0
+    stopped = False
+    for _ in range(24):
+        eng.step()
+        _, n = eng.accept()
+        m = int(n.cpu()[0])
+        total += m
+        if m == 0:
+            stopped = True
+            break
+    assert stopped
+    state = eng.buffer(sd2.BUF_STATE).view(4, -1)[:, 0].cpu()
+    assert int(state[3]) == 1 and int(state[0]) + work.k + 1 > 48 and int(state[0]) <= 48
+    eng.check()
+    eng.close()
+
+
+def test_standalone_steering_and_swiglu():
+    work = W.WORKLOADS["tiny"]
+    st = W.make_steering_weights(work, 3, ln_jitter=0.2)
+    taps = W.make_taps(5, work.verifier.d_model, seed=4)
+    nb = work.drafter.n_layers * work.drafter.d_ffn
+    g, bias = sd2.steer(taps.cuda(), parity.to_device(st), work.steer_ln_eps, nb)
+    g_ref = steering.steering_vector(taps, st, work.steer_ln_eps)
+    b_ref = steering.steering_bias(g_ref, st, work.drafter.n_layers, work.drafter.d_ffn).reshape(5, -1)
+    assert parity.row_rel_err(g, g_ref) < parity.TOL
+    assert parity.row_rel_err(bias, b_ref) < parity.TOL
+    gen = torch.Generator().manual_seed(1)
+    gate, up = torch.randn(7, 96, generator=gen), torch.randn(7, 96, generator=gen)
+    bb = torch.randn(3, 96, generator=gen)
+    seq = torch.tensor([0, 1, 2, 0, 1, 2, 2], dtype=torch.int32)
+    h = sd2.swiglu_steered(gate.cuda(), up.cuda(), bb.cuda(), seq.cuda())
+    ref = (up + bb[seq.long()]) * omodel.silu(gate)
+    assert parity.row_rel_err(h, ref) < 1e-2
