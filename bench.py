@@ -1,0 +1,408 @@
+"""Benchmark of the SD^2 hot path: one draft-and-verify iteration (steering, k drafter steps, the
+verifier over k+1 rows, acceptance and rollback) per step, on synthetic inputs.
+
+Default workload: a Llama-3-8B-shaped verifier with a Llama-3.2-1B-shaped drafter, batch 1,
+prompt 512 uniform-random ids, k = 5, T = 1.0 (random-init bf16 weights N(0, 0.02^2)).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference] [--workload NAME]
+
+Prints one JSON line. `value` is emitted tokens per second per sequence (N > 1: summed over the
+N independent replicas). The reference arm times the CPU oracle on a bounded slice of the same
+workload (a few decoder layers, scaled to the full depth).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import torch  # noqa: E402
+
+from paper_2511_09844_gb300 import workloads as W  # noqa: E402
+
+METRIC = "steered-SD emitted tokens/sec/sequence at 1 GB300; verify-step HBM GB/s vs 8 TB/s"
+NOMINAL_HBM_GBS = 8000.0
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=32)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="llama8b_1b", choices=sorted(W.WORKLOADS))
+    ap.add_argument("--seed", type=int, default=1234)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    return ap.parse_args()
+
+
+def measured_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return json.load(f), "measured"
+    except OSError:
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0}, "fallback"
+
+
+def workload_config(work, n_gpus, extra=None):
+    cfg = {"workload": work.name + ": " + work.description, "batch_per_gpu": work.batch,
+           "prompt_len": list(work.prompt_len), "k": work.k, "temperature": work.temperatures[-1],
+           "gen_tokens": work.gen_tokens, "parallelism": f"replicas x{n_gpus}",
+           "l2": "no flush: the weights streamed every step (%.1f GB) exceed the 126 MB L2" % (
+               2e-9 * (work.verifier.param_count() + work.drafter.param_count()))}
+    if extra:
+        cfg.update(extra)
+    return cfg
+
+
+# ---------------------------------------------------------------------------------------------
+# clocks sampled during the timed region
+# ---------------------------------------------------------------------------------------------
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+        self.lines = []
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except OSError:
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def __exit__(self, *a):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in self.lines:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx.append(float(parts[2]))
+            except ValueError:
+                continue
+            for name, flag in zip(names, parts[5:9]):
+                if flag.lower().startswith("active"):
+                    reasons.add(name)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ---------------------------------------------------------------------------------------------
+# our arm
+# ---------------------------------------------------------------------------------------------
+def make_device_weights(work, seed, device):
+    vw = W.make_lm_weights(work.verifier, seed, device=device)
+    dw = W.make_lm_weights(work.drafter, seed + 1, device=device)
+    st = W.make_steering_weights(work, seed + 2, device=device)
+    return vw, dw, st
+
+
+def run_ours(args, rank, world, local_rank):
+    from paper_2511_09844_gb300 import build as _build
+    from paper_2511_09844_gb300 import sd2
+    _build.build()
+    torch.cuda.set_device(local_rank)
+    dev = f"cuda:{local_rank}"
+    work = W.WORKLOADS[args.workload]
+    B, k, V = work.batch, work.k, work.verifier.vocab
+    temp = work.temperatures[-1]
+    prompts = W.make_prompts(V, B, work.prompt_len, seed=7 + rank)
+    steps_total = args.warmup + 2 * args.steps + 2
+    max_ctx = max(len(p) for p in prompts) + steps_total * (k + 1) + k + 8
+    vw, dw, st = make_device_weights(work, args.seed, dev)
+    stream = torch.cuda.current_stream()
+    eng = sd2.SD2Engine(work, vw, dw, st, max_batch=B, max_ctx=max_ctx,
+                        max_prefill_tokens=sum(len(p) for p in prompts), stream=stream)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    eng.prefill(prompts, [temp] * B, seed=args.seed + rank)
+    torch.cuda.synchronize()
+    prefill_s = time.perf_counter() - t0
+
+    tok_all = torch.zeros((args.steps, B, k + 1), dtype=torch.int32, device=dev)
+    n_all = torch.zeros((args.steps, B), dtype=torch.int32, device=dev)
+
+    def one_step(i):
+        eng.step()
+        eng.accept(tok_all[i], n_all[i])
+
+    for i in range(args.warmup):
+        one_step(i % args.steps)
+    torch.cuda.synchronize()
+    n_all.zero_()
+    barrier(world)
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(local_rank) as clocks:
+        torch.cuda.synchronize()
+        ev0.record(stream)
+        for i in range(args.steps):
+            one_step(i)
+        ev1.record(stream)
+        torch.cuda.synchronize()
+    barrier(world)
+    ms = ev0.elapsed_time(ev1)
+    emitted = int(n_all.sum().item())
+    ms_max, emitted_all = reduce_max_sum(ms, emitted, world)
+    value = emitted_all / B / (ms_max / 1e3)
+    tau = emitted / (args.steps * B)
+
+    # end to end through the public API: step, accept, read the emitted tokens back into pinned
+    # host memory every step (the per-step work of a serving loop; no per-step host input exists)
+    h_tok = torch.empty((B, k + 1), dtype=torch.int32, pin_memory=True)
+    h_n = torch.empty(B, dtype=torch.int32, pin_memory=True)
+    e2e_emitted = 0
+    torch.cuda.synchronize()
+    barrier(world)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        eng.step()
+        tok, n = eng.accept()
+        h_tok.copy_(tok, non_blocking=True)
+        h_n.copy_(n, non_blocking=True)
+        stream.synchronize()
+        e2e_emitted += int(h_n.sum())
+    e2e_s = time.perf_counter() - t0
+    e2e_s_max, e2e_all = reduce_max_sum(e2e_s * 1e3, e2e_emitted, world)
+    e2e_value = e2e_all / B / (e2e_s_max / 1e3)
+
+    # one more pass with per-launch CUDA events on the engine's stream (no graphs) for the
+    # roofline of the dominant kernel and the per-stage bandwidth
+    prof_steps = min(args.steps, 8)
+    eng.profile(True)
+    for _ in range(prof_steps):
+        eng.step()
+        eng.accept()
+    prof = eng.profile_read()
+    eng.profile(False)
+    eng.check()
+    peaks, peak_src = measured_peaks()
+    hbm = float(peaks["hbm_gbs"])
+    g = prof["gemm"]
+    gemm_gbs = g["bytes"] / (g["ms"] / 1e3) / 1e9 if g["ms"] else 0.0
+    ver, dra = prof["verify"], prof["draft"]
+    verify_gbs = ver["bytes"] / (ver["ms"] / 1e3) / 1e9 if ver["ms"] else 0.0
+    draft_gbs = dra["bytes"] / (dra["ms"] / 1e3) / 1e9 if dra["ms"] else 0.0
+    launches_per_step = sum(v["launches"] for name, v in prof.items()
+                            if name in ("gemm", "attention", "accept", "sample", "other")) / prof_steps
+    step_ms_prof = sum(v["ms"] for name, v in prof.items() if name in ("verify", "draft", "steer")) / prof_steps
+    gemm_share = g["ms"] / max(1e-9, sum(prof[c]["ms"] for c in ("gemm", "attention", "accept", "sample", "other")))
+    eng.close()
+    keep = (vw, dw, st) if (rank == 0 and world == 1 and not args.no_cpu_baseline) else None
+    del vw, dw, st
+
+    line = {
+        "metric": METRIC, "value": round(value, 3), "unit": "tokens/s/sequence", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_max / args.steps, 4),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic: random-init bf16 weights N(0, 0.02^2), uniform-random prompt ids",
+        "config": workload_config(work, world, {"max_ctx": max_ctx}),
+        "tau": round(tau, 4),
+        "tokens_per_s_at_paper_tau": {"tau": 5.00, "value": round(5.00 / (ms_max / args.steps / 1e3), 2)},
+        "prefill_s": round(prefill_s, 3),
+        "e2e": {"value": round(e2e_value, 3), "unit": "tokens/s/sequence", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": int(h_tok.numel() * 4 + h_n.numel() * 4)},
+        "roofline": {"bound": "hbm", "kernel": "weight-streaming GEMM (all projections + lm_head)",
+                     "achieved": round(gemm_gbs, 1), "peak": hbm, "unit": "GB/s",
+                     "frac": round(gemm_gbs / hbm, 4), "traffic": None,
+                     "peak_source": f"{peak_src} hbm_gbs (MEASURED_PEAKS.json)" if peak_src == "measured" else
+                     "fallback 6800 GB/s", "time_share": round(gemm_share, 4),
+                     "timing": f"CUDA events per launch on the engine stream over {prof_steps} profiled steps"},
+        "stages": {"verify_gbs": round(verify_gbs, 1), "verify_frac_of_8tbs": round(verify_gbs / NOMINAL_HBM_GBS, 4),
+                   "verify_frac_of_measured": round(verify_gbs / hbm, 4),
+                   "verify_ms": round(ver["ms"] / max(1, ver["launches"]), 4),
+                   "draft_step_gbs": round(draft_gbs, 1), "draft_step_frac_of_measured": round(draft_gbs / hbm, 4),
+                   "draft_step_ms": round(dra["ms"] / max(1, dra["launches"]), 4),
+                   "steer_ms": round(prof["steer"]["ms"] / max(1, prof["steer"]["launches"]), 4),
+                   "profiled_step_ms": round(step_ms_prof, 4)},
+        "gpu_launches": int(round(launches_per_step * args.steps)),
+        "clocks": clocks.summary(),
+    }
+    return line, work, tau, keep
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def reduce_max_sum(ms, count, world):
+    if world == 1:
+        return ms, count
+    import torch.distributed as dist
+    t = torch.tensor([ms], dtype=torch.float64, device="cuda")
+    c = torch.tensor([count], dtype=torch.float64, device="cuda")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    dist.all_reduce(c, op=dist.ReduceOp.SUM)
+    return float(t.item()), int(c.item())
+
+
+# ---------------------------------------------------------------------------------------------
+# the oracle on the host cores (reference arm and cpu_baseline)
+# ---------------------------------------------------------------------------------------------
+class OracleSlices:
+    """The oracle on two slices of the workload (1 and 2 decoder layers per model, same widths,
+    same context); the difference prices one layer, which scales the slice to the full depth.
+    Weights: the first layers of the given models (copied to the host), or freshly generated."""
+
+    def __init__(self, work, seed, weights=None):
+        import dataclasses
+        self.work = work
+        self.context = work.prompt_len[0]
+        two_v = dataclasses.replace(work.verifier, n_layers=2)
+        two_d = dataclasses.replace(work.drafter, n_layers=2)
+        if weights is None:
+            sw2 = dataclasses.replace(work, verifier=two_v, drafter=two_d)
+            vw, dw, st = (W.make_lm_weights(two_v, seed), W.make_lm_weights(two_d, seed + 1),
+                          W.make_steering_weights(sw2, seed + 2))
+        else:
+            vw, dw, st = weights
+
+        def host(w, n):
+            return {"embed": w["embed"].cpu(), "final_norm": w["final_norm"].cpu(), "lm_head": w["lm_head"].cpu(),
+                    "layers": [{k: v.cpu() for k, v in lw.items()} for lw in w["layers"][:n]]}
+
+        vh, dh = host(vw, 2), host(dw, 2)
+        F = work.drafter.d_ffn
+        sth = {k: v.cpu() for k, v in st.items()}
+        self.slices = []
+        for n in (1, 2):
+            vs = dataclasses.replace(work.verifier, n_layers=n)
+            ds = dataclasses.replace(work.drafter, n_layers=n)
+            sw = dataclasses.replace(work, verifier=vs, drafter=ds)
+            v_n = dict(vh, layers=vh["layers"][:n])
+            d_n = dict(dh, layers=dh["layers"][:n])
+            st_n = dict(sth, w_s=sth["w_s"][:n * F])
+            self.slices.append((sw, v_n, d_n, st_n))
+        self.prompt = W.make_prompts(work.verifier.vocab, 1, (self.context, self.context), seed=7)[0]
+        self.seed = seed
+
+    def _iteration(self, sl):
+        from oracle.sd import OracleSD
+        sw, vw, dw, st = sl
+        ora = OracleSD(sw, vw, dw, st, self.seed)
+        ora.prefill([self.prompt], [self.work.temperatures[-1]], forced_first=[1])
+        t0 = time.perf_counter()
+        out = ora.stage(0, 1)
+        emitted, j = ora.accept(0, 1, out)
+        ora.commit(0, emitted, j, out["taps"])
+        return time.perf_counter() - t0
+
+    def estimate(self):
+        """(seconds per iteration scaled to full depth, seconds of CPU work measured)."""
+        t1 = self._iteration(self.slices[0])
+        t2 = self._iteration(self.slices[1])
+        per_pair = max(0.0, t2 - t1)                       # one verifier layer + one drafter layer (x k)
+        fixed = max(0.0, t1 - per_pair)
+        work = self.work
+        vcost = work.verifier.param_count() / work.verifier.n_layers
+        dcost = work.k * work.drafter.param_count() / work.drafter.n_layers
+        v_share = vcost / (vcost + dcost)
+        full = fixed + per_pair * (v_share * work.verifier.n_layers + (1 - v_share) * work.drafter.n_layers)
+        return full, t1 + t2
+
+    def sample_text(self, measured, tau):
+        w = self.work
+        return (f"oracle iterations (fp32, full recompute, no KV cache) on 1- and 2-layer slices of the "
+                f"same shapes at context {self.context}, scaled to {w.verifier.n_layers} verifier + "
+                f"{w.drafter.n_layers} drafter layers; {round(measured, 1)} s of CPU work; tau {round(tau, 3)}")
+
+
+def run_reference(args, rank, world):
+    if rank != 0:
+        return None
+    work = W.WORKLOADS[args.workload]
+    sl = OracleSlices(work, args.seed)
+    tau = float(os.environ.get("SD2_REFERENCE_TAU", "1.0"))
+    for _ in range(args.warmup):
+        sl.estimate()
+    per_step, cpu_s = [], 0.0
+    t_start = time.perf_counter()
+    for _ in range(args.steps):
+        est, measured = sl.estimate()
+        per_step.append(est)
+        cpu_s += measured
+        if time.perf_counter() - t_start > 150:      # keep the arm within a few minutes
+            break
+    t_iter = statistics.median(per_step)
+    value = tau / t_iter
+    return {
+        "impl": "reference", "metric": METRIC, "value": round(value, 6), "unit": "tokens/s/sequence",
+        "n_gpus": world, "steps": len(per_step), "warmup": args.warmup, "ms_per_step": round(t_iter * 1e3, 2),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+        "data": "synthetic: random-init weights N(0, 0.02^2), uniform-random prompt ids",
+        "config": workload_config(work, 1),
+        "cpu_baseline": {"value": round(value, 6), "unit": "tokens/s/sequence", "cores": torch.get_num_threads(),
+                         "kind": "oracle", "sample": sl.sample_text(cpu_s, tau)},
+        "e2e": {"value": round(value, 6), "unit": "tokens/s/sequence", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+
+
+def cpu_baseline(work, seed, tau, weights=None):
+    sl = OracleSlices(work, seed, weights)
+    est, measured = sl.estimate()
+    return {"value": round(tau / est, 6), "unit": "tokens/s/sequence", "cores": torch.get_num_threads(),
+            "kind": "oracle", "seconds_per_iteration": round(est, 3), "sample": sl.sample_text(measured, tau)}
+
+
+def main():
+    args = parse()
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        backend = "nccl" if args.impl == "ours" else "gloo"
+        if backend == "nccl":
+            torch.cuda.set_device(local_rank)
+        dist.init_process_group(backend)
+    if args.impl == "reference":
+        line = run_reference(args, rank, world)
+    else:
+        line, work, tau, keep = run_ours(args, rank, world, local_rank)
+        if keep is not None:
+            line["cpu_baseline"] = cpu_baseline(work, args.seed, tau, keep)
+    if rank == 0 and line is not None:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

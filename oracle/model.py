@@ -93,7 +93,7 @@ def forward(shape, w: Dict, tokens: Sequence[int], bias: Optional[torch.Tensor] 
     tok = torch.as_tensor(list(tokens), dtype=torch.long)
     T = tok.numel()
     pos = torch.arange(T)
-    x = w["embed"].float()[tok]
+    x = w["embed"][tok].float()
     taps = {}
     H, Hkv, hd = shape.n_heads, shape.n_kv_heads, shape.head_dim
     for li, lw in enumerate(w["layers"]):
