@@ -193,6 +193,25 @@ sd2_status sd2_steer(const float* d_taps, int32_t B, int32_t d_v, const void* w_
 sd2_status sd2_swiglu_steered(const float* d_gate, const float* d_up, const float* d_bias,
                               const int32_t* d_seq, int32_t M, int32_t F, void* d_h, void* stream);
 
+/* The acceptance of sd2_accept_logits without any device allocation by the caller or by the
+ * library. (An addition of this library: the paper has no counterpart.) It is for callers that
+ * cannot call cudaMalloc, for example code living in a process whose device memory is owned by
+ * another component's allocator, or a loop that must not risk the device-wide synchronisation a
+ * cudaMalloc/cudaFree can cause. Arguments and outputs are those of sd2_accept_logits, minus the
+ * workspace: the scratch is a fixed 256 KiB device array inside the library, held on every GPU
+ * that loads it until the process exits. The tables take 16*B*(2k+1) + 28*B + 68 bytes; requests
+ * above 262144 bytes (256 KiB) return SD2_ECAPACITY (B = 256 with k = 16 needs 142404 bytes).
+ *   - The first call on each device looks up the array's device address (cudaGetSymbolAddress)
+ *     with that device current; make that first call before any stream capture.
+ *   - Every call on a device shares the one array and leaves its contents behind; the call
+ *     clears what must start at zero. Calls whose GPU work overlaps (other streams, other host
+ *     threads) race on the array: order them on one stream.
+ *   - Errors: the status, with the text in sd2_last_error(NULL). */
+sd2_status sd2_accept_logits_noalloc(const void* d_target, const void* d_draft, int32_t dtype,
+                                     const int32_t* d_xhat, const float* d_temperature, int32_t B,
+                                     int32_t k, int32_t V, uint64_t seed, uint32_t step,
+                                     int32_t* d_tokens, int32_t* d_n, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

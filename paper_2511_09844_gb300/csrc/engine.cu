@@ -434,6 +434,11 @@ void add_groups(std::vector<int>& r0, std::vector<int>& nr, std::vector<int>& sq
 
 }  // namespace
 
+namespace sd2 {
+// Sets the text sd2_last_error(NULL) returns, for context-free entry points in other files.
+void record_last_error(const std::string& m) { g_last_error = m; }
+}  // namespace sd2
+
 // ------------------------------------------------------------------------------------------------
 // C ABI
 // ------------------------------------------------------------------------------------------------

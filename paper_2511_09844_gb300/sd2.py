@@ -26,7 +26,8 @@ PROFILE_CLASSES = ["gemm", "attention", "accept", "sample", "other", "verify", "
 
 EXPORTS = ["sd2_init", "sd2_prefill", "sd2_step", "sd2_accept", "sd2_check", "sd2_free", "sd2_last_error",
            "sd2_set_graphs", "sd2_debug_buffer", "sd2_profile", "sd2_profile_read", "sd2_accept_workspace_bytes",
-           "sd2_accept_logits", "sd2_steer_workspace_bytes", "sd2_steer", "sd2_swiglu_steered"]
+           "sd2_accept_logits", "sd2_steer_workspace_bytes", "sd2_steer", "sd2_swiglu_steered",
+           "sd2_accept_logits_noalloc"]
 
 
 class LMConfig(ctypes.Structure):
