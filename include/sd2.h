@@ -187,6 +187,24 @@ sd2_status sd2_steer(const float* d_taps, int32_t B, int32_t d_v, const void* w_
                      const void* ln_beta, float ln_eps, int32_t d_g, const void* w_s, int32_t n_bias,
                      float* d_g_out, float* d_bias, void* d_workspace, size_t workspace_bytes, void* stream);
 
+/* Weight-streaming GEMM of the decoder on caller buffers, Y[m, n] = sum_k X[m, k] W[n, k]:
+ *   d_x [M, ldx] bf16 (first K columns used), d_w [N, K] bf16 (nn.Linear layout).
+ *   epilogue 0: d_out[m*ldo + n] = Y (f32); 1: d_out[m*ldo + n] += Y (the residual add);
+ *   2: the steered SwiGLU of Eq. 2 with d_w = W_gate, d_w_up = W_up (both [N, K]):
+ *      d_h[m*N + f] = bf16((up + d_bias[seq[m]*ld_bias + f]) * SiLU(gate)), d_bias/d_seq optional.
+ *   impl 0: tensor cores (tcgen05, TMA) where the shape allows (K % 64 == 0; N % 128 == 0, or
+ *   N % 64 == 0 for epilogue 2), else CUDA cores; 1: CUDA cores; 2: tensor cores or SD2_EINVAL.
+ *   d_workspace: sd2_gemm_workspace_bytes(M) bytes, 256-byte aligned, for impl 0 and 2. */
+size_t sd2_gemm_workspace_bytes(int32_t M);
+sd2_status sd2_gemm(const void* d_x, int32_t ldx, int32_t M, int32_t K, const void* d_w, const void* d_w_up,
+                    int32_t N, int32_t epilogue, float* d_out, int32_t ldo, void* d_h, const float* d_bias,
+                    const int32_t* d_seq, int32_t ld_bias, int32_t impl, void* d_workspace,
+                    size_t workspace_bytes, void* stream);
+
+/* Choose the GEMM of a context: 0 tensor cores where the shape allows (default), 1 CUDA cores.
+ * Drops captured graphs. */
+sd2_status sd2_set_gemm_impl(sd2_ctx* ctx, int32_t impl);
+
 /* Steered SwiGLU activation of Eq. 2 on caller buffers (the injection step of a2):
  *   h[m, f] = (up[m, f] + bias[seq[m], f]) * SiLU(gate[m, f]) as bf16, with gate/up [M, F] f32,
  *   bias [*, F] f32 (row seq[m]; d_seq may be null for bias row 0), h [M, F] bf16. */

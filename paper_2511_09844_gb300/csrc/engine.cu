@@ -91,6 +91,10 @@ struct sd2_ctx {
   float *taps = nullptr, *g_pre = nullptr, *g = nullptr, *bias = nullptr;
   void *a = nullptr, *attn = nullptr, *h = nullptr, *g_bf = nullptr, *hml_in = nullptr;
   size_t part_elems = 0;
+  float* gemm_ws = nullptr;     // tensor-core GEMM: split-tile partials
+  int* gemm_cnt = nullptr;      // tensor-core GEMM: per-tile arrival counters (zero between launches)
+  size_t gemm_cnt_len = 0;
+  int gemm_impl = 0;            // 0 tensor cores where the shape allows, 1 CUDA cores
   unsigned long long* samp_slot = nullptr;
   int* samp_counter = nullptr;
   AcceptScratch as{};
@@ -228,6 +232,16 @@ struct FwdOut {
   long long ld_logits = 0;
 };
 
+// The tensor-core GEMM's scratch and the implementation choice, attached to every GEMM launch.
+GemmArgs& tc(sd2_ctx* c, GemmArgs& g) {
+  g.ws = c->gemm_ws;
+  g.counters = c->gemm_cnt;
+  g.counters_len = c->gemm_cnt_len;
+  g.err = c->errw;
+  g.impl = c->gemm_impl;
+  return g;
+}
+
 double gemm_bytes(int M, int N, int K, int out_bytes) {
   return 2.0 * N * K + 2.0 * M * K + static_cast<double>(out_bytes) * M * N;
 }
@@ -258,7 +272,7 @@ sd2_status forward(sd2_ctx* c, const Model& m, const Plan& p, const FwdOut& o) {
     g.seg[1] = {m.W(l, SD2_W_K), Hkv * hd};
     g.seg[2] = {m.W(l, SD2_W_V), Hkv * hd};
     g.nseg = 3; g.epi = EPI_STORE; g.out = c->qkv; g.ldo = m.qkv_width();
-    CK(timed(c, PC_GEMM, gemm_bytes(M, m.qkv_width(), d, 4), [&] { return gemm(g, c->st); }));
+    CK(timed(c, PC_GEMM, gemm_bytes(M, m.qkv_width(), d, 4), [&] { return gemm(tc(c, g), c->st); }));
     CK(timed(c, PC_OTHER, 0, [&] {
       return rope_append(c->qkv, m.rope_cs, M, H, Hkv, hd, p.seq, p.pos, p.valid, m.cache(), l, c->q, c->st);
     }));
@@ -274,7 +288,7 @@ sd2_status forward(sd2_ctx* c, const Model& m, const Plan& p, const FwdOut& o) {
     GemmArgs go{};
     go.x = c->attn; go.ldx = H * hd; go.M = M; go.K = H * hd;
     go.seg[0] = {m.W(l, SD2_W_O), d}; go.nseg = 1; go.epi = EPI_ADD; go.out = c->x; go.ldo = d;
-    CK(timed(c, PC_GEMM, gemm_bytes(M, d, H * hd, 8), [&] { return gemm(go, c->st); }));
+    CK(timed(c, PC_GEMM, gemm_bytes(M, d, H * hd, 8), [&] { return gemm(tc(c, go), c->st); }));
     CK(timed(c, PC_OTHER, 0, [&] {
       return rmsnorm(c->x, nullptr, m.W(l, SD2_W_MLP_NORM), mc.norm_eps, M, d, c->a, nullptr, nullptr, 0, c->st);
     }));
@@ -284,11 +298,11 @@ sd2_status forward(sd2_ctx* c, const Model& m, const Plan& p, const FwdOut& o) {
     gu.epi = EPI_SWIGLU; gu.out_bf = c->h; gu.ldh = F;
     gu.bias = o.bias ? o.bias + static_cast<size_t>(l) * F : nullptr;
     gu.ld_bias = L * F; gu.row_seq = p.seq;
-    CK(timed(c, PC_GEMM, gemm_bytes(M, 2 * F, d, 1), [&] { return gemm(gu, c->st); }));
+    CK(timed(c, PC_GEMM, gemm_bytes(M, 2 * F, d, 1), [&] { return gemm(tc(c, gu), c->st); }));
     GemmArgs gd{};
     gd.x = c->h; gd.ldx = F; gd.M = M; gd.K = F;
     gd.seg[0] = {m.W(l, SD2_W_DOWN), d}; gd.nseg = 1; gd.epi = EPI_ADD; gd.out = c->x; gd.ldo = d;
-    CK(timed(c, PC_GEMM, gemm_bytes(M, d, F, 8), [&] { return gemm(gd, c->st); }));
+    CK(timed(c, PC_GEMM, gemm_bytes(M, d, F, 8), [&] { return gemm(tc(c, gd), c->st); }));
   }
   if (o.n_logit_rows > 0 || tap_mask(L)) {
     const int nr = o.n_logit_rows > 0 ? o.n_logit_rows : M;
@@ -301,7 +315,7 @@ sd2_status forward(sd2_ctx* c, const Model& m, const Plan& p, const FwdOut& o) {
     gl.x = c->a; gl.ldx = d; gl.M = o.n_logit_rows; gl.K = d;
     gl.seg[0] = {m.lm_head, mc.vocab}; gl.nseg = 1; gl.epi = EPI_STORE; gl.out = o.logits;
     gl.ldo = static_cast<int>(o.ld_logits);
-    CK(timed(c, PC_GEMM, gemm_bytes(o.n_logit_rows, mc.vocab, d, 4), [&] { return gemm(gl, c->st); }));
+    CK(timed(c, PC_GEMM, gemm_bytes(o.n_logit_rows, mc.vocab, d, 4), [&] { return gemm(tc(c, gl), c->st); }));
   }
   return SD2_OK;
 }
@@ -316,14 +330,14 @@ sd2_status steer(sd2_ctx* c, const int* row_idx) {
   GemmArgs g{};
   g.x = c->hml_in; g.ldx = 3 * dv; g.M = B; g.K = 3 * dv;
   g.seg[0] = {c->w_hml, dg}; g.nseg = 1; g.epi = EPI_STORE; g.out = c->g_pre; g.ldo = dg;
-  CK(timed(c, PC_GEMM, gemm_bytes(B, dg, 3 * dv, 4), [&] { return gemm(g, c->st); }));
+  CK(timed(c, PC_GEMM, gemm_bytes(B, dg, 3 * dv, 4), [&] { return gemm(tc(c, g), c->st); }));
   CK(timed(c, PC_OTHER, 0, [&] {
     return layernorm(c->g_pre, c->ln_g, c->ln_b, c->cfg.steer_ln_eps, B, dg, c->g, c->g_bf, c->st);
   }));
   GemmArgs gs{};
   gs.x = c->g_bf; gs.ldx = dg; gs.M = B; gs.K = dg;
   gs.seg[0] = {c->w_s, nb}; gs.nseg = 1; gs.epi = EPI_STORE; gs.out = c->bias; gs.ldo = nb;
-  CK(timed(c, PC_GEMM, gemm_bytes(B, nb, dg, 4), [&] { return gemm(gs, c->st); }));
+  CK(timed(c, PC_GEMM, gemm_bytes(B, nb, dg, 4), [&] { return gemm(tc(c, gs), c->st); }));
   return SD2_OK;
 }
 
@@ -514,6 +528,10 @@ sd2_status sd2_init(const sd2_config* cfg, const sd2_weights* w, void* stream, s
     ALLOC(c->g, static_cast<size_t>(maxB) * cfg->d_steer);
     ALLOC(c->g_bf, static_cast<size_t>(maxB) * cfg->d_steer * 2);
     ALLOC(c->bias, static_cast<size_t>(maxB) * cfg->drafter.n_layers * cfg->drafter.d_ffn);
+    c->gemm_cnt_len = 1 << 20;
+    ALLOC(c->gemm_ws, gemm_tc_workspace_floats(R));
+    ALLOC(c->gemm_cnt, c->gemm_cnt_len);
+    CK(cudaMemset(c->gemm_cnt, 0, sizeof(int) * c->gemm_cnt_len));
     ALLOC(c->samp_slot, maxB);
     ALLOC(c->samp_counter, maxB);
     void* acc;
@@ -698,6 +716,14 @@ sd2_status sd2_set_graphs(sd2_ctx* c, int32_t enable) {
   return SD2_OK;
 }
 
+sd2_status sd2_set_gemm_impl(sd2_ctx* c, int32_t impl) {
+  if (!c) return fail(nullptr, SD2_EINVAL, "null context");
+  if (impl != 0 && impl != 1) return fail(c, SD2_EINVAL, "impl must be 0 (tensor cores) or 1 (CUDA cores)");
+  c->gemm_impl = impl;
+  drop_graphs(c);
+  return SD2_OK;
+}
+
 sd2_status sd2_free(sd2_ctx* c) {
   if (!c) return SD2_OK;
   if (c->st) cudaStreamSynchronize(c->st);
@@ -814,6 +840,51 @@ sd2_status sd2_steer(const float* d_taps, int32_t B, int32_t d_v, const void* w_
   gs.x = g_bf; gs.ldx = d_g; gs.M = B; gs.K = d_g;
   gs.seg[0] = {w_s, n_bias}; gs.nseg = 1; gs.epi = EPI_STORE; gs.out = d_bias; gs.ldo = n_bias;
   CK(gemm(gs, st));
+  return SD2_OK;
+}
+
+size_t sd2_gemm_workspace_bytes(int32_t M) {
+  if (M < 1) return 0;
+  return ((gemm_tc_workspace_floats(M) * 4 + 255) / 256 + (static_cast<size_t>(1 << 20) * 4) / 256) * 256;
+}
+
+sd2_status sd2_gemm(const void* d_x, int32_t ldx, int32_t M, int32_t K, const void* d_w, const void* d_w_up,
+                    int32_t N, int32_t epilogue, float* d_out, int32_t ldo, void* d_h, const float* d_bias,
+                    const int32_t* d_seq, int32_t ld_bias, int32_t impl, void* d_workspace, size_t workspace_bytes,
+                    void* stream) {
+  sd2_ctx* c = nullptr;
+  if (!d_x || !d_w || M < 1 || K < 8 || K % 8 || ldx < K || ldx % 8 || N < 1)
+    return fail(nullptr, SD2_EINVAL, "bad GEMM shape or null input");
+  if (epilogue < EPI_STORE || epilogue > EPI_SWIGLU) return fail(nullptr, SD2_EINVAL, "unknown epilogue");
+  if (epilogue == EPI_SWIGLU ? (!d_w_up || !d_h) : (!d_out || ldo < N))
+    return fail(nullptr, SD2_EINVAL, "missing output for the epilogue");
+  if (impl < 0 || impl > 2) return fail(nullptr, SD2_EINVAL, "impl must be 0, 1 or 2");
+  GemmArgs g{};
+  g.x = d_x; g.ldx = ldx; g.M = M; g.K = K;
+  g.seg[0] = {d_w, N};
+  g.nseg = 1;
+  if (epilogue == EPI_SWIGLU) { g.seg[1] = {d_w_up, N}; g.nseg = 2; }
+  g.epi = epilogue; g.out = d_out; g.ldo = ldo; g.out_bf = d_h; g.ldh = N;
+  g.bias = d_bias; g.ld_bias = ld_bias; g.row_seq = d_seq;
+  g.impl = impl == 1 ? 1 : 0;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if (impl != 1) {
+    if (!d_workspace || workspace_bytes < sd2_gemm_workspace_bytes(M))
+      return fail(nullptr, SD2_EINVAL, "tensor-core GEMM needs sd2_gemm_workspace_bytes(M) of workspace");
+    if (reinterpret_cast<uintptr_t>(d_workspace) & 255) return fail(nullptr, SD2_EINVAL, "workspace not 256-aligned");
+    const size_t ws_bytes = (gemm_tc_workspace_floats(M) * 4 + 255) / 256 * 256;
+    g.ws = static_cast<float*>(d_workspace);
+    g.counters = reinterpret_cast<int*>(static_cast<char*>(d_workspace) + ws_bytes);
+    g.counters_len = 1 << 20;
+    g.err = nullptr;
+    if (impl == 2 && !gemm_tc_supported(g))
+      return fail(nullptr, SD2_EINVAL, "shape not supported by the tensor-core GEMM (K % 64, rows % 128)");
+    CK(cudaMemsetAsync(g.counters, 0, sizeof(int) * g.counters_len, st));
+    static unsigned* err_word = nullptr;  // a device word for the timeout flag of standalone calls
+    if (!err_word) CK(cudaMalloc(&err_word, sizeof(unsigned)));
+    g.err = err_word;
+  }
+  CK(gemm(g, st));
   return SD2_OK;
 }
 

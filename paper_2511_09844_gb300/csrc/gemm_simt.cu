@@ -108,6 +108,12 @@ __global__ void __launch_bounds__(kThreads) gemm_simt_kernel(const GemmArgs a, i
 }  // namespace
 
 cudaError_t gemm(const GemmArgs& a, cudaStream_t st) {
+  if (a.ws && a.counters && a.impl != 1 && gemm_tc_supported(a))
+    return gemm_tc(a, a.ws, a.counters, a.counters_len, a.err, st);
+  return gemm_simt(a, st);
+}
+
+cudaError_t gemm_simt(const GemmArgs& a, cudaStream_t st) {
   int n_total = 0;
   for (int s = 0; s < a.nseg; ++s) n_total += a.seg[s].rows;
   const int n_units = (a.epi == EPI_SWIGLU) ? a.seg[0].rows : (n_total + 1) / 2;

@@ -34,8 +34,22 @@ struct GemmArgs {
   const float* bias;
   int ld_bias;
   const int* row_seq;
+  // tensor-core path: fp32 split-tile partials, per-tile arrival counters (zero between
+  // launches), the device error word; impl 0 = tensor cores when the shape allows, 1 = CUDA cores
+  float* ws;
+  int* counters;
+  size_t counters_len;
+  unsigned* err;
+  int impl;
 };
+// Dispatches to the tcgen05 kernel (gemm_tc.cu) when ws is set, impl != 1 and gemm_tc_supported
+// holds, else to the CUDA-core kernel (gemm_simt.cu).
 cudaError_t gemm(const GemmArgs& a, cudaStream_t st);
+bool gemm_tc_supported(const GemmArgs& a);
+cudaError_t gemm_tc(const GemmArgs& a, float* ws, int* counters, size_t counters_len, unsigned* err, cudaStream_t st);
+int gemm_tc_token_tile(int M);
+size_t gemm_tc_workspace_floats(int max_M);
+cudaError_t gemm_simt(const GemmArgs& a, cudaStream_t st);
 
 // ---------------------------------------------------------------- decoder elementwise
 // x[m] = embed[tok[m]] (f32), a[m] = bf16(RMSNorm(x[m]) * gamma); ids are clamped to [0, vocab).

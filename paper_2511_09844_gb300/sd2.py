@@ -27,7 +27,7 @@ PROFILE_CLASSES = ["gemm", "attention", "accept", "sample", "other", "verify", "
 EXPORTS = ["sd2_init", "sd2_prefill", "sd2_step", "sd2_accept", "sd2_check", "sd2_free", "sd2_last_error",
            "sd2_set_graphs", "sd2_debug_buffer", "sd2_profile", "sd2_profile_read", "sd2_accept_workspace_bytes",
            "sd2_accept_logits", "sd2_steer_workspace_bytes", "sd2_steer", "sd2_swiglu_steered",
-           "sd2_accept_logits_noalloc"]
+           "sd2_accept_logits_noalloc", "sd2_gemm_workspace_bytes", "sd2_gemm", "sd2_set_gemm_impl"]
 
 
 class LMConfig(ctypes.Structure):
@@ -83,8 +83,16 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
     lib.sd2_steer.argtypes = [c_void_p, c_int32, c_int32, c_void_p, c_void_p, c_void_p, c_float, c_int32, c_void_p,
                               c_int32, c_void_p, c_void_p, c_void_p, c_size_t, c_void_p]
     lib.sd2_swiglu_steered.argtypes = [c_void_p, c_void_p, c_void_p, c_void_p, c_int32, c_int32, c_void_p, c_void_p]
+    lib.sd2_gemm_workspace_bytes.argtypes = [c_int32]
+    lib.sd2_gemm_workspace_bytes.restype = c_size_t
+    lib.sd2_gemm.argtypes = [c_void_p, c_int32, c_int32, c_int32, c_void_p, c_void_p, c_int32, c_int32, c_void_p,
+                             c_int32, c_void_p, c_void_p, c_void_p, c_int32, c_int32, c_void_p, c_size_t, c_void_p]
+    lib.sd2_set_gemm_impl.argtypes = [c_void_p, c_int32]
+    lib.sd2_accept_logits_noalloc.argtypes = [c_void_p, c_void_p, c_int32, c_void_p, c_void_p, c_int32, c_int32,
+                                              c_int32, c_uint64, c_uint32, c_void_p, c_void_p, c_void_p]
     for name in EXPORTS:
-        if name not in ("sd2_last_error", "sd2_accept_workspace_bytes", "sd2_steer_workspace_bytes"):
+        if name not in ("sd2_last_error", "sd2_accept_workspace_bytes", "sd2_steer_workspace_bytes",
+                        "sd2_gemm_workspace_bytes"):
             getattr(lib, name).restype = c_int32
     _LIB = lib
     return lib
@@ -209,6 +217,10 @@ class SD2Engine:
         torch.cuda.synchronize()
         return torch.as_tensor(_DeviceView(p.value, n.value, typestr), device="cuda").clone()
 
+    def set_gemm_impl(self, impl: int):
+        """0: tensor-core GEMM where the shape allows (default); 1: CUDA-core GEMM."""
+        self._call(self.lib.sd2_set_gemm_impl(self.ctx, impl))
+
     def profile(self, enable: bool):
         self._call(self.lib.sd2_profile(self.ctx, 1 if enable else 0))
 
@@ -270,3 +282,23 @@ def swiglu_steered(gate: torch.Tensor, up: torch.Tensor, bias: Optional[torch.Te
     h = torch.empty((M, F), dtype=torch.bfloat16, device=gate.device)
     _check(lib, lib.sd2_swiglu_steered(_ptr(gate), _ptr(up), _ptr(bias), _ptr(seq), M, F, _ptr(h), _stream(stream)))
     return h
+
+
+def gemm(x: torch.Tensor, w: torch.Tensor, epilogue: int = 0, out: Optional[torch.Tensor] = None,
+         w_up: Optional[torch.Tensor] = None, bias: Optional[torch.Tensor] = None,
+         seq: Optional[torch.Tensor] = None, impl: int = 0, stream=None):
+    """Standalone weight-streaming GEMM (sd2_gemm). epilogue 0: returns X W^T (f32); 1: adds it into
+    `out`; 2: steered SwiGLU with w = W_gate, w_up = W_up, returns bf16 [M, N]."""
+    lib = load_library()
+    M, K = x.shape
+    N = w.shape[0]
+    h = None
+    if epilogue == 0 and out is None:
+        out = torch.empty((M, N), dtype=torch.float32, device=x.device)
+    if epilogue == 2:
+        h = torch.empty((M, N), dtype=torch.bfloat16, device=x.device)
+    ws = torch.empty(lib.sd2_gemm_workspace_bytes(M), dtype=torch.uint8, device=x.device)
+    _check(lib, lib.sd2_gemm(_ptr(x), x.stride(0), M, K, _ptr(w), _ptr(w_up), N, epilogue, _ptr(out),
+                             0 if out is None else out.stride(0), _ptr(h), _ptr(bias), _ptr(seq),
+                             0 if bias is None else bias.stride(0), impl, _ptr(ws), ws.numel(), _stream(stream)))
+    return h if epilogue == 2 else out
