@@ -27,6 +27,8 @@ constexpr int smem_bytes() {
 
 template <int HD>
 __global__ void __launch_bounds__(kWarps * 32) attn_kernel(const AttnArgs a) {
+  pdl_trigger();
+  pdl_wait();
   constexpr int DPL = HD / 32;        // output dims per lane
   constexpr int KS = HD + 8;          // padded smem row (bf16 elements)
   extern __shared__ __align__(16) unsigned char smem[];
@@ -158,6 +160,8 @@ __global__ void __launch_bounds__(kWarps * 32) attn_kernel(const AttnArgs a) {
 // Merge the splits of one (row, head): out = sum_s acc_s e^{m_s - M} / sum_s l_s e^{m_s - M}.
 template <int HD>
 __global__ void __launch_bounds__(HD) attn_merge_kernel(const AttnArgs a) {
+  pdl_trigger();
+  pdl_wait();
   const int row = blockIdx.x / a.H, h = blockIdx.x % a.H;
   const int ns = min(a.n_splits, a.row_pos[row] / a.chunk + 1);
   const float* p = a.part + (static_cast<size_t>(row) * a.H + h) * a.n_splits * (HD + 2);
@@ -182,10 +186,10 @@ cudaError_t launch(const AttnArgs& a, cudaStream_t st) {
     configured = true;
   }
   dim3 grid(a.n_groups, a.kv.Hkv, a.n_splits);
-  attn_kernel<HD><<<grid, kWarps * 32, smem_bytes<HD>(), st>>>(a);
+  { const cudaError_t e_ = launch_pdl(attn_kernel<HD>, dim3(grid), dim3(kWarps * 32), smem_bytes<HD>(), st, a); if (e_ != cudaSuccess) return e_; }
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess || a.n_splits == 1) return e;
-  attn_merge_kernel<HD><<<a.M * a.H, HD, 0, st>>>(a);
+  { const cudaError_t e_ = launch_pdl(attn_merge_kernel<HD>, dim3(a.M * a.H), dim3(HD), 0, st, a); if (e_ != cudaSuccess) return e_; }
   return cudaGetLastError();
 }
 

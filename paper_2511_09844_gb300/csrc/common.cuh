@@ -164,6 +164,15 @@ __device__ __forceinline__ float packed_key(unsigned long long p) {
   return unord_f32(static_cast<uint32_t>(p >> 32));
 }
 
+// ------------------------------------------------------------------------------------------
+// Programmatic dependent launch: every kernel of the hot path is launched so that it may start
+// while its predecessor finishes. pdl_trigger lets the successor be scheduled; pdl_wait blocks
+// until the predecessor grid has completed and its writes are visible. A kernel touches no
+// global memory written by earlier kernels, and writes none, before pdl_wait.
+// ------------------------------------------------------------------------------------------
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
 // Device error word bits (latched; read and cleared by the host).
 enum { ERR_NONFINITE = 1, ERR_TIMEOUT = 2 };
 

@@ -17,7 +17,7 @@
 #include <string>
 #include <vector>
 
-#include "../../include/sd2.h"
+#include "sd2.h"
 #include "common.cuh"
 #include "kernels.h"
 #include "state.h"
@@ -879,7 +879,9 @@ sd2_status sd2_gemm(const void* d_x, int32_t ldx, int32_t M, int32_t K, const vo
     g.err = nullptr;
     if (impl == 2 && !gemm_tc_supported(g))
       return fail(nullptr, SD2_EINVAL, "shape not supported by the tensor-core GEMM (K % 64, rows % 128)");
-    CK(cudaMemsetAsync(g.counters, 0, sizeof(int) * g.counters_len, st));
+    const size_t tiles = static_cast<size_t>(epilogue == EPI_SWIGLU ? (N + 63) / 64 : (N + 127) / 128) *
+                         ((M + gemm_tc_token_tile(M) - 1) / gemm_tc_token_tile(M));
+    CK(cudaMemsetAsync(g.counters, 0, sizeof(int) * std::min(tiles, g.counters_len), st));
     static unsigned* err_word = nullptr;  // a device word for the timeout flag of standalone calls
     if (!err_word) CK(cudaMalloc(&err_word, sizeof(unsigned)));
     g.err = err_word;

@@ -32,6 +32,8 @@ __device__ __forceinline__ const bf16* seg_row(const GemmArgs& a, int n) {
 
 template <int EPI>
 __global__ void __launch_bounds__(kThreads) gemm_simt_kernel(const GemmArgs a, int n_units, int n_total) {
+  pdl_trigger();
+  pdl_wait();
   const int lane = threadIdx.x & 31;
   const int warp = (blockIdx.x * kThreads + threadIdx.x) >> 5;
   const int n_warps = (gridDim.x * kThreads) >> 5;
@@ -122,9 +124,9 @@ cudaError_t gemm_simt(const GemmArgs& a, cudaStream_t st) {
   const int cap = 152 * 8;
   if (blocks > cap) blocks = cap;
   switch (a.epi) {
-    case EPI_STORE: gemm_simt_kernel<EPI_STORE><<<blocks, kThreads, 0, st>>>(a, n_units, n_total); break;
-    case EPI_ADD: gemm_simt_kernel<EPI_ADD><<<blocks, kThreads, 0, st>>>(a, n_units, n_total); break;
-    default: gemm_simt_kernel<EPI_SWIGLU><<<blocks, kThreads, 0, st>>>(a, n_units, n_total); break;
+    case EPI_STORE: { const cudaError_t e_ = launch_pdl(gemm_simt_kernel<EPI_STORE>, dim3(blocks), dim3(kThreads), 0, st, a, n_units, n_total); if (e_ != cudaSuccess) return e_; } break;
+    case EPI_ADD: { const cudaError_t e_ = launch_pdl(gemm_simt_kernel<EPI_ADD>, dim3(blocks), dim3(kThreads), 0, st, a, n_units, n_total); if (e_ != cudaSuccess) return e_; } break;
+    default: { const cudaError_t e_ = launch_pdl(gemm_simt_kernel<EPI_SWIGLU>, dim3(blocks), dim3(kThreads), 0, st, a, n_units, n_total); if (e_ != cudaSuccess) return e_; } break;
   }
   return cudaGetLastError();
 }

@@ -219,7 +219,7 @@ __device__ __forceinline__ void finish_chunk(const TcArgs& a, int wt, int tt, in
   }
 }
 
-__global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_constant__ TcArgs a) {
+__global__ void __launch_bounds__(kThreads, 2) gemm_tc_kernel(const __grid_constant__ TcArgs a) {
   extern __shared__ unsigned char smem_raw[];
   unsigned char* smem =
       reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -264,31 +264,63 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
   const long long lo = cta_lo(c, U, G), hi = cta_lo(c + 1, U, G);
   volatile int* abort_flag = flags;
 
+  pdl_trigger();                             // the next kernel may start its own prologue
   if (warp == 0) {
     if (lane == 0) {
-      uint32_t j = 0;
-      bool ok = true;
-      for (long long u = lo; u < hi && ok;) {
-        const Seg sg = segment(u, hi, a.KB);
-        const int wt = sg.tile % a.n_wtiles, tt = sg.tile / a.n_wtiles;
-        int seg = 0, row0 = wt * kWRows;
+      // Stage use j loads k-block (lo + j) of this CTA's range: the weight half first, then the
+      // token half. Weights never depend on earlier kernels, so the first stages' weight tiles
+      // are requested before waiting for the predecessor grid. Cursors advance one k-block at a
+      // time (no divisions in the issue loop: this one thread feeds the whole SM).
+      const uint32_t n_units = static_cast<uint32_t>(hi - lo);
+      struct Cursor {
+        int tile, kb, wt, tt, seg, row0;
+      };
+      auto locate = [&](Cursor& c) {
+        c.wt = c.tile % a.n_wtiles;
+        c.tt = c.tile / a.n_wtiles;
+        c.seg = 0;
+        c.row0 = c.wt * kWRows;
         if (!a.swiglu)
-          while (seg + 1 < a.nseg && row0 >= a.seg_rows[seg]) row0 -= a.seg_rows[seg++];
-        for (int i = 0; i < sg.nkb; ++i, ++j) {
-          const uint32_t s = j % S;
-          if (!wait_bar(empty0 + 8 * s, ((j / S) & 1) ^ 1, abort_flag, a.err)) { ok = false; break; }
-          const uint32_t dst = smem_u32(smem + static_cast<size_t>(s) * stage_bytes);
-          mbar_expect_tx(full0 + 8 * s, stage_bytes);
-          const int k0 = (sg.kb + i) * kBK;
-          if (a.swiglu) {
-            tma_load_2d(dst, &a.mapA[0], k0, wt * 64, full0 + 8 * s);
-            tma_load_2d(dst + a_bytes / 2, &a.mapA[1], k0, wt * 64, full0 + 8 * s);
-          } else {
-            tma_load_2d(dst, &a.mapA[seg], k0, row0, full0 + 8 * s);
-          }
-          tma_load_2d(dst + a_bytes, &a.mapB, k0, tt * NT, full0 + 8 * s);
+          while (c.seg + 1 < a.nseg && c.row0 >= a.seg_rows[c.seg]) c.row0 -= a.seg_rows[c.seg++];
+      };
+      auto advance = [&](Cursor& c) {
+        if (++c.kb == a.KB) { c.kb = 0; ++c.tile; locate(c); }
+      };
+      Cursor ca, cb;
+      ca.tile = static_cast<int>(lo / a.KB);
+      ca.kb = static_cast<int>(lo % a.KB);
+      locate(ca);
+      cb = ca;
+      auto load_a = [&](uint32_t j, const Cursor& c) {
+        const uint32_t s = j % S;
+        const uint32_t dst = smem_u32(smem + static_cast<size_t>(s) * stage_bytes);
+        if (a.swiglu) {
+          tma_load_2d(dst, &a.mapA[0], c.kb * kBK, c.wt * 64, full0 + 8 * s);
+          tma_load_2d(dst + a_bytes / 2, &a.mapA[1], c.kb * kBK, c.wt * 64, full0 + 8 * s);
+        } else {
+          tma_load_2d(dst, &a.mapA[c.seg], c.kb * kBK, c.row0, full0 + 8 * s);
         }
-        u += sg.nkb;
+      };
+      auto load_b = [&](uint32_t j, const Cursor& c) {
+        const uint32_t s = j % S;
+        const uint32_t dst = smem_u32(smem + static_cast<size_t>(s) * stage_bytes);
+        tma_load_2d(dst + a_bytes, &a.mapB, c.kb * kBK, c.tt * NT, full0 + 8 * s);
+      };
+      const uint32_t pre = n_units < static_cast<uint32_t>(S) ? n_units : static_cast<uint32_t>(S);
+      for (uint32_t j = 0; j < pre; ++j, advance(ca)) {   // first use of each stage: no wait
+        mbar_expect_tx(full0 + 8 * j, stage_bytes);
+        load_a(j, ca);
+      }
+      pdl_wait();
+      for (uint32_t j = 0; j < pre; ++j, advance(cb)) load_b(j, cb);
+      uint32_t j = pre;
+      bool ok = true;
+      for (; j < n_units; ++j, advance(ca)) {
+        const uint32_t s = j % S;
+        if (!wait_bar(empty0 + 8 * s, ((j / S) & 1) ^ 1, abort_flag, a.err)) { ok = false; break; }
+        mbar_expect_tx(full0 + 8 * s, stage_bytes);
+        load_a(j, ca);
+        load_b(j, ca);
       }
       if (!ok) {  // let the loads already issued land before the CTA exits
         const uint32_t done = static_cast<uint32_t>(flags[3]);
@@ -330,6 +362,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
     const int q = warp & 3;                   // TMEM lane quarter of this warp
     const int r = q * 32 + lane;              // weight row within the tile
     const bool leader = (warp == 2 && lane == 0);
+    pdl_wait();                              // outputs, residuals and biases come from earlier kernels
     uint32_t segi = 0;
     for (long long u = lo; u < hi; ++segi) {
       const Seg sg = segment(u, hi, a.KB);
@@ -370,13 +403,13 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
         if (lane == 0) mbar_arrive(tempty0 + 8 * acc);
         const long long t_lo = static_cast<long long>(sg.tile) * a.KB, t_hi = t_lo + a.KB;
         const int c1 = cta_of(t_lo, U, G), c2 = cta_of(t_hi - 1, U, G);
-        __threadfence();
-        named_bar_epi();
+        named_bar_epi();                       // every partial row of this CTA is written
         if (leader) {
+          __threadfence();                     // release them (cumulative over the barrier)
           const int old = atomicAdd(&a.counters[sg.tile], 1);
           const bool last = (old == c2 - c1);
           if (last) a.counters[sg.tile] = 0;
-          __threadfence();
+          __threadfence();                     // acquire the other CTAs' partials
           flags[2] = last ? 1 : 0;
         }
         named_bar_epi();
@@ -386,6 +419,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
             float v[16];
 #pragma unroll
             for (int j = 0; j < 16; ++j) v[j] = 0.f;
+#pragma unroll 8
             for (int cc = c1; cc <= c2; ++cc) {
               const int sl = (cta_lo(cc, U, G) / a.KB == sg.tile) ? 0 : 1;
               const float* src = a.ws + ((static_cast<size_t>(cc) * 2 + sl) * kWRows + r) * NT + ch * 16;
@@ -476,6 +510,7 @@ int sm_count() {
 }
 
 constexpr int kSmemBudget = 227 * 1024;
+constexpr int kSmemShared = 110 * 1024;
 
 }  // namespace
 
@@ -522,7 +557,10 @@ cudaError_t gemm_tc(const GemmArgs& g, float* ws, int* counters, size_t counters
   a.ws = ws; a.counters = counters; a.err = err;
   const int stage_bytes = (kWRows + a.NT) * kBK * 2;
   const int fixed = 1024 + 64 * 17 * 4 + 64 + 8 * (2 * 16 + 6);
-  int S = (kSmemBudget - fixed) / stage_bytes;
+  // Up to NT = 128 the ring fits in half an SM's shared memory (and the two accumulators in half
+  // of TMEM), so the next GEMM's CTA can start on the same SM while this one drains.
+  int S = (kSmemShared - fixed) / stage_bytes;
+  if (a.NT > 128 || S < 3) S = (kSmemBudget - fixed) / stage_bytes;
   if (S > 8) S = 8;
   if (S < 2) return cudaErrorInvalidValue;
   a.stages = S;
@@ -533,11 +571,15 @@ cudaError_t gemm_tc(const GemmArgs& g, float* ws, int* counters, size_t counters
     if (e != cudaSuccess) return e;
     configured = true;
   }
+  // At least kMinUnits k-blocks (kMinUnits x 16 KB of weights) per CTA: fewer CTAs share a
+  // tile, so the last one to arrive sums fewer partials.
+  constexpr long long kMinUnits = 8;
   long long G = sm_count();
+  const long long g_cap = (a.units + kMinUnits - 1) / kMinUnits;
+  if (G > g_cap) G = g_cap;
   if (G > a.units) G = a.units;
   if (G > 512) G = 512;
-  gemm_tc_kernel<<<static_cast<int>(G), kThreads, smem, st>>>(a);
-  return cudaGetLastError();
+  return launch_pdl(gemm_tc_kernel, dim3(static_cast<unsigned>(G)), dim3(kThreads), static_cast<size_t>(smem), st, a);
 }
 
 }  // namespace sd2

@@ -6,7 +6,26 @@
 #include <stddef.h>
 #include <stdint.h>
 
+#include <utility>
+
 namespace sd2 {
+
+// Launch with programmatic stream serialisation (see pdl_wait / pdl_trigger in common.cuh).
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                       Args&&... args) {
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
 
 // ---------------------------------------------------------------- weight-streaming GEMM
 // Y[m, n] = sum_k X[m, k] W[n, k] for m < M, with W the row concatenation of up to three

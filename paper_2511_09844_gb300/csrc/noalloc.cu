@@ -15,7 +15,7 @@
 #include <mutex>
 #include <string>
 
-#include "../../include/sd2.h"
+#include "sd2.h"
 #include "common.cuh"
 #include "kernels.h"
 

@@ -33,6 +33,8 @@ __device__ __forceinline__ void write_normed(const float* xr, const bf16* gamma,
 
 __global__ void __launch_bounds__(kNormThreads) embed_rmsnorm_kernel(const int* tok, const bf16* embed, const bf16* gamma,
                                                                       float eps, int d, int vocab, float* x, bf16* a) {
+  pdl_trigger();
+  pdl_wait();
   __shared__ float red[32];
   const int m = blockIdx.x;
   const int t = min(max(tok[m], 0), vocab - 1);  // ids outside the vocabulary read row 0 / V-1
@@ -51,6 +53,8 @@ __global__ void __launch_bounds__(kNormThreads) embed_rmsnorm_kernel(const int* 
 __global__ void __launch_bounds__(kNormThreads) rmsnorm_kernel(const float* x, const int* rows, const bf16* gamma,
                                                                 float eps, int d, bf16* a, float* tap,
                                                                 const int* tap_row, int tap_mask) {
+  pdl_trigger();
+  pdl_wait();
   __shared__ float red[32];
   const int i = blockIdx.x;
   const int src = rows ? rows[i] : i;
@@ -73,6 +77,8 @@ __global__ void __launch_bounds__(kNormThreads) rmsnorm_kernel(const float* x, c
 // One CTA per row; thread t handles rotation pairs (head, i) with i < hd/2 over all q, k, v heads.
 __global__ void rope_append_kernel(const float* qkv, const float* cs, int H, int Hkv, int hd, const int* row_seq,
                                    const int* row_pos, const int* row_valid, KVCache kv, int layer, float* q) {
+  pdl_trigger();
+  pdl_wait();
   const int m = blockIdx.x;
   const int half = hd / 2;
   const int nh = H + 2 * Hkv;
@@ -111,6 +117,8 @@ __global__ void rope_append_kernel(const float* qkv, const float* cs, int H, int
 
 __global__ void __launch_bounds__(kNormThreads) layernorm_kernel(const float* x, const bf16* gamma, const bf16* beta,
                                                                   float eps, int d, float* g, bf16* g_bf) {
+  pdl_trigger();
+  pdl_wait();
   __shared__ float red[32];
   const int b = blockIdx.x;
   const float* xr = x + static_cast<size_t>(b) * d;
@@ -133,6 +141,8 @@ __global__ void __launch_bounds__(kNormThreads) layernorm_kernel(const float* x,
 
 __global__ void swiglu_kernel(const float* gate, const float* up, const float* bias, const int* seq, int M, int F,
                               bf16* h) {
+  pdl_trigger();
+  pdl_wait();
   const size_t n = static_cast<size_t>(M) * F;
   for (size_t idx = blockIdx.x * static_cast<size_t>(blockDim.x) + threadIdx.x; idx < n;
        idx += static_cast<size_t>(gridDim.x) * blockDim.x) {
@@ -145,6 +155,8 @@ __global__ void swiglu_kernel(const float* gate, const float* up, const float* b
 }
 
 __global__ void gather_rows_bf16_kernel(const float* src, int ld_src, const int* idx, int width, bf16* out) {
+  pdl_trigger();
+  pdl_wait();
   const int b = blockIdx.x;
   const float* s = src + static_cast<size_t>(b) * ld_src + static_cast<size_t>(idx ? idx[b] : 0) * width;
   for (int j = threadIdx.x; j < width; j += blockDim.x)
@@ -156,17 +168,17 @@ __global__ void gather_rows_bf16_kernel(const float* src, int ld_src, const int*
 cudaError_t embed_rmsnorm(const int* tok, const void* embed, const void* gamma, float eps, int M, int d, int vocab,
                           float* x, void* a, cudaStream_t st) {
   if (M <= 0) return cudaSuccess;
-  embed_rmsnorm_kernel<<<M, kNormThreads, 0, st>>>(tok, static_cast<const bf16*>(embed),
+  { const cudaError_t e_ = launch_pdl(embed_rmsnorm_kernel, dim3(M), dim3(kNormThreads), 0, st, tok, static_cast<const bf16*>(embed),
                                                    static_cast<const bf16*>(gamma), eps, d, vocab, x,
-                                                   static_cast<bf16*>(a));
+                                                   static_cast<bf16*>(a)); if (e_ != cudaSuccess) return e_; }
   return cudaGetLastError();
 }
 
 cudaError_t rmsnorm(const float* x, const int* rows, const void* gamma, float eps, int M, int d, void* a, float* tap,
                     const int* tap_row, int tap_mask, cudaStream_t st) {
   if (M <= 0) return cudaSuccess;
-  rmsnorm_kernel<<<M, kNormThreads, 0, st>>>(x, rows, static_cast<const bf16*>(gamma), eps, d, static_cast<bf16*>(a),
-                                             tap, tap_row, tap_mask);
+  { const cudaError_t e_ = launch_pdl(rmsnorm_kernel, dim3(M), dim3(kNormThreads), 0, st, x, rows, static_cast<const bf16*>(gamma), eps, d, static_cast<bf16*>(a),
+                                             tap, tap_row, tap_mask); if (e_ != cudaSuccess) return e_; }
   return cudaGetLastError();
 }
 
@@ -174,15 +186,15 @@ cudaError_t rope_append(const float* qkv, const float* rope_cs, int M, int H, in
                         const int* row_pos, const int* row_valid, const KVCache& kv, int layer, float* q,
                         cudaStream_t st) {
   if (M <= 0) return cudaSuccess;
-  rope_append_kernel<<<M, 256, 0, st>>>(qkv, rope_cs, H, Hkv, hd, row_seq, row_pos, row_valid, kv, layer, q);
+  { const cudaError_t e_ = launch_pdl(rope_append_kernel, dim3(M), dim3(256), 0, st, qkv, rope_cs, H, Hkv, hd, row_seq, row_pos, row_valid, kv, layer, q); if (e_ != cudaSuccess) return e_; }
   return cudaGetLastError();
 }
 
 cudaError_t layernorm(const float* x, const void* gamma, const void* beta, float eps, int B, int d, float* g,
                       void* g_bf, cudaStream_t st) {
   if (B <= 0) return cudaSuccess;
-  layernorm_kernel<<<B, kNormThreads, 0, st>>>(x, static_cast<const bf16*>(gamma), static_cast<const bf16*>(beta), eps,
-                                               d, g, static_cast<bf16*>(g_bf));
+  { const cudaError_t e_ = launch_pdl(layernorm_kernel, dim3(B), dim3(kNormThreads), 0, st, x, static_cast<const bf16*>(gamma), static_cast<const bf16*>(beta), eps,
+                                               d, g, static_cast<bf16*>(g_bf)); if (e_ != cudaSuccess) return e_; }
   return cudaGetLastError();
 }
 
@@ -192,14 +204,14 @@ cudaError_t swiglu(const float* gate, const float* up, const float* bias, const 
   const size_t n = static_cast<size_t>(M) * F;
   int blocks = static_cast<int>((n + 255) / 256);
   if (blocks > 152 * 16) blocks = 152 * 16;
-  swiglu_kernel<<<blocks, 256, 0, st>>>(gate, up, bias, seq, M, F, static_cast<bf16*>(h));
+  { const cudaError_t e_ = launch_pdl(swiglu_kernel, dim3(blocks), dim3(256), 0, st, gate, up, bias, seq, M, F, static_cast<bf16*>(h)); if (e_ != cudaSuccess) return e_; }
   return cudaGetLastError();
 }
 
 cudaError_t gather_rows_bf16(const float* src, int ld_src, const int* idx, int width, int B, void* out,
                              cudaStream_t st) {
   if (B <= 0) return cudaSuccess;
-  gather_rows_bf16_kernel<<<B, 256, 0, st>>>(src, ld_src, idx, width, static_cast<bf16*>(out));
+  { const cudaError_t e_ = launch_pdl(gather_rows_bf16_kernel, dim3(B), dim3(256), 0, st, src, ld_src, idx, width, static_cast<bf16*>(out)); if (e_ != cudaSuccess) return e_; }
   return cudaGetLastError();
 }
 

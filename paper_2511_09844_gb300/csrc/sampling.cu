@@ -91,6 +91,8 @@ template <typename T>
 __global__ void __launch_bounds__(kThreads) rowmax_kernel(const T* target, const T* draft, int B, int k, int V,
                                                           const float* temp, const int* stopped,
                                                           unsigned long long* rowkey, unsigned* err) {
+  pdl_trigger();
+  pdl_wait();
   __shared__ unsigned long long red[32];
   const RowRef rr = row_ref(blockIdx.x, B, k, V);
   if (stopped && stopped[rr.b]) return;
@@ -124,6 +126,8 @@ __global__ void __launch_bounds__(kThreads) rowsum_kernel(const T* target, const
                                                           const float* temp, const int* stopped,
                                                           const unsigned long long* rowkey,
                                                           unsigned long long* rowsum) {
+  pdl_trigger();
+  pdl_wait();
   __shared__ unsigned long long red[32];
   const RowRef rr = row_ref(blockIdx.x, B, k, V);
   if (stopped && stopped[rr.b]) return;
@@ -163,6 +167,8 @@ __global__ void decide_kernel(const T* target, const T* draft, const int* xhat, 
                               unsigned long long seed, const int* step_ptr, unsigned step, const int* stopped,
                               const unsigned long long* rowkey, const unsigned long long* rowsum, int* tokens, int* n,
                               AcceptScratch s) {
+  pdl_trigger();
+  pdl_wait();
   const int b = blockIdx.x * blockDim.x + threadIdx.x;
   if (b >= B) return;
   s.slot[2 * b] = 0ull;
@@ -217,6 +223,8 @@ __global__ void __launch_bounds__(kThreads) resample_kernel(const T* target, con
                                                             unsigned step, const unsigned long long* rowkey,
                                                             const unsigned long long* rowsum, int* tokens, int* n,
                                                             AcceptScratch s) {
+  pdl_trigger();
+  pdl_wait();
   __shared__ unsigned long long red[32];
   __shared__ bool last;
   const int b = blockIdx.x;
@@ -287,6 +295,8 @@ __global__ void __launch_bounds__(kThreads) sample_kernel(const float* logits, l
                                                           const int* step_ptr, unsigned step, int* out, int ld_out,
                                                           int* out2, int ld_out2, unsigned long long* slot,
                                                           int* counter, unsigned* err) {
+  pdl_trigger();
+  pdl_wait();
   __shared__ unsigned long long red[32];
   __shared__ bool last;
   const int b = blockIdx.x;
@@ -345,12 +355,12 @@ cudaError_t accept_typed(const T* target, const T* draft, const int* xhat, const
   const int S = (V + kPerCta - 1) / kPerCta;
   cudaError_t e = cudaMemsetAsync(s.rowkey, 0, sizeof(unsigned long long) * 2 * R, st);  // rowkey + rowsum
   if (e != cudaSuccess) return e;
-  rowmax_kernel<T><<<dim3(R, S), kThreads, 0, st>>>(target, draft, B, k, V, temp, stopped, s.rowkey, err);
-  rowsum_kernel<T><<<dim3(R, S), kThreads, 0, st>>>(target, draft, B, k, V, temp, stopped, s.rowkey, s.rowsum);
-  decide_kernel<T><<<(B + 127) / 128, 128, 0, st>>>(target, draft, xhat, temp, B, k, V, seed, step_ptr, step, stopped,
-                                                    s.rowkey, s.rowsum, tokens, n, s);
-  resample_kernel<T><<<dim3(B, S), kThreads, 0, st>>>(target, draft, temp, B, k, V, seed, step_ptr, step, s.rowkey,
-                                                      s.rowsum, tokens, n, s);
+  { const cudaError_t e_ = launch_pdl(rowmax_kernel<T>, dim3(dim3(R, S)), dim3(kThreads), 0, st, target, draft, B, k, V, temp, stopped, s.rowkey, err); if (e_ != cudaSuccess) return e_; }
+  { const cudaError_t e_ = launch_pdl(rowsum_kernel<T>, dim3(dim3(R, S)), dim3(kThreads), 0, st, target, draft, B, k, V, temp, stopped, s.rowkey, s.rowsum); if (e_ != cudaSuccess) return e_; }
+  { const cudaError_t e_ = launch_pdl(decide_kernel<T>, dim3((B + 127) / 128), dim3(128), 0, st, target, draft, xhat, temp, B, k, V, seed, step_ptr, step, stopped,
+                                                    s.rowkey, s.rowsum, tokens, n, s); if (e_ != cudaSuccess) return e_; }
+  { const cudaError_t e_ = launch_pdl(resample_kernel<T>, dim3(dim3(B, S)), dim3(kThreads), 0, st, target, draft, temp, B, k, V, seed, step_ptr, step, s.rowkey,
+                                                      s.rowsum, tokens, n, s); if (e_ != cudaSuccess) return e_; }
   return cudaGetLastError();
 }
 
@@ -389,8 +399,8 @@ cudaError_t sample_rows(const float* logits, long long ld, int B, int V, const f
                         int ld_out2, unsigned long long* slot, int* counter, unsigned* err, cudaStream_t st) {
   if (B <= 0) return cudaSuccess;
   const int S = (V + kPerCta - 1) / kPerCta;
-  sample_kernel<<<dim3(B, S), kThreads, 0, st>>>(logits, ld, V, temp, seed, purpose, i, step_ptr, step, out, ld_out,
-                                                 out2, ld_out2, slot, counter, err);
+  { const cudaError_t e_ = launch_pdl(sample_kernel, dim3(dim3(B, S)), dim3(kThreads), 0, st, logits, ld, V, temp, seed, purpose, i, step_ptr, step, out, ld_out,
+                                                 out2, ld_out2, slot, counter, err); if (e_ != cudaSuccess) return e_; }
   return cudaGetLastError();
 }
 

@@ -10,6 +10,8 @@
 //   verifier         rows b(k+1)+t = [x_{n-1}, draft 1..k] at positions n-1+t
 //   commit (j kept)  n += j+1; D = min(n_old + j, n_old + k - 1); verifier cache = n-1 positions
 //                    implicitly (it only ever reads positions below each row's own).
+#include "common.cuh"
+#include "kernels.h"
 #include "state.h"
 
 namespace sd2 {
@@ -21,6 +23,8 @@ __device__ __forceinline__ void put(int* tok, int* pos, int* seq, int* valid, in
 
 __global__ void plan_kernel(int mode, int i, int B, int k, int max_ctx, const int* state, int maxB,
                             const int* committed, const int* xhat, int* tok, int* pos, int* seq, int* valid) {
+  pdl_trigger();
+  pdl_wait();
   const int b = blockIdx.x * blockDim.x + threadIdx.x;
   if (b >= B) return;
   const int n = state[b], D = state[maxB + b], stop = state[3 * maxB + b];
@@ -44,6 +48,8 @@ __global__ void plan_kernel(int mode, int i, int B, int k, int max_ctx, const in
 
 __global__ void commit_kernel(int B, int k, int max_ctx, int* state, int maxB, int* committed, const int* tokens,
                               const int* n_out, int* iter) {
+  pdl_trigger();
+  pdl_wait();
   const int b = blockIdx.x * blockDim.x + threadIdx.x;
   if (b == 0) *iter += 1;
   if (b >= B) return;
@@ -62,6 +68,8 @@ __global__ void commit_kernel(int B, int k, int max_ctx, int* state, int maxB, i
 // After the prefill sample: committed[b] = prompt + first token; n = len+1, D = len, j = 0.
 __global__ void prefill_init_kernel(int B, int max_ctx, const int* prompts, const int* cu, const int* first,
                                     int* state, int maxB, int* committed, int* first_out) {
+  pdl_trigger();
+  pdl_wait();
   const int b = blockIdx.x;
   const int off = cu[b], len = cu[b + 1] - cu[b];
   int* cb = committed + static_cast<size_t>(b) * max_ctx;
@@ -80,20 +88,20 @@ __global__ void prefill_init_kernel(int B, int max_ctx, const int* prompts, cons
 
 cudaError_t plan_rows(int mode, int i, int B, int k, int max_ctx, const int* state, int maxB, const int* committed,
                       const int* xhat, int* tok, int* pos, int* seq, int* valid, cudaStream_t st) {
-  plan_kernel<<<(B + 127) / 128, 128, 0, st>>>(mode, i, B, k, max_ctx, state, maxB, committed, xhat, tok, pos, seq,
-                                                valid);
+  { const cudaError_t e_ = launch_pdl(plan_kernel, dim3((B + 127) / 128), dim3(128), 0, st, mode, i, B, k, max_ctx, state, maxB, committed, xhat, tok, pos, seq,
+                                                valid); if (e_ != cudaSuccess) return e_; }
   return cudaGetLastError();
 }
 
 cudaError_t commit(int B, int k, int max_ctx, int* state, int maxB, int* committed, const int* tokens, const int* n_out,
                    int* iter, cudaStream_t st) {
-  commit_kernel<<<(B + 127) / 128, 128, 0, st>>>(B, k, max_ctx, state, maxB, committed, tokens, n_out, iter);
+  { const cudaError_t e_ = launch_pdl(commit_kernel, dim3((B + 127) / 128), dim3(128), 0, st, B, k, max_ctx, state, maxB, committed, tokens, n_out, iter); if (e_ != cudaSuccess) return e_; }
   return cudaGetLastError();
 }
 
 cudaError_t prefill_init(int B, int max_ctx, const int* prompts, const int* cu, const int* first, int* state, int maxB,
                          int* committed, int* first_out, cudaStream_t st) {
-  prefill_init_kernel<<<B, 256, 0, st>>>(B, max_ctx, prompts, cu, first, state, maxB, committed, first_out);
+  { const cudaError_t e_ = launch_pdl(prefill_init_kernel, dim3(B), dim3(256), 0, st, B, max_ctx, prompts, cu, first, state, maxB, committed, first_out); if (e_ != cudaSuccess) return e_; }
   return cudaGetLastError();
 }
 
