@@ -194,12 +194,10 @@ sd2_status sd2_steer(const float* d_taps, int32_t B, int32_t d_v, const void* w_
  *      d_h[m*N + f] = bf16((up + d_bias[seq[m]*ld_bias + f]) * SiLU(gate)), d_bias/d_seq optional.
  *   impl 0: tensor cores (tcgen05, TMA) where the shape allows (K % 64 == 0; N % 128 == 0, or
  *   N % 64 == 0 for epilogue 2), else CUDA cores; 1: CUDA cores; 2: tensor cores or SD2_EINVAL.
- *   d_workspace: sd2_gemm_workspace_bytes(M) bytes, 256-byte aligned, for impl 0 and 2. */
-size_t sd2_gemm_workspace_bytes(int32_t M);
+ *   No device memory is allocated except, once, a 4-byte error word. */
 sd2_status sd2_gemm(const void* d_x, int32_t ldx, int32_t M, int32_t K, const void* d_w, const void* d_w_up,
                     int32_t N, int32_t epilogue, float* d_out, int32_t ldo, void* d_h, const float* d_bias,
-                    const int32_t* d_seq, int32_t ld_bias, int32_t impl, void* d_workspace,
-                    size_t workspace_bytes, void* stream);
+                    const int32_t* d_seq, int32_t ld_bias, int32_t impl, void* stream);
 
 /* Choose the GEMM of a context: 0 tensor cores where the shape allows (default), 1 CUDA cores.
  * Drops captured graphs. */

@@ -6,7 +6,8 @@
 // 16-byte reads of eight lanes hit distinct banks), and each warp runs an online softmax for up
 // to 8 query vectors (query rows x the heads sharing the KV head). Every K/V byte of the split
 // is read from HBM once per CTA, whatever the number of rows in the group. With several splits
-// the partial (max, sum, accumulator) triples are merged by a second kernel.
+// each CTA stores its partial (max, sum, accumulator) triples, and the last CTA of the
+// (group, KV head) to arrive merges them in split order.
 #include <math.h>
 
 #include "common.cuh"
@@ -155,26 +156,52 @@ __global__ void __launch_bounds__(kWarps * 32) attn_kernel(const AttnArgs a) {
       for (int d = 0; d < DPL; ++d) p[2 + lane * DPL + d] = acc[j][d];
     }
   }
-}
+  if (a.n_splits == 1) return;
 
-// Merge the splits of one (row, head): out = sum_s acc_s e^{m_s - M} / sum_s l_s e^{m_s - M}.
-template <int HD>
-__global__ void __launch_bounds__(HD) attn_merge_kernel(const AttnArgs a) {
-  pdl_trigger();
-  pdl_wait();
-  const int row = blockIdx.x / a.H, h = blockIdx.x % a.H;
-  const int ns = min(a.n_splits, a.row_pos[row] / a.chunk + 1);
-  const float* p = a.part + (static_cast<size_t>(row) * a.H + h) * a.n_splits * (HD + 2);
-  float M = -INFINITY;
-  for (int s = 0; s < ns; ++s) M = fmaxf(M, p[s * (HD + 2)]);
-  float L = 0.f, o = 0.f;
-  for (int s = 0; s < ns; ++s) {
-    const float* ps = p + s * (HD + 2);
-    const float w = __expf(ps[0] - M);
-    L += ps[1] * w;
-    o += ps[2 + threadIdx.x] * w;
+  // The splits that run for this group are those starting at or before its last position.
+  __shared__ int last_flag;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int old;
+    asm volatile("atom.acq_rel.gpu.global.add.s32 %0, [%1], 1;"
+                 : "=r"(old)
+                 : "l"(a.counters + static_cast<size_t>(g) * Hkv + kvh)
+                 : "memory");
+    const int n_used = pmax / a.chunk + 1;
+    last_flag = (old == n_used - 1) ? 1 : 0;
+    if (last_flag) a.counters[static_cast<size_t>(g) * Hkv + kvh] = 0;
   }
-  static_cast<bf16*>(a.out)[static_cast<size_t>(row) * a.H * HD + h * HD + threadIdx.x] = __float2bfloat16_rn(o / L);
+  __syncthreads();
+  if (!last_flag) return;
+  // merge: out = sum_s acc_s e^{m_s - M} / sum_s l_s e^{m_s - M} for every (row, head) here
+  float* sM = sQ;                 // the queries are no longer needed
+  float* sL = sQ + kMaxQV;
+  if (threadIdx.x < nqv) {
+    const int qv = threadIdx.x;
+    const int row = r0 + qv / G, h = kvh * G + qv % G;
+    const int ns = min(a.n_splits, a.row_pos[row] / a.chunk + 1);
+    const float* p = a.part + (static_cast<size_t>(row) * a.H + h) * a.n_splits * (HD + 2);
+    float M = -INFINITY;
+    for (int s2 = 0; s2 < ns; ++s2) M = fmaxf(M, __ldcg(p + s2 * (HD + 2)));
+    float L = 0.f;
+    for (int s2 = 0; s2 < ns; ++s2) L += __ldcg(p + s2 * (HD + 2) + 1) * __expf(__ldcg(p + s2 * (HD + 2)) - M);
+    sM[qv] = M;
+    sL[qv] = 1.f / L;
+  }
+  __syncthreads();
+  for (int idx = threadIdx.x; idx < nqv * HD; idx += blockDim.x) {
+    const int qv = idx / HD, d = idx % HD;
+    const int row = r0 + qv / G, h = kvh * G + qv % G;
+    const int ns = min(a.n_splits, a.row_pos[row] / a.chunk + 1);
+    const float* p = a.part + (static_cast<size_t>(row) * a.H + h) * a.n_splits * (HD + 2);
+    const float M = sM[qv];
+    float o = 0.f;
+    for (int s2 = 0; s2 < ns; ++s2) {
+      const float* ps = p + s2 * (HD + 2);
+      o += __ldcg(ps + 2 + d) * __expf(__ldcg(ps) - M);
+    }
+    static_cast<bf16*>(a.out)[static_cast<size_t>(row) * a.H * HD + h * HD + d] = __float2bfloat16_rn(o * sL[qv]);
+  }
 }
 
 template <int HD>
@@ -187,9 +214,6 @@ cudaError_t launch(const AttnArgs& a, cudaStream_t st) {
   }
   dim3 grid(a.n_groups, a.kv.Hkv, a.n_splits);
   { const cudaError_t e_ = launch_pdl(attn_kernel<HD>, dim3(grid), dim3(kWarps * 32), smem_bytes<HD>(), st, a); if (e_ != cudaSuccess) return e_; }
-  cudaError_t e = cudaGetLastError();
-  if (e != cudaSuccess || a.n_splits == 1) return e;
-  { const cudaError_t e_ = launch_pdl(attn_merge_kernel<HD>, dim3(a.M * a.H), dim3(HD), 0, st, a); if (e_ != cudaSuccess) return e_; }
   return cudaGetLastError();
 }
 

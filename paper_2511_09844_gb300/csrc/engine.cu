@@ -91,10 +91,9 @@ struct sd2_ctx {
   float *taps = nullptr, *g_pre = nullptr, *g = nullptr, *bias = nullptr;
   void *a = nullptr, *attn = nullptr, *h = nullptr, *g_bf = nullptr, *hml_in = nullptr;
   size_t part_elems = 0;
-  float* gemm_ws = nullptr;     // tensor-core GEMM: split-tile partials
-  int* gemm_cnt = nullptr;      // tensor-core GEMM: per-tile arrival counters (zero between launches)
-  size_t gemm_cnt_len = 0;
   int gemm_impl = 0;            // 0 tensor cores where the shape allows, 1 CUDA cores
+  int* attn_cnt = nullptr;      // attention split arrivals per (row group, KV head), zero between launches
+  size_t attn_cnt_len = 0;
   unsigned long long* samp_slot = nullptr;
   int* samp_counter = nullptr;
   AcceptScratch as{};
@@ -232,11 +231,8 @@ struct FwdOut {
   long long ld_logits = 0;
 };
 
-// The tensor-core GEMM's scratch and the implementation choice, attached to every GEMM launch.
+// The error word and the implementation choice, attached to every GEMM launch.
 GemmArgs& tc(sd2_ctx* c, GemmArgs& g) {
-  g.ws = c->gemm_ws;
-  g.counters = c->gemm_cnt;
-  g.counters_len = c->gemm_cnt_len;
   g.err = c->errw;
   g.impl = c->gemm_impl;
   return g;
@@ -271,15 +267,16 @@ sd2_status forward(sd2_ctx* c, const Model& m, const Plan& p, const FwdOut& o) {
     g.seg[0] = {m.W(l, SD2_W_Q), H * hd};
     g.seg[1] = {m.W(l, SD2_W_K), Hkv * hd};
     g.seg[2] = {m.W(l, SD2_W_V), Hkv * hd};
-    g.nseg = 3; g.epi = EPI_STORE; g.out = c->qkv; g.ldo = m.qkv_width();
+    g.nseg = 3; g.epi = EPI_QKV; g.out = c->qkv; g.ldo = m.qkv_width();
+    g.q_out = c->q; g.kv_pool = m.kv_pool; g.kv_table = m.table; g.kv_bt_stride = m.bt_stride;
+    g.kv_n_blocks = m.n_blocks; g.n_heads = H; g.n_kv_heads = Hkv; g.head_dim = hd; g.layer = l;
+    g.rope_cs = m.rope_cs; g.row_pos = p.pos; g.row_valid = p.valid; g.row_seq = p.seq;
     CK(timed(c, PC_GEMM, gemm_bytes(M, m.qkv_width(), d, 4), [&] { return gemm(tc(c, g), c->st); }));
-    CK(timed(c, PC_OTHER, 0, [&] {
-      return rope_append(c->qkv, m.rope_cs, M, H, Hkv, hd, p.seq, p.pos, p.valid, m.cache(), l, c->q, c->st);
-    }));
     AttnArgs at{};
     at.q = c->q; at.kv = m.cache(); at.layer = l; at.row_pos = p.pos;
     at.grp_row0 = p.g_row0; at.grp_nrows = p.g_nrows; at.grp_seq = p.g_seq; at.n_groups = p.n_groups;
     at.M = M; at.H = H; at.hd = hd; at.n_splits = p.n_splits; at.chunk = p.chunk; at.part = c->part; at.out = c->attn;
+    at.counters = c->attn_cnt;
     double kvb = 0;
     if (c->prof && !c->h_n.empty()) {
       for (int b = 0; b < c->B; ++b) kvb += 2.0 * 2.0 * Hkv * hd * (c->h_n[b] + 16);
@@ -528,10 +525,9 @@ sd2_status sd2_init(const sd2_config* cfg, const sd2_weights* w, void* stream, s
     ALLOC(c->g, static_cast<size_t>(maxB) * cfg->d_steer);
     ALLOC(c->g_bf, static_cast<size_t>(maxB) * cfg->d_steer * 2);
     ALLOC(c->bias, static_cast<size_t>(maxB) * cfg->drafter.n_layers * cfg->drafter.d_ffn);
-    c->gemm_cnt_len = 1 << 20;
-    ALLOC(c->gemm_ws, gemm_tc_workspace_floats(R));
-    ALLOC(c->gemm_cnt, c->gemm_cnt_len);
-    CK(cudaMemset(c->gemm_cnt, 0, sizeof(int) * c->gemm_cnt_len));
+    c->attn_cnt_len = static_cast<size_t>(maxB) * 17 * 64;
+    ALLOC(c->attn_cnt, c->attn_cnt_len);
+    CK(cudaMemset(c->attn_cnt, 0, sizeof(int) * c->attn_cnt_len));
     ALLOC(c->samp_slot, maxB);
     ALLOC(c->samp_counter, maxB);
     void* acc;
@@ -613,6 +609,9 @@ sd2_status sd2_prefill(sd2_ctx* c, int32_t batch, const int32_t* d_tokens, const
   std::vector<int> cu(h_cu_lens, h_cu_lens + batch + 1);
   const int o_cu = push(cu);
   if ((int)st.size() > c->statics_cap) return fail(c, SD2_ECAPACITY, "plan tables exceed their buffer");
+  const size_t max_groups = std::max(std::max(d1r0.size(), dnr0.size()), sr0.size());
+  if (max_groups * static_cast<size_t>(std::max(c->V.c.n_kv_heads, c->D.c.n_kv_heads)) > c->attn_cnt_len)
+    return fail(c, SD2_ECAPACITY, "attention counter table too small for this batch");
   CK(cudaMemcpyAsync(c->statics, st.data(), st.size() * sizeof(int), cudaMemcpyHostToDevice, c->st));
   std::vector<float> temps(h_temperature, h_temperature + batch);
   CK(cudaMemcpyAsync(c->temp, temps.data(), batch * sizeof(float), cudaMemcpyHostToDevice, c->st));
@@ -843,15 +842,9 @@ sd2_status sd2_steer(const float* d_taps, int32_t B, int32_t d_v, const void* w_
   return SD2_OK;
 }
 
-size_t sd2_gemm_workspace_bytes(int32_t M) {
-  if (M < 1) return 0;
-  return ((gemm_tc_workspace_floats(M) * 4 + 255) / 256 + (static_cast<size_t>(1 << 20) * 4) / 256) * 256;
-}
-
 sd2_status sd2_gemm(const void* d_x, int32_t ldx, int32_t M, int32_t K, const void* d_w, const void* d_w_up,
                     int32_t N, int32_t epilogue, float* d_out, int32_t ldo, void* d_h, const float* d_bias,
-                    const int32_t* d_seq, int32_t ld_bias, int32_t impl, void* d_workspace, size_t workspace_bytes,
-                    void* stream) {
+                    const int32_t* d_seq, int32_t ld_bias, int32_t impl, void* stream) {
   sd2_ctx* c = nullptr;
   if (!d_x || !d_w || M < 1 || K < 8 || K % 8 || ldx < K || ldx % 8 || N < 1)
     return fail(nullptr, SD2_EINVAL, "bad GEMM shape or null input");
@@ -867,26 +860,15 @@ sd2_status sd2_gemm(const void* d_x, int32_t ldx, int32_t M, int32_t K, const vo
   g.epi = epilogue; g.out = d_out; g.ldo = ldo; g.out_bf = d_h; g.ldh = N;
   g.bias = d_bias; g.ld_bias = ld_bias; g.row_seq = d_seq;
   g.impl = impl == 1 ? 1 : 0;
-  cudaStream_t st = static_cast<cudaStream_t>(stream);
-  if (impl != 1) {
-    if (!d_workspace || workspace_bytes < sd2_gemm_workspace_bytes(M))
-      return fail(nullptr, SD2_EINVAL, "tensor-core GEMM needs sd2_gemm_workspace_bytes(M) of workspace");
-    if (reinterpret_cast<uintptr_t>(d_workspace) & 255) return fail(nullptr, SD2_EINVAL, "workspace not 256-aligned");
-    const size_t ws_bytes = (gemm_tc_workspace_floats(M) * 4 + 255) / 256 * 256;
-    g.ws = static_cast<float*>(d_workspace);
-    g.counters = reinterpret_cast<int*>(static_cast<char*>(d_workspace) + ws_bytes);
-    g.counters_len = 1 << 20;
-    g.err = nullptr;
-    if (impl == 2 && !gemm_tc_supported(g))
-      return fail(nullptr, SD2_EINVAL, "shape not supported by the tensor-core GEMM (K % 64, rows % 128)");
-    const size_t tiles = static_cast<size_t>(epilogue == EPI_SWIGLU ? (N + 63) / 64 : (N + 127) / 128) *
-                         ((M + gemm_tc_token_tile(M) - 1) / gemm_tc_token_tile(M));
-    CK(cudaMemsetAsync(g.counters, 0, sizeof(int) * std::min(tiles, g.counters_len), st));
-    static unsigned* err_word = nullptr;  // a device word for the timeout flag of standalone calls
-    if (!err_word) CK(cudaMalloc(&err_word, sizeof(unsigned)));
-    g.err = err_word;
+  static unsigned* err_word = nullptr;  // timeout flag of context-free tensor-core launches
+  if (!err_word) {
+    CK(cudaMalloc(&err_word, sizeof(unsigned)));
+    CK(cudaMemset(err_word, 0, sizeof(unsigned)));
   }
-  CK(gemm(g, st));
+  g.err = err_word;
+  if (impl == 2 && !gemm_tc_supported(g))
+    return fail(nullptr, SD2_EINVAL, "shape not supported by the tensor-core GEMM (K % 64, rows % 128)");
+  CK(gemm(g, static_cast<cudaStream_t>(stream)));
   return SD2_OK;
 }
 

@@ -110,9 +110,18 @@ __global__ void __launch_bounds__(kThreads) gemm_simt_kernel(const GemmArgs a, i
 }  // namespace
 
 cudaError_t gemm(const GemmArgs& a, cudaStream_t st) {
-  if (a.ws && a.counters && a.impl != 1 && gemm_tc_supported(a))
-    return gemm_tc(a, a.ws, a.counters, a.counters_len, a.err, st);
-  return gemm_simt(a, st);
+  if (a.impl != 1 && a.err && gemm_tc_supported(a)) return gemm_tc(a, a.err, st);
+  if (a.epi != EPI_QKV) return gemm_simt(a, st);
+  // CUDA-core path of the QKV epilogue: projections to `out`, then the rotary/append kernel
+  GemmArgs s = a;
+  s.epi = EPI_STORE;
+  cudaError_t e = gemm_simt(s, st);
+  if (e != cudaSuccess) return e;
+  KVCache kv;
+  kv.pool = a.kv_pool; kv.table = a.kv_table; kv.bt_stride = a.kv_bt_stride; kv.n_blocks = a.kv_n_blocks;
+  kv.Hkv = a.n_kv_heads; kv.hd = a.head_dim;
+  return rope_append(a.out, a.rope_cs, a.M, a.n_heads, a.n_kv_heads, a.head_dim, a.row_seq, a.row_pos, a.row_valid, kv,
+                     a.layer, a.q_out, st);
 }
 
 cudaError_t gemm_simt(const GemmArgs& a, cudaStream_t st) {
@@ -124,6 +133,7 @@ cudaError_t gemm_simt(const GemmArgs& a, cudaStream_t st) {
   const int cap = 152 * 8;
   if (blocks > cap) blocks = cap;
   switch (a.epi) {
+    case EPI_QKV:
     case EPI_STORE: { const cudaError_t e_ = launch_pdl(gemm_simt_kernel<EPI_STORE>, dim3(blocks), dim3(kThreads), 0, st, a, n_units, n_total); if (e_ != cudaSuccess) return e_; } break;
     case EPI_ADD: { const cudaError_t e_ = launch_pdl(gemm_simt_kernel<EPI_ADD>, dim3(blocks), dim3(kThreads), 0, st, a, n_units, n_total); if (e_ != cudaSuccess) return e_; } break;
     default: { const cudaError_t e_ = launch_pdl(gemm_simt_kernel<EPI_SWIGLU>, dim3(blocks), dim3(kThreads), 0, st, a, n_units, n_total); if (e_ != cudaSuccess) return e_; } break;

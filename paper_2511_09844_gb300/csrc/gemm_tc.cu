@@ -7,14 +7,17 @@
 // tokens are K-major bf16 tiles of 64 elements (128 bytes) per stage, loaded by TMA with the
 // 128-byte swizzle that the UMMA shared-memory descriptors expect.
 //
-// Work split: the weight stream of a launch is U = tiles x (K/64) k-blocks; a persistent grid of
-// G <= #SMs CTAs takes contiguous ranges of U/G k-blocks (stream-K), so every SM streams the same
-// number of weight bytes whatever the matrix shape. A tile split across CTAs is finished by the
-// last CTA to arrive on its counter, which sums the fp32 partials in k order (deterministic; no
-// CTA ever waits on another).
+// Work split. A launch has T = (weight tiles) x (token tiles) output tiles of K/64 k-blocks each.
+// When T is small (few, tall weight matrices) each tile's K range is split over sp <= 8 CTAs
+// that form one thread-block cluster; their fp32 partial tiles are summed in rank order through
+// distributed shared memory, so no partial ever leaves the SMs and no CTA waits on global
+// atomics. When T is large, sp = 1 and each CTA streams whole tiles, double-buffering its TMEM
+// accumulator across tiles. Either way ~152 CTAs stream at once, and with the stage ring kept
+// within half an SM's shared memory a second CTA (the next kernel's, under programmatic
+// dependent launch) can start on the same SM and prefetch its weights.
 //
 // Warp roles (192 threads): warp 0 issues TMA loads into a ring of stages, warp 1 issues the
-// MMAs (one thread) and owns the TMEM allocation, warps 2-5 read the two TMEM accumulators back
+// MMAs (one thread) and owns the TMEM allocation, warps 2-5 read the TMEM accumulators back
 // (each warp its 32-lane quarter) and run the epilogue. Every wait is bounded by a clock budget;
 // on expiry the kernel records ERR_TIMEOUT, drains what it issued and returns.
 #include <cuda.h>
@@ -51,9 +54,17 @@ struct TcArgs {
   const float* bias;
   int ld_bias;
   const int* row_seq;
-  float* ws;
-  int* counters;
+  int sp;            // CTAs per tile (cluster size); 1 = whole tiles, persistent
+  int tiles;
   unsigned* err;
+  // EPI_QKV
+  float* q_out;
+  bf16* kv_pool;
+  const int* kv_table;
+  int kv_bt_stride, kv_n_blocks, n_heads, n_kv_heads, head_dim, layer;
+  const float* rope_cs;
+  const int* row_pos;
+  const int* row_valid;
 };
 
 // ------------------------------------------------------------------------------ PTX wrappers
@@ -161,82 +172,123 @@ __device__ __forceinline__ bool wait_bar_budget(uint32_t bar, uint32_t parity, l
   return true;
 }
 
-struct Seg {
-  int tile, kb, nkb;
-};
-__device__ __forceinline__ Seg segment(long long u, long long hi, int KB) {
-  Seg s;
-  s.tile = static_cast<int>(u / KB);
-  s.kb = static_cast<int>(u % KB);
-  s.nkb = static_cast<int>(min(static_cast<long long>(KB - s.kb), hi - u));
-  return s;
+// ------------------------------------------------------------------------------ cluster helpers
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
 }
-__device__ __forceinline__ long long cta_lo(long long c, long long U, long long G) { return c * U / G; }
-// The CTA whose range holds unit x (ranges are non-empty because G <= U).
-__device__ __forceinline__ int cta_of(long long x, long long U, long long G) {
-  long long c = x * G / U;
-  while (c + 1 < G && cta_lo(c + 1, U, G) <= x) ++c;
-  while (c > 0 && cta_lo(c, U, G) > x) --c;
-  return static_cast<int>(c);
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+// fp32 at shared-memory address `saddr` of CTA `rank` of this cluster
+__device__ __forceinline__ float ld_dsmem(uint32_t saddr, uint32_t rank) {
+  uint32_t remote;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(saddr), "r"(rank));
+  float v;
+  asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(remote) : "memory");
+  return v;
 }
 
-// Epilogue of 16 token columns j0..j0+15 of one weight row r of the tile.
+constexpr int kXS = 17;   // padded row of the epilogue exchange buffer (128 rows x 16 columns)
+
+// ------------------------------------------------------------------------------ epilogue stores
+// One output value of weight row `row` of tile (wt, tt) for token m (m < M).
+__device__ __forceinline__ void emit_plain(const TcArgs& a, int wt, int row, int m, float v) {
+  float* o = a.out + static_cast<size_t>(m) * a.ldo + wt * kWRows + row;
+  if (a.epi == EPI_ADD) *o += v;
+  else *o = v;
+}
+// Eq. 2 for feature f of the tile (gate row f, up row f + 64).
+__device__ __forceinline__ void emit_swiglu(const TcArgs& a, int wt, int f, int m, float gate, float up) {
+  const int feat = wt * 64 + f;
+  if (a.bias) up += a.bias[static_cast<size_t>(a.row_seq ? a.row_seq[m] : 0) * a.ld_bias + feat];
+  a.out_bf[static_cast<size_t>(m) * a.ldh + feat] = __float2bfloat16_rn(up * (gate / (1.f + __expf(-gate))));
+}
+// Tile rows are whole heads of [q | k | v]; q and k are rotated with their rotate-half partner
+// (row +- hd/2 of the same head), q goes to q_out and k, v of valid rows to the paged cache.
+__device__ __forceinline__ void emit_qkv(const TcArgs& a, int wt, int row, int m, float v, float vp) {
+  const int hd = a.head_dim, half = hd >> 1;
+  const int n = wt * kWRows + row;
+  const int head = n / hd, i = n % hd;
+  const int pos = a.row_pos[m];
+  float o = v;
+  if (head < a.n_heads + a.n_kv_heads) {
+    const int ir = (i < half) ? i : i - half;
+    const float2 cs = reinterpret_cast<const float2*>(a.rope_cs)[static_cast<size_t>(pos) * half + ir];
+    o = (i < half) ? v * cs.x - vp * cs.y : v * cs.x + vp * cs.y;
+  }
+  if (head < a.n_heads) {
+    a.q_out[(static_cast<size_t>(m) * a.n_heads + head) * hd + i] = o;
+  } else if (a.row_valid[m]) {
+    const int kvi = (head - a.n_heads) / a.n_kv_heads;            // 0: K, 1: V
+    const int kvh = (head - a.n_heads) % a.n_kv_heads;
+    const int blk = a.kv_table[static_cast<size_t>(a.row_seq[m]) * a.kv_bt_stride + (pos >> 4)];
+    a.kv_pool[((static_cast<size_t>(a.layer) * a.kv_n_blocks + blk) * 2 + kvi) * a.n_kv_heads * 16 * hd +
+              static_cast<size_t>(kvh) * 16 * hd + (pos & 15) * hd + i] = __float2bfloat16_rn(o);
+  }
+}
+__device__ __forceinline__ int partner_row(const TcArgs& a, int row) {
+  const int half = a.head_dim >> 1;
+  return ((row % a.head_dim) < half) ? row + half : row - half;
+}
+
+// Whole-tile epilogue: thread r holds weight row r for 16 token columns j0..j0+15; rows that
+// need another row (SwiGLU pairs, rotate-half partners) are exchanged through shared memory.
 __device__ __forceinline__ void finish_chunk(const TcArgs& a, int wt, int tt, int r, int j0, const float (&v)[16],
                                              float* xbuf) {
   const int m0 = tt * a.NT + j0;
-  if (a.swiglu) {
-    // rows 0..63: gate of feature f0 + r; rows 64..127: up of the same features
-    constexpr int XS = 17;
-    if (r >= 64)
+  if (a.epi == EPI_QKV || a.swiglu) {
 #pragma unroll
-      for (int j = 0; j < 16; ++j) xbuf[(r - 64) * XS + j] = v[j];
+    for (int j = 0; j < 16; ++j) xbuf[r * kXS + j] = v[j];
     named_bar_epi();
-    if (r < 64) {
-      const int f = wt * 64 + r;
+    if (a.swiglu) {
+      if (r < 64)
 #pragma unroll
-      for (int j = 0; j < 16; ++j) {
-        const int m = m0 + j;
-        if (m < a.M) {
-          float up = xbuf[r * XS + j];
-          if (a.bias) up += a.bias[static_cast<size_t>(a.row_seq ? a.row_seq[m] : 0) * a.ld_bias + f];
-          const float g = v[j];
-          a.out_bf[static_cast<size_t>(m) * a.ldh + f] = __float2bfloat16_rn(up * (g / (1.f + __expf(-g))));
-        }
-      }
+        for (int j = 0; j < 16; ++j)
+          if (m0 + j < a.M) emit_swiglu(a, wt, r, m0 + j, v[j], xbuf[(r + 64) * kXS + j]);
+    } else {
+      const int p = partner_row(a, r);
+#pragma unroll
+      for (int j = 0; j < 16; ++j)
+        if (m0 + j < a.M) emit_qkv(a, wt, r, m0 + j, v[j], xbuf[p * kXS + j]);
     }
     named_bar_epi();
     return;
   }
-  const int n = wt * kWRows + r;
 #pragma unroll
-  for (int j = 0; j < 16; ++j) {
-    const int m = m0 + j;
-    if (m < a.M) {
-      float* o = a.out + static_cast<size_t>(m) * a.ldo + n;
-      if (a.epi == EPI_ADD) *o += v[j];
-      else *o = v[j];
-    }
-  }
+  for (int j = 0; j < 16; ++j)
+    if (m0 + j < a.M) emit_plain(a, wt, r, m0 + j, v[j]);
+}
+
+// Sum over the cluster's ranks (in rank order) of element (row, col) of their partial tiles.
+__device__ __forceinline__ float cluster_sum(uint32_t red, int NT1, int row, int col, int sp) {
+  const uint32_t addr = red + static_cast<uint32_t>((row * NT1 + col) * 4);
+  float v = 0.f;
+  for (int q = 0; q < sp; ++q) v += ld_dsmem(addr, static_cast<uint32_t>(q));
+  return v;
 }
 
 __global__ void __launch_bounds__(kThreads, 2) gemm_tc_kernel(const __grid_constant__ TcArgs a) {
   extern __shared__ unsigned char smem_raw[];
   unsigned char* smem =
       reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-  const int S = a.stages, NT = a.NT;
+  const int S = a.stages, NT = a.NT, sp = a.sp;
   const uint32_t a_bytes = kWRows * kBK * 2;
   const uint32_t b_bytes = static_cast<uint32_t>(NT) * kBK * 2;
   const uint32_t stage_bytes = a_bytes + b_bytes;
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + static_cast<size_t>(S) * stage_bytes);
   // bars: full[S], empty[S], tfull[2], tempty[2], drain
   float* xbuf = reinterpret_cast<float*>(bars + 2 * S + 6);
-  volatile int* flags = reinterpret_cast<volatile int*>(xbuf + 64 * 17);
-  // flags: [0] abort, [1] TMEM base, [2] last-arrival decision, [3] stages consumed, [4] go
+  volatile int* flags = reinterpret_cast<volatile int*>(xbuf + kWRows * kXS);
+  // flags: [0] abort, [1] TMEM base, [3] stages consumed, [4] go
   const uint32_t full0 = smem_u32(bars), empty0 = full0 + 8 * S, tfull0 = empty0 + 8 * S, tempty0 = tfull0 + 16,
                  drain = tempty0 + 16;
+  const uint32_t red = smem_u32(smem);   // the split-K partial tile reuses the drained stage ring
+  const int NT1 = NT + 1;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   uint32_t ncols = 32;
-  while (ncols < static_cast<uint32_t>(2 * NT)) ncols <<= 1;
+  while (ncols < static_cast<uint32_t>((sp == 1 ? 2 : 1) * NT)) ncols <<= 1;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
@@ -248,7 +300,7 @@ __global__ void __launch_bounds__(kThreads, 2) gemm_tc_kernel(const __grid_const
     mbar_init(tempty0, 4);
     mbar_init(tempty0 + 8, 4);
     mbar_init(drain, 1);
-    flags[0] = 0; flags[2] = 0; flags[3] = 0; flags[4] = 0;
+    flags[0] = 0; flags[3] = 0; flags[4] = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   if (warp == 1) {
@@ -259,19 +311,23 @@ __global__ void __launch_bounds__(kThreads, 2) gemm_tc_kernel(const __grid_const
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = static_cast<uint32_t>(flags[1]);
-
-  const long long G = gridDim.x, U = a.units, c = blockIdx.x;
-  const long long lo = cta_lo(c, U, G), hi = cta_lo(c + 1, U, G);
   volatile int* abort_flag = flags;
+
+  // This CTA's segments: sp > 1 -> one K-slice of tile blockIdx.x / sp; sp == 1 -> whole tiles
+  // blockIdx.x, blockIdx.x + gridDim.x, ...
+  const int rank = sp > 1 ? static_cast<int>(cluster_rank()) : 0;
+  const int first_tile = sp > 1 ? static_cast<int>(blockIdx.x) / sp : static_cast<int>(blockIdx.x);
+  const int tile_step = sp > 1 ? a.tiles : static_cast<int>(gridDim.x);
+  const int kb_lo = rank * a.KB / sp, kb_hi = (rank + 1) * a.KB / sp;
+  const int nkb = kb_hi - kb_lo;
 
   pdl_trigger();                             // the next kernel may start its own prologue
   if (warp == 0) {
     if (lane == 0) {
-      // Stage use j loads k-block (lo + j) of this CTA's range: the weight half first, then the
-      // token half. Weights never depend on earlier kernels, so the first stages' weight tiles
-      // are requested before waiting for the predecessor grid. Cursors advance one k-block at a
-      // time (no divisions in the issue loop: this one thread feeds the whole SM).
-      const uint32_t n_units = static_cast<uint32_t>(hi - lo);
+      // Stage use j loads k-block (kb_lo + j % nkb) of the CTA's (j / nkb)-th tile: the weight
+      // half first, then the token half. Weights never depend on earlier kernels, so the first
+      // stages' weight tiles are requested before waiting for the predecessor grid. Cursors
+      // advance one k-block at a time (no divisions in the issue loop).
       struct Cursor {
         int tile, kb, wt, tt, seg, row0;
       };
@@ -284,13 +340,16 @@ __global__ void __launch_bounds__(kThreads, 2) gemm_tc_kernel(const __grid_const
           while (c.seg + 1 < a.nseg && c.row0 >= a.seg_rows[c.seg]) c.row0 -= a.seg_rows[c.seg++];
       };
       auto advance = [&](Cursor& c) {
-        if (++c.kb == a.KB) { c.kb = 0; ++c.tile; locate(c); }
+        if (++c.kb == kb_hi) { c.kb = kb_lo; c.tile += tile_step; if (c.tile < a.tiles) locate(c); }
       };
-      Cursor ca, cb;
-      ca.tile = static_cast<int>(lo / a.KB);
-      ca.kb = static_cast<int>(lo % a.KB);
-      locate(ca);
-      cb = ca;
+      int n_my_tiles = 0;
+      for (int t = first_tile; t < a.tiles; t += tile_step) ++n_my_tiles;
+      const uint32_t n_units = static_cast<uint32_t>(n_my_tiles * nkb);
+      Cursor ca;
+      ca.tile = first_tile;
+      ca.kb = kb_lo;
+      if (ca.tile < a.tiles) locate(ca);
+      Cursor cb = ca;
       auto load_a = [&](uint32_t j, const Cursor& c) {
         const uint32_t s = j % S;
         const uint32_t dst = smem_u32(smem + static_cast<size_t>(s) * stage_bytes);
@@ -332,13 +391,12 @@ __global__ void __launch_bounds__(kThreads, 2) gemm_tc_kernel(const __grid_const
       const uint32_t idesc = idesc_bf16(kWRows, NT);
       uint32_t j = 0, segi = 0;
       bool ok = true;
-      for (long long u = lo; u < hi && ok; ++segi) {
-        const Seg sg = segment(u, hi, a.KB);
+      for (int t = first_tile; t < a.tiles && ok; t += tile_step, ++segi) {
         const uint32_t acc = segi & 1;
         if (!wait_bar(tempty0 + 8 * acc, ((segi >> 1) & 1) ^ 1, abort_flag, a.err)) break;
         tc_fence_after();
         const uint32_t d = tmem + acc * NT;
-        for (int i = 0; i < sg.nkb; ++i, ++j) {
+        for (int i = 0; i < nkb; ++i, ++j) {
           const uint32_t s = j % S;
           if (!wait_bar(full0 + 8 * s, (j / S) & 1, abort_flag, a.err)) { ok = false; break; }
           tc_fence_after();
@@ -352,90 +410,81 @@ __global__ void __launch_bounds__(kThreads, 2) gemm_tc_kernel(const __grid_const
         }
         if (!ok) break;
         mma_commit(tfull0 + 8 * acc);
-        u += sg.nkb;
       }
       mma_commit(drain);                      // all MMAs issued by this thread have completed
       wait_bar_budget(drain, 0, kDrainCycles);
     }
-    __syncwarp();
   } else {
     const int q = warp & 3;                   // TMEM lane quarter of this warp
     const int r = q * 32 + lane;              // weight row within the tile
     const bool leader = (warp == 2 && lane == 0);
     pdl_wait();                              // outputs, residuals and biases come from earlier kernels
     uint32_t segi = 0;
-    for (long long u = lo; u < hi; ++segi) {
-      const Seg sg = segment(u, hi, a.KB);
+    for (int t = first_tile; t < a.tiles; t += tile_step, ++segi) {
       const uint32_t acc = segi & 1;
       if (leader) flags[4] = wait_bar(tfull0 + 8 * acc, (segi >> 1) & 1, abort_flag, a.err) ? 1 : 0;
       named_bar_epi();
       const bool go = flags[4] != 0;
       tc_fence_after();
       if (!go) break;
-      const int wt = sg.tile % a.n_wtiles, tt = sg.tile / a.n_wtiles;
+      const int wt = t % a.n_wtiles, tt = t / a.n_wtiles;
       const uint32_t tbase = tmem + (static_cast<uint32_t>(q * 32) << 16) + acc * NT;
-      const bool full_tile = (sg.kb == 0 && sg.nkb == a.KB);
       const int nchunk = NT / 16;
-      const int rows_left = a.M - tt * NT;    // token columns of this tile that exist
-      if (full_tile) {
+      const int cols = min(NT, a.M - tt * NT);   // token columns of this tile that exist
+      if (sp == 1) {
         for (int ch = 0; ch < nchunk; ++ch) {
-          if (ch * 16 >= rows_left) break;
+          if (ch * 16 >= cols) break;
           float v[16];
           tmem_ld16(tbase + ch * 16, v);
           finish_chunk(a, wt, tt, r, ch * 16, v, xbuf);
         }
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(tempty0 + 8 * acc);
       } else {
-        // partial of a split tile: store it, then the last CTA to arrive sums them in k order
-        const int slot = (u == lo) ? 0 : 1;
-        float* wsrow = a.ws + ((static_cast<size_t>(c) * 2 + slot) * kWRows + r) * NT;
+        // this CTA's K-slice partial -> shared memory, summed across the cluster below
+        float* rp = reinterpret_cast<float*>(smem) + r * NT1;
         for (int ch = 0; ch < nchunk; ++ch) {
           float v[16];
           tmem_ld16(tbase + ch * 16, v);
 #pragma unroll
-          for (int j = 0; j < 16; j += 4)
-            *reinterpret_cast<float4*>(wsrow + ch * 16 + j) = make_float4(v[j], v[j + 1], v[j + 2], v[j + 3]);
+          for (int jj = 0; jj < 16; ++jj) rp[ch * 16 + jj] = v[jj];
         }
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(tempty0 + 8 * acc);
-        const long long t_lo = static_cast<long long>(sg.tile) * a.KB, t_hi = t_lo + a.KB;
-        const int c1 = cta_of(t_lo, U, G), c2 = cta_of(t_hi - 1, U, G);
-        named_bar_epi();                       // every partial row of this CTA is written
-        if (leader) {
-          __threadfence();                     // release them (cumulative over the barrier)
-          const int old = atomicAdd(&a.counters[sg.tile], 1);
-          const bool last = (old == c2 - c1);
-          if (last) a.counters[sg.tile] = 0;
-          __threadfence();                     // acquire the other CTAs' partials
-          flags[2] = last ? 1 : 0;
-        }
-        named_bar_epi();
-        if (flags[2]) {
-          for (int ch = 0; ch < nchunk; ++ch) {
-            if (ch * 16 >= rows_left) break;
-            float v[16];
-#pragma unroll
-            for (int j = 0; j < 16; ++j) v[j] = 0.f;
-#pragma unroll 8
-            for (int cc = c1; cc <= c2; ++cc) {
-              const int sl = (cta_lo(cc, U, G) / a.KB == sg.tile) ? 0 : 1;
-              const float* src = a.ws + ((static_cast<size_t>(cc) * 2 + sl) * kWRows + r) * NT + ch * 16;
-#pragma unroll
-              for (int j = 0; j < 16; j += 4) {
-                const float4 t = __ldcg(reinterpret_cast<const float4*>(src + j));
-                v[j] += t.x; v[j + 1] += t.y; v[j + 2] += t.z; v[j + 3] += t.w;
-              }
-            }
-            finish_chunk(a, wt, tt, r, ch * 16, v, xbuf);
-          }
-        }
-        named_bar_epi();
       }
-      u += sg.nkb;
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(tempty0 + 8 * acc);
     }
+  }
+
+  if (sp > 1) {
+    // Split-K reduction across the cluster: rank q finishes its share of the tile's rows
+    // (features for SwiGLU), summing the partials of ranks 0..sp-1 in order.
+    __syncwarp();
+    cluster_sync_all();                       // every rank's partial is in its shared memory
+    if (warp >= 2 && flags[0] == 0) {
+      const int tid = threadIdx.x - 64;
+      const int t = first_tile;
+      const int wt = t % a.n_wtiles, tt = t / a.n_wtiles;
+      const int cols = min(NT, a.M - tt * NT);
+      if (a.swiglu) {
+        const int f_lo = rank * 64 / sp, nf = (rank + 1) * 64 / sp - f_lo;
+        for (int e = tid; e < nf * cols; e += 128) {
+          const int f = f_lo + e % nf, col = e / nf;
+          emit_swiglu(a, wt, f, tt * NT + col, cluster_sum(red, NT1, f, col, sp),
+                      cluster_sum(red, NT1, f + 64, col, sp));
+        }
+      } else {
+        const int r_lo = rank * kWRows / sp, nr = (rank + 1) * kWRows / sp - r_lo;
+        for (int e = tid; e < nr * cols; e += 128) {
+          const int row = r_lo + e % nr, col = e / nr;
+          const float v = cluster_sum(red, NT1, row, col, sp);
+          if (a.epi == EPI_QKV)
+            emit_qkv(a, wt, row, tt * NT + col, v, cluster_sum(red, NT1, partner_row(a, row), col, sp));
+          else
+            emit_plain(a, wt, row, tt * NT + col, v);
+        }
+      }
+    }
+    __syncwarp();
+    cluster_sync_all();                       // no rank leaves while others read its partial
   }
 
   tc_fence_before();
@@ -519,21 +568,18 @@ int gemm_tc_token_tile(int M) {
   return nt > 256 ? 256 : (nt < 16 ? 16 : nt);
 }
 
-size_t gemm_tc_workspace_floats(int max_M) {
-  return static_cast<size_t>(512) * 2 * kWRows * gemm_tc_token_tile(max_M);
-}
 
 bool gemm_tc_supported(const GemmArgs& g) {
   if (g.K % kBK != 0 || g.K < kBK || g.M < 1 || g.ldx % 8 != 0) return false;
   if (reinterpret_cast<uintptr_t>(g.x) & 15) return false;
+  if (g.epi == EPI_QKV && (g.head_dim != 64 && g.head_dim != 128)) return false;
   if (g.epi == EPI_SWIGLU) return g.nseg == 2 && g.seg[0].rows == g.seg[1].rows && g.seg[0].rows % 64 == 0;
   for (int s = 0; s < g.nseg; ++s)
     if (g.seg[s].rows % kWRows != 0) return false;
   return true;
 }
 
-cudaError_t gemm_tc(const GemmArgs& g, float* ws, int* counters, size_t counters_len, unsigned* err,
-                    cudaStream_t st) {
+cudaError_t gemm_tc(const GemmArgs& g, unsigned* err, cudaStream_t st) {
   TcArgs a{};  // built on the host; passed by value as the kernel parameter
   a.nseg = g.nseg;
   a.swiglu = (g.epi == EPI_SWIGLU) ? 1 : 0;
@@ -549,20 +595,33 @@ cudaError_t gemm_tc(const GemmArgs& g, float* ws, int* counters, size_t counters
   a.M = g.M; a.K = g.K; a.KB = g.K / kBK;
   a.n_wtiles = a.swiglu ? g.seg[0].rows / 64 : N / kWRows;
   a.n_ttiles = (g.M + a.NT - 1) / a.NT;
-  const long long tiles = static_cast<long long>(a.n_wtiles) * a.n_ttiles;
-  if (static_cast<size_t>(tiles) > counters_len) return cudaErrorInvalidValue;
-  a.units = tiles * a.KB;
+  a.tiles = a.n_wtiles * a.n_ttiles;
   a.epi = g.epi; a.out = g.out; a.ldo = g.ldo; a.out_bf = static_cast<bf16*>(g.out_bf); a.ldh = g.ldh;
   a.bias = g.bias; a.ld_bias = g.ld_bias; a.row_seq = g.row_seq;
-  a.ws = ws; a.counters = counters; a.err = err;
+  a.err = err;
+  a.q_out = g.q_out; a.kv_pool = static_cast<bf16*>(g.kv_pool); a.kv_table = g.kv_table;
+  a.kv_bt_stride = g.kv_bt_stride; a.kv_n_blocks = g.kv_n_blocks; a.n_heads = g.n_heads;
+  a.n_kv_heads = g.n_kv_heads; a.head_dim = g.head_dim; a.layer = g.layer; a.rope_cs = g.rope_cs;
+  a.row_pos = g.row_pos; a.row_valid = g.row_valid;
+  // Split each tile's K over sp CTAs of a cluster when there are fewer tiles than SMs.
+  const int sms = sm_count();
+  int sp = 1;
+  if (a.tiles < sms && a.NT <= 128) {
+    sp = sms / a.tiles;
+    if (sp > 8) sp = 8;
+    if (sp > a.KB) sp = a.KB;
+    if (sp < 1) sp = 1;
+  }
+  a.sp = sp;
   const int stage_bytes = (kWRows + a.NT) * kBK * 2;
-  const int fixed = 1024 + 64 * 17 * 4 + 64 + 8 * (2 * 16 + 6);
-  // Up to NT = 128 the ring fits in half an SM's shared memory (and the two accumulators in half
-  // of TMEM), so the next GEMM's CTA can start on the same SM while this one drains.
+  const int fixed = 1024 + kWRows * kXS * 4 + 64 + 8 * (2 * 16 + 6);
+  // Up to NT = 128 the ring fits in half an SM's shared memory (and the accumulators in half of
+  // TMEM), so the next GEMM's CTA can start on the same SM while this one drains.
   int S = (kSmemShared - fixed) / stage_bytes;
   if (a.NT > 128 || S < 3) S = (kSmemBudget - fixed) / stage_bytes;
   if (S > 8) S = 8;
   if (S < 2) return cudaErrorInvalidValue;
+  if (sp > 1 && S * stage_bytes < kWRows * (a.NT + 1) * 4) return cudaErrorInvalidValue;  // partial tile
   a.stages = S;
   const int smem = fixed + S * stage_bytes;
   static bool configured = false;
@@ -571,15 +630,9 @@ cudaError_t gemm_tc(const GemmArgs& g, float* ws, int* counters, size_t counters
     if (e != cudaSuccess) return e;
     configured = true;
   }
-  // At least kMinUnits k-blocks (kMinUnits x 16 KB of weights) per CTA: fewer CTAs share a
-  // tile, so the last one to arrive sums fewer partials.
-  constexpr long long kMinUnits = 8;
-  long long G = sm_count();
-  const long long g_cap = (a.units + kMinUnits - 1) / kMinUnits;
-  if (G > g_cap) G = g_cap;
-  if (G > a.units) G = a.units;
-  if (G > 512) G = 512;
-  return launch_pdl(gemm_tc_kernel, dim3(static_cast<unsigned>(G)), dim3(kThreads), static_cast<size_t>(smem), st, a);
+  const int grid = sp > 1 ? a.tiles * sp : std::min(a.tiles, 2 * sms);
+  return launch_pdl_cluster(gemm_tc_kernel, dim3(static_cast<unsigned>(grid)), dim3(kThreads),
+                            static_cast<size_t>(smem), st, sp, a);
 }
 
 }  // namespace sd2

@@ -27,6 +27,31 @@ cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t s
   return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
 }
 
+// The same with a 1-D thread-block cluster of `cluster` CTAs (1 = no cluster).
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl_cluster(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                               int cluster, Args&&... args) {
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  int n = 1;
+  if (cluster > 1) {
+    attr[1].id = cudaLaunchAttributeClusterDimension;
+    attr[1].val.clusterDim.x = static_cast<unsigned>(cluster);
+    attr[1].val.clusterDim.y = 1;
+    attr[1].val.clusterDim.z = 1;
+    n = 2;
+  }
+  cfg.attrs = attr;
+  cfg.numAttrs = n;
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
+
 // ---------------------------------------------------------------- weight-streaming GEMM
 // Y[m, n] = sum_k X[m, k] W[n, k] for m < M, with W the row concatenation of up to three
 // bf16 segments (e.g. W_q | W_k | W_v). X is bf16 with row stride ldx; K % 8 == 0.
@@ -35,6 +60,8 @@ enum GemmEpilogue {
   EPI_ADD = 1,      // out[m*ldo + n] += y (f32 residual stream)
   EPI_SWIGLU = 2,   // Eq. 2: h[m*ldh + f] = bf16((up + bias[seq[m]*ld_bias + f]) * SiLU(gate));
                     //   segments: seg0 = W_gate [F, K], seg1 = W_up [F, K]
+  EPI_QKV = 3,      // segments W_q | W_k | W_v: rotary embedding on q and k, q -> q_out [M, H, hd] f32,
+                    //   k and v of valid rows -> the paged KV cache of `layer` at (row_seq, row_pos)
 };
 struct GemmSeg {
   const void* w;
@@ -53,21 +80,25 @@ struct GemmArgs {
   const float* bias;
   int ld_bias;
   const int* row_seq;
-  // tensor-core path: fp32 split-tile partials, per-tile arrival counters (zero between
-  // launches), the device error word; impl 0 = tensor cores when the shape allows, 1 = CUDA cores
-  float* ws;
-  int* counters;
-  size_t counters_len;
+  // the device error word (bounded waits) and the implementation: 0 = tensor cores when the
+  // shape allows, 1 = CUDA cores
   unsigned* err;
   int impl;
+  // EPI_QKV
+  float* q_out;
+  void* kv_pool;
+  const int* kv_table;
+  int kv_bt_stride, kv_n_blocks, n_heads, n_kv_heads, head_dim, layer;
+  const float* rope_cs;
+  const int* row_pos;
+  const int* row_valid;
 };
-// Dispatches to the tcgen05 kernel (gemm_tc.cu) when ws is set, impl != 1 and gemm_tc_supported
-// holds, else to the CUDA-core kernel (gemm_simt.cu).
+// Dispatches to the tcgen05 kernel (gemm_tc.cu) when impl != 1 and gemm_tc_supported holds, else
+// to the CUDA-core kernel (gemm_simt.cu).
 cudaError_t gemm(const GemmArgs& a, cudaStream_t st);
 bool gemm_tc_supported(const GemmArgs& a);
-cudaError_t gemm_tc(const GemmArgs& a, float* ws, int* counters, size_t counters_len, unsigned* err, cudaStream_t st);
+cudaError_t gemm_tc(const GemmArgs& a, unsigned* err, cudaStream_t st);
 int gemm_tc_token_tile(int M);
-size_t gemm_tc_workspace_floats(int max_M);
 cudaError_t gemm_simt(const GemmArgs& a, cudaStream_t st);
 
 // ---------------------------------------------------------------- decoder elementwise
@@ -103,7 +134,8 @@ cudaError_t gather_rows_bf16(const float* src, int ld_src, const int* idx, int w
 // Causal paged attention for query rows grouped by sequence: group g covers rows
 // grp_row0[g] .. +grp_nrows[g] of sequence grp_seq[g]; row r attends to cache positions
 // 0..row_pos[r]. The context is cut into splits of `chunk` positions (a multiple of 64);
-// with n_splits == 1 the result goes straight to out, otherwise partials are merged.
+// with n_splits == 1 the result goes straight to out, otherwise the last split of each
+// (group, KV head) to finish merges the partials.
 struct AttnArgs {
   const float* q;        // [M, H, hd] rotated queries
   KVCache kv;
@@ -115,6 +147,7 @@ struct AttnArgs {
   int n_groups, M, H, hd;
   int n_splits, chunk;
   float* part;           // [M, H, n_splits, hd + 2] scratch (n_splits > 1)
+  int* counters;         // [n_groups, Hkv] arrival counts of the splits, zero between launches
   void* out;             // [M, H * hd] bf16
 };
 cudaError_t attention(const AttnArgs& a, cudaStream_t st);

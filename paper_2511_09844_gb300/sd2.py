@@ -27,7 +27,7 @@ PROFILE_CLASSES = ["gemm", "attention", "accept", "sample", "other", "verify", "
 EXPORTS = ["sd2_init", "sd2_prefill", "sd2_step", "sd2_accept", "sd2_check", "sd2_free", "sd2_last_error",
            "sd2_set_graphs", "sd2_debug_buffer", "sd2_profile", "sd2_profile_read", "sd2_accept_workspace_bytes",
            "sd2_accept_logits", "sd2_steer_workspace_bytes", "sd2_steer", "sd2_swiglu_steered",
-           "sd2_accept_logits_noalloc", "sd2_gemm_workspace_bytes", "sd2_gemm", "sd2_set_gemm_impl"]
+           "sd2_accept_logits_noalloc", "sd2_gemm", "sd2_set_gemm_impl"]
 
 
 class LMConfig(ctypes.Structure):
@@ -83,16 +83,13 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
     lib.sd2_steer.argtypes = [c_void_p, c_int32, c_int32, c_void_p, c_void_p, c_void_p, c_float, c_int32, c_void_p,
                               c_int32, c_void_p, c_void_p, c_void_p, c_size_t, c_void_p]
     lib.sd2_swiglu_steered.argtypes = [c_void_p, c_void_p, c_void_p, c_void_p, c_int32, c_int32, c_void_p, c_void_p]
-    lib.sd2_gemm_workspace_bytes.argtypes = [c_int32]
-    lib.sd2_gemm_workspace_bytes.restype = c_size_t
     lib.sd2_gemm.argtypes = [c_void_p, c_int32, c_int32, c_int32, c_void_p, c_void_p, c_int32, c_int32, c_void_p,
-                             c_int32, c_void_p, c_void_p, c_void_p, c_int32, c_int32, c_void_p, c_size_t, c_void_p]
+                             c_int32, c_void_p, c_void_p, c_void_p, c_int32, c_int32, c_void_p]
     lib.sd2_set_gemm_impl.argtypes = [c_void_p, c_int32]
     lib.sd2_accept_logits_noalloc.argtypes = [c_void_p, c_void_p, c_int32, c_void_p, c_void_p, c_int32, c_int32,
                                               c_int32, c_uint64, c_uint32, c_void_p, c_void_p, c_void_p]
     for name in EXPORTS:
-        if name not in ("sd2_last_error", "sd2_accept_workspace_bytes", "sd2_steer_workspace_bytes",
-                        "sd2_gemm_workspace_bytes"):
+        if name not in ("sd2_last_error", "sd2_accept_workspace_bytes", "sd2_steer_workspace_bytes"):
             getattr(lib, name).restype = c_int32
     _LIB = lib
     return lib
@@ -297,8 +294,7 @@ def gemm(x: torch.Tensor, w: torch.Tensor, epilogue: int = 0, out: Optional[torc
         out = torch.empty((M, N), dtype=torch.float32, device=x.device)
     if epilogue == 2:
         h = torch.empty((M, N), dtype=torch.bfloat16, device=x.device)
-    ws = torch.empty(lib.sd2_gemm_workspace_bytes(M), dtype=torch.uint8, device=x.device)
     _check(lib, lib.sd2_gemm(_ptr(x), x.stride(0), M, K, _ptr(w), _ptr(w_up), N, epilogue, _ptr(out),
                              0 if out is None else out.stride(0), _ptr(h), _ptr(bias), _ptr(seq),
-                             0 if bias is None else bias.stride(0), impl, _ptr(ws), ws.numel(), _stream(stream)))
+                             0 if bias is None else bias.stride(0), impl, _stream(stream)))
     return h if epilogue == 2 else out

@@ -53,7 +53,7 @@ class ParityReport:
 
 
 def run(work, vw, dw, st, prompts, temps, seed, n_steps, max_ctx=None, graphs=True, tol=TOL,
-        check_taps=True) -> ParityReport:
+        check_taps=True, gemm_impl=0) -> ParityReport:
     """Run prefill + n_steps iterations on the GPU and check each against the oracle."""
     B, k, V = len(prompts), work.k, work.verifier.vocab
     if max_ctx is None:
@@ -62,6 +62,7 @@ def run(work, vw, dw, st, prompts, temps, seed, n_steps, max_ctx=None, graphs=Tr
     eng = sd2.SD2Engine(work, *dev, max_batch=B, max_ctx=max_ctx,
                         max_prefill_tokens=sum(len(p) for p in prompts))
     eng.set_graphs(graphs)
+    eng.set_gemm_impl(gemm_impl)
     rep = ParityReport()
     try:
         first = eng.prefill(prompts, temps, seed).cpu().tolist()

@@ -13,12 +13,14 @@ from paper_2511_09844_gb300 import workloads as W
 pytestmark = pytest.mark.gpu
 
 
+@pytest.mark.parametrize("gemm_impl", [0, 1])
 @pytest.mark.parametrize("temp", [0.0, 1.0])
-def test_tiny_single_sequence(temp):
+def test_tiny_single_sequence(temp, gemm_impl):
+    """gemm_impl 0: tensor-core GEMM with fused epilogues; 1: CUDA-core GEMM + separate kernels."""
     work = parity.tiny_work()
     vw, dw, st = parity.tiny_weights(work)
     prompts = W.make_prompts(work.verifier.vocab, 1, (32, 32), seed=7)
-    rep = parity.run(work, vw, dw, st, prompts, [temp], seed=1234, n_steps=8)
+    rep = parity.run(work, vw, dw, st, prompts, [temp], seed=1234, n_steps=8, gemm_impl=gemm_impl)
     assert rep.blocks == 8 and rep.decisions > 8 * work.k
 
 
