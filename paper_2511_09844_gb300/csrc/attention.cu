@@ -20,10 +20,13 @@ constexpr int kTile = 64;
 constexpr int kWarps = 8;
 constexpr int kQPW = 8;               // query vectors per warp
 constexpr int kMaxQV = kWarps * kQPW;  // per CTA
+constexpr int kMaxMergeSplits = 64;     // context splits one merge handles (weights in smem)
 
 template <int HD>
 constexpr int smem_bytes() {
-  return 2 * kTile * (HD + 8) * 2 + kMaxQV * HD * 4;
+  return (2 * kTile * (HD + 8) * 2 + kMaxQV * HD * 4) > (2 * kMaxQV * kMaxMergeSplits * 4)
+             ? (2 * kTile * (HD + 8) * 2 + kMaxQV * HD * 4)
+             : (2 * kMaxQV * kMaxMergeSplits * 4);
 }
 
 template <int HD>
@@ -173,36 +176,48 @@ __global__ void __launch_bounds__(kWarps * 32) attn_kernel(const AttnArgs a) {
   }
   __syncthreads();
   if (!last_flag) return;
-  // merge: out = sum_s acc_s e^{m_s - M} / sum_s l_s e^{m_s - M} for every (row, head) here
-  float* sM = sQ;                 // the queries are no longer needed
-  float* sL = sQ + kMaxQV;
+  // merge: out = sum_s acc_s e^{m_s - M} / sum_s l_s e^{m_s - M} for every (row, head) here.
+  // (1) every thread gathers (m_s, l_s) pairs into shared memory, (2) one thread per query
+  // vector turns them into split weights, (3) all threads form the weighted sums over hd with
+  // coalesced loads. At most kMaxMergeSplits splits, so the weights fit in shared memory.
+  float* sW = reinterpret_cast<float*>(smem);               // [kMaxQV][n_splits] weights
+  float* sL = sW + kMaxQV * kMaxMergeSplits;                 // [kMaxQV][n_splits] sums
+  const int NS = a.n_splits;
+  for (int idx = threadIdx.x; idx < nqv * NS; idx += blockDim.x) {
+    const int qv = idx / NS, s2 = idx % NS;
+    const int row = r0 + qv / G, h = kvh * G + qv % G;
+    const int ns = min(NS, a.row_pos[row] / a.chunk + 1);
+    const float* ps = a.part + ((static_cast<size_t>(row) * a.H + h) * NS + s2) * (HD + 2);
+    sW[qv * NS + s2] = s2 < ns ? __ldcg(ps) : -INFINITY;
+    sL[qv * NS + s2] = s2 < ns ? __ldcg(ps + 1) : 0.f;
+  }
+  __syncthreads();
   if (threadIdx.x < nqv) {
     const int qv = threadIdx.x;
-    const int row = r0 + qv / G, h = kvh * G + qv % G;
-    const int ns = min(a.n_splits, a.row_pos[row] / a.chunk + 1);
-    const float* p = a.part + (static_cast<size_t>(row) * a.H + h) * a.n_splits * (HD + 2);
     float M = -INFINITY;
-    for (int s2 = 0; s2 < ns; ++s2) M = fmaxf(M, __ldcg(p + s2 * (HD + 2)));
+    for (int s2 = 0; s2 < NS; ++s2) M = fmaxf(M, sW[qv * NS + s2]);
     float L = 0.f;
-    for (int s2 = 0; s2 < ns; ++s2) L += __ldcg(p + s2 * (HD + 2) + 1) * __expf(__ldcg(p + s2 * (HD + 2)) - M);
-    sM[qv] = M;
-    sL[qv] = 1.f / L;
+    for (int s2 = 0; s2 < NS; ++s2) {
+      const float w = __expf(sW[qv * NS + s2] - M);          // exp(-inf) = 0 for absent splits
+      sW[qv * NS + s2] = w;
+      L += sL[qv * NS + s2] * w;
+    }
+    const float inv = 1.f / L;
+    for (int s2 = 0; s2 < NS; ++s2) sW[qv * NS + s2] *= inv;
   }
   __syncthreads();
   for (int idx = threadIdx.x; idx < nqv * HD; idx += blockDim.x) {
     const int qv = idx / HD, d = idx % HD;
     const int row = r0 + qv / G, h = kvh * G + qv % G;
-    const int ns = min(a.n_splits, a.row_pos[row] / a.chunk + 1);
-    const float* p = a.part + (static_cast<size_t>(row) * a.H + h) * a.n_splits * (HD + 2);
-    const float M = sM[qv];
+    const int ns = min(NS, a.row_pos[row] / a.chunk + 1);
+    const float* p = a.part + (static_cast<size_t>(row) * a.H + h) * NS * (HD + 2) + 2 + d;
     float o = 0.f;
-    for (int s2 = 0; s2 < ns; ++s2) {
-      const float* ps = p + s2 * (HD + 2);
-      o += __ldcg(ps + 2 + d) * __expf(__ldcg(ps) - M);
-    }
-    static_cast<bf16*>(a.out)[static_cast<size_t>(row) * a.H * HD + h * HD + d] = __float2bfloat16_rn(o * sL[qv]);
+#pragma unroll 4
+    for (int s2 = 0; s2 < ns; ++s2) o += sW[qv * NS + s2] * __ldcg(p + static_cast<size_t>(s2) * (HD + 2));
+    static_cast<bf16*>(a.out)[static_cast<size_t>(row) * a.H * HD + h * HD + d] = __float2bfloat16_rn(o);
   }
 }
+
 
 template <int HD>
 cudaError_t launch(const AttnArgs& a, cudaStream_t st) {
@@ -221,6 +236,7 @@ cudaError_t launch(const AttnArgs& a, cudaStream_t st) {
 
 cudaError_t attention(const AttnArgs& a, cudaStream_t st) {
   if (a.n_groups <= 0) return cudaSuccess;
+  if (a.n_splits > kMaxMergeSplits || a.chunk % kTile != 0) return cudaErrorInvalidValue;
   if (a.hd == 128) return launch<128>(a, st);
   if (a.hd == 64) return launch<64>(a, st);
   return cudaErrorInvalidValue;

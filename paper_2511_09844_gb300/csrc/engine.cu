@@ -434,6 +434,9 @@ void drop_graphs(sd2_ctx* c) {
   c->g_step = c->g_accept = nullptr;
 }
 
+// Context positions per attention split: 64-position tiles, at most 64 splits.
+int attn_chunk(int max_ctx) { return 64 * std::max(1, (max_ctx + 64 * 64 - 1) / (64 * 64)); }
+
 // Attention row groups: consecutive rows of one sequence, at most `cap` rows per group.
 void add_groups(std::vector<int>& r0, std::vector<int>& nr, std::vector<int>& sq, int row0, int rows, int seq, int cap) {
   for (int t = 0; t < rows; t += cap) {
@@ -496,7 +499,7 @@ sd2_status sd2_init(const sd2_config* cfg, const sd2_weights* w, void* stream, s
   const int fmax = std::max(cfg->verifier.d_ffn, cfg->drafter.d_ffn);
   const int qkvmax = std::max(c->V.qkv_width(), c->D.qkv_width());
   const int hmax = std::max(cfg->verifier.n_heads * cfg->verifier.head_dim, cfg->drafter.n_heads * cfg->drafter.head_dim);
-  const int splits = (cfg->max_ctx + 63) / 64;
+  const int splits = (cfg->max_ctx + attn_chunk(cfg->max_ctx) - 1) / attn_chunk(cfg->max_ctx);
   const int hdmax = std::max(cfg->verifier.head_dim, cfg->drafter.head_dim);
   const int headsmax = std::max(cfg->verifier.n_heads, cfg->drafter.n_heads);
   auto go = [&]() -> sd2_status {
@@ -624,11 +627,11 @@ sd2_status sd2_prefill(sd2_ctx* c, int32_t batch, const int32_t* d_tokens, const
   Plan pd = pv;
   pd.n_groups = (int)dr0.size(); pd.g_row0 = S + o_dr0; pd.g_nrows = S + o_dnr; pd.g_seq = S + o_dsq;
   // step-shape plans (rows filled on the device each step)
-  const int splits = (c->cfg.max_ctx + 63) / 64;
+  const int chunk = attn_chunk(c->cfg.max_ctx), splits = (c->cfg.max_ctx + chunk - 1) / chunk;
   auto step_plan = [&](int M, int ng, int o0, int o1, int o2) {
     Plan p;
     p.M = M; p.tok = c->row_tok; p.pos = c->row_pos; p.seq = c->row_seq; p.valid = c->row_valid;
-    p.n_groups = ng; p.g_row0 = S + o0; p.g_nrows = S + o1; p.g_seq = S + o2; p.n_splits = splits; p.chunk = 64;
+    p.n_groups = ng; p.g_row0 = S + o0; p.g_nrows = S + o1; p.g_seq = S + o2; p.n_splits = splits; p.chunk = chunk;
     return p;
   };
   c->p_d1 = step_plan(2 * batch, (int)d1r0.size(), o_d1r0, o_d1nr, o_d1sq);
