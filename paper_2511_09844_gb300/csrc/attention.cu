@@ -1,13 +1,20 @@
 // Causal attention over the paged KV cache, grouped by sequence (verifier block of k+1 rows,
 // drafter rows, or prompt rows) and by KV head (grouped-query attention).
 //
-// One CTA = (row group of one sequence, KV head, split of the context). It stages the split's
-// K and V in 64-position tiles in shared memory (rows padded by 16 bytes so that the per-lane
-// 16-byte reads of eight lanes hit distinct banks), and each warp runs an online softmax for up
-// to 8 query vectors (query rows x the heads sharing the KV head). Every K/V byte of the split
-// is read from HBM once per CTA, whatever the number of rows in the group. With several splits
-// each CTA stores its partial (max, sum, accumulator) triples, and the last CTA of the
-// (group, KV head) to arrive merges them in split order.
+// One CTA = (row group of one sequence, KV head, split of the context). Its query vectors (query
+// rows x the heads sharing the KV head, at most 64) are the M side of two small contractions per
+// 64-position tile, both on the tensor cores with mma.sync m16n8k16 (bf16 in, f32 accumulate):
+//   scores S = Q K^T      warp w owns positions 8w .. 8w+7 of the tile, every query tile
+//   online softmax        4 threads per query row: running max/sum, P = e^{S - m} in bf16
+//   O = O * corr + P V    warp w owns 8 (hd 64) or 16 (hd 128) output dimensions
+// The contractions are tiny (M <= 64); the kernel is bound by the latency of its loads, so the
+// block ids of the split, the row positions and the queries are all fetched together, and K/V
+// tiles are staged with cp.async (zero-filled past the last position), the next tile in flight
+// while the current one is used. Every K/V byte of the split is read from HBM once per CTA.
+//
+// With several splits each CTA stores partial records [acc(hd) | max | sum | pad] (16-byte
+// aligned), and the last CTA of the (group, KV head) to arrive merges them: split weights first,
+// then the weighted sums with 16-byte loads, eight splits in flight at a time.
 #include <math.h>
 
 #include "common.cuh"
@@ -16,155 +23,315 @@
 namespace sd2 {
 namespace {
 
-constexpr int kTile = 64;
+constexpr int kTile = 64;               // positions per K/V tile
 constexpr int kWarps = 8;
-constexpr int kQPW = 8;               // query vectors per warp
-constexpr int kMaxQV = kWarps * kQPW;  // per CTA
+constexpr int kThreads = kWarps * 32;
+constexpr int kMaxQV = 64;              // query vectors per CTA
 constexpr int kMaxMergeSplits = 64;     // context splits one merge handles (weights in smem)
+constexpr int kMaxSmem = 200 * 1024;   // dynamic shared memory opt-in (static arrays come on top)
 
 template <int HD>
-constexpr int smem_bytes() {
-  return (2 * kTile * (HD + 8) * 2 + kMaxQV * HD * 4) > (2 * kMaxQV * kMaxMergeSplits * 4)
-             ? (2 * kTile * (HD + 8) * 2 + kMaxQV * HD * 4)
-             : (2 * kMaxQV * kMaxMergeSplits * 4);
+struct AttnSmem {
+  static constexpr int KS = HD + 8;                     // Q/K/V row stride, bf16 (conflict-free fragments)
+  static constexpr int SS = kTile + 8;                  // score row stride, f32
+  static constexpr int PS = kTile + 8;                  // probability row stride, bf16
+  static constexpr int REC = HD + 4;                    // partial record, f32
+  static constexpr int ROW_BYTES = 4 * kMaxQV * 4;      // position, correction, max, sum per query
+  static constexpr int Q_BYTES = kMaxQV * KS * 2;
+  static constexpr int S_BYTES = kMaxQV * SS * 4;
+  static constexpr int P_BYTES = kMaxQV * PS * 2;
+  static constexpr int KV_TILE = 2 * kTile * KS * 2;    // K and V of one tile
+  static constexpr int KV_OFF = ROW_BYTES + Q_BYTES + S_BYTES + P_BYTES;
+  static constexpr int MERGE_BYTES = 2 * kMaxQV * kMaxMergeSplits * 4;
+  static_assert(Q_BYTES + S_BYTES + P_BYTES + KV_TILE >= MERGE_BYTES, "merge arrays overlay the tile buffers");
+  __host__ __device__ static int nbuf(int chunk) { return chunk > kTile ? 2 : 1; }
+  static size_t bytes(int chunk) {
+    return static_cast<size_t>(KV_OFF) + static_cast<size_t>(nbuf(chunk)) * KV_TILE +
+           ((static_cast<size_t>(chunk / 16) * 4 + 15) & ~static_cast<size_t>(15));
+  }
+};
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ uint32_t ld_u32(const bf16* p) { return *reinterpret_cast<const uint32_t*>(p); }
+__device__ __forceinline__ uint32_t pack_bf2(float x, float y) {
+  const __nv_bfloat162 h = __floats2bfloat162_rn(x, y);
+  return *reinterpret_cast<const uint32_t*>(&h);
+}
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, bool valid) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(valid ? 16 : 0)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
+
+// D(16x8, f32) += A(16x16, bf16, row-major) * B(16x8, bf16, column-major)
+__device__ __forceinline__ void mma_bf16(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
+                                         uint32_t b0, uint32_t b1) {
+  asm("mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+      "{%0,%1,%2,%3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr)
+               : "memory");
+}
+__device__ __forceinline__ void ldsm_x2_t(uint32_t addr, uint32_t& r0, uint32_t& r1) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x2.trans.shared.b16 {%0,%1}, [%2];"
+               : "=r"(r0), "=r"(r1)
+               : "r"(addr)
+               : "memory");
 }
 
 template <int HD>
-__global__ void __launch_bounds__(kWarps * 32) attn_kernel(const AttnArgs a) {
+__global__ void __launch_bounds__(kThreads, 2) attn_kernel(const AttnArgs a) {
+  using L = AttnSmem<HD>;
+  constexpr int KS = L::KS, SS = L::SS, PS = L::PS, REC = L::REC;
+  constexpr int NT = HD / 64;  // n8 tiles of output dimensions per warp
   pdl_trigger();
   pdl_wait();
-  constexpr int DPL = HD / 32;        // output dims per lane
-  constexpr int KS = HD + 8;          // padded smem row (bf16 elements)
   extern __shared__ __align__(16) unsigned char smem[];
-  bf16* sK = reinterpret_cast<bf16*>(smem);
-  bf16* sV = sK + kTile * KS;
-  float* sQ = reinterpret_cast<float*>(sV + kTile * KS);
+  int* sPos = reinterpret_cast<int*>(smem);
+  float* sCorr = reinterpret_cast<float*>(smem) + kMaxQV;
+  float* sM = sCorr + kMaxQV;
+  float* sL = sM + kMaxQV;
+  bf16* sQ = reinterpret_cast<bf16*>(smem + L::ROW_BYTES);
+  float* sS = reinterpret_cast<float*>(smem + L::ROW_BYTES + L::Q_BYTES);
+  bf16* sP = reinterpret_cast<bf16*>(smem + L::ROW_BYTES + L::Q_BYTES + L::S_BYTES);
+  unsigned char* sKV = smem + L::KV_OFF;
+  int* sBlk = reinterpret_cast<int*>(sKV + L::nbuf(a.chunk) * L::KV_TILE);
+  __shared__ int sPmax[2];
+  __shared__ int last_flag;
 
   const int g = blockIdx.x, kvh = blockIdx.y, split = blockIdx.z;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int g8 = lane >> 2, t4 = lane & 3;
   const int r0 = a.grp_row0[g], nr = a.grp_nrows[g], seq = a.grp_seq[g];
-  const int Hkv = a.kv.Hkv, G = a.H / Hkv;
-  const int nqv = nr * G;
-  int pmax = 0;
-  for (int i = 0; i < nr; ++i) pmax = max(pmax, a.row_pos[r0 + i]);
+  const int Hkv = a.kv.Hkv, G = a.H / Hkv, nqv = nr * G;
   const int lo = split * a.chunk;
-  if (lo > pmax) return;
+
+  // Independent loads, all in flight together: block ids of the split, row positions, queries.
+  {
+    const int* table = a.kv.table + static_cast<size_t>(seq) * a.kv.bt_stride + (lo >> 4);
+    const int nblk = min(a.chunk >> 4, a.kv.bt_stride - (lo >> 4));
+    for (int i = tid; i < nblk; i += kThreads) sBlk[i] = table[i];
+  }
+  int pq = -1;
+  if (tid < nqv) pq = __ldcg(a.row_pos + r0 + tid / G);
+  constexpr int QC = HD / 4;                        // float4 per query vector
+  constexpr int QPT = kMaxQV * QC / kThreads;
+  float4 qr[QPT];
+#pragma unroll
+  for (int u = 0; u < QPT; ++u) {
+    const int idx = tid + u * kThreads, qv = idx / QC, c = idx % QC;
+    qr[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (qv < nqv)
+      qr[u] = __ldcg(reinterpret_cast<const float4*>(
+                         a.q + (static_cast<size_t>(r0 + qv / G) * a.H + kvh * G + qv % G) * HD) + c);
+  }
+  if (tid < kMaxQV) sPos[tid] = pq;
+#pragma unroll
+  for (int u = 0; u < QPT; ++u) {
+    const int idx = tid + u * kThreads, qv = idx / QC, c = idx % QC;
+    *reinterpret_cast<uint2*>(sQ + qv * KS + c * 4) = make_uint2(pack_bf2(qr[u].x, qr[u].y), pack_bf2(qr[u].z, qr[u].w));
+  }
+  const int wmax = __reduce_max_sync(0xffffffffu, pq);
+  if (warp < 2 && lane == 0) sPmax[warp] = wmax;
+  __syncthreads();
+  const int pmax = max(sPmax[0], sPmax[1]);
+  if (lo > pmax) return;  // the split starts after every row of the group
   const int hi = min(lo + a.chunk, pmax + 1);
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int ntiles = (hi - lo + kTile - 1) / kTile;
+  const int nmt = (nqv + 15) >> 4;
 
-  // queries of the group -> shared memory
-  for (int idx = threadIdx.x; idx < nqv * (HD / 4); idx += blockDim.x) {
-    const int qv = idx / (HD / 4), c = idx % (HD / 4);
-    const int row = r0 + qv / G, h = kvh * G + qv % G;
-    reinterpret_cast<float4*>(sQ)[qv * (HD / 4) + c] =
-        reinterpret_cast<const float4*>(a.q + (static_cast<size_t>(row) * a.H + h) * HD)[c];
-  }
-
-  float m_run[kQPW], l_run[kQPW], acc[kQPW][DPL];
-  int pos_r[kQPW];
-#pragma unroll
-  for (int j = 0; j < kQPW; ++j) {
-    m_run[j] = -INFINITY;
-    l_run[j] = 0.f;
-#pragma unroll
-    for (int d = 0; d < DPL; ++d) acc[j][d] = 0.f;
-    const int qv = warp + kWarps * j;
-    pos_r[j] = qv < nqv ? a.row_pos[r0 + qv / G] : -1;
-  }
-  const float scale = rsqrtf(static_cast<float>(HD));
   const bf16* pool = static_cast<const bf16*>(a.kv.pool);
   const size_t head_stride = static_cast<size_t>(16) * HD;
   const size_t blk_stride = static_cast<size_t>(2) * Hkv * head_stride;
-  const int* table = a.kv.table + static_cast<size_t>(seq) * a.kv.bt_stride;
-
-  for (int t0 = lo; t0 < hi; t0 += kTile) {
-    __syncthreads();
-    // stage K and V rows t0 .. t0+63 (zeros beyond hi)
-    constexpr int CPR = HD / 8;  // 16-byte chunks per row
-    for (int idx = threadIdx.x; idx < kTile * CPR; idx += blockDim.x) {
-      const int t = idx / CPR, c = idx % CPR;
+  const bf16* layer_base = pool + static_cast<size_t>(a.layer) * a.kv.n_blocks * blk_stride + kvh * head_stride;
+  // positions t0 .. t0+63 of tile i -> buffer i & 1 (zero-filled at and beyond hi)
+  auto issue_tile = [&](int i) {
+    bf16* dK = reinterpret_cast<bf16*>(sKV + (i & 1) * L::KV_TILE);
+    bf16* dV = dK + kTile * KS;
+    const int t0 = lo + i * kTile;
+#pragma unroll
+    for (int u = 0; u < kTile * (HD / 8) / kThreads; ++u) {
+      const int idx = tid + u * kThreads, t = idx / (HD / 8), c = idx % (HD / 8);
       const int p = t0 + t;
-      uint4 kvk = make_uint4(0, 0, 0, 0), kvv = make_uint4(0, 0, 0, 0);
-      if (p < hi) {
-        const int blk = table[p >> 4];
-        const bf16* base = pool + (static_cast<size_t>(a.layer) * a.kv.n_blocks + blk) * blk_stride +
-                           kvh * head_stride + (p & 15) * HD;
-        kvk = __ldg(reinterpret_cast<const uint4*>(base) + c);
-        kvv = __ldg(reinterpret_cast<const uint4*>(base + Hkv * head_stride) + c);
+      const bool ok = p < hi;
+      const bf16* src = layer_base;
+      if (ok) src += static_cast<size_t>(sBlk[(p - lo) >> 4]) * blk_stride + static_cast<size_t>(p & 15) * HD + c * 8;
+      cp_async16(smem_u32(dK + t * KS + c * 8), src, ok);
+      cp_async16(smem_u32(dV + t * KS + c * 8), ok ? src + Hkv * head_stride : layer_base, ok);
+    }
+    cp_async_commit();
+  };
+
+  const float scale = rsqrtf(static_cast<float>(HD));
+  const int srow = tid >> 2, squart = tid & 3;  // softmax: query row, quarter of the tile
+  float m_run = -INFINITY, l_run = 0.f;
+  float acc[4][NT][4];
+#pragma unroll
+  for (int mt = 0; mt < 4; ++mt)
+#pragma unroll
+    for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) acc[mt][nt][e] = 0.f;
+
+  issue_tile(0);
+  for (int i = 0; i < ntiles; ++i) {
+    cp_async_wait_all();
+    __syncthreads();  // tile i visible to all; every warp is past tile i-1, so its buffer is free
+    if (i + 1 < ntiles) issue_tile(i + 1);
+    const int t0 = lo + i * kTile;
+    const bf16* sK = reinterpret_cast<const bf16*>(sKV + (i & 1) * L::KV_TILE);
+    const bf16* sV = sK + kTile * KS;
+
+    // (1) S = Q K^T * scale, causal and range masks
+    {
+      const int n0 = warp * 8;
+      uint32_t kb[HD / 16][2];
+#pragma unroll
+      for (int kk = 0; kk < HD / 16; ++kk) {
+        const bf16* p = sK + (n0 + g8) * KS + kk * 16 + 2 * t4;
+        kb[kk][0] = ld_u32(p);
+        kb[kk][1] = ld_u32(p + 8);
       }
-      *reinterpret_cast<uint4*>(sK + t * KS + c * 8) = kvk;
-      *reinterpret_cast<uint4*>(sV + t * KS + c * 8) = kvv;
+      const int pc = t0 + n0 + 2 * t4;
+#pragma unroll
+      for (int mt = 0; mt < 4; ++mt) {
+        if (mt < nmt) {
+          float c[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+          for (int kk = 0; kk < HD / 16; ++kk) {
+            const bf16* qa = sQ + (mt * 16 + g8) * KS + kk * 16 + 2 * t4;
+            mma_bf16(c, ld_u32(qa), ld_u32(qa + 8 * KS), ld_u32(qa + 8), ld_u32(qa + 8 * KS + 8), kb[kk][0], kb[kk][1]);
+          }
+          const int qv = mt * 16 + g8;
+          const int pa = sPos[qv], pb = sPos[qv + 8];
+          float2 s_a, s_b;
+          s_a.x = (pc < hi && pc <= pa) ? c[0] * scale : -INFINITY;
+          s_a.y = (pc + 1 < hi && pc + 1 <= pa) ? c[1] * scale : -INFINITY;
+          s_b.x = (pc < hi && pc <= pb) ? c[2] * scale : -INFINITY;
+          s_b.y = (pc + 1 < hi && pc + 1 <= pb) ? c[3] * scale : -INFINITY;
+          *reinterpret_cast<float2*>(sS + qv * SS + n0 + 2 * t4) = s_a;
+          *reinterpret_cast<float2*>(sS + (qv + 8) * SS + n0 + 2 * t4) = s_b;
+        }
+      }
     }
     __syncthreads();
 
+    // (2) online softmax: P = e^{S - m_new} (bf16), corr = e^{m_old - m_new}
+    if (srow < nmt * 16) {  // whole warps: nmt * 64 threads
+      const float4* sr = reinterpret_cast<const float4*>(sS + srow * SS + squart * 16);
+      float v[16];
 #pragma unroll
-    for (int j = 0; j < kQPW; ++j) {
-      const int qv = warp + kWarps * j;
-      if (qv >= nqv) break;
-      if (pos_r[j] < t0) continue;  // whole tile after this row's position
-      const float* q = sQ + qv * HD;
-      float s0 = 0.f, s1 = 0.f;
-#pragma unroll 4
-      for (int c = 0; c < HD / 8; ++c) {
-        const float4 qa = reinterpret_cast<const float4*>(q)[2 * c];
-        const float4 qb = reinterpret_cast<const float4*>(q)[2 * c + 1];
-        const uint4 k0 = *reinterpret_cast<const uint4*>(sK + lane * KS + c * 8);
-        const uint4 k1 = *reinterpret_cast<const uint4*>(sK + (lane + 32) * KS + c * 8);
-        s0 = fmaf(qa.x, bf_lo(k0.x), s0); s0 = fmaf(qa.y, bf_hi(k0.x), s0);
-        s0 = fmaf(qa.z, bf_lo(k0.y), s0); s0 = fmaf(qa.w, bf_hi(k0.y), s0);
-        s0 = fmaf(qb.x, bf_lo(k0.z), s0); s0 = fmaf(qb.y, bf_hi(k0.z), s0);
-        s0 = fmaf(qb.z, bf_lo(k0.w), s0); s0 = fmaf(qb.w, bf_hi(k0.w), s0);
-        s1 = fmaf(qa.x, bf_lo(k1.x), s1); s1 = fmaf(qa.y, bf_hi(k1.x), s1);
-        s1 = fmaf(qa.z, bf_lo(k1.y), s1); s1 = fmaf(qa.w, bf_hi(k1.y), s1);
-        s1 = fmaf(qb.x, bf_lo(k1.z), s1); s1 = fmaf(qb.y, bf_hi(k1.z), s1);
-        s1 = fmaf(qb.z, bf_lo(k1.w), s1); s1 = fmaf(qb.w, bf_hi(k1.w), s1);
+      for (int u = 0; u < 4; ++u) {
+        const float4 f = sr[u];
+        v[4 * u] = f.x; v[4 * u + 1] = f.y; v[4 * u + 2] = f.z; v[4 * u + 3] = f.w;
       }
-      const int p0 = t0 + lane, p1 = t0 + lane + 32;
-      s0 = (p0 < hi && p0 <= pos_r[j]) ? s0 * scale : -INFINITY;
-      s1 = (p1 < hi && p1 <= pos_r[j]) ? s1 * scale : -INFINITY;
-      const float mt = warp_max(fmaxf(s0, s1));
-      const float m_new = fmaxf(m_run[j], mt);
-      const float corr = __expf(m_run[j] - m_new);
-      const float e0 = __expf(s0 - m_new), e1 = __expf(s1 - m_new);
-      l_run[j] = l_run[j] * corr + warp_sum(e0 + e1);
-      m_run[j] = m_new;
+      float mx = v[0];
 #pragma unroll
-      for (int d = 0; d < DPL; ++d) acc[j][d] *= corr;
-      const int tmax = min(32, hi - t0);
-      for (int t = 0; t < tmax; ++t) {
-        const float w0 = __shfl_sync(0xffffffffu, e0, t);
-        const float w1 = __shfl_sync(0xffffffffu, e1, t);
-        const bf16* v0 = sV + t * KS + lane * DPL;
-        const bf16* v1 = sV + (t + 32) * KS + lane * DPL;
+      for (int u = 1; u < 16; ++u) mx = fmaxf(mx, v[u]);
+      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
+      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
+      const float m_new = fmaxf(m_run, mx);
+      const float m_use = m_new == -INFINITY ? 0.f : m_new;  // a row with nothing visible yet
+      const float corr = __expf(m_run - m_use);
+      uint32_t pk[8];
+      float sum = 0.f;
 #pragma unroll
-        for (int d = 0; d < DPL; ++d)
-          acc[j][d] = fmaf(w0, bf2f(v0[d]), fmaf(w1, bf2f(v1[d]), acc[j][d]));
+      for (int u = 0; u < 8; ++u) {
+        const __nv_bfloat162 h = __floats2bfloat162_rn(__expf(v[2 * u] - m_use), __expf(v[2 * u + 1] - m_use));
+        sum += __low2float(h) + __high2float(h);
+        pk[u] = *reinterpret_cast<const uint32_t*>(&h);
+      }
+      uint4* dst = reinterpret_cast<uint4*>(sP + srow * PS + squart * 16);
+      dst[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+      dst[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+      sum += __shfl_xor_sync(0xffffffffu, sum, 1);
+      sum += __shfl_xor_sync(0xffffffffu, sum, 2);
+      l_run = l_run * corr + sum;
+      m_run = m_new;
+      if (squart == 0) sCorr[srow] = corr;
+    }
+    __syncthreads();
+
+    // (3) O = O * corr + P V over this warp's output dimensions
+    {
+      const int d0 = warp * 8 * NT;
+      uint32_t vb[kTile / 16][NT][2];
+#pragma unroll
+      for (int kk = 0; kk < kTile / 16; ++kk) {
+        const int row = kk * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
+        if constexpr (NT == 2) {
+          ldsm_x4_t(smem_u32(sV + row * KS + d0 + (lane >> 4) * 8), vb[kk][0][0], vb[kk][0][1], vb[kk][1][0], vb[kk][1][1]);
+        } else {
+          ldsm_x2_t(smem_u32(sV + row * KS + d0), vb[kk][0][0], vb[kk][0][1]);
+        }
+      }
+#pragma unroll
+      for (int mt = 0; mt < 4; ++mt) {
+        if (mt < nmt) {
+          const float ca = sCorr[mt * 16 + g8], cb = sCorr[mt * 16 + g8 + 8];
+#pragma unroll
+          for (int nt = 0; nt < NT; ++nt) {
+            acc[mt][nt][0] *= ca; acc[mt][nt][1] *= ca;
+            acc[mt][nt][2] *= cb; acc[mt][nt][3] *= cb;
+          }
+#pragma unroll
+          for (int kk = 0; kk < kTile / 16; ++kk) {
+            const bf16* pa = sP + (mt * 16 + g8) * PS + kk * 16 + 2 * t4;
+            const uint32_t a0 = ld_u32(pa), a1 = ld_u32(pa + 8 * PS), a2 = ld_u32(pa + 8), a3 = ld_u32(pa + 8 * PS + 8);
+#pragma unroll
+            for (int nt = 0; nt < NT; ++nt) mma_bf16(acc[mt][nt], a0, a1, a2, a3, vb[kk][nt][0], vb[kk][nt][1]);
+          }
+        }
       }
     }
   }
 
+  if (srow < nmt * 16 && squart == 0) { sM[srow] = m_run; sL[srow] = l_run; }
+  __syncthreads();
+  const int NS = a.n_splits;
+  {
+    const int d0 = warp * 8 * NT;
 #pragma unroll
-  for (int j = 0; j < kQPW; ++j) {
-    const int qv = warp + kWarps * j;
-    if (qv >= nqv) break;
-    const int row = r0 + qv / G, h = kvh * G + qv % G;
-    if (a.n_splits == 1) {
-      const float inv = 1.f / l_run[j];
-      bf16* o = static_cast<bf16*>(a.out) + static_cast<size_t>(row) * a.H * HD + h * HD + lane * DPL;
+    for (int mt = 0; mt < 4; ++mt) {
+      if (mt >= nmt) break;
 #pragma unroll
-      for (int d = 0; d < DPL; ++d) o[d] = __float2bfloat16_rn(acc[j][d] * inv);
-    } else {
-      float* p = a.part + ((static_cast<size_t>(row) * a.H + h) * a.n_splits + split) * (HD + 2);
-      if (lane == 0) { p[0] = m_run[j]; p[1] = l_run[j]; }
+      for (int half = 0; half < 2; ++half) {
+        const int qv = mt * 16 + g8 + 8 * half;
+        if (qv >= nqv) continue;
+        const size_t rh = static_cast<size_t>(r0 + qv / G) * a.H + kvh * G + qv % G;
 #pragma unroll
-      for (int d = 0; d < DPL; ++d) p[2 + lane * DPL + d] = acc[j][d];
+        for (int nt = 0; nt < NT; ++nt) {
+          const int d = d0 + nt * 8 + 2 * t4;
+          const float x = acc[mt][nt][2 * half], y = acc[mt][nt][2 * half + 1];
+          if (NS == 1) {
+            const float inv = 1.f / sL[qv];
+            *reinterpret_cast<__nv_bfloat162*>(static_cast<bf16*>(a.out) + rh * HD + d) =
+                __floats2bfloat162_rn(x * inv, y * inv);
+          } else {
+            *reinterpret_cast<float2*>(a.part + (rh * NS + split) * REC + d) = make_float2(x, y);
+          }
+        }
+      }
     }
   }
-  if (a.n_splits == 1) return;
+  if (NS == 1) return;
+  if (tid < nqv) {
+    const size_t rh = static_cast<size_t>(r0 + tid / G) * a.H + kvh * G + tid % G;
+    *reinterpret_cast<float2*>(a.part + (rh * NS + split) * REC + HD) = make_float2(sM[tid], sL[tid]);
+  }
 
   // The splits that run for this group are those starting at or before its last position.
-  __shared__ int last_flag;
+  __threadfence();
   __syncthreads();
-  if (threadIdx.x == 0) {
+  if (tid == 0) {
     int old;
     asm volatile("atom.acq_rel.gpu.global.add.s32 %0, [%1], 1;"
                  : "=r"(old)
@@ -176,67 +343,78 @@ __global__ void __launch_bounds__(kWarps * 32) attn_kernel(const AttnArgs a) {
   }
   __syncthreads();
   if (!last_flag) return;
-  // merge: out = sum_s acc_s e^{m_s - M} / sum_s l_s e^{m_s - M} for every (row, head) here.
-  // (1) every thread gathers (m_s, l_s) pairs into shared memory, (2) one thread per query
-  // vector turns them into split weights, (3) all threads form the weighted sums over hd with
-  // coalesced loads. At most kMaxMergeSplits splits, so the weights fit in shared memory.
-  float* sW = reinterpret_cast<float*>(smem);               // [kMaxQV][n_splits] weights
-  float* sL = sW + kMaxQV * kMaxMergeSplits;                 // [kMaxQV][n_splits] sums
-  const int NS = a.n_splits;
-  for (int idx = threadIdx.x; idx < nqv * NS; idx += blockDim.x) {
-    const int qv = idx / NS, s2 = idx % NS;
-    const int row = r0 + qv / G, h = kvh * G + qv % G;
-    const int ns = min(NS, a.row_pos[row] / a.chunk + 1);
-    const float* ps = a.part + ((static_cast<size_t>(row) * a.H + h) * NS + s2) * (HD + 2);
-    sW[qv * NS + s2] = s2 < ns ? __ldcg(ps) : -INFINITY;
-    sL[qv * NS + s2] = s2 < ns ? __ldcg(ps + 1) : 0.f;
-  }
-  __syncthreads();
-  if (threadIdx.x < nqv) {
-    const int qv = threadIdx.x;
-    float M = -INFINITY;
-    for (int s2 = 0; s2 < NS; ++s2) M = fmaxf(M, sW[qv * NS + s2]);
-    float L = 0.f;
-    for (int s2 = 0; s2 < NS; ++s2) {
-      const float w = __expf(sW[qv * NS + s2] - M);          // exp(-inf) = 0 for absent splits
-      sW[qv * NS + s2] = w;
-      L += sL[qv * NS + s2] * w;
-    }
-    const float inv = 1.f / L;
-    for (int s2 = 0; s2 < NS; ++s2) sW[qv * NS + s2] *= inv;
-  }
-  __syncthreads();
-  for (int idx = threadIdx.x; idx < nqv * HD; idx += blockDim.x) {
-    const int qv = idx / HD, d = idx % HD;
-    const int row = r0 + qv / G, h = kvh * G + qv % G;
-    const int ns = min(NS, a.row_pos[row] / a.chunk + 1);
-    const float* p = a.part + (static_cast<size_t>(row) * a.H + h) * NS * (HD + 2) + 2 + d;
-    float o = 0.f;
+
+  // merge: out = sum_s acc_s e^{m_s - M} / sum_s l_s e^{m_s - M} for every query vector here
+  float* sW = reinterpret_cast<float*>(smem + L::ROW_BYTES);  // [kMaxQV][NS] weights (over the tile buffers)
+  float* sLs = sW + kMaxQV * kMaxMergeSplits;                  // [kMaxQV][NS] sums
 #pragma unroll 4
-    for (int s2 = 0; s2 < ns; ++s2) o += sW[qv * NS + s2] * __ldcg(p + static_cast<size_t>(s2) * (HD + 2));
-    static_cast<bf16*>(a.out)[static_cast<size_t>(row) * a.H * HD + h * HD + d] = __float2bfloat16_rn(o);
+  for (int idx = tid; idx < nqv * NS; idx += kThreads) {
+    const int qv = idx / NS, s2 = idx % NS;
+    const int ns = min(NS, sPos[qv] / a.chunk + 1);
+    const size_t rh = static_cast<size_t>(r0 + qv / G) * a.H + kvh * G + qv % G;
+    float2 ml = make_float2(-INFINITY, 0.f);
+    if (s2 < ns) ml = __ldcg(reinterpret_cast<const float2*>(a.part + (rh * NS + s2) * REC + HD));
+    sW[qv * NS + s2] = ml.x;
+    sLs[qv * NS + s2] = ml.y;
+  }
+  __syncthreads();
+  if (tid < nqv) {
+    float M = -INFINITY;
+    for (int s2 = 0; s2 < NS; ++s2) M = fmaxf(M, sW[tid * NS + s2]);
+    float Lsum = 0.f;
+    for (int s2 = 0; s2 < NS; ++s2) {
+      const float w = __expf(sW[tid * NS + s2] - M);  // absent splits: e^{-inf} = 0
+      sW[tid * NS + s2] = w;
+      Lsum += sLs[tid * NS + s2] * w;
+    }
+    const float inv = 1.f / Lsum;
+    for (int s2 = 0; s2 < NS; ++s2) sW[tid * NS + s2] *= inv;
+  }
+  __syncthreads();
+  for (int e = tid; e < nqv * (HD / 4); e += kThreads) {
+    const int qv = e / (HD / 4), d4 = e % (HD / 4);
+    const int ns = min(NS, sPos[qv] / a.chunk + 1);
+    const size_t rh = static_cast<size_t>(r0 + qv / G) * a.H + kvh * G + qv % G;
+    const float* p = a.part + rh * NS * REC + d4 * 4;
+    const float* w = sW + qv * NS;
+    float4 o = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int s0 = 0; s0 < ns; s0 += 8) {
+      float4 v[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u)
+        v[u] = s0 + u < ns ? __ldcg(reinterpret_cast<const float4*>(p + static_cast<size_t>(s0 + u) * REC))
+                           : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const float wu = s0 + u < ns ? w[s0 + u] : 0.f;
+        o.x = fmaf(wu, v[u].x, o.x); o.y = fmaf(wu, v[u].y, o.y);
+        o.z = fmaf(wu, v[u].z, o.z); o.w = fmaf(wu, v[u].w, o.w);
+      }
+    }
+    *reinterpret_cast<uint2*>(static_cast<bf16*>(a.out) + rh * HD + d4 * 4) =
+        make_uint2(pack_bf2(o.x, o.y), pack_bf2(o.z, o.w));
   }
 }
-
 
 template <int HD>
 cudaError_t launch(const AttnArgs& a, cudaStream_t st) {
   static bool configured = false;
   if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(attn_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes<HD>());
+    const cudaError_t e = cudaFuncSetAttribute(attn_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, kMaxSmem);
     if (e != cudaSuccess) return e;
     configured = true;
   }
-  dim3 grid(a.n_groups, a.kv.Hkv, a.n_splits);
-  { const cudaError_t e_ = launch_pdl(attn_kernel<HD>, dim3(grid), dim3(kWarps * 32), smem_bytes<HD>(), st, a); if (e_ != cudaSuccess) return e_; }
-  return cudaGetLastError();
+  const size_t smem = AttnSmem<HD>::bytes(a.chunk);
+  if (smem > static_cast<size_t>(kMaxSmem)) return cudaErrorInvalidValue;
+  return launch_pdl(attn_kernel<HD>, dim3(a.n_groups, a.kv.Hkv, a.n_splits), dim3(kThreads), smem, st, a);
 }
 
 }  // namespace
 
 cudaError_t attention(const AttnArgs& a, cudaStream_t st) {
   if (a.n_groups <= 0) return cudaSuccess;
-  if (a.n_splits > kMaxMergeSplits || a.chunk % kTile != 0) return cudaErrorInvalidValue;
+  if (a.n_splits < 1 || a.n_splits > kMaxMergeSplits || a.chunk <= 0 || a.chunk % kTile != 0) return cudaErrorInvalidValue;
+  if (a.kv.Hkv <= 0 || a.H % a.kv.Hkv != 0 || a.H / a.kv.Hkv > kMaxQV) return cudaErrorInvalidValue;
   if (a.hd == 128) return launch<128>(a, st);
   if (a.hd == 64) return launch<64>(a, st);
   return cudaErrorInvalidValue;

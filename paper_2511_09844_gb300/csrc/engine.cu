@@ -517,7 +517,7 @@ sd2_status sd2_init(const sd2_config* cfg, const sd2_weights* w, void* stream, s
     ALLOC(c->qkv, static_cast<size_t>(R) * qkvmax);
     ALLOC(c->q, static_cast<size_t>(R) * hmax);
     ALLOC(c->attn, static_cast<size_t>(R) * hmax * 2);
-    c->part_elems = static_cast<size_t>(step_rows) * headsmax * splits * (hdmax + 2);
+    c->part_elems = static_cast<size_t>(step_rows) * headsmax * splits * (hdmax + 4);
     ALLOC(c->part, c->part_elems);
     ALLOC(c->h, static_cast<size_t>(R) * fmax * 2);
     ALLOC(c->logits_t, static_cast<size_t>(maxB) * (k + 1) * Vv);

@@ -146,7 +146,7 @@ struct AttnArgs {
   const int* grp_seq;
   int n_groups, M, H, hd;
   int n_splits, chunk;
-  float* part;           // [M, H, n_splits, hd + 2] scratch (n_splits > 1)
+  float* part;           // [M, H, n_splits, hd + 4] scratch (n_splits > 1): acc[hd], max, sum, pad
   int* counters;         // [n_groups, Hkv] arrival counts of the splits, zero between launches
   void* out;             // [M, H * hd] bf16
 };
