@@ -1,20 +1,22 @@
 // Causal attention over the paged KV cache, grouped by sequence (verifier block of k+1 rows,
 // drafter rows, or prompt rows) and by KV head (grouped-query attention).
 //
-// One CTA = (row group of one sequence, KV head, split of the context). Its query vectors (query
+// One CTA = (split of the context, row group of one sequence, KV head). Its query vectors (query
 // rows x the heads sharing the KV head, at most 64) are the M side of two small contractions per
 // 64-position tile, both on the tensor cores with mma.sync m16n8k16 (bf16 in, f32 accumulate):
 //   scores S = Q K^T      warp w owns positions 8w .. 8w+7 of the tile, every query tile
 //   online softmax        4 threads per query row: running max/sum, P = e^{S - m} in bf16
 //   O = O * corr + P V    warp w owns 8 (hd 64) or 16 (hd 128) output dimensions
-// The contractions are tiny (M <= 64); the kernel is bound by the latency of its loads, so the
-// block ids of the split, the row positions and the queries are all fetched together, and K/V
-// tiles are staged with cp.async (zero-filled past the last position), the next tile in flight
-// while the current one is used. Every K/V byte of the split is read from HBM once per CTA.
+// The contractions are tiny (M <= 64); the kernel is bound by the latency of its loads. The block
+// ids of the split are read before the programmatic wait (they are fixed before the step starts),
+// the row positions and queries are fetched together after it, and K/V tiles are staged with
+// cp.async (zero-filled past the last position), two tiles in flight. Every K/V byte of the split
+// is read from HBM once per CTA.
 //
-// With several splits each CTA stores partial records [acc(hd) | max | sum | pad] (16-byte
-// aligned), and the last CTA of the (group, KV head) to arrive merges them: split weights first,
-// then the weighted sums with 16-byte loads, eight splits in flight at a time.
+// The splits of one (row group, KV head) form a thread-block cluster (at most 8). Each CTA leaves
+// its partial (accumulator, max, sum) in shared memory; after a cluster barrier, rank r merges
+// the r-th share of the group's outputs, reading every split's partial through distributed shared
+// memory, so no partial goes through global memory and the merge is spread over the cluster.
 #include <math.h>
 
 #include "common.cuh"
@@ -27,28 +29,35 @@ constexpr int kTile = 64;               // positions per K/V tile
 constexpr int kWarps = 8;
 constexpr int kThreads = kWarps * 32;
 constexpr int kMaxQV = 64;              // query vectors per CTA
-constexpr int kMaxMergeSplits = 64;     // context splits one merge handles (weights in smem)
+constexpr int kMaxSplits = 8;           // context splits = CTAs of one cluster (portable size)
 constexpr int kMaxSmem = 200 * 1024;   // dynamic shared memory opt-in (static arrays come on top)
 
 template <int HD>
-struct AttnSmem {
+struct AttnCfg {
   static constexpr int KS = HD + 8;                     // Q/K/V row stride, bf16 (conflict-free fragments)
   static constexpr int SS = kTile + 8;                  // score row stride, f32
   static constexpr int PS = kTile + 8;                  // probability row stride, bf16
-  static constexpr int REC = HD + 4;                    // partial record, f32
-  static constexpr int ROW_BYTES = 4 * kMaxQV * 4;      // position, correction, max, sum per query
-  static constexpr int Q_BYTES = kMaxQV * KS * 2;
-  static constexpr int S_BYTES = kMaxQV * SS * 4;
-  static constexpr int P_BYTES = kMaxQV * PS * 2;
+  static constexpr int REC = HD + 4;                    // partial accumulator row, f32
+  // per query vector: position, correction, max, sum; per (query vector, split): max, sum / weight
+  static constexpr int ROW_BYTES = 4 * kMaxQV * 4 + 2 * kMaxQV * kMaxSplits * 4;
   static constexpr int KV_TILE = 2 * kTile * KS * 2;    // K and V of one tile
-  static constexpr int KV_OFF = ROW_BYTES + Q_BYTES + S_BYTES + P_BYTES;
-  static constexpr int MERGE_BYTES = 2 * kMaxQV * kMaxMergeSplits * 4;
-  static_assert(Q_BYTES + S_BYTES + P_BYTES + KV_TILE >= MERGE_BYTES, "merge arrays overlay the tile buffers");
-  __host__ __device__ static int nbuf(int chunk) { return chunk > kTile ? 2 : 1; }
-  static size_t bytes(int chunk) {
-    return static_cast<size_t>(KV_OFF) + static_cast<size_t>(nbuf(chunk)) * KV_TILE +
-           ((static_cast<size_t>(chunk / 16) * 4 + 15) & ~static_cast<size_t>(15));
+  __host__ __device__ static int qrows(int max_rows, int G) {
+    const int r = ((max_rows * G + 15) / 16) * 16;
+    return r < kMaxQV ? r : kMaxQV;
   }
+  __host__ __device__ static int nbuf(int chunk) { return chunk > kTile ? 2 : 1; }
+  __host__ __device__ static size_t q_off() { return ROW_BYTES; }
+  __host__ __device__ static size_t s_off(int qr) { return q_off() + static_cast<size_t>(qr) * KS * 2; }
+  __host__ __device__ static size_t p_off(int qr) { return s_off(qr) + static_cast<size_t>(qr) * SS * 4; }
+  __host__ __device__ static size_t kv_off(int qr) { return p_off(qr) + static_cast<size_t>(qr) * PS * 2; }
+  __host__ __device__ static size_t blk_off(int qr, int chunk) {
+    return kv_off(qr) + static_cast<size_t>(nbuf(chunk)) * KV_TILE;
+  }
+  static size_t bytes(int qr, int chunk) {
+    return blk_off(qr, chunk) + ((static_cast<size_t>(chunk / 16) * 4 + 15) & ~static_cast<size_t>(15));
+  }
+  // the partial accumulators [qr][REC] overlay Q, S and P once the tiles are done
+  static_assert(2 * KS + SS * 4 + PS * 2 >= REC * 4, "partials fit over the tile working set");
 };
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
@@ -64,7 +73,8 @@ __device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, bool v
                : "memory");
 }
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
 
 // D(16x8, f32) += A(16x16, bf16, row-major) * B(16x8, bf16, column-major)
 __device__ __forceinline__ void mma_bf16(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
@@ -89,37 +99,42 @@ __device__ __forceinline__ void ldsm_x2_t(uint32_t addr, uint32_t& r0, uint32_t&
 
 template <int HD>
 __global__ void __launch_bounds__(kThreads, 2) attn_kernel(const AttnArgs a) {
-  using L = AttnSmem<HD>;
-  constexpr int KS = L::KS, SS = L::SS, PS = L::PS, REC = L::REC;
+  using C = AttnCfg<HD>;
+  constexpr int KS = C::KS, SS = C::SS, PS = C::PS, REC = C::REC;
   constexpr int NT = HD / 64;  // n8 tiles of output dimensions per warp
   pdl_trigger();
-  pdl_wait();
   extern __shared__ __align__(16) unsigned char smem[];
+  __shared__ int sPmax[2];
+
+  const int split = blockIdx.x, g = blockIdx.y, kvh = blockIdx.z;
+  const int NS = a.n_splits;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int g8 = lane >> 2, t4 = lane & 3;
+  const int Hkv = a.kv.Hkv, G = a.H / Hkv;
+  const int QR = C::qrows(a.max_rows, G);
   int* sPos = reinterpret_cast<int*>(smem);
   float* sCorr = reinterpret_cast<float*>(smem) + kMaxQV;
   float* sM = sCorr + kMaxQV;
   float* sL = sM + kMaxQV;
-  bf16* sQ = reinterpret_cast<bf16*>(smem + L::ROW_BYTES);
-  float* sS = reinterpret_cast<float*>(smem + L::ROW_BYTES + L::Q_BYTES);
-  bf16* sP = reinterpret_cast<bf16*>(smem + L::ROW_BYTES + L::Q_BYTES + L::S_BYTES);
-  unsigned char* sKV = smem + L::KV_OFF;
-  int* sBlk = reinterpret_cast<int*>(sKV + L::nbuf(a.chunk) * L::KV_TILE);
-  __shared__ int sPmax[2];
-  __shared__ int last_flag;
+  float* sWm = sL + kMaxQV;                 // [kMaxQV][kMaxSplits] split maxima, then weights
+  float* sWl = sWm + kMaxQV * kMaxSplits;   // [kMaxQV][kMaxSplits] split sums
+  bf16* sQ = reinterpret_cast<bf16*>(smem + C::q_off());
+  float* sS = reinterpret_cast<float*>(smem + C::s_off(QR));
+  bf16* sP = reinterpret_cast<bf16*>(smem + C::p_off(QR));
+  unsigned char* sKV = smem + C::kv_off(QR);
+  int* sBlk = reinterpret_cast<int*>(smem + C::blk_off(QR, a.chunk));
 
-  const int g = blockIdx.x, kvh = blockIdx.y, split = blockIdx.z;
-  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int g8 = lane >> 2, t4 = lane & 3;
+  // The plan tables and the block table are written before the step's first kernel, so they are
+  // read before the wait; everything the preceding kernels write is read after it.
   const int r0 = a.grp_row0[g], nr = a.grp_nrows[g], seq = a.grp_seq[g];
-  const int Hkv = a.kv.Hkv, G = a.H / Hkv, nqv = nr * G;
+  const int nqv = nr * G;
   const int lo = split * a.chunk;
-
-  // Independent loads, all in flight together: block ids of the split, row positions, queries.
   {
     const int* table = a.kv.table + static_cast<size_t>(seq) * a.kv.bt_stride + (lo >> 4);
     const int nblk = min(a.chunk >> 4, a.kv.bt_stride - (lo >> 4));
     for (int i = tid; i < nblk; i += kThreads) sBlk[i] = table[i];
   }
+  pdl_wait();
   int pq = -1;
   if (tid < nqv) pq = __ldcg(a.row_pos + r0 + tid / G);
   constexpr int QC = HD / 4;                        // float4 per query vector
@@ -137,15 +152,18 @@ __global__ void __launch_bounds__(kThreads, 2) attn_kernel(const AttnArgs a) {
 #pragma unroll
   for (int u = 0; u < QPT; ++u) {
     const int idx = tid + u * kThreads, qv = idx / QC, c = idx % QC;
-    *reinterpret_cast<uint2*>(sQ + qv * KS + c * 4) = make_uint2(pack_bf2(qr[u].x, qr[u].y), pack_bf2(qr[u].z, qr[u].w));
+    if (qv < QR)
+      *reinterpret_cast<uint2*>(sQ + qv * KS + c * 4) =
+          make_uint2(pack_bf2(qr[u].x, qr[u].y), pack_bf2(qr[u].z, qr[u].w));
   }
   const int wmax = __reduce_max_sync(0xffffffffu, pq);
   if (warp < 2 && lane == 0) sPmax[warp] = wmax;
   __syncthreads();
   const int pmax = max(sPmax[0], sPmax[1]);
-  if (lo > pmax) return;  // the split starts after every row of the group
+  // A split that starts after every row of the group has no tiles; it still takes part in the
+  // cluster's merge with an empty partial.
   const int hi = min(lo + a.chunk, pmax + 1);
-  const int ntiles = (hi - lo + kTile - 1) / kTile;
+  const int ntiles = hi > lo ? (hi - lo + kTile - 1) / kTile : 0;
   const int nmt = (nqv + 15) >> 4;
 
   const bf16* pool = static_cast<const bf16*>(a.kv.pool);
@@ -154,7 +172,7 @@ __global__ void __launch_bounds__(kThreads, 2) attn_kernel(const AttnArgs a) {
   const bf16* layer_base = pool + static_cast<size_t>(a.layer) * a.kv.n_blocks * blk_stride + kvh * head_stride;
   // positions t0 .. t0+63 of tile i -> buffer i & 1 (zero-filled at and beyond hi)
   auto issue_tile = [&](int i) {
-    bf16* dK = reinterpret_cast<bf16*>(sKV + (i & 1) * L::KV_TILE);
+    bf16* dK = reinterpret_cast<bf16*>(sKV + (i & 1) * C::KV_TILE);
     bf16* dV = dK + kTile * KS;
     const int t0 = lo + i * kTile;
 #pragma unroll
@@ -181,13 +199,16 @@ __global__ void __launch_bounds__(kThreads, 2) attn_kernel(const AttnArgs a) {
 #pragma unroll
       for (int e = 0; e < 4; ++e) acc[mt][nt][e] = 0.f;
 
-  issue_tile(0);
+  // two tiles in flight: tiles 0 and 1 now, tile i+1 at the top of iteration i >= 1
+  if (ntiles > 0) issue_tile(0);
+  if (ntiles > 1) issue_tile(1);
   for (int i = 0; i < ntiles; ++i) {
-    cp_async_wait_all();
+    if (i == 0 && ntiles > 1) cp_async_wait<1>();
+    else cp_async_wait<0>();
     __syncthreads();  // tile i visible to all; every warp is past tile i-1, so its buffer is free
-    if (i + 1 < ntiles) issue_tile(i + 1);
+    if (i >= 1 && i + 1 < ntiles) issue_tile(i + 1);
     const int t0 = lo + i * kTile;
-    const bf16* sK = reinterpret_cast<const bf16*>(sKV + (i & 1) * L::KV_TILE);
+    const bf16* sK = reinterpret_cast<const bf16*>(sKV + (i & 1) * C::KV_TILE);
     const bf16* sV = sK + kTile * KS;
 
     // (1) S = Q K^T * scale, causal and range masks
@@ -295,10 +316,9 @@ __global__ void __launch_bounds__(kThreads, 2) attn_kernel(const AttnArgs a) {
   }
 
   if (srow < nmt * 16 && squart == 0) { sM[srow] = m_run; sL[srow] = l_run; }
-  __syncthreads();
-  const int NS = a.n_splits;
-  {
-    const int d0 = warp * 8 * NT;
+  __syncthreads();  // also: every warp is done with the tile working set that the partials overlay
+  const int d0 = warp * 8 * NT;
+  if (NS == 1) {
 #pragma unroll
     for (int mt = 0; mt < 4; ++mt) {
       if (mt >= nmt) break;
@@ -307,93 +327,83 @@ __global__ void __launch_bounds__(kThreads, 2) attn_kernel(const AttnArgs a) {
         const int qv = mt * 16 + g8 + 8 * half;
         if (qv >= nqv) continue;
         const size_t rh = static_cast<size_t>(r0 + qv / G) * a.H + kvh * G + qv % G;
+        const float inv = 1.f / sL[qv];
 #pragma unroll
-        for (int nt = 0; nt < NT; ++nt) {
-          const int d = d0 + nt * 8 + 2 * t4;
-          const float x = acc[mt][nt][2 * half], y = acc[mt][nt][2 * half + 1];
-          if (NS == 1) {
-            const float inv = 1.f / sL[qv];
-            *reinterpret_cast<__nv_bfloat162*>(static_cast<bf16*>(a.out) + rh * HD + d) =
-                __floats2bfloat162_rn(x * inv, y * inv);
-          } else {
-            *reinterpret_cast<float2*>(a.part + (rh * NS + split) * REC + d) = make_float2(x, y);
-          }
-        }
+        for (int nt = 0; nt < NT; ++nt)
+          *reinterpret_cast<__nv_bfloat162*>(static_cast<bf16*>(a.out) + rh * HD + d0 + nt * 8 + 2 * t4) =
+              __floats2bfloat162_rn(acc[mt][nt][2 * half] * inv, acc[mt][nt][2 * half + 1] * inv);
       }
     }
-  }
-  if (NS == 1) return;
-  if (tid < nqv) {
-    const size_t rh = static_cast<size_t>(r0 + tid / G) * a.H + kvh * G + tid % G;
-    *reinterpret_cast<float2*>(a.part + (rh * NS + split) * REC + HD) = make_float2(sM[tid], sL[tid]);
+    return;
   }
 
-  // The splits that run for this group are those starting at or before its last position.
-  __threadfence();
-  __syncthreads();
-  if (tid == 0) {
-    int old;
-    asm volatile("atom.acq_rel.gpu.global.add.s32 %0, [%1], 1;"
-                 : "=r"(old)
-                 : "l"(a.counters + static_cast<size_t>(g) * Hkv + kvh)
-                 : "memory");
-    const int n_used = pmax / a.chunk + 1;
-    last_flag = (old == n_used - 1) ? 1 : 0;
-    if (last_flag) a.counters[static_cast<size_t>(g) * Hkv + kvh] = 0;
+  // Split merge across the cluster (rank = split): out = sum_s acc_s e^{m_s - M} / sum_s l_s e^{m_s - M}.
+  // Each CTA publishes its partial in shared memory; rank r then finishes the r-th share of the
+  // group's (query vector, 4 dimensions) elements, reading the partials of every split.
+  float* sAcc = reinterpret_cast<float*>(smem + C::q_off());  // [QR][REC]
+#pragma unroll
+  for (int mt = 0; mt < 4; ++mt) {
+    if (mt >= nmt) break;
+#pragma unroll
+    for (int half = 0; half < 2; ++half) {
+      const int qv = mt * 16 + g8 + 8 * half;
+#pragma unroll
+      for (int nt = 0; nt < NT; ++nt)
+        *reinterpret_cast<float2*>(sAcc + qv * REC + d0 + nt * 8 + 2 * t4) =
+            make_float2(acc[mt][nt][2 * half], acc[mt][nt][2 * half + 1]);
+    }
   }
-  __syncthreads();
-  if (!last_flag) return;
-
-  // merge: out = sum_s acc_s e^{m_s - M} / sum_s l_s e^{m_s - M} for every query vector here
-  float* sW = reinterpret_cast<float*>(smem + L::ROW_BYTES);  // [kMaxQV][NS] weights (over the tile buffers)
-  float* sLs = sW + kMaxQV * kMaxMergeSplits;                  // [kMaxQV][NS] sums
-#pragma unroll 4
-  for (int idx = tid; idx < nqv * NS; idx += kThreads) {
-    const int qv = idx / NS, s2 = idx % NS;
-    const int ns = min(NS, sPos[qv] / a.chunk + 1);
-    const size_t rh = static_cast<size_t>(r0 + qv / G) * a.H + kvh * G + qv % G;
-    float2 ml = make_float2(-INFINITY, 0.f);
-    if (s2 < ns) ml = __ldcg(reinterpret_cast<const float2*>(a.part + (rh * NS + s2) * REC + HD));
-    sW[qv * NS + s2] = ml.x;
-    sLs[qv * NS + s2] = ml.y;
+  cluster_sync_all();  // every split's partial is in its shared memory
+  for (int t = tid; t < nqv * NS; t += kThreads) {
+    const int qv = t / NS, s2 = t % NS;
+    const int ns = min(NS, sPos[qv] / a.chunk + 1);  // splits that start at or before this row
+    float m = -INFINITY, l = 0.f;
+    if (s2 < ns) {
+      m = ld_dsmem(smem_u32(sM + qv), s2);
+      l = ld_dsmem(smem_u32(sL + qv), s2);
+    }
+    sWm[qv * kMaxSplits + s2] = m;
+    sWl[qv * kMaxSplits + s2] = l;
   }
   __syncthreads();
   if (tid < nqv) {
+    float* wm = sWm + tid * kMaxSplits;
+    const float* wl = sWl + tid * kMaxSplits;
     float M = -INFINITY;
-    for (int s2 = 0; s2 < NS; ++s2) M = fmaxf(M, sW[tid * NS + s2]);
+    for (int s2 = 0; s2 < NS; ++s2) M = fmaxf(M, wm[s2]);
     float Lsum = 0.f;
     for (int s2 = 0; s2 < NS; ++s2) {
-      const float w = __expf(sW[tid * NS + s2] - M);  // absent splits: e^{-inf} = 0
-      sW[tid * NS + s2] = w;
-      Lsum += sLs[tid * NS + s2] * w;
+      const float w = __expf(wm[s2] - M);  // absent splits: e^{-inf} = 0
+      wm[s2] = w;
+      Lsum += wl[s2] * w;
     }
     const float inv = 1.f / Lsum;
-    for (int s2 = 0; s2 < NS; ++s2) sW[tid * NS + s2] *= inv;
+    for (int s2 = 0; s2 < NS; ++s2) wm[s2] *= inv;
   }
   __syncthreads();
-  for (int e = tid; e < nqv * (HD / 4); e += kThreads) {
+  const int E4 = nqv * (HD / 4);
+  const int e_hi = (split + 1) * E4 / NS;
+  const uint32_t acc_base = smem_u32(sAcc);
+  for (int e = split * E4 / NS + tid; e < e_hi; e += kThreads) {
     const int qv = e / (HD / 4), d4 = e % (HD / 4);
     const int ns = min(NS, sPos[qv] / a.chunk + 1);
-    const size_t rh = static_cast<size_t>(r0 + qv / G) * a.H + kvh * G + qv % G;
-    const float* p = a.part + rh * NS * REC + d4 * 4;
-    const float* w = sW + qv * NS;
+    const uint32_t addr = acc_base + static_cast<uint32_t>((qv * REC + d4 * 4) * 4);
+    float4 v[kMaxSplits];
+#pragma unroll
+    for (int s2 = 0; s2 < kMaxSplits; ++s2)
+      v[s2] = s2 < ns ? ld_dsmem_v4(addr, s2) : make_float4(0.f, 0.f, 0.f, 0.f);
     float4 o = make_float4(0.f, 0.f, 0.f, 0.f);
-    for (int s0 = 0; s0 < ns; s0 += 8) {
-      float4 v[8];
 #pragma unroll
-      for (int u = 0; u < 8; ++u)
-        v[u] = s0 + u < ns ? __ldcg(reinterpret_cast<const float4*>(p + static_cast<size_t>(s0 + u) * REC))
-                           : make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll
-      for (int u = 0; u < 8; ++u) {
-        const float wu = s0 + u < ns ? w[s0 + u] : 0.f;
-        o.x = fmaf(wu, v[u].x, o.x); o.y = fmaf(wu, v[u].y, o.y);
-        o.z = fmaf(wu, v[u].z, o.z); o.w = fmaf(wu, v[u].w, o.w);
-      }
+    for (int s2 = 0; s2 < kMaxSplits; ++s2) {
+      const float w = s2 < ns ? sWm[qv * kMaxSplits + s2] : 0.f;
+      o.x = fmaf(w, v[s2].x, o.x); o.y = fmaf(w, v[s2].y, o.y);
+      o.z = fmaf(w, v[s2].z, o.z); o.w = fmaf(w, v[s2].w, o.w);
     }
+    const size_t rh = static_cast<size_t>(r0 + qv / G) * a.H + kvh * G + qv % G;
     *reinterpret_cast<uint2*>(static_cast<bf16*>(a.out) + rh * HD + d4 * 4) =
         make_uint2(pack_bf2(o.x, o.y), pack_bf2(o.z, o.w));
   }
+  cluster_sync_all();  // no CTA leaves while another still reads its shared memory
 }
 
 template <int HD>
@@ -404,17 +414,20 @@ cudaError_t launch(const AttnArgs& a, cudaStream_t st) {
     if (e != cudaSuccess) return e;
     configured = true;
   }
-  const size_t smem = AttnSmem<HD>::bytes(a.chunk);
+  const int qr = AttnCfg<HD>::qrows(a.max_rows, a.H / a.kv.Hkv);
+  const size_t smem = AttnCfg<HD>::bytes(qr, a.chunk);
   if (smem > static_cast<size_t>(kMaxSmem)) return cudaErrorInvalidValue;
-  return launch_pdl(attn_kernel<HD>, dim3(a.n_groups, a.kv.Hkv, a.n_splits), dim3(kThreads), smem, st, a);
+  return launch_pdl_cluster(attn_kernel<HD>, dim3(a.n_splits, a.n_groups, a.kv.Hkv), dim3(kThreads), smem, st,
+                            a.n_splits, a);
 }
 
 }  // namespace
 
 cudaError_t attention(const AttnArgs& a, cudaStream_t st) {
   if (a.n_groups <= 0) return cudaSuccess;
-  if (a.n_splits < 1 || a.n_splits > kMaxMergeSplits || a.chunk <= 0 || a.chunk % kTile != 0) return cudaErrorInvalidValue;
-  if (a.kv.Hkv <= 0 || a.H % a.kv.Hkv != 0 || a.H / a.kv.Hkv > kMaxQV) return cudaErrorInvalidValue;
+  if (a.n_splits < 1 || a.n_splits > kMaxSplits || a.chunk <= 0 || a.chunk % kTile != 0) return cudaErrorInvalidValue;
+  if (a.kv.Hkv <= 0 || a.H % a.kv.Hkv != 0 || a.max_rows < 1 || a.max_rows * (a.H / a.kv.Hkv) > kMaxQV)
+    return cudaErrorInvalidValue;
   if (a.hd == 128) return launch<128>(a, st);
   if (a.hd == 64) return launch<64>(a, st);
   return cudaErrorInvalidValue;

@@ -173,6 +173,39 @@ __device__ __forceinline__ float packed_key(unsigned long long p) {
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 __device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 
+// ------------------------------------------------------------------------------------------
+// Thread-block clusters: rank, full barrier (release/acquire), and loads from the shared memory
+// of another CTA of the cluster (distributed shared memory).
+// ------------------------------------------------------------------------------------------
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+__device__ __forceinline__ uint32_t dsmem_addr(uint32_t saddr, uint32_t rank) {
+  uint32_t remote;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(saddr), "r"(rank));
+  return remote;
+}
+// fp32 at shared-memory address `saddr` of CTA `rank` of this cluster
+__device__ __forceinline__ float ld_dsmem(uint32_t saddr, uint32_t rank) {
+  float v;
+  asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(dsmem_addr(saddr, rank)) : "memory");
+  return v;
+}
+// four fp32 (16-byte aligned) at `saddr` of CTA `rank`
+__device__ __forceinline__ float4 ld_dsmem_v4(uint32_t saddr, uint32_t rank) {
+  float4 v;
+  asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
+               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+               : "r"(dsmem_addr(saddr, rank))
+               : "memory");
+  return v;
+}
+
 // Device error word bits (latched; read and cleared by the host).
 enum { ERR_NONFINITE = 1, ERR_TIMEOUT = 2 };
 

@@ -60,6 +60,7 @@ struct Plan {
   const int* g_nrows = nullptr;
   const int* g_seq = nullptr;
   int n_splits = 1, chunk = 64;
+  int max_rows = 1;  // rows of the largest attention group
 };
 
 struct ProfRec {
@@ -87,13 +88,10 @@ struct sd2_ctx {
   int* statics = nullptr;  // group tables and row lists of the step shapes, then prefill's
   int statics_cap = 0;
   // activations
-  float *x = nullptr, *qkv = nullptr, *q = nullptr, *part = nullptr, *logits_t = nullptr, *logits_d = nullptr;
+  float *x = nullptr, *qkv = nullptr, *q = nullptr, *logits_t = nullptr, *logits_d = nullptr;
   float *taps = nullptr, *g_pre = nullptr, *g = nullptr, *bias = nullptr;
   void *a = nullptr, *attn = nullptr, *h = nullptr, *g_bf = nullptr, *hml_in = nullptr;
-  size_t part_elems = 0;
   int gemm_impl = 0;            // 0 tensor cores where the shape allows, 1 CUDA cores
-  int* attn_cnt = nullptr;      // attention split arrivals per (row group, KV head), zero between launches
-  size_t attn_cnt_len = 0;
   unsigned long long* samp_slot = nullptr;
   int* samp_counter = nullptr;
   AcceptScratch as{};
@@ -275,8 +273,7 @@ sd2_status forward(sd2_ctx* c, const Model& m, const Plan& p, const FwdOut& o) {
     AttnArgs at{};
     at.q = c->q; at.kv = m.cache(); at.layer = l; at.row_pos = p.pos;
     at.grp_row0 = p.g_row0; at.grp_nrows = p.g_nrows; at.grp_seq = p.g_seq; at.n_groups = p.n_groups;
-    at.M = M; at.H = H; at.hd = hd; at.n_splits = p.n_splits; at.chunk = p.chunk; at.part = c->part; at.out = c->attn;
-    at.counters = c->attn_cnt;
+    at.M = M; at.H = H; at.hd = hd; at.n_splits = p.n_splits; at.chunk = p.chunk; at.max_rows = p.max_rows; at.out = c->attn;
     double kvb = 0;
     if (c->prof && !c->h_n.empty()) {
       for (int b = 0; b < c->B; ++b) kvb += 2.0 * 2.0 * Hkv * hd * (c->h_n[b] + 16);
@@ -434,8 +431,8 @@ void drop_graphs(sd2_ctx* c) {
   c->g_step = c->g_accept = nullptr;
 }
 
-// Context positions per attention split: 64-position tiles, at most 64 splits.
-int attn_chunk(int max_ctx) { return 64 * std::max(1, (max_ctx + 64 * 64 - 1) / (64 * 64)); }
+// Context positions per attention split: whole 64-position tiles, at most 8 splits (one cluster).
+int attn_chunk(int max_ctx) { return 64 * std::max(1, (max_ctx + 8 * 64 - 1) / (8 * 64)); }
 
 // Attention row groups: consecutive rows of one sequence, at most `cap` rows per group.
 void add_groups(std::vector<int>& r0, std::vector<int>& nr, std::vector<int>& sq, int row0, int rows, int seq, int cap) {
@@ -499,9 +496,6 @@ sd2_status sd2_init(const sd2_config* cfg, const sd2_weights* w, void* stream, s
   const int fmax = std::max(cfg->verifier.d_ffn, cfg->drafter.d_ffn);
   const int qkvmax = std::max(c->V.qkv_width(), c->D.qkv_width());
   const int hmax = std::max(cfg->verifier.n_heads * cfg->verifier.head_dim, cfg->drafter.n_heads * cfg->drafter.head_dim);
-  const int splits = (cfg->max_ctx + attn_chunk(cfg->max_ctx) - 1) / attn_chunk(cfg->max_ctx);
-  const int hdmax = std::max(cfg->verifier.head_dim, cfg->drafter.head_dim);
-  const int headsmax = std::max(cfg->verifier.n_heads, cfg->drafter.n_heads);
   auto go = [&]() -> sd2_status {
     ALLOC(c->state, 4 * maxB);
     ALLOC(c->committed, static_cast<size_t>(maxB) * cfg->max_ctx);
@@ -517,8 +511,6 @@ sd2_status sd2_init(const sd2_config* cfg, const sd2_weights* w, void* stream, s
     ALLOC(c->qkv, static_cast<size_t>(R) * qkvmax);
     ALLOC(c->q, static_cast<size_t>(R) * hmax);
     ALLOC(c->attn, static_cast<size_t>(R) * hmax * 2);
-    c->part_elems = static_cast<size_t>(step_rows) * headsmax * splits * (hdmax + 4);
-    ALLOC(c->part, c->part_elems);
     ALLOC(c->h, static_cast<size_t>(R) * fmax * 2);
     ALLOC(c->logits_t, static_cast<size_t>(maxB) * (k + 1) * Vv);
     ALLOC(c->logits_d, static_cast<size_t>(maxB) * k * Vv);
@@ -528,9 +520,6 @@ sd2_status sd2_init(const sd2_config* cfg, const sd2_weights* w, void* stream, s
     ALLOC(c->g, static_cast<size_t>(maxB) * cfg->d_steer);
     ALLOC(c->g_bf, static_cast<size_t>(maxB) * cfg->d_steer * 2);
     ALLOC(c->bias, static_cast<size_t>(maxB) * cfg->drafter.n_layers * cfg->drafter.d_ffn);
-    c->attn_cnt_len = static_cast<size_t>(maxB) * 17 * 64;
-    ALLOC(c->attn_cnt, c->attn_cnt_len);
-    CK(cudaMemset(c->attn_cnt, 0, sizeof(int) * c->attn_cnt_len));
     ALLOC(c->samp_slot, maxB);
     ALLOC(c->samp_counter, maxB);
     void* acc;
@@ -612,9 +601,6 @@ sd2_status sd2_prefill(sd2_ctx* c, int32_t batch, const int32_t* d_tokens, const
   std::vector<int> cu(h_cu_lens, h_cu_lens + batch + 1);
   const int o_cu = push(cu);
   if ((int)st.size() > c->statics_cap) return fail(c, SD2_ECAPACITY, "plan tables exceed their buffer");
-  const size_t max_groups = std::max(std::max(d1r0.size(), dnr0.size()), sr0.size());
-  if (max_groups * static_cast<size_t>(std::max(c->V.c.n_kv_heads, c->D.c.n_kv_heads)) > c->attn_cnt_len)
-    return fail(c, SD2_ECAPACITY, "attention counter table too small for this batch");
   CK(cudaMemcpyAsync(c->statics, st.data(), st.size() * sizeof(int), cudaMemcpyHostToDevice, c->st));
   std::vector<float> temps(h_temperature, h_temperature + batch);
   CK(cudaMemcpyAsync(c->temp, temps.data(), batch * sizeof(float), cudaMemcpyHostToDevice, c->st));
@@ -623,20 +609,22 @@ sd2_status sd2_prefill(sd2_ctx* c, int32_t batch, const int32_t* d_tokens, const
   Plan pv;
   pv.M = total; pv.tok = d_tokens; pv.pos = S + o_pos; pv.seq = S + o_seq; pv.valid = S + o_valid;
   pv.n_groups = (int)vr0.size(); pv.g_row0 = S + o_vr0; pv.g_nrows = S + o_vnr; pv.g_seq = S + o_vsq;
-  pv.n_splits = 1; pv.chunk = ((maxlen + 63) / 64) * 64;
+  pv.n_splits = 1; pv.chunk = ((maxlen + 63) / 64) * 64; pv.max_rows = std::min(maxlen, c->V.group_rows());
   Plan pd = pv;
   pd.n_groups = (int)dr0.size(); pd.g_row0 = S + o_dr0; pd.g_nrows = S + o_dnr; pd.g_seq = S + o_dsq;
+  pd.max_rows = std::min(maxlen, c->D.group_rows());
   // step-shape plans (rows filled on the device each step)
   const int chunk = attn_chunk(c->cfg.max_ctx), splits = (c->cfg.max_ctx + chunk - 1) / chunk;
-  auto step_plan = [&](int M, int ng, int o0, int o1, int o2) {
+  auto step_plan = [&](int M, int ng, int o0, int o1, int o2, int rows) {
     Plan p;
+    p.max_rows = rows;
     p.M = M; p.tok = c->row_tok; p.pos = c->row_pos; p.seq = c->row_seq; p.valid = c->row_valid;
     p.n_groups = ng; p.g_row0 = S + o0; p.g_nrows = S + o1; p.g_seq = S + o2; p.n_splits = splits; p.chunk = chunk;
     return p;
   };
-  c->p_d1 = step_plan(2 * batch, (int)d1r0.size(), o_d1r0, o_d1nr, o_d1sq);
-  c->p_dn = step_plan(batch, (int)dnr0.size(), o_dnr0, o_dnnr, o_dnsq);
-  c->p_v = step_plan(batch * (k + 1), (int)sr0.size(), o_sr0, o_snr, o_ssq);
+  c->p_d1 = step_plan(2 * batch, (int)d1r0.size(), o_d1r0, o_d1nr, o_d1sq, std::min(2, c->D.group_rows()));
+  c->p_dn = step_plan(batch, (int)dnr0.size(), o_dnr0, o_dnnr, o_dnsq, 1);
+  c->p_v = step_plan(batch * (k + 1), (int)sr0.size(), o_sr0, o_snr, o_ssq, std::min(k + 1, c->V.group_rows()));
   c->logit_rows_d1 = S + o_lr1;
 
   // verifier over the prompts: logits of each last row -> row b*(k+1) of the target buffer

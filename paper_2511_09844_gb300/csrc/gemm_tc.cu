@@ -172,24 +172,6 @@ __device__ __forceinline__ bool wait_bar_budget(uint32_t bar, uint32_t parity, l
   return true;
 }
 
-// ------------------------------------------------------------------------------ cluster helpers
-__device__ __forceinline__ uint32_t cluster_rank() {
-  uint32_t r;
-  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
-  return r;
-}
-__device__ __forceinline__ void cluster_sync_all() {
-  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
-}
-// fp32 at shared-memory address `saddr` of CTA `rank` of this cluster
-__device__ __forceinline__ float ld_dsmem(uint32_t saddr, uint32_t rank) {
-  uint32_t remote;
-  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(saddr), "r"(rank));
-  float v;
-  asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(remote) : "memory");
-  return v;
-}
-
 constexpr int kXS = 17;   // padded row of the epilogue exchange buffer (128 rows x 16 columns)
 
 // ------------------------------------------------------------------------------ epilogue stores

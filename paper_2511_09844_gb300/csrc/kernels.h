@@ -145,9 +145,8 @@ struct AttnArgs {
   const int* grp_nrows;
   const int* grp_seq;
   int n_groups, M, H, hd;
-  int n_splits, chunk;
-  float* part;           // [M, H, n_splits, hd + 4] scratch (n_splits > 1): acc[hd], max, sum, pad
-  int* counters;         // [n_groups, Hkv] arrival counts of the splits, zero between launches
+  int n_splits, chunk;   // context splits (<= 8, one cluster) of `chunk` positions (a multiple of 64)
+  int max_rows;          // upper bound of grp_nrows (max_rows x heads per KV head <= 64)
   void* out;             // [M, H * hd] bf16
 };
 cudaError_t attention(const AttnArgs& a, cudaStream_t st);
