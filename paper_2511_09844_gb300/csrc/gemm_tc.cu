@@ -96,6 +96,21 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map
       "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(bar)
       : "memory");
 }
+// L2 policy for data read exactly once per step (the weights): evicted first, so the 17+ GB
+// streamed every step do not flush the kernels' code, activations and caches out of L2.
+__device__ __forceinline__ uint64_t l2_evict_first() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+__device__ __forceinline__ void tma_load_2d_stream(uint32_t dst, const CUtensorMap* map, int c0, int c1, uint32_t bar,
+                                                   uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1, {%2, "
+      "%3}], [%4], %5;" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(bar), "l"(policy)
+      : "memory");
+}
 __device__ __forceinline__ void tmem_alloc(uint32_t dst_smem, uint32_t ncols) {
   asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst_smem), "r"(ncols)
                : "memory");
@@ -327,6 +342,7 @@ __global__ void __launch_bounds__(kThreads, 2) gemm_tc_kernel(const __grid_const
       int n_my_tiles = 0;
       for (int t = first_tile; t < a.tiles; t += tile_step) ++n_my_tiles;
       const uint32_t n_units = static_cast<uint32_t>(n_my_tiles * nkb);
+      const uint64_t wpol = l2_evict_first();
       Cursor ca;
       ca.tile = first_tile;
       ca.kb = kb_lo;
@@ -336,10 +352,10 @@ __global__ void __launch_bounds__(kThreads, 2) gemm_tc_kernel(const __grid_const
         const uint32_t s = j % S;
         const uint32_t dst = smem_u32(smem + static_cast<size_t>(s) * stage_bytes);
         if (a.swiglu) {
-          tma_load_2d(dst, &a.mapA[0], c.kb * kBK, c.wt * 64, full0 + 8 * s);
-          tma_load_2d(dst + a_bytes / 2, &a.mapA[1], c.kb * kBK, c.wt * 64, full0 + 8 * s);
+          tma_load_2d_stream(dst, &a.mapA[0], c.kb * kBK, c.wt * 64, full0 + 8 * s, wpol);
+          tma_load_2d_stream(dst + a_bytes / 2, &a.mapA[1], c.kb * kBK, c.wt * 64, full0 + 8 * s, wpol);
         } else {
-          tma_load_2d(dst, &a.mapA[c.seg], c.kb * kBK, c.row0, full0 + 8 * s);
+          tma_load_2d_stream(dst, &a.mapA[c.seg], c.kb * kBK, c.row0, full0 + 8 * s, wpol);
         }
       };
       auto load_b = [&](uint32_t j, const Cursor& c) {
