@@ -206,6 +206,13 @@ __device__ __forceinline__ float4 ld_dsmem_v4(uint32_t saddr, uint32_t rank) {
   return v;
 }
 
+// four fp32 stored to `saddr` (16-byte aligned) of CTA `rank`
+__device__ __forceinline__ void st_dsmem_v4(uint32_t saddr, uint32_t rank, float x, float y, float z, float w) {
+  asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(dsmem_addr(saddr, rank)), "f"(x), "f"(y),
+               "f"(z), "f"(w)
+               : "memory");
+}
+
 // Device error word bits (latched; read and cleared by the host).
 enum { ERR_NONFINITE = 1, ERR_TIMEOUT = 2 };
 

@@ -9,9 +9,11 @@
 //
 // Work split. A launch has T = (weight tiles) x (token tiles) output tiles of K/64 k-blocks each.
 // When T is small (few, tall weight matrices) each tile's K range is split over sp <= 8 CTAs
-// that form one thread-block cluster; their fp32 partial tiles are summed in rank order through
-// distributed shared memory, so no partial ever leaves the SMs and no CTA waits on global
-// atomics. When T is large, sp = 1 and each CTA streams whole tiles, double-buffering its TMEM
+// that form one thread-block cluster. The tile's rows are kept in pairs (SwiGLU gate/up, rotary
+// partners), and each rank owns a share of the pairs: every rank stores its fp32 partial of each
+// pair into the owner's shared memory (distributed shared memory), one cluster barrier later the
+// owner sums the partials in rank order from its own shared memory and runs the epilogue. No
+// partial leaves the SMs, no CTA waits on a remote load, and no CTA waits on global atomics. When T is large, sp = 1 and each CTA streams whole tiles, double-buffering its TMEM
 // accumulator across tiles. Either way ~152 CTAs stream at once, and with the stage ring kept
 // within half an SM's shared memory a second CTA (the next kernel's, under programmatic
 // dependent launch) can start on the same SM and prefetch its weights.
@@ -258,13 +260,23 @@ __device__ __forceinline__ void finish_chunk(const TcArgs& a, int wt, int tt, in
     if (m0 + j < a.M) emit_plain(a, wt, r, m0 + j, v[j]);
 }
 
-// Sum over the cluster's ranks (in rank order) of element (row, col) of their partial tiles.
-__device__ __forceinline__ float cluster_sum(uint32_t red, int NT1, int row, int col, int sp) {
-  const uint32_t addr = red + static_cast<uint32_t>((row * NT1 + col) * 4);
-  float v = 0.f;
-  for (int q = 0; q < sp; ++q) v += ld_dsmem(addr, static_cast<uint32_t>(q));
-  return v;
+// Split-K pairs: the 128 rows of a tile as 64 pairs whose members one epilogue needs together.
+// SwiGLU: (gate f, up f) = rows (p, p + 64); QKV with hd = 128: rotate-half partners (i, i + 64);
+// QKV with hd = 64 (two heads per tile): (64h + i, 64h + i + 32); plain outputs: (p, p + 64).
+__device__ __forceinline__ bool pairs_of_32(const TcArgs& a) { return a.epi == EPI_QKV && a.head_dim == 64; }
+__device__ __forceinline__ int pair_of(const TcArgs& a, int row) {
+  return pairs_of_32(a) ? (row >> 6) * 32 + (row & 31) : (row & 63);
 }
+__device__ __forceinline__ int member_of(const TcArgs& a, int row) {
+  return pairs_of_32(a) ? ((row >> 5) & 1) : (row >> 6);
+}
+__device__ __forceinline__ int pair_row(const TcArgs& a, int p, int m) {
+  return pairs_of_32(a) ? (p >> 5) * 64 + m * 32 + (p & 31) : p + 64 * m;
+}
+// Rank r of sp owns pairs [64 r / sp, 64 (r + 1) / sp); its receive buffer holds, per source
+// rank q and owned pair lp, both members' NT columns: [q][lp][member][NT] floats.
+__device__ __forceinline__ int pair_owner(int p, int sp) { return ((p + 1) * sp - 1) / 64; }
+__device__ __forceinline__ int pairs_max(int sp) { return (64 + sp - 1) / sp; }
 
 __global__ void __launch_bounds__(kThreads, 2) gemm_tc_kernel(const __grid_constant__ TcArgs a) {
   extern __shared__ unsigned char smem_raw[];
@@ -274,15 +286,16 @@ __global__ void __launch_bounds__(kThreads, 2) gemm_tc_kernel(const __grid_const
   const uint32_t a_bytes = kWRows * kBK * 2;
   const uint32_t b_bytes = static_cast<uint32_t>(NT) * kBK * 2;
   const uint32_t stage_bytes = a_bytes + b_bytes;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + static_cast<size_t>(S) * stage_bytes);
+  const int npmax = pairs_max(sp);
+  const uint32_t recv_bytes = sp > 1 ? static_cast<uint32_t>(sp * npmax * 2 * NT * 4) : 0u;
+  float* recv = reinterpret_cast<float*>(smem + static_cast<size_t>(S) * stage_bytes);  // split-K partials in
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + static_cast<size_t>(S) * stage_bytes + recv_bytes);
   // bars: full[S], empty[S], tfull[2], tempty[2], drain
   float* xbuf = reinterpret_cast<float*>(bars + 2 * S + 6);
   volatile int* flags = reinterpret_cast<volatile int*>(xbuf + kWRows * kXS);
   // flags: [0] abort, [1] TMEM base, [3] stages consumed, [4] go
   const uint32_t full0 = smem_u32(bars), empty0 = full0 + 8 * S, tfull0 = empty0 + 8 * S, tempty0 = tfull0 + 16,
                  drain = tempty0 + 16;
-  const uint32_t red = smem_u32(smem);   // the split-K partial tile reuses the drained stage ring
-  const int NT1 = NT + 1;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   uint32_t ncols = 32;
   while (ncols < static_cast<uint32_t>((sp == 1 ? 2 : 1) * NT)) ncols <<= 1;
@@ -437,13 +450,19 @@ __global__ void __launch_bounds__(kThreads, 2) gemm_tc_kernel(const __grid_const
           finish_chunk(a, wt, tt, r, ch * 16, v, xbuf);
         }
       } else {
-        // this CTA's K-slice partial -> shared memory, summed across the cluster below
-        float* rp = reinterpret_cast<float*>(smem) + r * NT1;
+        // this CTA's K-slice partial of row r -> the receive buffer of the rank owning its pair
+        const int p = pair_of(a, r), mem = member_of(a, r);
+        const int owner = pair_owner(p, sp);
+        const int lp = p - owner * 64 / sp;
+        const uint32_t dst = smem_u32(recv) + static_cast<uint32_t>((((rank * npmax + lp) * 2 + mem) * NT) * 4);
         for (int ch = 0; ch < nchunk; ++ch) {
+          if (ch * 16 >= cols) break;
           float v[16];
           tmem_ld16(tbase + ch * 16, v);
 #pragma unroll
-          for (int jj = 0; jj < 16; ++jj) rp[ch * 16 + jj] = v[jj];
+          for (int k4 = 0; k4 < 4; ++k4)
+            st_dsmem_v4(dst + static_cast<uint32_t>((ch * 16 + 4 * k4) * 4), static_cast<uint32_t>(owner), v[4 * k4],
+                        v[4 * k4 + 1], v[4 * k4 + 2], v[4 * k4 + 3]);
         }
       }
       tc_fence_before();
@@ -453,36 +472,37 @@ __global__ void __launch_bounds__(kThreads, 2) gemm_tc_kernel(const __grid_const
   }
 
   if (sp > 1) {
-    // Split-K reduction across the cluster: rank q finishes its share of the tile's rows
-    // (features for SwiGLU), summing the partials of ranks 0..sp-1 in order.
+    // Split-K reduction: after the barrier every partial of this rank's pairs is in its own
+    // receive buffer; sum them in rank order and run the epilogue. Nothing remote is read, so no
+    // second barrier is needed before the CTA leaves.
     __syncwarp();
-    cluster_sync_all();                       // every rank's partial is in its shared memory
+    cluster_sync_all();
     if (warp >= 2 && flags[0] == 0) {
       const int tid = threadIdx.x - 64;
       const int t = first_tile;
       const int wt = t % a.n_wtiles, tt = t / a.n_wtiles;
       const int cols = min(NT, a.M - tt * NT);
-      if (a.swiglu) {
-        const int f_lo = rank * 64 / sp, nf = (rank + 1) * 64 / sp - f_lo;
-        for (int e = tid; e < nf * cols; e += 128) {
-          const int f = f_lo + e % nf, col = e / nf;
-          emit_swiglu(a, wt, f, tt * NT + col, cluster_sum(red, NT1, f, col, sp),
-                      cluster_sum(red, NT1, f + 64, col, sp));
+      const int p_lo = rank * 64 / sp, np = (rank + 1) * 64 / sp - p_lo;
+      for (int e = tid; e < np * cols; e += 128) {
+        const int lp = e % np, col = e / np;
+        const float* rv = recv + lp * 2 * NT + col;
+        float s0 = 0.f, s1 = 0.f;
+        for (int q = 0; q < sp; ++q) {
+          s0 += rv[q * npmax * 2 * NT];
+          s1 += rv[q * npmax * 2 * NT + NT];
         }
-      } else {
-        const int r_lo = rank * kWRows / sp, nr = (rank + 1) * kWRows / sp - r_lo;
-        for (int e = tid; e < nr * cols; e += 128) {
-          const int row = r_lo + e % nr, col = e / nr;
-          const float v = cluster_sum(red, NT1, row, col, sp);
-          if (a.epi == EPI_QKV)
-            emit_qkv(a, wt, row, tt * NT + col, v, cluster_sum(red, NT1, partner_row(a, row), col, sp));
-          else
-            emit_plain(a, wt, row, tt * NT + col, v);
+        const int p = p_lo + lp, m = tt * NT + col;
+        if (a.swiglu) {
+          emit_swiglu(a, wt, p, m, s0, s1);
+        } else if (a.epi == EPI_QKV) {
+          emit_qkv(a, wt, pair_row(a, p, 0), m, s0, s1);
+          emit_qkv(a, wt, pair_row(a, p, 1), m, s1, s0);
+        } else {
+          emit_plain(a, wt, pair_row(a, p, 0), m, s0);
+          emit_plain(a, wt, pair_row(a, p, 1), m, s1);
         }
       }
     }
-    __syncwarp();
-    cluster_sync_all();                       // no rank leaves while others read its partial
   }
 
   tc_fence_before();
@@ -612,14 +632,14 @@ cudaError_t gemm_tc(const GemmArgs& g, unsigned* err, cudaStream_t st) {
   }
   a.sp = sp;
   const int stage_bytes = (kWRows + a.NT) * kBK * 2;
-  const int fixed = 1024 + kWRows * kXS * 4 + 64 + 8 * (2 * 16 + 6);
+  const int recv = sp > 1 ? sp * ((64 + sp - 1) / sp) * 2 * a.NT * 4 : 0;   // split-K receive buffer
+  const int fixed = 1024 + recv + kWRows * kXS * 4 + 64 + 8 * (2 * 16 + 6);
   // Up to NT = 128 the ring fits in half an SM's shared memory (and the accumulators in half of
   // TMEM), so the next GEMM's CTA can start on the same SM while this one drains.
   int S = (kSmemShared - fixed) / stage_bytes;
   if (a.NT > 128 || S < 3) S = (kSmemBudget - fixed) / stage_bytes;
   if (S > 8) S = 8;
   if (S < 2) return cudaErrorInvalidValue;
-  if (sp > 1 && S * stage_bytes < kWRows * (a.NT + 1) * 4) return cudaErrorInvalidValue;  // partial tile
   a.stages = S;
   const int smem = fixed + S * stage_bytes;
   static bool configured = false;
