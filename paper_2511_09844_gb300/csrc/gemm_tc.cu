@@ -278,6 +278,69 @@ __device__ __forceinline__ int pair_row(const TcArgs& a, int p, int m) {
 __device__ __forceinline__ int pair_owner(int p, int sp) { return ((p + 1) * sp - 1) / 64; }
 __device__ __forceinline__ int pairs_max(int sp) { return (64 + sp - 1) / sp; }
 
+// The global operands of one output pair (pair p of tile wt, token m), loaded before its sums
+// are known: residuals (EPI_ADD), steering bias (SwiGLU), or position, rotary factors and KV
+// block (QKV; blk = -1 when the pair is a q head or the row writes no KV).
+struct PairOps {
+  float r0, r1, bias;
+  float2 cs;
+  int pos, blk;
+};
+__device__ __forceinline__ PairOps pair_ops(const TcArgs& a, int wt, int p, int m) {
+  PairOps o{0.f, 0.f, 0.f, make_float2(1.f, 0.f), 0, -1};
+  if (a.swiglu) {
+    if (a.bias) o.bias = a.bias[static_cast<size_t>(a.row_seq ? a.row_seq[m] : 0) * a.ld_bias + wt * 64 + p];
+  } else if (a.epi == EPI_QKV) {
+    const int hd = a.head_dim, half = hd >> 1;
+    const int n = wt * kWRows + pair_row(a, p, 0);
+    const int head = n / hd, i = n % hd;
+    o.pos = a.row_pos[m];
+    if (head < a.n_heads + a.n_kv_heads)
+      o.cs = reinterpret_cast<const float2*>(a.rope_cs)[static_cast<size_t>(o.pos) * half + i];
+    if (head >= a.n_heads && a.row_valid[m])
+      o.blk = a.kv_table[static_cast<size_t>(a.row_seq[m]) * a.kv_bt_stride + (o.pos >> 4)];
+  } else if (a.epi == EPI_ADD) {
+    const float* x = a.out + static_cast<size_t>(m) * a.ldo + wt * kWRows;
+    o.r0 = x[pair_row(a, p, 0)];
+    o.r1 = x[pair_row(a, p, 1)];
+  }
+  return o;
+}
+// Epilogue of one output pair from its split-K sums s0 (member 0) and s1 (member 1).
+__device__ __forceinline__ void pair_emit(const TcArgs& a, int wt, int p, int m, float s0, float s1, const PairOps& o) {
+  if (a.swiglu) {
+    const float up = s1 + o.bias;
+    a.out_bf[static_cast<size_t>(m) * a.ldh + wt * 64 + p] = __float2bfloat16_rn(up * (s0 / (1.f + __expf(-s0))));
+  } else if (a.epi == EPI_QKV) {
+    // members are rotate-half partners i < hd/2 and i + hd/2 of one head
+    const int hd = a.head_dim, half = hd >> 1;
+    const int n = wt * kWRows + pair_row(a, p, 0);
+    const int head = n / hd, i = n % hd;
+    float o0 = s0, o1 = s1;
+    if (head < a.n_heads + a.n_kv_heads) {
+      o0 = s0 * o.cs.x - s1 * o.cs.y;
+      o1 = s1 * o.cs.x + s0 * o.cs.y;
+    }
+    if (head < a.n_heads) {
+      float* q = a.q_out + (static_cast<size_t>(m) * a.n_heads + head) * hd;
+      q[i] = o0;
+      q[i + half] = o1;
+    } else if (o.blk >= 0) {
+      const int kvi = (head - a.n_heads) / a.n_kv_heads;            // 0: K, 1: V
+      const int kvh = (head - a.n_heads) % a.n_kv_heads;
+      bf16* dst = a.kv_pool + ((static_cast<size_t>(a.layer) * a.kv_n_blocks + o.blk) * 2 + kvi) * a.n_kv_heads * 16 * hd +
+                  static_cast<size_t>(kvh) * 16 * hd + (o.pos & 15) * hd;
+      dst[i] = __float2bfloat16_rn(o0);
+      dst[i + half] = __float2bfloat16_rn(o1);
+    }
+  } else {
+    float* x = a.out + static_cast<size_t>(m) * a.ldo + wt * kWRows;
+    const bool add = a.epi == EPI_ADD;
+    x[pair_row(a, p, 0)] = add ? o.r0 + s0 : s0;
+    x[pair_row(a, p, 1)] = add ? o.r1 + s1 : s1;
+  }
+}
+
 __global__ void __launch_bounds__(kThreads, 2) gemm_tc_kernel(const __grid_constant__ TcArgs a) {
   extern __shared__ unsigned char smem_raw[];
   unsigned char* smem =
@@ -332,6 +395,7 @@ __global__ void __launch_bounds__(kThreads, 2) gemm_tc_kernel(const __grid_const
   const int nkb = kb_hi - kb_lo;
 
   pdl_trigger();                             // the next kernel may start its own prologue
+  PairOps pf{};                              // split-K: operands of this thread's first output pair
   if (warp == 0) {
     if (lane == 0) {
       // Stage use j loads k-block (kb_lo + j % nkb) of the CTA's (j / nkb)-th tile: the weight
@@ -430,6 +494,12 @@ __global__ void __launch_bounds__(kThreads, 2) gemm_tc_kernel(const __grid_const
     const int r = q * 32 + lane;              // weight row within the tile
     const bool leader = (warp == 2 && lane == 0);
     pdl_wait();                              // outputs, residuals and biases come from earlier kernels
+    if (sp > 1) {                            // fetched while the main loop runs
+      const int wt = first_tile % a.n_wtiles, tt = first_tile / a.n_wtiles;
+      const int np = (rank + 1) * 64 / sp - rank * 64 / sp;
+      const int tid = threadIdx.x - 64;
+      if (tid < np * min(NT, a.M - tt * NT)) pf = pair_ops(a, wt, rank * 64 / sp + tid % np, tt * NT + tid / np);
+    }
     uint32_t segi = 0;
     for (int t = first_tile; t < a.tiles; t += tile_step, ++segi) {
       const uint32_t acc = segi & 1;
@@ -492,15 +562,7 @@ __global__ void __launch_bounds__(kThreads, 2) gemm_tc_kernel(const __grid_const
           s1 += rv[q * npmax * 2 * NT + NT];
         }
         const int p = p_lo + lp, m = tt * NT + col;
-        if (a.swiglu) {
-          emit_swiglu(a, wt, p, m, s0, s1);
-        } else if (a.epi == EPI_QKV) {
-          emit_qkv(a, wt, pair_row(a, p, 0), m, s0, s1);
-          emit_qkv(a, wt, pair_row(a, p, 1), m, s1, s0);
-        } else {
-          emit_plain(a, wt, pair_row(a, p, 0), m, s0);
-          emit_plain(a, wt, pair_row(a, p, 1), m, s1);
-        }
+        pair_emit(a, wt, p, m, s0, s1, e == tid ? pf : pair_ops(a, wt, p, m));
       }
     }
   }
