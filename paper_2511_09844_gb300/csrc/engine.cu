@@ -90,6 +90,7 @@ struct sd2_ctx {
   // activations
   float *x = nullptr, *qkv = nullptr, *q = nullptr, *logits_t = nullptr, *logits_d = nullptr;
   float *taps = nullptr, *g_pre = nullptr, *g = nullptr, *bias = nullptr;
+  float* ssq = nullptr;          // fused RMSNorm: [slices][max_rows] sums of squares of the residual stream
   void *a = nullptr, *attn = nullptr, *h = nullptr, *g_bf = nullptr, *hml_in = nullptr;
   int gemm_impl = 0;            // 0 tensor cores where the shape allows, 1 CUDA cores
   unsigned long long* samp_slot = nullptr;
@@ -240,10 +241,16 @@ double gemm_bytes(int M, int N, int K, int out_bytes) {
   return 2.0 * N * K + 2.0 * M * K + static_cast<double>(out_bytes) * M * N;
 }
 
+// Decoder forward pass over the rows of plan p. On the tensor-core path the RMSNorm in front of
+// each projection is fused into the GEMMs around it: the residual-adding GEMM (or the embedding)
+// that produces x also writes bf16(x * gamma) and per-slice sums of squares of x, and the next
+// GEMM scales its outputs by the row's rsqrt(mean(x^2) + eps). Otherwise separate RMSNorm
+// kernels run between the GEMMs.
 sd2_status forward(sd2_ctx* c, const Model& m, const Plan& p, const FwdOut& o) {
   const sd2_lm_config& mc = m.c;
   const int M = p.M, d = mc.d_model, H = mc.n_heads, Hkv = mc.n_kv_heads, hd = mc.head_dim, F = mc.d_ffn;
   const int L = mc.n_layers;
+  const int R = c->max_rows;
   auto tap_mask = [&](int layer_out) {
     int mask = 0;
     if (!o.taps) return 0;
@@ -251,15 +258,7 @@ sd2_status forward(sd2_ctx* c, const Model& m, const Plan& p, const FwdOut& o) {
       if (o.tap_layers[s] == layer_out) mask |= 1 << s;
     return mask;
   };
-  CK(timed(c, PC_OTHER, 0, [&] {
-    return embed_rmsnorm(p.tok, m.embed, m.W(0, SD2_W_ATTN_NORM), mc.norm_eps, M, d, mc.vocab, c->x, c->a, c->st);
-  }));
-  for (int l = 0; l < L; ++l) {
-    if (l > 0)
-      CK(timed(c, PC_OTHER, 0, [&] {
-        return rmsnorm(c->x, nullptr, m.W(l, SD2_W_ATTN_NORM), mc.norm_eps, M, d, c->a, o.taps, o.tap_row, tap_mask(l),
-                       c->st);
-      }));
+  auto qkv_args = [&](int l) {
     GemmArgs g{};
     g.x = c->a; g.ldx = d; g.M = M; g.K = d;
     g.seg[0] = {m.W(l, SD2_W_Q), H * hd};
@@ -269,6 +268,62 @@ sd2_status forward(sd2_ctx* c, const Model& m, const Plan& p, const FwdOut& o) {
     g.q_out = c->q; g.kv_pool = m.kv_pool; g.kv_table = m.table; g.kv_bt_stride = m.bt_stride;
     g.kv_n_blocks = m.n_blocks; g.n_heads = H; g.n_kv_heads = Hkv; g.head_dim = hd; g.layer = l;
     g.rope_cs = m.rope_cs; g.row_pos = p.pos; g.row_valid = p.valid; g.row_seq = p.seq;
+    return g;
+  };
+  auto o_args = [&](int l) {
+    GemmArgs g{};
+    g.x = c->attn; g.ldx = H * hd; g.M = M; g.K = H * hd;
+    g.seg[0] = {m.W(l, SD2_W_O), d}; g.nseg = 1; g.epi = EPI_ADD; g.out = c->x; g.ldo = d;
+    return g;
+  };
+  auto gu_args = [&](int l) {
+    GemmArgs g{};
+    g.x = c->a; g.ldx = d; g.M = M; g.K = d;
+    g.seg[0] = {m.W(l, SD2_W_GATE), F}; g.seg[1] = {m.W(l, SD2_W_UP), F}; g.nseg = 2;
+    g.epi = EPI_SWIGLU; g.out_bf = c->h; g.ldh = F;
+    g.bias = o.bias ? o.bias + static_cast<size_t>(l) * F : nullptr;
+    g.ld_bias = L * F; g.row_seq = p.seq;
+    return g;
+  };
+  auto down_args = [&](int l) {
+    GemmArgs g{};
+    g.x = c->h; g.ldx = F; g.M = M; g.K = F;
+    g.seg[0] = {m.W(l, SD2_W_DOWN), d}; g.nseg = 1; g.epi = EPI_ADD; g.out = c->x; g.ldo = d;
+    return g;
+  };
+  // producer / consumer halves of a fused RMSNorm with gamma
+  auto produce = [&](GemmArgs& g, const void* gamma) {
+    g.norm_gamma = gamma; g.norm_out = c->a; g.norm_ssq_out = c->ssq; g.ld_ssq = R;
+  };
+  auto consume = [&](GemmArgs& g, int parts) {
+    g.norm_ssq_in = c->ssq; g.norm_parts = parts; g.norm_d = d; g.norm_eps = mc.norm_eps; g.ld_ssq = R;
+  };
+  bool fused = c->gemm_impl == 0 && tap_mask(0) == 0 && d % 128 == 0;
+  if (fused) {
+    GemmArgs g0 = qkv_args(0), g1 = o_args(0), g2 = gu_args(0), g3 = down_args(0);
+    tc(c, g0); tc(c, g1); tc(c, g2); tc(c, g3);
+    consume(g0, 1); produce(g1, m.W(0, SD2_W_MLP_NORM)); consume(g2, 1); produce(g3, m.W(0, SD2_W_ATTN_NORM));
+    fused = gemm_tc_supported(g0) && gemm_tc_supported(g1) && gemm_tc_supported(g2) && gemm_tc_supported(g3) &&
+            gemm_norm_parts(g1) <= (d / 128 + 1) * 8 && gemm_norm_parts(g3) <= (d / 128 + 1) * 8;
+  }
+  int parts = 1;   // slices of the sums of squares the last producer wrote
+  if (fused) {
+    CK(timed(c, PC_OTHER, 0, [&] {
+      return embed_scaled(p.tok, m.embed, m.W(0, SD2_W_ATTN_NORM), M, d, mc.vocab, c->x, c->a, c->ssq, c->st);
+    }));
+  } else {
+    CK(timed(c, PC_OTHER, 0, [&] {
+      return embed_rmsnorm(p.tok, m.embed, m.W(0, SD2_W_ATTN_NORM), mc.norm_eps, M, d, mc.vocab, c->x, c->a, c->st);
+    }));
+  }
+  for (int l = 0; l < L; ++l) {
+    if (l > 0 && !fused)
+      CK(timed(c, PC_OTHER, 0, [&] {
+        return rmsnorm(c->x, nullptr, m.W(l, SD2_W_ATTN_NORM), mc.norm_eps, M, d, c->a, o.taps, o.tap_row, tap_mask(l),
+                       c->st);
+      }));
+    GemmArgs g = qkv_args(l);
+    if (fused) consume(g, parts);
     CK(timed(c, PC_GEMM, gemm_bytes(M, m.qkv_width(), d, 4), [&] { return gemm(tc(c, g), c->st); }));
     AttnArgs at{};
     at.q = c->q; at.kv = m.cache(); at.layer = l; at.row_pos = p.pos;
@@ -279,23 +334,25 @@ sd2_status forward(sd2_ctx* c, const Model& m, const Plan& p, const FwdOut& o) {
       for (int b = 0; b < c->B; ++b) kvb += 2.0 * 2.0 * Hkv * hd * (c->h_n[b] + 16);
     }
     CK(timed(c, PC_ATTN, kvb, [&] { return attention(at, c->st); }));
-    GemmArgs go{};
-    go.x = c->attn; go.ldx = H * hd; go.M = M; go.K = H * hd;
-    go.seg[0] = {m.W(l, SD2_W_O), d}; go.nseg = 1; go.epi = EPI_ADD; go.out = c->x; go.ldo = d;
+    GemmArgs go = o_args(l);
+    if (fused) {
+      produce(go, m.W(l, SD2_W_MLP_NORM));
+      parts = gemm_norm_parts(go);
+    }
     CK(timed(c, PC_GEMM, gemm_bytes(M, d, H * hd, 8), [&] { return gemm(tc(c, go), c->st); }));
-    CK(timed(c, PC_OTHER, 0, [&] {
-      return rmsnorm(c->x, nullptr, m.W(l, SD2_W_MLP_NORM), mc.norm_eps, M, d, c->a, nullptr, nullptr, 0, c->st);
-    }));
-    GemmArgs gu{};
-    gu.x = c->a; gu.ldx = d; gu.M = M; gu.K = d;
-    gu.seg[0] = {m.W(l, SD2_W_GATE), F}; gu.seg[1] = {m.W(l, SD2_W_UP), F}; gu.nseg = 2;
-    gu.epi = EPI_SWIGLU; gu.out_bf = c->h; gu.ldh = F;
-    gu.bias = o.bias ? o.bias + static_cast<size_t>(l) * F : nullptr;
-    gu.ld_bias = L * F; gu.row_seq = p.seq;
+    if (!fused)
+      CK(timed(c, PC_OTHER, 0, [&] {
+        return rmsnorm(c->x, nullptr, m.W(l, SD2_W_MLP_NORM), mc.norm_eps, M, d, c->a, nullptr, nullptr, 0, c->st);
+      }));
+    GemmArgs gu = gu_args(l);
+    if (fused) consume(gu, parts);
     CK(timed(c, PC_GEMM, gemm_bytes(M, 2 * F, d, 1), [&] { return gemm(tc(c, gu), c->st); }));
-    GemmArgs gd{};
-    gd.x = c->h; gd.ldx = F; gd.M = M; gd.K = F;
-    gd.seg[0] = {m.W(l, SD2_W_DOWN), d}; gd.nseg = 1; gd.epi = EPI_ADD; gd.out = c->x; gd.ldo = d;
+    GemmArgs gd = down_args(l);
+    if (fused && l + 1 < L) {
+      produce(gd, m.W(l + 1, SD2_W_ATTN_NORM));
+      gd.tap = o.taps; gd.tap_row = o.tap_row; gd.tap_mask = tap_mask(l + 1);
+      parts = gemm_norm_parts(gd);
+    }
     CK(timed(c, PC_GEMM, gemm_bytes(M, d, F, 8), [&] { return gemm(tc(c, gd), c->st); }));
   }
   if (o.n_logit_rows > 0 || tap_mask(L)) {
@@ -512,6 +569,7 @@ sd2_status sd2_init(const sd2_config* cfg, const sd2_weights* w, void* stream, s
     ALLOC(c->q, static_cast<size_t>(R) * hmax);
     ALLOC(c->attn, static_cast<size_t>(R) * hmax * 2);
     ALLOC(c->h, static_cast<size_t>(R) * fmax * 2);
+    ALLOC(c->ssq, static_cast<size_t>(R) * (dmax / 128 + 1) * 8);
     ALLOC(c->logits_t, static_cast<size_t>(maxB) * (k + 1) * Vv);
     ALLOC(c->logits_d, static_cast<size_t>(maxB) * k * Vv);
     ALLOC(c->taps, static_cast<size_t>(maxB) * (k + 1) * 3 * cfg->verifier.d_model);

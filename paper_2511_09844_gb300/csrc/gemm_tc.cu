@@ -67,6 +67,17 @@ struct TcArgs {
   const float* rope_cs;
   const int* row_pos;
   const int* row_valid;
+  // fused RMSNorm (see GemmArgs)
+  const bf16* norm_gamma;
+  bf16* norm_out;
+  float* norm_ssq_out;
+  float* tap;
+  const int* tap_row;
+  int tap_mask;
+  const float* norm_ssq_in;
+  int norm_parts, norm_d;
+  float norm_eps;
+  int ld_ssq;
 };
 
 // ------------------------------------------------------------------------------ PTX wrappers
@@ -189,6 +200,7 @@ __device__ __forceinline__ bool wait_bar_budget(uint32_t bar, uint32_t parity, l
   return true;
 }
 
+constexpr int kMaxNT = 256;  // token columns per tile
 constexpr int kXS = 17;   // padded row of the epilogue exchange buffer (128 rows x 16 columns)
 
 // ------------------------------------------------------------------------------ epilogue stores
@@ -232,11 +244,46 @@ __device__ __forceinline__ int partner_row(const TcArgs& a, int row) {
   return ((row % a.head_dim) < half) ? row + half : row - half;
 }
 
+// Fused RMSNorm, producer side: the updated residual x_new of output (token m, feature n) also
+// goes out as bf16(x_new * gamma[n]) and, for tap rows, into the tap slots.
+__device__ __forceinline__ void norm_produce(const TcArgs& a, int m, int n, float xn, float g) {
+  a.norm_out[static_cast<size_t>(m) * a.ldo + n] = __float2bfloat16_rn(xn * g);
+  if (a.tap_mask) {
+    const int tr = a.tap_row ? a.tap_row[m] : m;
+    if (tr >= 0)
+      for (int s = 0; s < 3; ++s)
+        if (a.tap_mask & (1 << s)) a.tap[(static_cast<size_t>(tr) * 3 + s) * a.ldo + n] = xn;
+  }
+}
+// Fused RMSNorm, consumer side: rs[c] = rsqrt(mean of x_new^2 + eps) of the token tile's columns,
+// from the producer's slices summed in a fixed order (8 strided partial sums, then a butterfly
+// over the 8 lanes). Called by the 128 epilogue threads (tid = 0..127).
+__device__ __forceinline__ void tile_rstd(const TcArgs& a, int tt, float* rs, int tid) {
+  const int cols = min(a.NT, a.M - tt * a.NT);
+  const int j = tid & 7;
+  for (int c0 = 0; c0 < cols; c0 += 16) {
+    const int c = c0 + (tid >> 3);
+    float s = 0.f;
+    if (c < cols) {
+      const float* src = a.norm_ssq_in + tt * a.NT + c;
+#pragma unroll 4
+      for (int p = j; p < a.norm_parts; p += 8) s += src[static_cast<size_t>(p) * a.ld_ssq];
+    }
+    s += __shfl_xor_sync(0xffffffffu, s, 1);
+    s += __shfl_xor_sync(0xffffffffu, s, 2);
+    s += __shfl_xor_sync(0xffffffffu, s, 4);
+    if (j == 0 && c < cols) rs[c] = rsqrtf(s / static_cast<float>(a.norm_d) + a.norm_eps);
+  }
+}
+
 // Whole-tile epilogue: thread r holds weight row r for 16 token columns j0..j0+15; rows that
 // need another row (SwiGLU pairs, rotate-half partners) are exchanged through shared memory.
-__device__ __forceinline__ void finish_chunk(const TcArgs& a, int wt, int tt, int r, int j0, const float (&v)[16],
-                                             float* xbuf) {
+__device__ __forceinline__ void finish_chunk(const TcArgs& a, int wt, int tt, int r, int j0, float (&v)[16],
+                                             float* xbuf, const float* rs) {
   const int m0 = tt * a.NT + j0;
+  if (a.norm_ssq_in)
+#pragma unroll
+    for (int j = 0; j < 16; ++j) v[j] *= rs[j0 + j];
   if (a.epi == EPI_QKV || a.swiglu) {
 #pragma unroll
     for (int j = 0; j < 16; ++j) xbuf[r * kXS + j] = v[j];
@@ -252,6 +299,34 @@ __device__ __forceinline__ void finish_chunk(const TcArgs& a, int wt, int tt, in
       for (int j = 0; j < 16; ++j)
         if (m0 + j < a.M) emit_qkv(a, wt, r, m0 + j, v[j], xbuf[p * kXS + j]);
     }
+    named_bar_epi();
+    return;
+  }
+  if (a.norm_out) {
+    // residual add, bf16(x_new * gamma), taps, and this tile's sums of squares per token
+    const int n = wt * kWRows + r;
+    const float g = __bfloat162float(a.norm_gamma[n]);
+#pragma unroll
+    for (int j = 0; j < 16; ++j) {
+      float sq = 0.f;
+      if (m0 + j < a.M) {
+        float* o = a.out + static_cast<size_t>(m0 + j) * a.ldo + n;
+        const float xn = *o + v[j];
+        *o = xn;
+        norm_produce(a, m0 + j, n, xn, g);
+        sq = xn * xn;
+      }
+      xbuf[r * kXS + j] = sq;
+    }
+    named_bar_epi();
+    const int jj = r >> 3, sg = r & 7;   // column jj, rows 16 sg .. 16 sg + 15
+    float s = 0.f;
+#pragma unroll
+    for (int i = 0; i < 16; ++i) s += xbuf[(sg * 16 + i) * kXS + jj];
+    s += __shfl_xor_sync(0xffffffffu, s, 1);
+    s += __shfl_xor_sync(0xffffffffu, s, 2);
+    s += __shfl_xor_sync(0xffffffffu, s, 4);
+    if (sg == 0 && m0 + jj < a.M) a.norm_ssq_out[static_cast<size_t>(wt) * a.ld_ssq + m0 + jj] = s;
     named_bar_epi();
     return;
   }
@@ -282,12 +357,12 @@ __device__ __forceinline__ int pairs_max(int sp) { return (64 + sp - 1) / sp; }
 // are known: residuals (EPI_ADD), steering bias (SwiGLU), or position, rotary factors and KV
 // block (QKV; blk = -1 when the pair is a q head or the row writes no KV).
 struct PairOps {
-  float r0, r1, bias;
+  float r0, r1, bias, g0, g1;
   float2 cs;
   int pos, blk;
 };
 __device__ __forceinline__ PairOps pair_ops(const TcArgs& a, int wt, int p, int m) {
-  PairOps o{0.f, 0.f, 0.f, make_float2(1.f, 0.f), 0, -1};
+  PairOps o{0.f, 0.f, 0.f, 0.f, 0.f, make_float2(1.f, 0.f), 0, -1};
   if (a.swiglu) {
     if (a.bias) o.bias = a.bias[static_cast<size_t>(a.row_seq ? a.row_seq[m] : 0) * a.ld_bias + wt * 64 + p];
   } else if (a.epi == EPI_QKV) {
@@ -303,11 +378,16 @@ __device__ __forceinline__ PairOps pair_ops(const TcArgs& a, int wt, int p, int 
     const float* x = a.out + static_cast<size_t>(m) * a.ldo + wt * kWRows;
     o.r0 = x[pair_row(a, p, 0)];
     o.r1 = x[pair_row(a, p, 1)];
+    if (a.norm_out) {
+      o.g0 = __bfloat162float(a.norm_gamma[wt * kWRows + pair_row(a, p, 0)]);
+      o.g1 = __bfloat162float(a.norm_gamma[wt * kWRows + pair_row(a, p, 1)]);
+    }
   }
   return o;
 }
-// Epilogue of one output pair from its split-K sums s0 (member 0) and s1 (member 1).
-__device__ __forceinline__ void pair_emit(const TcArgs& a, int wt, int p, int m, float s0, float s1, const PairOps& o) {
+// Epilogue of one output pair from its split-K sums s0 (member 0) and s1 (member 1). Returns the
+// pair's contribution to the token's sum of squares when it produces a fused RMSNorm.
+__device__ __forceinline__ float pair_emit(const TcArgs& a, int wt, int p, int m, float s0, float s1, const PairOps& o) {
   if (a.swiglu) {
     const float up = s1 + o.bias;
     a.out_bf[static_cast<size_t>(m) * a.ldh + wt * 64 + p] = __float2bfloat16_rn(up * (s0 / (1.f + __expf(-s0))));
@@ -336,9 +416,16 @@ __device__ __forceinline__ void pair_emit(const TcArgs& a, int wt, int p, int m,
   } else {
     float* x = a.out + static_cast<size_t>(m) * a.ldo + wt * kWRows;
     const bool add = a.epi == EPI_ADD;
-    x[pair_row(a, p, 0)] = add ? o.r0 + s0 : s0;
-    x[pair_row(a, p, 1)] = add ? o.r1 + s1 : s1;
+    const float x0 = add ? o.r0 + s0 : s0, x1 = add ? o.r1 + s1 : s1;
+    x[pair_row(a, p, 0)] = x0;
+    x[pair_row(a, p, 1)] = x1;
+    if (a.norm_out) {
+      norm_produce(a, m, wt * kWRows + pair_row(a, p, 0), x0, o.g0);
+      norm_produce(a, m, wt * kWRows + pair_row(a, p, 1), x1, o.g1);
+      return x0 * x0 + x1 * x1;
+    }
   }
+  return 0.f;
 }
 
 __global__ void __launch_bounds__(kThreads, 2) gemm_tc_kernel(const __grid_constant__ TcArgs a) {
@@ -357,6 +444,7 @@ __global__ void __launch_bounds__(kThreads, 2) gemm_tc_kernel(const __grid_const
   float* xbuf = reinterpret_cast<float*>(bars + 2 * S + 6);
   volatile int* flags = reinterpret_cast<volatile int*>(xbuf + kWRows * kXS);
   // flags: [0] abort, [1] TMEM base, [3] stages consumed, [4] go
+  float* rs = const_cast<float*>(reinterpret_cast<volatile float*>(flags + 16));   // [kMaxNT] fused-norm scales
   const uint32_t full0 = smem_u32(bars), empty0 = full0 + 8 * S, tfull0 = empty0 + 8 * S, tempty0 = tfull0 + 16,
                  drain = tempty0 + 16;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -501,14 +589,20 @@ __global__ void __launch_bounds__(kThreads, 2) gemm_tc_kernel(const __grid_const
       if (tid < np * min(NT, a.M - tt * NT)) pf = pair_ops(a, wt, rank * 64 / sp + tid % np, tt * NT + tid / np);
     }
     uint32_t segi = 0;
+    int rs_tt = -1;
     for (int t = first_tile; t < a.tiles; t += tile_step, ++segi) {
       const uint32_t acc = segi & 1;
+      const int wt = t % a.n_wtiles, tt = t / a.n_wtiles;
+      if (a.norm_ssq_in && tt != rs_tt) {    // RMSNorm scales of the token tile, while its MMAs run
+        named_bar_epi();                     // no thread still reads the previous tile's scales
+        tile_rstd(a, tt, rs, threadIdx.x - 64);
+        rs_tt = tt;
+      }
       if (leader) flags[4] = wait_bar(tfull0 + 8 * acc, (segi >> 1) & 1, abort_flag, a.err) ? 1 : 0;
       named_bar_epi();
       const bool go = flags[4] != 0;
       tc_fence_after();
       if (!go) break;
-      const int wt = t % a.n_wtiles, tt = t / a.n_wtiles;
       const uint32_t tbase = tmem + (static_cast<uint32_t>(q * 32) << 16) + acc * NT;
       const int nchunk = NT / 16;
       const int cols = min(NT, a.M - tt * NT);   // token columns of this tile that exist
@@ -517,7 +611,7 @@ __global__ void __launch_bounds__(kThreads, 2) gemm_tc_kernel(const __grid_const
           if (ch * 16 >= cols) break;
           float v[16];
           tmem_ld16(tbase + ch * 16, v);
-          finish_chunk(a, wt, tt, r, ch * 16, v, xbuf);
+          finish_chunk(a, wt, tt, r, ch * 16, v, xbuf, rs);
         }
       } else {
         // this CTA's K-slice partial of row r -> the receive buffer of the rank owning its pair
@@ -553,6 +647,7 @@ __global__ void __launch_bounds__(kThreads, 2) gemm_tc_kernel(const __grid_const
       const int wt = t % a.n_wtiles, tt = t / a.n_wtiles;
       const int cols = min(NT, a.M - tt * NT);
       const int p_lo = rank * 64 / sp, np = (rank + 1) * 64 / sp - p_lo;
+      float* sq = reinterpret_cast<float*>(smem);   // [cols][np] fused-norm sums of squares (drained ring)
       for (int e = tid; e < np * cols; e += 128) {
         const int lp = e % np, col = e / np;
         const float* rv = recv + lp * 2 * NT + col;
@@ -561,8 +656,21 @@ __global__ void __launch_bounds__(kThreads, 2) gemm_tc_kernel(const __grid_const
           s0 += rv[q * npmax * 2 * NT];
           s1 += rv[q * npmax * 2 * NT + NT];
         }
+        if (a.norm_ssq_in) {
+          s0 *= rs[col];
+          s1 *= rs[col];
+        }
         const int p = p_lo + lp, m = tt * NT + col;
-        pair_emit(a, wt, p, m, s0, s1, e == tid ? pf : pair_ops(a, wt, p, m));
+        const float q2 = pair_emit(a, wt, p, m, s0, s1, e == tid ? pf : pair_ops(a, wt, p, m));
+        if (a.norm_out) sq[col * np + lp] = q2;
+      }
+      if (a.norm_out) {   // this rank's slice of the tile: sums of squares per token, in pair order
+        named_bar_epi();
+        for (int c = tid; c < cols; c += 128) {
+          float ssum = 0.f;
+          for (int lp = 0; lp < np; ++lp) ssum += sq[c * np + lp];
+          a.norm_ssq_out[static_cast<size_t>(wt * sp + rank) * a.ld_ssq + tt * NT + c] = ssum;
+        }
       }
     }
   }
@@ -641,7 +749,34 @@ int sm_count() {
 constexpr int kSmemBudget = 227 * 1024;
 constexpr int kSmemShared = 110 * 1024;
 
+// CTAs per tile: split each tile's K over up to 8 CTAs of a cluster when there are fewer tiles
+// than SMs (and the token tile is at most 128 wide).
+int split_factor(int tiles, int NT, int KB) {
+  const int sms = sm_count();
+  int sp = 1;
+  if (tiles < sms && NT <= 128) {
+    sp = sms / tiles;
+    if (sp > 8) sp = 8;
+    if (sp > KB) sp = KB;
+    if (sp < 1) sp = 1;
+  }
+  return sp;
+}
+
+int n_out_rows(const GemmArgs& g) {
+  int N = 0;
+  for (int s = 0; s < g.nseg; ++s) N += g.seg[s].rows;
+  return N;
+}
+
 }  // namespace
+
+int gemm_norm_parts(const GemmArgs& g) {
+  const int NT = gemm_tc_token_tile(g.M);
+  const int n_wtiles = n_out_rows(g) / kWRows;
+  const int tiles = n_wtiles * ((g.M + NT - 1) / NT);
+  return n_wtiles * split_factor(tiles, NT, g.K / kBK);
+}
 
 int gemm_tc_token_tile(int M) {
   int nt = ((M + 15) / 16) * 16;
@@ -653,6 +788,9 @@ bool gemm_tc_supported(const GemmArgs& g) {
   if (g.K % kBK != 0 || g.K < kBK || g.M < 1 || g.ldx % 8 != 0) return false;
   if (reinterpret_cast<uintptr_t>(g.x) & 15) return false;
   if (g.epi == EPI_QKV && (g.head_dim != 64 && g.head_dim != 128)) return false;
+  if (g.norm_out && (g.epi != EPI_ADD || !g.norm_gamma || !g.norm_ssq_out)) return false;
+  if (g.tap_mask && (!g.norm_out || !g.tap)) return false;
+  if (g.norm_ssq_in && (g.epi == EPI_ADD || g.norm_parts < 1 || g.norm_d < 1)) return false;
   if (g.epi == EPI_SWIGLU) return g.nseg == 2 && g.seg[0].rows == g.seg[1].rows && g.seg[0].rows % 64 == 0;
   for (int s = 0; s < g.nseg; ++s)
     if (g.seg[s].rows % kWRows != 0) return false;
@@ -683,19 +821,15 @@ cudaError_t gemm_tc(const GemmArgs& g, unsigned* err, cudaStream_t st) {
   a.kv_bt_stride = g.kv_bt_stride; a.kv_n_blocks = g.kv_n_blocks; a.n_heads = g.n_heads;
   a.n_kv_heads = g.n_kv_heads; a.head_dim = g.head_dim; a.layer = g.layer; a.rope_cs = g.rope_cs;
   a.row_pos = g.row_pos; a.row_valid = g.row_valid;
-  // Split each tile's K over sp CTAs of a cluster when there are fewer tiles than SMs.
-  const int sms = sm_count();
-  int sp = 1;
-  if (a.tiles < sms && a.NT <= 128) {
-    sp = sms / a.tiles;
-    if (sp > 8) sp = 8;
-    if (sp > a.KB) sp = a.KB;
-    if (sp < 1) sp = 1;
-  }
+  a.norm_gamma = static_cast<const bf16*>(g.norm_gamma); a.norm_out = static_cast<bf16*>(g.norm_out);
+  a.norm_ssq_out = g.norm_ssq_out; a.tap = g.tap; a.tap_row = g.tap_row; a.tap_mask = g.tap_mask;
+  a.norm_ssq_in = g.norm_ssq_in; a.norm_parts = g.norm_parts; a.norm_d = g.norm_d; a.norm_eps = g.norm_eps;
+  a.ld_ssq = g.ld_ssq;
+  const int sp = split_factor(a.tiles, a.NT, a.KB);
   a.sp = sp;
   const int stage_bytes = (kWRows + a.NT) * kBK * 2;
   const int recv = sp > 1 ? sp * ((64 + sp - 1) / sp) * 2 * a.NT * 4 : 0;   // split-K receive buffer
-  const int fixed = 1024 + recv + kWRows * kXS * 4 + 64 + 8 * (2 * 16 + 6);
+  const int fixed = 1024 + recv + kWRows * kXS * 4 + 64 + kMaxNT * 4 + 8 * (2 * 16 + 6);
   // Up to NT = 128 the ring fits in half an SM's shared memory (and the accumulators in half of
   // TMEM), so the next GEMM's CTA can start on the same SM while this one drains.
   int S = (kSmemShared - fixed) / stage_bytes;
@@ -710,7 +844,7 @@ cudaError_t gemm_tc(const GemmArgs& g, unsigned* err, cudaStream_t st) {
     if (e != cudaSuccess) return e;
     configured = true;
   }
-  const int grid = sp > 1 ? a.tiles * sp : std::min(a.tiles, 2 * sms);
+  const int grid = sp > 1 ? a.tiles * sp : std::min(a.tiles, 2 * sm_count());
   return launch_pdl_cluster(gemm_tc_kernel, dim3(static_cast<unsigned>(grid)), dim3(kThreads),
                             static_cast<size_t>(smem), st, sp, a);
 }

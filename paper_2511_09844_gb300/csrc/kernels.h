@@ -92,7 +92,27 @@ struct GemmArgs {
   const float* rope_cs;
   const int* row_pos;
   const int* row_valid;
+  // RMSNorm fused across GEMMs (tensor-core path only). Producer (EPI_ADD with norm_out set):
+  // besides x_new = out + y it writes norm_out[m * ldo + n] = bf16(x_new[m, n] * norm_gamma[n]),
+  // the sums of squares of x_new over its slices of n, norm_ssq_out[part * ld_ssq + m] for
+  // part < gemm_norm_parts(this launch), and x_new into tap slot s (tap_mask bit s) of rows with
+  // tap_row[m] >= 0: tap[(tap_row[m] * 3 + s) * ldo + n].
+  const void* norm_gamma;
+  void* norm_out;
+  float* norm_ssq_out;
+  float* tap;
+  const int* tap_row;
+  int tap_mask;
+  // Consumer (norm_ssq_in set): each output of token m is scaled by
+  // rsqrt(sum_{p < norm_parts} norm_ssq_in[p * ld_ssq + m] / norm_d + norm_eps), the RMSNorm of
+  // the producer's x_new, before the epilogue (the GEMM's input being bf16(x_new * gamma)).
+  const float* norm_ssq_in;
+  int norm_parts, norm_d;
+  float norm_eps;
+  int ld_ssq;
 };
+// Number of sums-of-squares slices a producer launch with these arguments writes.
+int gemm_norm_parts(const GemmArgs& a);
 // Dispatches to the tcgen05 kernel (gemm_tc.cu) when impl != 1 and gemm_tc_supported holds, else
 // to the CUDA-core kernel (gemm_simt.cu).
 cudaError_t gemm(const GemmArgs& a, cudaStream_t st);
@@ -105,6 +125,10 @@ cudaError_t gemm_simt(const GemmArgs& a, cudaStream_t st);
 // x[m] = embed[tok[m]] (f32), a[m] = bf16(RMSNorm(x[m]) * gamma); ids are clamped to [0, vocab).
 cudaError_t embed_rmsnorm(const int* tok, const void* embed, const void* gamma, float eps, int M, int d, int vocab,
                           float* x, void* a, cudaStream_t st);
+// Producer form for the fused RMSNorm: x[m] = embed[tok[m]], a[m] = bf16(x[m] * gamma) and
+// ssq[m] = sum_n x[m, n]^2 (one slice).
+cudaError_t embed_scaled(const int* tok, const void* embed, const void* gamma, int M, int d, int vocab, float* x,
+                         void* a, float* ssq, cudaStream_t st);
 // a[i] = bf16(RMSNorm(x[src(i)]) * gamma) for i < M, src(i) = rows ? rows[i] : i.
 // Taps: for each of up to 3 slots s with tap_mask bit s, tap[(tap_row[src] * 3 + s) * d] = x[src]
 // for source rows whose tap_row >= 0 (tap_row may be null = identity).

@@ -50,6 +50,31 @@ __global__ void __launch_bounds__(kNormThreads) embed_rmsnorm_kernel(const int* 
   write_normed(xr, gamma, inv, d, a + static_cast<size_t>(m) * d);
 }
 
+// Producer form of the fused RMSNorm: x, bf16(x * gamma) and the row's sum of squares.
+__global__ void __launch_bounds__(kNormThreads) embed_scaled_kernel(const int* tok, const bf16* embed, const bf16* gamma,
+                                                                    int d, int vocab, float* x, bf16* a, float* ssq) {
+  pdl_trigger();
+  pdl_wait();
+  __shared__ float red[32];
+  const int m = blockIdx.x;
+  const int t = min(max(tok[m], 0), vocab - 1);  // ids outside the vocabulary read row 0 / V-1
+  const bf16* er = embed + static_cast<size_t>(t) * d;
+  float* xr = x + static_cast<size_t>(m) * d;
+  bf16* ar = a + static_cast<size_t>(m) * d;
+  float ss = 0.f;
+  for (int j = threadIdx.x * 2; j < d; j += blockDim.x * 2) {
+    const __nv_bfloat162 e = *reinterpret_cast<const __nv_bfloat162*>(er + j);
+    const __nv_bfloat162 g = *reinterpret_cast<const __nv_bfloat162*>(gamma + j);
+    const float e0 = __low2float(e), e1 = __high2float(e);
+    xr[j] = e0;
+    xr[j + 1] = e1;
+    *reinterpret_cast<__nv_bfloat162*>(ar + j) = __floats2bfloat162_rn(e0 * __low2float(g), e1 * __high2float(g));
+    ss += e0 * e0 + e1 * e1;
+  }
+  ss = block_sum(ss, red);
+  if (threadIdx.x == 0) ssq[m] = ss;
+}
+
 __global__ void __launch_bounds__(kNormThreads) rmsnorm_kernel(const float* x, const int* rows, const bf16* gamma,
                                                                 float eps, int d, bf16* a, float* tap,
                                                                 const int* tap_row, int tap_mask) {
@@ -172,6 +197,13 @@ cudaError_t embed_rmsnorm(const int* tok, const void* embed, const void* gamma, 
                                                    static_cast<const bf16*>(gamma), eps, d, vocab, x,
                                                    static_cast<bf16*>(a)); if (e_ != cudaSuccess) return e_; }
   return cudaGetLastError();
+}
+
+cudaError_t embed_scaled(const int* tok, const void* embed, const void* gamma, int M, int d, int vocab, float* x,
+                         void* a, float* ssq, cudaStream_t st) {
+  if (M <= 0) return cudaSuccess;
+  return launch_pdl(embed_scaled_kernel, dim3(M), dim3(kNormThreads), 0, st, tok, static_cast<const bf16*>(embed),
+                    static_cast<const bf16*>(gamma), d, vocab, x, static_cast<bf16*>(a), ssq);
 }
 
 cudaError_t rmsnorm(const float* x, const int* rows, const void* gamma, float eps, int M, int d, void* a, float* tap,
