@@ -750,12 +750,14 @@ constexpr int kSmemBudget = 227 * 1024;
 constexpr int kSmemShared = 110 * 1024;
 
 // CTAs per tile: split each tile's K over up to 8 CTAs of a cluster when there are fewer tiles
-// than SMs (and the token tile is at most 128 wide).
+// than SMs (and the token tile is at most 128 wide), aiming at about 1.5 CTAs per SM: two CTAs
+// share an SM's shared memory, so more weight bytes are in flight per SM, while part of the SMs
+// stay free for the next kernel's CTAs to start and prefetch.
 int split_factor(int tiles, int NT, int KB) {
   const int sms = sm_count();
   int sp = 1;
   if (tiles < sms && NT <= 128) {
-    sp = sms / tiles;
+    sp = (3 * sms / 2 + tiles / 2) / tiles;
     if (sp > 8) sp = 8;
     if (sp > KB) sp = KB;
     if (sp < 1) sp = 1;
