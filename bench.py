@@ -198,8 +198,19 @@ def run_ours(args, rank, world, local_rank):
     e2e_s_max, e2e_all = reduce_max_sum(e2e_s * 1e3, e2e_emitted, world)
     e2e_value = e2e_all / B / (e2e_s_max / 1e3)
 
+    # stage times inside the captured step (event nodes between the stages, graph replay as above)
+    stage_steps = min(args.steps, 8)
+    eng.stage_timing(True)
+    st_ms = {"steer": 0.0, "draft": 0.0, "verify": 0.0}
+    for _ in range(stage_steps):
+        eng.step()
+        eng.accept()
+        for key, v in eng.stage_read().items():
+            st_ms[key] += v / stage_steps
+    eng.stage_timing(False)
+
     # one more pass with per-launch CUDA events on the engine's stream (no graphs) for the
-    # roofline of the dominant kernel and the per-stage bandwidth
+    # roofline of the dominant kernel
     prof_steps = min(args.steps, 8)
     eng.profile(True)
     for _ in range(prof_steps):
@@ -213,8 +224,10 @@ def run_ours(args, rank, world, local_rank):
     g = prof["gemm"]
     gemm_gbs = g["bytes"] / (g["ms"] / 1e3) / 1e9 if g["ms"] else 0.0
     ver, dra = prof["verify"], prof["draft"]
-    verify_gbs = ver["bytes"] / (ver["ms"] / 1e3) / 1e9 if ver["ms"] else 0.0
-    draft_gbs = dra["bytes"] / (dra["ms"] / 1e3) / 1e9 if dra["ms"] else 0.0
+    verify_bytes = ver["bytes"] / max(1, ver["launches"])      # weights streamed by one verify (a3)
+    draft_bytes = dra["bytes"] / max(1, dra["launches"])       # weights streamed by one drafter step (a2)
+    verify_gbs = verify_bytes / (st_ms["verify"] / 1e3) / 1e9 if st_ms["verify"] else 0.0
+    draft_gbs = draft_bytes / (st_ms["draft"] / k / 1e3) / 1e9 if st_ms["draft"] else 0.0
     launches_per_step = sum(v["launches"] for name, v in prof.items()
                             if name in ("gemm", "attention", "accept", "sample", "other")) / prof_steps
     step_ms_prof = sum(v["ms"] for name, v in prof.items() if name in ("verify", "draft", "steer")) / prof_steps
@@ -240,12 +253,14 @@ def run_ours(args, rank, world, local_rank):
                      "peak_source": f"{peak_src} hbm_gbs (MEASURED_PEAKS.json)" if peak_src == "measured" else
                      "fallback 6800 GB/s", "time_share": round(gemm_share, 4),
                      "timing": f"CUDA events per launch on the engine stream over {prof_steps} profiled steps"},
-        "stages": {"verify_gbs": round(verify_gbs, 1), "verify_frac_of_8tbs": round(verify_gbs / NOMINAL_HBM_GBS, 4),
+        "stages": {"timing": f"CUDA event nodes between the stages of the captured step, mean of {stage_steps} steps",
+                   "bytes": "weights streamed per stage (verify: all layers + lm_head; draft step: all layers + lm_head)",
+                   "verify_ms": round(st_ms["verify"], 4), "verify_gb": round(verify_bytes / 1e9, 3),
+                   "verify_gbs": round(verify_gbs, 1), "verify_frac_of_8tbs": round(verify_gbs / NOMINAL_HBM_GBS, 4),
                    "verify_frac_of_measured": round(verify_gbs / hbm, 4),
-                   "verify_ms": round(ver["ms"] / max(1, ver["launches"]), 4),
+                   "draft_step_ms": round(st_ms["draft"] / k, 4), "draft_step_gb": round(draft_bytes / 1e9, 3),
                    "draft_step_gbs": round(draft_gbs, 1), "draft_step_frac_of_measured": round(draft_gbs / hbm, 4),
-                   "draft_step_ms": round(dra["ms"] / max(1, dra["launches"]), 4),
-                   "steer_ms": round(prof["steer"]["ms"] / max(1, prof["steer"]["launches"]), 4),
+                   "steer_ms": round(st_ms["steer"], 4),
                    "profiled_step_ms": round(step_ms_prof, 4)},
         "gpu_launches": int(round(launches_per_step * args.steps)),
         "clocks": clocks.summary(),

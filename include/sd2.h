@@ -153,6 +153,15 @@ sd2_status sd2_debug_buffer(const sd2_ctx* ctx, int32_t which, void** d_ptr, int
 sd2_status sd2_profile(sd2_ctx* ctx, int32_t enable);
 sd2_status sd2_profile_read(sd2_ctx* ctx, int64_t* launches, double* ms, double* bytes, int32_t n_classes);
 
+/* Stage timing inside the captured step: with it enabled, every following sd2_step records CUDA
+ * events (external event nodes in the graph) before the steering stage (a1), between the k
+ * drafter steps (a2) and around the verifier forward (a3); the kernels between them run exactly
+ * as in an untimed step. Toggling re-captures the step graph. sd2_stage_read waits for the ctx
+ * stream and writes the last step's milliseconds: ms[0] steering, ms[1] all k drafter steps,
+ * ms[2] verifier forward. SD2_ESTATE when no timed step has run. */
+sd2_status sd2_stage_timing(sd2_ctx* ctx, int32_t enable);
+sd2_status sd2_stage_read(sd2_ctx* ctx, double* ms);
+
 /* ---------------------------------------------------------------------------------------------
  * Standalone kernels (no context): the acceptance and steering steps on caller buffers.
  * ------------------------------------------------------------------------------------------- */

@@ -105,6 +105,9 @@ struct sd2_ctx {
   cudaGraphExec_t g_step = nullptr, g_accept = nullptr;
   // profiling
   bool prof = false;
+  bool stage_on = false;                  // stage markers inside the step (graph event nodes)
+  bool stage_done = false;
+  std::vector<cudaEvent_t> stage_ev;      // [k + 3]: before steer, after steer, after draft i, after verify
   std::vector<ProfRec> recs;
   std::vector<cudaEvent_t> ev_pool;
   std::vector<int> h_n;  // host copy of committed lengths while profiling
@@ -401,11 +404,16 @@ sd2_status run_step(sd2_ctx* c) {
   auto stage_end = [&](int cls, double bytes) {
     if (c->prof) { s1 = take_event(c); cudaEventRecord(s1, c->st); c->recs.push_back({cls, bytes, s0, s1}); }
   };
+  auto mark = [&](int i) {
+    if (c->stage_on) cudaEventRecordWithFlags(c->stage_ev[i], c->st, cudaEventRecordExternal);
+  };
+  mark(0);
   stage_begin();
   sd2_status s = steer(c, c->state + 2 * c->maxB);
   if (s != SD2_OK) return s;
   stage_end(PC_STEER, 2.0 * c->cfg.d_steer * 3 * c->V.c.d_model +
                           2.0 * c->cfg.d_steer * c->D.c.n_layers * static_cast<double>(c->D.c.d_ffn));
+  mark(1);
   for (int i = 1; i <= k; ++i) {
     stage_begin();
     const Plan& p = (i == 1) ? c->p_d1 : c->p_dn;
@@ -429,6 +437,7 @@ sd2_status run_step(sd2_ctx* c) {
                                                   static_cast<double>(c->D.c.n_heads) * c->D.c.head_dim * c->D.c.d_model +
                                                   3.0 * c->D.c.d_model * c->D.c.d_ffn) +
                             2.0 * V * c->D.c.d_model);
+    mark(1 + i);
   }
   stage_begin();
   CK(timed(c, PC_OTHER, 0, [&] {
@@ -449,6 +458,7 @@ sd2_status run_step(sd2_ctx* c) {
                                                  static_cast<double>(c->V.c.n_heads) * c->V.c.head_dim * c->V.c.d_model +
                                                  3.0 * c->V.c.d_model * c->V.c.d_ffn) +
                           2.0 * V * c->V.c.d_model);
+  mark(k + 2);
   return SD2_OK;
 }
 
@@ -725,6 +735,7 @@ sd2_status sd2_step(sd2_ctx* c) {
   } else if ((s = run_step(c)) != SD2_OK) {
     return s;
   }
+  if (c->stage_on) c->stage_done = true;
   c->phase = 2;
   return SD2_OK;
 }
@@ -779,6 +790,8 @@ sd2_status sd2_free(sd2_ctx* c) {
   for (void* p : c->allocs) cudaFree(p);
   for (auto& r : c->recs) { cudaEventDestroy(r.e0); cudaEventDestroy(r.e1); }
   for (auto e : c->ev_pool) cudaEventDestroy(e);
+  for (auto e : c->stage_ev)
+    if (e) cudaEventDestroy(e);
   if (c->cap_st) cudaStreamDestroy(c->cap_st);
   delete c;
   return SD2_OK;
@@ -807,6 +820,34 @@ sd2_status sd2_profile(sd2_ctx* c, int32_t enable) {
   c->prof = enable != 0;
   for (auto& r : c->recs) { c->ev_pool.push_back(r.e0); c->ev_pool.push_back(r.e1); }
   c->recs.clear();
+  return SD2_OK;
+}
+
+sd2_status sd2_stage_timing(sd2_ctx* c, int32_t enable) {
+  if (!c) return fail(nullptr, SD2_EINVAL, "null context");
+  const bool on = enable != 0;
+  if (on && c->stage_ev.empty()) {
+    c->stage_ev.resize(c->cfg.k + 3, nullptr);
+    for (auto& e : c->stage_ev) CK(cudaEventCreate(&e));
+  }
+  if (on != c->stage_on) drop_graphs(c);
+  c->stage_on = on;
+  c->stage_done = false;
+  return SD2_OK;
+}
+
+sd2_status sd2_stage_read(sd2_ctx* c, double* ms) {
+  if (!c || !ms) return fail(c, SD2_EINVAL, "null argument");
+  if (!c->stage_on || !c->stage_done) return fail(c, SD2_ESTATE, "no step has run with stage timing on");
+  CK(cudaStreamSynchronize(c->st));
+  const int k = c->cfg.k;
+  float t = 0;
+  CK(cudaEventElapsedTime(&t, c->stage_ev[0], c->stage_ev[1]));
+  ms[0] = t;
+  CK(cudaEventElapsedTime(&t, c->stage_ev[1], c->stage_ev[k + 1]));
+  ms[1] = t;
+  CK(cudaEventElapsedTime(&t, c->stage_ev[k + 1], c->stage_ev[k + 2]));
+  ms[2] = t;
   return SD2_OK;
 }
 

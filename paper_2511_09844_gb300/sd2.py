@@ -27,7 +27,7 @@ PROFILE_CLASSES = ["gemm", "attention", "accept", "sample", "other", "verify", "
 EXPORTS = ["sd2_init", "sd2_prefill", "sd2_step", "sd2_accept", "sd2_check", "sd2_free", "sd2_last_error",
            "sd2_set_graphs", "sd2_debug_buffer", "sd2_profile", "sd2_profile_read", "sd2_accept_workspace_bytes",
            "sd2_accept_logits", "sd2_steer_workspace_bytes", "sd2_steer", "sd2_swiglu_steered",
-           "sd2_accept_logits_noalloc", "sd2_gemm", "sd2_set_gemm_impl"]
+           "sd2_accept_logits_noalloc", "sd2_gemm", "sd2_set_gemm_impl", "sd2_stage_timing", "sd2_stage_read"]
 
 
 class LMConfig(ctypes.Structure):
@@ -74,6 +74,8 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
     lib.sd2_debug_buffer.argtypes = [c_void_p, c_int32, POINTER(c_void_p), POINTER(c_int64), POINTER(c_int32)]
     lib.sd2_profile.argtypes = [c_void_p, c_int32]
     lib.sd2_profile_read.argtypes = [c_void_p, POINTER(c_int64), POINTER(c_double), POINTER(c_double), c_int32]
+    lib.sd2_stage_timing.argtypes = [c_void_p, c_int32]
+    lib.sd2_stage_read.argtypes = [c_void_p, POINTER(c_double)]
     lib.sd2_accept_workspace_bytes.argtypes = [c_int32, c_int32]
     lib.sd2_accept_workspace_bytes.restype = c_size_t
     lib.sd2_accept_logits.argtypes = [c_void_p, c_void_p, c_int32, c_void_p, c_void_p, c_int32, c_int32, c_int32,
@@ -226,6 +228,16 @@ class SD2Engine:
         la, ms, by = (c_int64 * n)(), (c_double * n)(), (c_double * n)()
         self._call(self.lib.sd2_profile_read(self.ctx, la, ms, by, n))
         return {name: {"launches": la[i], "ms": ms[i], "bytes": by[i]} for i, name in enumerate(PROFILE_CLASSES)}
+
+    def stage_timing(self, enable: bool):
+        """Record stage events inside the captured step (steering, k drafter steps, verify)."""
+        self._call(self.lib.sd2_stage_timing(self.ctx, 1 if enable else 0))
+
+    def stage_read(self):
+        """Milliseconds of the last timed step: (steering, all k drafter steps, verify)."""
+        ms = (c_double * 3)()
+        self._call(self.lib.sd2_stage_read(self.ctx, ms))
+        return {"steer": ms[0], "draft": ms[1], "verify": ms[2]}
 
     def close(self):
         if getattr(self, "ctx", None) is not None and self.ctx.value:

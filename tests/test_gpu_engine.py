@@ -70,6 +70,36 @@ def test_graphs_and_direct_launches_agree():
             assert torch.equal(ta[b, :na[b]], tb[b, :nb[b]])
 
 
+def test_stage_timing_keeps_results():
+    """Stage event nodes in the captured step change no output; the stage times are positive."""
+    work = parity.tiny_work()
+    vw, dw, st = parity.tiny_weights(work, seed=5)
+    prompts = W.make_prompts(work.verifier.vocab, 2, (30, 40), seed=11)
+    outs = []
+    for timed in (False, True):
+        dev = [parity.to_device(x) for x in (vw, dw, st)]
+        eng = sd2.SD2Engine(work, *dev, max_batch=2, max_ctx=120, max_prefill_tokens=80)
+        eng.prefill(prompts, [1.0, 0.0], seed=9)
+        if timed:
+            with pytest.raises(sd2.SD2Error):
+                eng.stage_read()                       # nothing timed yet
+            eng.stage_timing(True)
+        toks = []
+        for _ in range(5):
+            eng.step()
+            t, n = eng.accept()
+            toks.append((t.cpu().clone(), n.cpu().clone()))
+            if timed:
+                ms = eng.stage_read()
+                assert ms["steer"] > 0 and ms["draft"] > 0 and ms["verify"] > 0
+        outs.append(toks)
+        eng.close()
+    for (ta, na), (tb, nb) in zip(*outs):
+        assert torch.equal(na, nb)
+        for b in range(2):
+            assert torch.equal(ta[b, :na[b]], tb[b, :nb[b]])
+
+
 def test_capacity_stop_and_call_order():
     work = parity.tiny_work()
     vw, dw, st = parity.tiny_weights(work)
