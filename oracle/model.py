@@ -53,20 +53,27 @@ def rotary(x: torch.Tensor, pos: torch.Tensor, theta: float) -> torch.Tensor:
     return torch.cat([x1 * cos - x2 * sin, x2 * cos + x1 * sin], dim=-1)
 
 
-def causal_attention(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor) -> torch.Tensor:
+def causal_attention(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, row_block: int = 1024) -> torch.Tensor:
     """softmax(q k^T / sqrt(hd) + causal mask) v with grouped KV heads.
 
     q: [T, H, hd], k and v: [T, H_kv, hd]; query head h reads KV head h // (H / H_kv).
+    Query rows are independent by this definition, so they are taken `row_block` at a time (row
+    r attends to keys 0..r; each block reads the keys up to its last row), which bounds the score
+    matrix at long context without changing any row's softmax.
     """
     T, H, hd = q.shape
     rep = H // k.shape[1]
     k = k.repeat_interleave(rep, dim=1)
     v = v.repeat_interleave(rep, dim=1)
-    scores = torch.einsum("thd,shd->hts", q, k) / math.sqrt(hd)
-    mask = torch.ones(T, T, dtype=torch.bool).triu(1)
-    scores = scores.masked_fill(mask[None], float("-inf"))
-    probs = torch.softmax(scores, dim=-1)
-    return torch.einsum("hts,shd->thd", probs, v)
+    out = torch.empty(T, H, hd, dtype=q.dtype)
+    for r0 in range(0, T, row_block):
+        r1 = min(T, r0 + row_block)
+        scores = torch.einsum("thd,shd->hts", q[r0:r1], k[:r1]) / math.sqrt(hd)
+        mask = torch.arange(r1)[None, :] > torch.arange(r0, r1)[:, None]    # key after the query row
+        scores = scores.masked_fill(mask[None], float("-inf"))
+        probs = torch.softmax(scores, dim=-1)
+        out[r0:r1] = torch.einsum("hts,shd->thd", probs, v[:r1])
+    return out
 
 
 def silu(x: torch.Tensor) -> torch.Tensor:

@@ -163,3 +163,14 @@ def test_tap_layers_follow_appendix():
     assert W.default_tap_layers(64) == (62, 32, 3)
     assert W.default_tap_layers(4) == (2, 2, 3)
     assert W.default_tap_layers(2) == (1, 1, 2)
+
+
+def test_attention_row_blocks_do_not_change_rows():
+    """Query rows are independent: any row blocking gives the same output as one block."""
+    g = torch.Generator().manual_seed(3)
+    q = torch.randn(97, 4, 16, generator=g)
+    k = torch.randn(97, 2, 16, generator=g)
+    v = torch.randn(97, 2, 16, generator=g)
+    whole = model.causal_attention(q, k, v, row_block=10 ** 9)
+    for blk in (1, 13, 64):
+        assert torch.allclose(model.causal_attention(q, k, v, row_block=blk), whole, atol=1e-6, rtol=0)
