@@ -41,6 +41,13 @@ def parse():
     ap.add_argument("--workload", default="llama8b_1b", choices=sorted(W.WORKLOADS))
     ap.add_argument("--seed", type=int, default=1234)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--depth", default=None,
+                    help="profiling aid: 'LV,LD' keeps the first LV verifier and LD drafter layers of the "
+                         "workload (same widths, context and batch) so that an ncu capture holds a few GB; the "
+                         "JSON line's config names the depth")
+    ap.add_argument("--pretrained", action="store_true",
+                    help="the unsteered pretrained drafter (no steering stage, no bias): the baseline SD^2 "
+                         "is compared with")
     return ap.parse_args()
 
 
@@ -123,6 +130,17 @@ class ClockSampler:
 # ---------------------------------------------------------------------------------------------
 # our arm
 # ---------------------------------------------------------------------------------------------
+def bench_workload(args):
+    """The named workload; with --depth, its models cut to their first layers (profiling aid)."""
+    import dataclasses
+    work = W.WORKLOADS[args.workload]
+    if args.depth:
+        lv, ld = (int(x) for x in args.depth.split(","))
+        work = dataclasses.replace(work, verifier=dataclasses.replace(work.verifier, n_layers=lv),
+                                   drafter=dataclasses.replace(work.drafter, n_layers=ld))
+    return work
+
+
 def make_device_weights(work, seed, device):
     vw = W.make_lm_weights(work.verifier, seed, device=device)
     dw = W.make_lm_weights(work.drafter, seed + 1, device=device)
@@ -136,16 +154,17 @@ def run_ours(args, rank, world, local_rank):
     _build.build()
     torch.cuda.set_device(local_rank)
     dev = f"cuda:{local_rank}"
-    work = W.WORKLOADS[args.workload]
+    work = bench_workload(args)
     B, k, V = work.batch, work.k, work.verifier.vocab
     temp = work.temperatures[-1]
     prompts = W.make_prompts(V, B, work.prompt_len, seed=7 + rank)
-    steps_total = args.warmup + 2 * args.steps + 2
+    steps_total = args.warmup + 2 * args.steps + 2 * min(args.steps, 8) + 2
     max_ctx = max(len(p) for p in prompts) + steps_total * (k + 1) + k + 8
     vw, dw, st = make_device_weights(work, args.seed, dev)
     stream = torch.cuda.current_stream()
     eng = sd2.SD2Engine(work, vw, dw, st, max_batch=B, max_ctx=max_ctx,
-                        max_prefill_tokens=sum(len(p) for p in prompts), stream=stream)
+                        max_prefill_tokens=sum(len(p) for p in prompts), stream=stream,
+                        steering=not args.pretrained)
     torch.cuda.synchronize()
     t0 = time.perf_counter()
     eng.prefill(prompts, [temp] * B, seed=args.seed + rank)
@@ -241,7 +260,13 @@ def run_ours(args, rank, world, local_rank):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_max / args.steps, 4),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic: random-init bf16 weights N(0, 0.02^2), uniform-random prompt ids",
-        "config": workload_config(work, world, {"max_ctx": max_ctx}),
+        "config": workload_config(work, world, dict({"max_ctx": max_ctx},
+                                                    **({"depth": f"{work.verifier.n_layers} verifier + "
+                                                                 f"{work.drafter.n_layers} drafter layers "
+                                                                 "(profiling aid, not the workload)"}
+                                                       if args.depth else {}),
+                                                    **({"drafter": "pretrained, unsteered (no steering stage)"}
+                                                       if args.pretrained else {}))),
         "tau": round(tau, 4),
         "tokens_per_s_at_paper_tau": {"tau": 5.00, "value": round(5.00 / (ms_max / args.steps / 1e3), 2)},
         "prefill_s": round(prefill_s, 3),

@@ -74,6 +74,9 @@ typedef struct {
   int32_t max_ctx;                   /* per-sequence token capacity (prompt + generated + k + 2) */
   int32_t max_prefill_tokens;        /* most prompt tokens one sd2_prefill may carry in total */
   int32_t kv_block;                  /* paged KV-cache block size in tokens; must be 16 */
+  int32_t no_steering;               /* 0: SD^2 (Eq. 2 biases in every drafter MLP). 1: the pretrained
+                                        drafter alone, the baseline the paper compares with: no steering
+                                        stage and no bias (the steering weights may then be null) */
 } sd2_config;
 
 typedef struct {

@@ -409,8 +409,8 @@ sd2_status run_step(sd2_ctx* c) {
   };
   mark(0);
   stage_begin();
-  sd2_status s = steer(c, c->state + 2 * c->maxB);
-  if (s != SD2_OK) return s;
+  sd2_status s = SD2_OK;
+  if (!c->cfg.no_steering && (s = steer(c, c->state + 2 * c->maxB)) != SD2_OK) return s;
   stage_end(PC_STEER, 2.0 * c->cfg.d_steer * 3 * c->V.c.d_model +
                           2.0 * c->cfg.d_steer * c->D.c.n_layers * static_cast<double>(c->D.c.d_ffn));
   mark(1);
@@ -422,7 +422,7 @@ sd2_status run_step(sd2_ctx* c) {
                        c->committed, c->xhat, c->row_tok, c->row_pos, c->row_seq, c->row_valid, c->st);
     }));
     FwdOut o;
-    o.bias = c->bias;
+    o.bias = c->cfg.no_steering ? nullptr : c->bias;
     o.logit_rows = (i == 1) ? c->logit_rows_d1 : nullptr;
     o.n_logit_rows = B;
     o.logits = c->logits_d + static_cast<size_t>(i - 1) * V;
@@ -540,7 +540,7 @@ sd2_status sd2_init(const sd2_config* cfg, const sd2_weights* w, void* stream, s
   for (int t = 0; t < 3; ++t)
     if (cfg->tap_layers[t] < 1 || cfg->tap_layers[t] > cfg->verifier.n_layers)
       return fail(nullptr, SD2_EINVAL, "tap_layers must be 1-based verifier layers");
-  if (!aligned16(w->w_hml) || !aligned16(w->w_s) || !w->steer_ln_gamma || !w->steer_ln_beta)
+  if (!cfg->no_steering && (!aligned16(w->w_hml) || !aligned16(w->w_s) || !w->steer_ln_gamma || !w->steer_ln_beta))
     return fail(nullptr, SD2_EINVAL, "steering weights null or not 16-byte aligned");
 
   c = new sd2_ctx();
@@ -707,10 +707,9 @@ sd2_status sd2_prefill(sd2_ctx* c, int32_t batch, const int32_t* d_tokens, const
   CK(prefill_init(batch, c->cfg.max_ctx, d_tokens, S + o_cu, c->first, c->state, c->maxB, c->committed, d_first_token,
                   c->st));
   // steering from the last prompt row (j = 0 -> tap row b*(k+1)), then the drafter prefill
-  s = steer(c, c->state + 2 * c->maxB);
-  if (s != SD2_OK) return s;
+  if (!c->cfg.no_steering && (s = steer(c, c->state + 2 * c->maxB)) != SD2_OK) return s;
   FwdOut od;
-  od.bias = c->bias;
+  od.bias = c->cfg.no_steering ? nullptr : c->bias;
   s = forward(c, c->D, pd, od);
   if (s != SD2_OK) return s;
   const int one = 1;

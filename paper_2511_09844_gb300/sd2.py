@@ -39,7 +39,7 @@ class LMConfig(ctypes.Structure):
 class Config(ctypes.Structure):
     _fields_ = [("verifier", LMConfig), ("drafter", LMConfig), ("d_steer", c_int32), ("tap_layers", c_int32 * 3),
                 ("steer_ln_eps", c_float), ("k", c_int32), ("max_batch", c_int32), ("max_ctx", c_int32),
-                ("max_prefill_tokens", c_int32), ("kv_block", c_int32)]
+                ("max_prefill_tokens", c_int32), ("kv_block", c_int32), ("no_steering", c_int32)]
 
 
 class LMWeights(ctypes.Structure):
@@ -133,7 +133,7 @@ class SD2Engine:
     """One SD^2 context: borrowed weights, device-resident state, and the four hot-path calls."""
 
     def __init__(self, work: PairWorkload, verifier_w: dict, drafter_w: dict, steer_w: dict, max_batch: int,
-                 max_ctx: int, max_prefill_tokens: int, stream=None):
+                 max_ctx: int, max_prefill_tokens: int, stream=None, steering: bool = True):
         self.lib = load_library()
         self.work = work
         self.k = work.k
@@ -150,14 +150,16 @@ class SD2Engine:
         cfg.max_ctx = max_ctx
         cfg.max_prefill_tokens = max_prefill_tokens
         cfg.kv_block = work.kv_block
+        cfg.no_steering = 0 if steering else 1     # False: the pretrained drafter, no steering stage
         self.cfg = cfg
         w = Weights()
         w.verifier = self._lm_weights(verifier_w)
         w.drafter = self._lm_weights(drafter_w)
-        w.w_hml = _ptr(steer_w["w_hml"])
-        w.steer_ln_gamma = _ptr(steer_w["ln_gamma"])
-        w.steer_ln_beta = _ptr(steer_w["ln_beta"])
-        w.w_s = _ptr(steer_w["w_s"])
+        if steer_w is not None:
+            w.w_hml = _ptr(steer_w["w_hml"])
+            w.steer_ln_gamma = _ptr(steer_w["ln_gamma"])
+            w.steer_ln_beta = _ptr(steer_w["ln_beta"])
+            w.w_s = _ptr(steer_w["w_s"])
         self.stream = stream if stream is not None else torch.cuda.current_stream()
         ctx = c_void_p()
         _check(self.lib, self.lib.sd2_init(ctypes.byref(cfg), ctypes.byref(w), _stream(self.stream), ctypes.byref(ctx)))

@@ -53,14 +53,17 @@ class ParityReport:
 
 
 def run(work, vw, dw, st, prompts, temps, seed, n_steps, max_ctx=None, graphs=True, tol=TOL,
-        check_taps=True, gemm_impl=0) -> ParityReport:
-    """Run prefill + n_steps iterations on the GPU and check each against the oracle."""
+        check_taps=True, gemm_impl=0, steering=True) -> ParityReport:
+    """Run prefill + n_steps iterations on the GPU and check each against the oracle.
+
+    steering=False runs the engine's pretrained-drafter mode (no steering stage, no bias); the
+    oracle then needs W_s = 0 (its biases are exactly zero, the unsteered drafter)."""
     B, k, V = len(prompts), work.k, work.verifier.vocab
     if max_ctx is None:
         max_ctx = max(len(p) for p in prompts) + n_steps * (k + 1) + k + 4
     dev = (to_device(vw), to_device(dw), to_device(st))
     eng = sd2.SD2Engine(work, *dev, max_batch=B, max_ctx=max_ctx,
-                        max_prefill_tokens=sum(len(p) for p in prompts))
+                        max_prefill_tokens=sum(len(p) for p in prompts), steering=steering)
     eng.set_graphs(graphs)
     eng.set_gemm_impl(gemm_impl)
     rep = ParityReport()
@@ -79,7 +82,7 @@ def run(work, vw, dw, st, prompts, temps, seed, n_steps, max_ctx=None, graphs=Tr
             rep.decisions += 1
         g0 = eng.buffer(sd2.BUF_G).view(B, -1)
         b0 = eng.buffer(sd2.BUF_BIAS).view(B, -1)
-        for b in range(B):
+        for b in range(B if steering else 0):
             rep.note("g", row_rel_err(g0[b], ora.gs[ora.seqs[b].cur_bias]))
             rep.note("bias", row_rel_err(b0[b], ora.biases[ora.seqs[b].cur_bias].reshape(-1)))
         for step in range(1, n_steps + 1):
@@ -101,8 +104,9 @@ def run(work, vw, dw, st, prompts, temps, seed, n_steps, max_ctx=None, graphs=Tr
                     continue
                 s = ora.seqs[b]
                 assert int(state_before[0, b]) == len(s.tokens)
-                rep.note("g", row_rel_err(gg[b], ora.gs[s.cur_bias]))
-                rep.note("bias", row_rel_err(bb[b], ora.biases[s.cur_bias].reshape(-1)))
+                if steering:
+                    rep.note("g", row_rel_err(gg[b], ora.gs[s.cur_bias]))
+                    rep.note("bias", row_rel_err(bb[b], ora.biases[s.cur_bias].reshape(-1)))
                 xb = [int(x) for x in xh[b]]
                 out = ora.stage(b, step, forced_xhat=xb)
                 rep.note("draft_logits", row_rel_err(drf[b], out["draft"]))

@@ -70,6 +70,18 @@ def test_graphs_and_direct_launches_agree():
             assert torch.equal(ta[b, :na[b]], tb[b, :nb[b]])
 
 
+@pytest.mark.parametrize("temp", [0.0, 1.0])
+def test_pretrained_drafter_mode(temp):
+    """no_steering: the drafter runs without the steering stage and biases; the oracle with W_s = 0
+    (biases exactly zero) is the unsteered drafter, so every logit and decision must match it."""
+    work = parity.tiny_work()
+    vw, dw, _ = parity.tiny_weights(work, seed=6)
+    st0 = W.make_steering_weights(work, 8, std=0.02, ln_jitter=0.1, zero_ws=True)
+    prompts = W.make_prompts(work.verifier.vocab, 1, (32, 32), seed=12)
+    rep = parity.run(work, vw, dw, st0, prompts, [temp], seed=99, n_steps=6, steering=False)
+    assert rep.blocks == 6
+
+
 def test_stage_timing_keeps_results():
     """Stage event nodes in the captured step change no output; the stage times are positive."""
     work = parity.tiny_work()
