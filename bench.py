@@ -130,6 +130,20 @@ class ClockSampler:
 # ---------------------------------------------------------------------------------------------
 # our arm
 # ---------------------------------------------------------------------------------------------
+def gemm_traffic(algorithmic_bytes_per_launch):
+    """DRAM bytes per GEMM launch from the committed ncu record, if it was taken on this source."""
+    import hashlib
+    rec_path = os.path.join(os.path.dirname(os.path.abspath(__file__)), "profiles", "gemm_tc_traffic.json")
+    try:
+        rec = json.load(open(rec_path))
+        src = os.path.join(os.path.dirname(os.path.abspath(__file__)), rec["source"])
+        if hashlib.sha256(open(src, "rb").read()).hexdigest() != rec["source_sha256"]:
+            return None
+        return round(algorithmic_bytes_per_launch * float(rec["dram_bytes_per_algorithmic_byte"]))
+    except (OSError, KeyError, ValueError):
+        return None
+
+
 def bench_workload(args):
     """The named workload; with --depth, its models cut to their first layers (profiling aid)."""
     import dataclasses
@@ -274,7 +288,11 @@ def run_ours(args, rank, world, local_rank):
                 "d2h_bytes_per_step": int(h_tok.numel() * 4 + h_n.numel() * 4)},
         "roofline": {"bound": "hbm", "kernel": "weight-streaming GEMM (all projections + lm_head)",
                      "achieved": round(gemm_gbs, 1), "peak": hbm, "unit": "GB/s",
-                     "frac": round(gemm_gbs / hbm, 4), "traffic": None,
+                     "frac": round(gemm_gbs / hbm, 4),
+                     "traffic": gemm_traffic(g["bytes"] / max(1, g["launches"])),
+                     "traffic_note": "bytes per launch (mean over the GEMM launches): algorithmic bytes x the "
+                                     "DRAM/algorithmic ratio ncu measured on this kernel source "
+                                     "(profiles/gemm_tc_traffic.json); null if the source changed since",
                      "peak_source": f"{peak_src} hbm_gbs (MEASURED_PEAKS.json)" if peak_src == "measured" else
                      "fallback 6800 GB/s", "time_share": round(gemm_share, 4),
                      "timing": f"CUDA events per launch on the engine stream over {prof_steps} profiled steps"},
