@@ -29,7 +29,7 @@ constexpr int kTile = 64;               // positions per K/V tile
 constexpr int kWarps = 8;
 constexpr int kThreads = kWarps * 32;
 constexpr int kMaxQV = 64;              // query vectors per CTA
-constexpr int kMaxSplits = 8;           // context splits = CTAs of one cluster (portable size)
+constexpr int kMaxSplits = 16;          // context splits = CTAs of one cluster (16: non-portable size)
 constexpr int kMaxSmem = 200 * 1024;   // dynamic shared memory opt-in (static arrays come on top)
 
 template <int HD>
@@ -407,13 +407,38 @@ __global__ void __launch_bounds__(kThreads, 2) attn_kernel(const AttnArgs a) {
 }
 
 template <int HD>
+cudaError_t configure() {
+  static cudaError_t e = [] {
+    cudaError_t r = cudaFuncSetAttribute(attn_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, kMaxSmem);
+    if (r == cudaSuccess) r = cudaFuncSetAttribute(attn_kernel<HD>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    return r;
+  }();
+  return e;
+}
+
+// Whether clusters of n CTAs of the largest step-shape attention CTA can be scheduled.
+template <int HD>
+bool clusters_fit(int n) {
+  if (configure<HD>() != cudaSuccess) return false;
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3(n, 1, 1);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = AttnCfg<HD>::bytes(kMaxQV, 2 * kTile);
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = static_cast<unsigned>(n);
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  int clusters = 0;
+  return cudaOccupancyMaxActiveClusters(&clusters, attn_kernel<HD>, &cfg) == cudaSuccess && clusters > 0;
+}
+
+template <int HD>
 cudaError_t launch(const AttnArgs& a, cudaStream_t st) {
-  static bool configured = false;
-  if (!configured) {
-    const cudaError_t e = cudaFuncSetAttribute(attn_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, kMaxSmem);
-    if (e != cudaSuccess) return e;
-    configured = true;
-  }
+  const cudaError_t e = configure<HD>();
+  if (e != cudaSuccess) return e;
   const int qr = AttnCfg<HD>::qrows(a.max_rows, a.H / a.kv.Hkv);
   const size_t smem = AttnCfg<HD>::bytes(qr, a.chunk);
   if (smem > static_cast<size_t>(kMaxSmem)) return cudaErrorInvalidValue;
@@ -422,6 +447,11 @@ cudaError_t launch(const AttnArgs& a, cudaStream_t st) {
 }
 
 }  // namespace
+
+int attention_max_splits() {
+  static const int n = (clusters_fit<128>(kMaxSplits) && clusters_fit<64>(kMaxSplits)) ? kMaxSplits : 8;
+  return n;
+}
 
 cudaError_t attention(const AttnArgs& a, cudaStream_t st) {
   if (a.n_groups <= 0) return cudaSuccess;

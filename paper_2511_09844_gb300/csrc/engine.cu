@@ -498,8 +498,12 @@ void drop_graphs(sd2_ctx* c) {
   c->g_step = c->g_accept = nullptr;
 }
 
-// Context positions per attention split: whole 64-position tiles, at most 8 splits (one cluster).
-int attn_chunk(int max_ctx) { return 64 * std::max(1, (max_ctx + 8 * 64 - 1) / (8 * 64)); }
+// Context positions per attention split: whole 64-position tiles, at most attention_max_splits()
+// splits (one cluster).
+int attn_chunk(int max_ctx) {
+  const int span = 64 * attention_max_splits();
+  return 64 * std::max(1, (max_ctx + span - 1) / span);
+}
 
 // Attention row groups: consecutive rows of one sequence, at most `cap` rows per group.
 void add_groups(std::vector<int>& r0, std::vector<int>& nr, std::vector<int>& sq, int row0, int rows, int seq, int cap) {

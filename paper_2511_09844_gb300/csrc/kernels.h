@@ -169,11 +169,14 @@ struct AttnArgs {
   const int* grp_nrows;
   const int* grp_seq;
   int n_groups, M, H, hd;
-  int n_splits, chunk;   // context splits (<= 8, one cluster) of `chunk` positions (a multiple of 64)
+  int n_splits, chunk;   // context splits (<= attention_max_splits(), one cluster) of `chunk` positions (a multiple of 64)
   int max_rows;          // upper bound of grp_nrows (max_rows x heads per KV head <= 64)
   void* out;             // [M, H * hd] bf16
 };
 cudaError_t attention(const AttnArgs& a, cudaStream_t st);
+// Most context splits (= CTAs of one cluster) attention takes on this device: 16 where clusters of
+// 16 CTAs can be scheduled, else 8.
+int attention_max_splits();
 
 // ---------------------------------------------------------------- sampling / acceptance
 // Scratch layout used by the acceptance kernels for R = B(2k+1) rows and B sequences.
