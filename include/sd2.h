@@ -215,6 +215,12 @@ sd2_status sd2_gemm(const void* d_x, int32_t ldx, int32_t M, int32_t K, const vo
  * Drops captured graphs. */
 sd2_status sd2_set_gemm_impl(sd2_ctx* ctx, int32_t impl);
 
+/* Run each drafter step's decoder layers as one persistent cooperative kernel (1, wherever the
+ * drafter's shape and the step's rows allow it: at most 16 rows, d_model <= 2048) or as one kernel
+ * per projection and attention (0, the default: faster on GB300 at batch 1). Either way the same
+ * arithmetic of a2. Only with the tensor-core GEMM (sd2_set_gemm_impl 0). Drops captured graphs. */
+sd2_status sd2_set_drafter_chain(sd2_ctx* ctx, int32_t enable);
+
 /* Steered SwiGLU activation of Eq. 2 on caller buffers (the injection step of a2):
  *   h[m, f] = (up[m, f] + bias[seq[m], f]) * SiLU(gate[m, f]) as bf16, with gate/up [M, F] f32,
  *   bias [*, F] f32 (row seq[m]; d_seq may be null for bias row 0), h [M, F] bf16. */

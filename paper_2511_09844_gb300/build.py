@@ -17,7 +17,7 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 OUT_DIR = os.path.join(PKG, "_lib")
 LIB = os.path.join(OUT_DIR, "libsd2.so")
-SOURCES = ["engine.cu", "gemm_simt.cu", "gemm_tc.cu", "attention.cu", "norm.cu", "sampling.cu", "state.cu", "noalloc.cu"]
+SOURCES = ["engine.cu", "gemm_simt.cu", "gemm_tc.cu", "attention.cu", "norm.cu", "sampling.cu", "state.cu", "noalloc.cu", "chain.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-fno-strict-aliasing",
          "--expt-relaxed-constexpr", "-I", os.path.join(ROOT, "include")]

@@ -91,6 +91,9 @@ struct sd2_ctx {
   float *x = nullptr, *qkv = nullptr, *q = nullptr, *logits_t = nullptr, *logits_d = nullptr;
   float *taps = nullptr, *g_pre = nullptr, *g = nullptr, *bias = nullptr;
   float* ssq = nullptr;          // fused RMSNorm: [slices][max_rows] sums of squares of the residual stream
+  ChainPlan chain{};             // the drafter's persistent layer chain (chain.cu), when its shape allows
+  bool chain_ok = false;
+  bool use_chain = false;        // measured slower than the per-kernel path on GB300 (off by default)
   void *a = nullptr, *attn = nullptr, *h = nullptr, *g_bf = nullptr, *hml_in = nullptr;
   int gemm_impl = 0;            // 0 tensor cores where the shape allows, 1 CUDA cores
   unsigned long long* samp_slot = nullptr;
@@ -244,6 +247,55 @@ double gemm_bytes(int M, int N, int K, int out_bytes) {
   return 2.0 * N * K + 2.0 * M * K + static_cast<double>(out_bytes) * M * N;
 }
 
+// Final RMSNorm (with the last tap) and lm_head over the logit rows, from the residual stream c->x.
+sd2_status head(sd2_ctx* c, const Model& m, const Plan& p, const FwdOut& o) {
+  const sd2_lm_config& mc = m.c;
+  const int M = p.M, d = mc.d_model, L = mc.n_layers;
+  int mask = 0;
+  if (o.taps)
+    for (int s = 0; s < 3; ++s)
+      if (o.tap_layers[s] == L) mask |= 1 << s;
+  if (o.n_logit_rows > 0 || mask) {
+    const int nr = o.n_logit_rows > 0 ? o.n_logit_rows : M;
+    CK(timed(c, PC_OTHER, 0, [&] {
+      return rmsnorm(c->x, o.logit_rows, m.final_norm, mc.norm_eps, nr, d, c->a, o.taps, o.tap_row, mask, c->st);
+    }));
+  }
+  if (o.n_logit_rows > 0) {
+    GemmArgs gl{};
+    gl.x = c->a; gl.ldx = d; gl.M = o.n_logit_rows; gl.K = d;
+    gl.seg[0] = {m.lm_head, mc.vocab}; gl.nseg = 1; gl.epi = EPI_STORE; gl.out = o.logits;
+    gl.ldo = static_cast<int>(o.ld_logits);
+    CK(timed(c, PC_GEMM, gemm_bytes(o.n_logit_rows, mc.vocab, d, 4), [&] { return gemm(tc(c, gl), c->st); }));
+  }
+  return SD2_OK;
+}
+
+// The drafter's layers over plan p in one persistent launch (chain.cu), then the head. Used for
+// the drafter steps when the chain takes their shape; forward() otherwise.
+bool chain_takes(sd2_ctx* c, const Plan& p) {
+  if (!c->chain_ok || !c->use_chain || c->gemm_impl != 0) return false;
+  ChainRun r;
+  r.M = p.M; r.n_splits = p.n_splits; r.chunk = p.chunk; r.max_rows = p.max_rows;
+  return chain_supported(c->chain, r);
+}
+sd2_status forward_chain(sd2_ctx* c, const Model& m, const Plan& p, const FwdOut& o) {
+  ChainRun r;
+  r.M = p.M; r.tok = p.tok; r.row_pos = p.pos; r.row_seq = p.seq; r.row_valid = p.valid;
+  r.grp_row0 = p.g_row0; r.grp_nrows = p.g_nrows; r.grp_seq = p.g_seq; r.n_groups = p.n_groups;
+  r.n_splits = p.n_splits; r.chunk = p.chunk; r.max_rows = p.max_rows;
+  r.bias = o.bias; r.ld_bias = m.c.n_layers * m.c.d_ffn;
+  r.x_out = c->x; r.err = c->errw;
+  double bytes = 0;
+  if (c->prof) {
+    const sd2_lm_config& mc = m.c;
+    bytes = 2.0 * mc.n_layers * (static_cast<double>(mc.d_model) * m.qkv_width() +
+                                 static_cast<double>(mc.n_heads) * mc.head_dim * mc.d_model + 3.0 * mc.d_model * mc.d_ffn);
+  }
+  CK(timed(c, PC_GEMM, bytes, [&] { return chain_forward(c->chain, r, c->st); }));
+  return head(c, m, p, o);
+}
+
 // Decoder forward pass over the rows of plan p. On the tensor-core path the RMSNorm in front of
 // each projection is fused into the GEMMs around it: the residual-adding GEMM (or the embedding)
 // that produces x also writes bf16(x * gamma) and per-slice sums of squares of x, and the next
@@ -358,20 +410,7 @@ sd2_status forward(sd2_ctx* c, const Model& m, const Plan& p, const FwdOut& o) {
     }
     CK(timed(c, PC_GEMM, gemm_bytes(M, d, F, 8), [&] { return gemm(tc(c, gd), c->st); }));
   }
-  if (o.n_logit_rows > 0 || tap_mask(L)) {
-    const int nr = o.n_logit_rows > 0 ? o.n_logit_rows : M;
-    CK(timed(c, PC_OTHER, 0, [&] {
-      return rmsnorm(c->x, o.logit_rows, m.final_norm, mc.norm_eps, nr, d, c->a, o.taps, o.tap_row, tap_mask(L), c->st);
-    }));
-  }
-  if (o.n_logit_rows > 0) {
-    GemmArgs gl{};
-    gl.x = c->a; gl.ldx = d; gl.M = o.n_logit_rows; gl.K = d;
-    gl.seg[0] = {m.lm_head, mc.vocab}; gl.nseg = 1; gl.epi = EPI_STORE; gl.out = o.logits;
-    gl.ldo = static_cast<int>(o.ld_logits);
-    CK(timed(c, PC_GEMM, gemm_bytes(o.n_logit_rows, mc.vocab, d, 4), [&] { return gemm(tc(c, gl), c->st); }));
-  }
-  return SD2_OK;
+  return head(c, m, p, o);
 }
 
 // a1: g = LN(W_hml [h; m; l]) at each sequence's steering row, biases = W_s g.
@@ -427,7 +466,7 @@ sd2_status run_step(sd2_ctx* c) {
     o.n_logit_rows = B;
     o.logits = c->logits_d + static_cast<size_t>(i - 1) * V;
     o.ld_logits = static_cast<long long>(k) * V;
-    s = forward(c, c->D, p, o);
+    s = chain_takes(c, p) ? forward_chain(c, c->D, p, o) : forward(c, c->D, p, o);
     if (s != SD2_OK) return s;
     CK(timed(c, PC_SAMPLE, 4.0 * B * V, [&] {
       return sample_rows(o.logits, o.ld_logits, B, V, c->temp, c->seed, RNG_DRAFT, i, c->iter, 0, c->xhat + (i - 1), k,
@@ -607,6 +646,15 @@ sd2_status sd2_init(const sd2_config* cfg, const sd2_weights* w, void* stream, s
     CK(cudaMemset(c->state, 0, sizeof(int) * 4 * maxB));
     CK(cudaMemset(c->taps, 0, sizeof(float) * static_cast<size_t>(maxB) * (k + 1) * 3 * cfg->verifier.d_model));
     CK(cudaStreamCreateWithFlags(&c->cap_st, cudaStreamNonBlocking));
+    // the drafter's persistent layer chain, when its shape allows (the step plans stay within it)
+    const sd2_lm_config& dc = cfg->drafter;
+    if (chain_plan(c->chain, dc.n_layers, dc.d_model, dc.n_heads, dc.n_kv_heads, dc.head_dim, dc.d_ffn, dc.vocab,
+                   dc.norm_eps, attention_max_splits())) {
+      unsigned char* block;
+      ALLOC(block, chain_device_bytes(c->chain));
+      CK(chain_prepare(c->chain, c->D.w.data(), c->D.embed, c->D.cache(), c->D.rope_cs, block));
+      c->chain_ok = true;
+    }
     return SD2_OK;
   };
   if ((s = go()) != SD2_OK) {
@@ -782,6 +830,13 @@ sd2_status sd2_set_gemm_impl(sd2_ctx* c, int32_t impl) {
   if (!c) return fail(nullptr, SD2_EINVAL, "null context");
   if (impl != 0 && impl != 1) return fail(c, SD2_EINVAL, "impl must be 0 (tensor cores) or 1 (CUDA cores)");
   c->gemm_impl = impl;
+  drop_graphs(c);
+  return SD2_OK;
+}
+
+sd2_status sd2_set_drafter_chain(sd2_ctx* c, int32_t enable) {
+  if (!c) return fail(nullptr, SD2_EINVAL, "null context");
+  c->use_chain = enable != 0;
   drop_graphs(c);
   return SD2_OK;
 }

@@ -121,6 +121,11 @@ cudaError_t gemm_tc(const GemmArgs& a, unsigned* err, cudaStream_t st);
 int gemm_tc_token_tile(int M);
 cudaError_t gemm_simt(const GemmArgs& a, cudaStream_t st);
 
+// 2-D bf16 TMA map (CUtensorMap, 128 bytes) of a row-major [rows, K] weight: boxes of box_rows x 64
+// elements with the 128-byte swizzle (gemm_tc.cu).
+bool encode_weight_map(void* map, const void* w, int rows, int K, int box_rows);
+int sm_count_cached();
+
 // ---------------------------------------------------------------- decoder elementwise
 // x[m] = embed[tok[m]] (f32), a[m] = bf16(RMSNorm(x[m]) * gamma); ids are clamped to [0, vocab).
 cudaError_t embed_rmsnorm(const int* tok, const void* embed, const void* gamma, float eps, int M, int d, int vocab,
@@ -177,6 +182,45 @@ cudaError_t attention(const AttnArgs& a, cudaStream_t st);
 // Most context splits (= CTAs of one cluster) attention takes on this device: 16 where clusters of
 // 16 CTAs can be scheduled, else 8.
 int attention_max_splits();
+
+// ---------------------------------------------------------------- persistent layer chain
+// Every decoder layer of one forward pass over at most 16 token rows in one cooperative launch
+// (chain.cu): the projections stream their weights through one TMA ring across grid-wide
+// barriers, split-K partials are summed by the phase that reads them, attention runs between.
+struct ChainPlan {                   // one decoder, prepared once
+  int L = 0, d = 0, H = 0, Hkv = 0, hd = 0, F = 0;
+  float eps = 0.f;
+  const void* embed = nullptr;       // bf16 [vocab, d]
+  int vocab = 0;
+  KVCache kv{};
+  const float* rope_cs = nullptr;    // float2 [max_ctx, hd / 2]
+  int n_cta = 0, sp_q = 0, sp_o = 0, sp_d = 0, max_splits = 0;
+  void* dev = nullptr;               // tensor maps and norm gains of every layer (chain_prepare)
+  float *xbuf = nullptr, *pq = nullptr, *po = nullptr, *pd = nullptr, *pa = nullptr;
+  void* h = nullptr;
+  unsigned* sync = nullptr;
+};
+// Shape checks and work split of a decoder; false if the chain does not take it.
+bool chain_plan(ChainPlan& p, int L, int d, int H, int Hkv, int hd, int F, int vocab, float eps, int max_splits);
+// Device bytes chain_prepare needs for p (tables + scratch).
+size_t chain_device_bytes(const ChainPlan& p);
+// Writes the tables into `block` (chain_device_bytes of 256-aligned device memory) and points the
+// scratch into it. w = host array of L * SD2_LAYER_SLOTS device weight pointers.
+cudaError_t chain_prepare(ChainPlan& p, const void* const* w, const void* embed, const KVCache& kv,
+                          const float* rope_cs, void* block);
+struct ChainRun {
+  int M = 0;                         // token rows (<= 16)
+  const int *tok = nullptr, *row_pos = nullptr, *row_seq = nullptr, *row_valid = nullptr;
+  const int *grp_row0 = nullptr, *grp_nrows = nullptr, *grp_seq = nullptr;
+  int n_groups = 0, n_splits = 1, chunk = 64, max_rows = 1;
+  const float* bias = nullptr;       // steering biases [seq][L * F] (Eq. 2), null for none
+  int ld_bias = 0;
+  float* x_out = nullptr;            // [M, d] residual stream after the last layer
+  unsigned* err = nullptr;
+};
+bool chain_supported(const ChainPlan& p, const ChainRun& r);
+cudaError_t chain_forward(const ChainPlan& p, const ChainRun& r, cudaStream_t st);
+
 
 // ---------------------------------------------------------------- sampling / acceptance
 // Scratch layout used by the acceptance kernels for R = B(2k+1) rows and B sequences.

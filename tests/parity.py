@@ -53,7 +53,7 @@ class ParityReport:
 
 
 def run(work, vw, dw, st, prompts, temps, seed, n_steps, max_ctx=None, graphs=True, tol=TOL,
-        check_taps=True, gemm_impl=0, steering=True) -> ParityReport:
+        check_taps=True, gemm_impl=0, steering=True, chain=False) -> ParityReport:
     """Run prefill + n_steps iterations on the GPU and check each against the oracle.
 
     steering=False runs the engine's pretrained-drafter mode (no steering stage, no bias); the
@@ -66,6 +66,7 @@ def run(work, vw, dw, st, prompts, temps, seed, n_steps, max_ctx=None, graphs=Tr
                         max_prefill_tokens=sum(len(p) for p in prompts), steering=steering)
     eng.set_graphs(graphs)
     eng.set_gemm_impl(gemm_impl)
+    eng.set_drafter_chain(chain)
     rep = ParityReport()
     try:
         first = eng.prefill(prompts, temps, seed).cpu().tolist()

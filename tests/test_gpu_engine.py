@@ -13,14 +13,15 @@ from paper_2511_09844_gb300 import workloads as W
 pytestmark = pytest.mark.gpu
 
 
-@pytest.mark.parametrize("gemm_impl", [0, 1])
+@pytest.mark.parametrize("gemm_impl,chain", [(0, True), (0, False), (1, False)])
 @pytest.mark.parametrize("temp", [0.0, 1.0])
-def test_tiny_single_sequence(temp, gemm_impl):
-    """gemm_impl 0: tensor-core GEMM with fused epilogues; 1: CUDA-core GEMM + separate kernels."""
+def test_tiny_single_sequence(temp, gemm_impl, chain):
+    """gemm_impl 0: tensor-core GEMM with fused epilogues, the drafter steps as one persistent
+    kernel (chain) or one kernel per projection; 1: CUDA-core GEMM + separate kernels."""
     work = parity.tiny_work()
     vw, dw, st = parity.tiny_weights(work)
     prompts = W.make_prompts(work.verifier.vocab, 1, (32, 32), seed=7)
-    rep = parity.run(work, vw, dw, st, prompts, [temp], seed=1234, n_steps=8, gemm_impl=gemm_impl)
+    rep = parity.run(work, vw, dw, st, prompts, [temp], seed=1234, n_steps=8, gemm_impl=gemm_impl, chain=chain)
     assert rep.blocks == 8 and rep.decisions > 8 * work.k
 
 

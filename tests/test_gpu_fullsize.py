@@ -55,6 +55,16 @@ def test_full_width_one_layer_slices(name, n_steps):
     assert rep.blocks == work.batch * n_steps
 
 
+def test_full_width_slice_drafter_chain():
+    """The drafter steps as one persistent kernel (chain.cu) at the 8B/1B pair's widths."""
+    work = _one_layer(W.WORKLOADS["llama8b_1b"])
+    work = dataclasses.replace(work, drafter=dataclasses.replace(W.WORKLOADS["llama8b_1b"].drafter, n_layers=2))
+    vw, dw, st = _weights(work, 23)
+    prompts = W.make_prompts(work.verifier.vocab, work.batch, work.prompt_len, seed=18)
+    rep = parity.run(work, vw, dw, st, prompts, _temps(work), seed=7, n_steps=2, chain=True)
+    assert rep.blocks == 2
+
+
 def test_long_context_verify_16k():
     """8B-shaped verify at a 16384-token context, batch 1 (one-layer slice, k = 1)."""
     work = _one_layer(W.WORKLOADS["llama8b_1b"], k=1, prompt_len=(16384, 16384))
