@@ -130,6 +130,44 @@ class ClockSampler:
 # ---------------------------------------------------------------------------------------------
 # our arm
 # ---------------------------------------------------------------------------------------------
+def accept_sweep(sd2, dev, hbm, B=256, k=16, V=152064, reps=10):
+    """The acceptance kernels (a4) alone at the sweep's largest point: bf16 logits N(0, 3^2) with a
+    boosted token per row, B = 256, k = 16, V = 152064 (2.57 GB of logits, larger than L2)."""
+    target, draft, xhat = W.make_sweep_logits(B, k, V, seed=11, device=dev)
+    temp = torch.ones(B, dtype=torch.float32, device=dev)
+    ws = torch.empty(sd2.load_library().sd2_accept_workspace_bytes(B, k), dtype=torch.uint8, device=dev)
+    for i in range(3):
+        sd2.accept_logits(target, draft, xhat, temp, seed=5, step=i + 1, workspace=ws)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for i in range(reps):
+        sd2.accept_logits(target, draft, xhat, temp, seed=5, step=i + 4, workspace=ws)
+    e1.record()
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / reps
+    logit_bytes = (target.numel() + draft.numel()) * 2
+    gbs = 2 * logit_bytes / (ms / 1e3) / 1e9          # two passes over every row: max, exact normaliser
+    del target, draft
+    # the normaliser pass evaluates the fixed-sequence exp (about 24 fp32 operations) and the
+    # 2^-45 fixed-point sum for every logit, the max pass about 8 operations: ALU-bound, not HBM
+    elems = B * (2 * k + 1) * V
+    ops = 32.0 * elems
+    alu_peak = sm_count_of(dev) * 128 * 2.07e9 / 1e12      # fp32 lanes x max SM clock, Tops/s
+    return {"B": B, "k": k, "V": V, "dtype": "bf16", "ms_per_call": round(ms, 4),
+            "logit_bytes": logit_bytes, "algorithmic_bytes": 2 * logit_bytes, "achieved_gbs": round(gbs, 1),
+            "frac_of_measured_hbm": round(gbs / hbm, 4),
+            "bound": "alu", "alu_tops": round(ops / (ms / 1e3) / 1e12, 2), "alu_peak_tops": round(alu_peak, 1),
+            "alu_frac": round(ops / (ms / 1e3) / 1e12 / alu_peak, 4),
+            "alu_note": "about 32 fp32/integer operations per logit over the two passes (exact fixed-sequence exp "
+                        "and 2^-45 fixed-point normaliser); peak = SMs x 128 lanes x 2.07 GHz",
+            "timing": f"CUDA events around {reps} calls of sd2_accept_logits, inputs larger than L2"}
+
+
+def sm_count_of(dev):
+    return torch.cuda.get_device_properties(dev).multi_processor_count
+
+
 def gemm_traffic(algorithmic_bytes_per_launch):
     """DRAM bytes per GEMM launch from the committed ncu record, if it was taken on this source."""
     import hashlib
@@ -268,6 +306,7 @@ def run_ours(args, rank, world, local_rank):
     eng.close()
     keep = (vw, dw, st) if (rank == 0 and world == 1 and not args.no_cpu_baseline) else None
     del vw, dw, st
+    sweep = accept_sweep(sd2, dev, hbm) if not args.depth else None
 
     line = {
         "metric": METRIC, "value": round(value, 3), "unit": "tokens/s/sequence", "n_gpus": world,
@@ -305,6 +344,7 @@ def run_ours(args, rank, world, local_rank):
                    "draft_step_gbs": round(draft_gbs, 1), "draft_step_frac_of_measured": round(draft_gbs / hbm, 4),
                    "steer_ms": round(st_ms["steer"], 4),
                    "profiled_step_ms": round(step_ms_prof, 4)},
+        "accept_sweep": sweep,
         "gpu_launches": int(round(launches_per_step * args.steps)),
         "clocks": clocks.summary(),
     }

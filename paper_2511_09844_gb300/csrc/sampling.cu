@@ -23,6 +23,7 @@ namespace {
 
 constexpr int kThreads = 256;
 constexpr int kPerCta = kThreads * 4 * 8;   // vocabulary entries per CTA (8 iterations of 4)
+constexpr int kStatsPerCta = kThreads * 8 * 8;   // the row-statistics passes: 8 iterations of 8
 enum { MODE_NONE = 0, MODE_DONE = 1, MODE_RESIDUAL = 2, MODE_BONUS = 3 };
 
 template <typename T>
@@ -36,6 +37,31 @@ template <>
 __device__ __forceinline__ void load4<bf16>(const bf16* row, int v, float z[4]) {
   const uint2 t = *reinterpret_cast<const uint2*>(row + v);
   z[0] = bf_lo(t.x); z[1] = bf_hi(t.x); z[2] = bf_lo(t.y); z[3] = bf_hi(t.y);
+}
+// 8 consecutive entries from v (n < 8 of them at the row's end; rows start 16-byte (f32) or 8-byte
+// (bf16) aligned)
+template <typename T>
+__device__ __forceinline__ void load8(const T* row, int v, int n, float z[8]);
+template <>
+__device__ __forceinline__ void load8<float>(const float* row, int v, int n, float z[8]) {
+  if (n >= 8) {
+    const float4 a = *reinterpret_cast<const float4*>(row + v), b = *reinterpret_cast<const float4*>(row + v + 4);
+    z[0] = a.x; z[1] = a.y; z[2] = a.z; z[3] = a.w; z[4] = b.x; z[5] = b.y; z[6] = b.z; z[7] = b.w;
+  } else {
+#pragma unroll
+    for (int j = 0; j < 8; ++j) z[j] = j < n ? row[v + j] : 0.f;
+  }
+}
+template <>
+__device__ __forceinline__ void load8<bf16>(const bf16* row, int v, int n, float z[8]) {
+  if (n >= 8) {    // rows are 8-byte aligned (V % 4 == 0): two 8-byte loads
+    const uint2 t = *reinterpret_cast<const uint2*>(row + v), u = *reinterpret_cast<const uint2*>(row + v + 4);
+    z[0] = bf_lo(t.x); z[1] = bf_hi(t.x); z[2] = bf_lo(t.y); z[3] = bf_hi(t.y);
+    z[4] = bf_lo(u.x); z[5] = bf_hi(u.x); z[6] = bf_lo(u.y); z[7] = bf_hi(u.y);
+  } else {
+#pragma unroll
+    for (int j = 0; j < 8; ++j) z[j] = j < n ? bf2f(row[v + j]) : 0.f;
+  }
 }
 template <typename T>
 __device__ __forceinline__ float load1(const T* row, int v);
@@ -101,14 +127,17 @@ __global__ void __launch_bounds__(kThreads) rowmax_kernel(const T* target, const
   if (greedy && rr.is_draft) return;
   const float invT = greedy ? 1.f : inv_temp(t);
   const T* row = (rr.is_draft ? draft : target) + rr.offset;
-  const int lo = blockIdx.y * kPerCta, hi = min(V, lo + kPerCta);
+  const int lo = blockIdx.y * kStatsPerCta, hi = min(V, lo + kStatsPerCta);
   unsigned long long best = 0;
   bool bad = false;
-  for (int v = lo + threadIdx.x * 4; v < hi; v += kThreads * 4) {
-    float z[4];
-    load4<T>(row, v, z);
+#pragma unroll 2
+  for (int v = lo + threadIdx.x * 8; v < hi; v += kThreads * 8) {
+    float z[8];
+    const int n = min(8, hi - v);
+    load8<T>(row, v, n, z);
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
+    for (int j = 0; j < 8; ++j) {
+      if (j >= n) break;
       bad |= !isfinite(z[j]);
       const float s = greedy ? z[j] : __fmul_rn(z[j], invT);
       const unsigned long long key = pack_key(s, v + j);
@@ -136,13 +165,16 @@ __global__ void __launch_bounds__(kThreads) rowsum_kernel(const T* target, const
   const float invT = inv_temp(t);
   const float m = packed_key(rowkey[blockIdx.x]);
   const T* row = (rr.is_draft ? draft : target) + rr.offset;
-  const int lo = blockIdx.y * kPerCta, hi = min(V, lo + kPerCta);
+  const int lo = blockIdx.y * kStatsPerCta, hi = min(V, lo + kStatsPerCta);
   unsigned long long acc = 0;
-  for (int v = lo + threadIdx.x * 4; v < hi; v += kThreads * 4) {
-    float z[4];
-    load4<T>(row, v, z);
+#pragma unroll 2
+  for (int v = lo + threadIdx.x * 8; v < hi; v += kThreads * 8) {
+    float z[8];
+    const int n = min(8, hi - v);
+    load8<T>(row, v, n, z);
 #pragma unroll
-    for (int j = 0; j < 4; ++j) acc += fixed45(exp_cw(__fsub_rn(__fmul_rn(z[j], invT), m)));
+    for (int j = 0; j < 8; ++j)
+      if (j < n) acc += fixed45(exp_cw(__fsub_rn(__fmul_rn(z[j], invT), m)));
   }
   acc = block_sum_u64(acc, red);
   if (threadIdx.x == 0 && acc) atomicAdd(&rowsum[blockIdx.x], acc);
@@ -353,10 +385,11 @@ cudaError_t accept_typed(const T* target, const T* draft, const int* xhat, const
                          int* n, const AcceptScratch& s, unsigned* err, cudaStream_t st) {
   const int R = B * (2 * k + 1);
   const int S = (V + kPerCta - 1) / kPerCta;
+  const int SS = (V + kStatsPerCta - 1) / kStatsPerCta;
   cudaError_t e = cudaMemsetAsync(s.rowkey, 0, sizeof(unsigned long long) * 2 * R, st);  // rowkey + rowsum
   if (e != cudaSuccess) return e;
-  { const cudaError_t e_ = launch_pdl(rowmax_kernel<T>, dim3(dim3(R, S)), dim3(kThreads), 0, st, target, draft, B, k, V, temp, stopped, s.rowkey, err); if (e_ != cudaSuccess) return e_; }
-  { const cudaError_t e_ = launch_pdl(rowsum_kernel<T>, dim3(dim3(R, S)), dim3(kThreads), 0, st, target, draft, B, k, V, temp, stopped, s.rowkey, s.rowsum); if (e_ != cudaSuccess) return e_; }
+  { const cudaError_t e_ = launch_pdl(rowmax_kernel<T>, dim3(dim3(R, SS)), dim3(kThreads), 0, st, target, draft, B, k, V, temp, stopped, s.rowkey, err); if (e_ != cudaSuccess) return e_; }
+  { const cudaError_t e_ = launch_pdl(rowsum_kernel<T>, dim3(dim3(R, SS)), dim3(kThreads), 0, st, target, draft, B, k, V, temp, stopped, s.rowkey, s.rowsum); if (e_ != cudaSuccess) return e_; }
   { const cudaError_t e_ = launch_pdl(decide_kernel<T>, dim3((B + 127) / 128), dim3(128), 0, st, target, draft, xhat, temp, B, k, V, seed, step_ptr, step, stopped,
                                                     s.rowkey, s.rowsum, tokens, n, s); if (e_ != cudaSuccess) return e_; }
   { const cudaError_t e_ = launch_pdl(resample_kernel<T>, dim3(dim3(B, S)), dim3(kThreads), 0, st, target, draft, temp, B, k, V, seed, step_ptr, step, s.rowkey,
