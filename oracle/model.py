@@ -89,10 +89,13 @@ def steered_swiglu(a: torch.Tensor, w_gate, w_up, w_down, bias: Optional[torch.T
 
 
 def forward(shape, w: Dict, tokens: Sequence[int], bias: Optional[torch.Tensor] = None,
-            tap_layers: Optional[Sequence[int]] = None, logit_rows: Optional[Sequence[int]] = None):
+            tap_layers: Optional[Sequence[int]] = None, logit_rows: Optional[Sequence[int]] = None,
+            bias_site: str = "mlp_up"):
     """Run the decoder over `tokens` (positions 0..T-1).
 
-    bias: None, or [T, L, d_ffn] fp32 steering biases b^(l) per position (Eq. 2).
+    bias: None, or [T, L, w] fp32 steering biases b^(l) per position. bias_site "mlp_up": w = d_ffn,
+      added to W_u a before the gating (Eq. 2); "after_mlp": w = d_model, added to the layer's output
+      f^(l) = x + MLP(...) (the "Inv. Bias after MLP" variant of Sec. 5).
     tap_layers: 1-based layers whose output residual stream is returned (App. A.2 order h, m, l).
     logit_rows: positions whose logits are computed (default: all).
     Returns (logits [R, V] fp32, taps [T, len(tap_layers), d] fp32 or None).
@@ -114,7 +117,12 @@ def forward(shape, w: Dict, tokens: Sequence[int], bias: Optional[torch.Tensor] 
         x = x + o @ lw["wo"].float().T
         a = rms_norm(x, lw["mlp_norm"], shape.norm_eps)
         b = None if bias is None else bias[:, li, :]
-        x = x + steered_swiglu(a, lw["w_gate"], lw["w_up"], lw["w_down"], b)
+        if bias_site == "mlp_up":
+            x = x + steered_swiglu(a, lw["w_gate"], lw["w_up"], lw["w_down"], b)
+        else:
+            x = x + steered_swiglu(a, lw["w_gate"], lw["w_up"], lw["w_down"], None)
+            if b is not None:
+                x = x + b
         taps[li + 1] = x
     hN = rms_norm(x, w["final_norm"], shape.norm_eps)
     if logit_rows is not None:

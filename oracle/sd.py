@@ -81,13 +81,14 @@ class OracleSD:
     def drafter_last(self, tokens: Sequence[int], bias_ids: Sequence[int]) -> torch.Tensor:
         """Drafter logits at the last position; position t computed under biases[bias_ids[t]]."""
         bias = torch.stack([self.biases[i] for i in bias_ids])
-        z, _ = model.forward(self.ds, self.dw, tokens, bias=bias, logit_rows=[len(tokens) - 1])
+        z, _ = model.forward(self.ds, self.dw, tokens, bias=bias, logit_rows=[len(tokens) - 1],
+                             bias_site=self.work.steering_site)
         return z[0]
 
     def _new_bias(self, taps_hml: torch.Tensor) -> int:
         g = steering.steering_vector(taps_hml, self.st, self.work.steer_ln_eps)
         self.gs.append(g)
-        self.biases.append(steering.steering_bias(g, self.st, self.ds.n_layers, self.ds.d_ffn))
+        self.biases.append(steering.steering_bias(g, self.st, self.ds.n_layers, self.work.bias_width))
         return len(self.biases) - 1
 
     # -- the loop -------------------------------------------------------------------------------

@@ -31,6 +31,7 @@ def steering_vector(taps_hml: torch.Tensor, st: dict, eps: float) -> torch.Tenso
     return layer_norm(cat @ st["w_hml"].float().T, st["ln_gamma"], st["ln_beta"], eps)
 
 
-def steering_bias(g: torch.Tensor, st: dict, n_layers: int, d_ffn: int) -> torch.Tensor:
-    """b^(l) = W_s^(l) g for every drafter layer: [..., L_D, F_D]."""
-    return (g.float() @ st["w_s"].float().T).reshape(*g.shape[:-1], n_layers, d_ffn)
+def steering_bias(g: torch.Tensor, st: dict, n_layers: int, width: int) -> torch.Tensor:
+    """b^(l) = W_s^(l) g for every drafter layer: [..., L_D, width] (width F_D for Eq. 2, d_D for the
+    after-MLP variant of Sec. 5)."""
+    return (g.float() @ st["w_s"].float().T).reshape(*g.shape[:-1], n_layers, width)

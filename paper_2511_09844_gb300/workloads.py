@@ -85,10 +85,19 @@ class PairWorkload:
     kv_block: int = 16
     steer_ln_eps: float = 1e-5
     description: str = ""
+    # where the steering bias enters the drafter: "mlp_up" is Eq. 2 (added to W_u a before the
+    # gating, F_D wide per layer); "after_mlp" is the "Inv. Bias after MLP" ablation of Sec. 5
+    # (added to each layer's output, d_D wide per layer)
+    steering_site: str = "mlp_up"
 
     @property
     def tap_layers(self) -> Tuple[int, int, int]:
         return default_tap_layers(self.verifier.n_layers)
+
+    @property
+    def bias_width(self) -> int:
+        """Steering bias entries per drafter layer."""
+        return self.drafter.d_ffn if self.steering_site == "mlp_up" else self.drafter.d_model
 
 
 TINY_V = LMShape(4, 256, 4, 4, 64, 1024, 4096, 10000.0, 1e-5)
@@ -178,13 +187,14 @@ def make_lm_weights(shape: LMShape, seed: int, device: str = "cpu", std: float =
 
 def make_steering_weights(work: PairWorkload, seed: int, device: str = "cpu", std: float = 0.02,
                           ln_jitter: float = 0.0, zero_ws: bool = False) -> dict:
-    """Random steering parameters: W_hml [d_g, 3 d_v], LayerNorm gain/shift [d_g], W_s [L_D*F_D, d_g].
+    """Random steering parameters: W_hml [d_g, 3 d_v], LayerNorm gain/shift [d_g], W_s [L_D*w, d_g]
+    with w = work.bias_width (F_D for Eq. 2, d_D for the after-MLP ablation).
 
-    W_s is one stacked matrix: rows l*F_D .. (l+1)*F_D-1 give the bias of drafter layer l.
+    W_s is one stacked matrix: rows l*w .. (l+1)*w-1 give the bias of drafter layer l.
     zero_ws=True gives the paper's W_s = 0 initialisation (Sec. 3.3).
     """
     dv, dg = work.verifier.d_model, work.d_steer
-    n_out = work.drafter.n_layers * work.drafter.d_ffn
+    n_out = work.drafter.n_layers * work.bias_width
     st = {"w_hml": _normal((dg, 3 * dv), std, seed * 1000 + 901, device)}
     if ln_jitter == 0.0:
         st["ln_gamma"] = torch.ones(dg, dtype=torch.bfloat16, device=device)

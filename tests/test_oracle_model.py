@@ -174,3 +174,30 @@ def test_attention_row_blocks_do_not_change_rows():
     whole = model.causal_attention(q, k, v, row_block=10 ** 9)
     for blk in (1, 13, 64):
         assert torch.allclose(model.causal_attention(q, k, v, row_block=blk), whole, atol=1e-6, rtol=0)
+
+
+def test_after_mlp_bias_site():
+    """The "Inv. Bias after MLP" variant (Sec. 5): b^(l) (d_model wide) is added to layer l's output
+    f^(l). A zero bias changes nothing; at the last layer the residual stream (the tap before the
+    final norm) moves by exactly b; a bias at layer l changes the input of every later layer; and
+    with Eq. 2's site the same d_model-wide tensor would not fit the MLP (widths differ)."""
+    vs = _small_pair()
+    w = W.make_lm_weights(vs, seed=8, norm_jitter=0.1)
+    toks = [5, 6, 7, 8, 9]
+    L = vs.n_layers
+    base, taps0 = model.forward(vs, w, toks, tap_layers=(1, 2, L))
+    zero = torch.zeros(len(toks), L, vs.d_model)
+    same, taps_z = model.forward(vs, w, toks, tap_layers=(1, 2, L), bias=zero, bias_site="after_mlp")
+    assert torch.equal(base, same) and torch.equal(taps0, taps_z)
+    g = torch.Generator().manual_seed(9)
+    b = zero.clone()
+    b[:, L - 1, :] = torch.randn(len(toks), vs.d_model, generator=g)
+    _, taps_b = model.forward(vs, w, toks, tap_layers=(1, 2, L), bias=b, bias_site="after_mlp")
+    assert torch.equal(taps_b[:, :2], taps0[:, :2])                      # earlier layers untouched
+    assert torch.allclose(taps_b[:, 2] - taps0[:, 2], b[:, L - 1], atol=1e-5, rtol=0)
+    b1 = zero.clone()
+    b1[:, 0, :] = 0.25
+    _, taps_1 = model.forward(vs, w, toks, tap_layers=(1, 2, L), bias=b1, bias_site="after_mlp")
+    assert torch.allclose(taps_1[:, 0] - taps0[:, 0], b1[:, 0], atol=1e-5, rtol=0)
+    assert (taps_1[:, 1] - taps0[:, 1] - b1[:, 0]).abs().max() > 1e-4   # layer 2 saw the shifted input
+    assert vs.d_model != vs.d_ffn
