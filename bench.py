@@ -45,6 +45,9 @@ def parse():
                     help="profiling aid: 'LV,LD' keeps the first LV verifier and LD drafter layers of the "
                          "workload (same widths, context and batch) so that an ncu capture holds a few GB; the "
                          "JSON line's config names the depth")
+    ap.add_argument("--steer-site", default="mlp_up", choices=["mlp_up", "after_mlp"],
+                    help="where the steering bias enters the drafter: mlp_up = Eq. 2 (SD^2), after_mlp = the "
+                         "'Inv. Bias after MLP' ablation of Sec. 5")
     ap.add_argument("--pretrained", action="store_true",
                     help="the unsteered pretrained drafter (no steering stage, no bias): the baseline SD^2 "
                          "is compared with")
@@ -186,6 +189,8 @@ def bench_workload(args):
     """The named workload; with --depth, its models cut to their first layers (profiling aid)."""
     import dataclasses
     work = W.WORKLOADS[args.workload]
+    if args.steer_site != work.steering_site:
+        work = dataclasses.replace(work, steering_site=args.steer_site)
     if args.depth:
         lv, ld = (int(x) for x in args.depth.split(","))
         work = dataclasses.replace(work, verifier=dataclasses.replace(work.verifier, n_layers=lv),
@@ -319,7 +324,9 @@ def run_ours(args, rank, world, local_rank):
                                                                  "(profiling aid, not the workload)"}
                                                        if args.depth else {}),
                                                     **({"drafter": "pretrained, unsteered (no steering stage)"}
-                                                       if args.pretrained else {}))),
+                                                       if args.pretrained else {}),
+                                                    **({"steering_site": "after the MLP (Sec. 5 ablation)"}
+                                                       if work.steering_site != "mlp_up" else {}))),
         "tau": round(tau, 4),
         "tokens_per_s_at_paper_tau": {"tau": 5.00, "value": round(5.00 / (ms_max / args.steps / 1e3), 2)},
         "prefill_s": round(prefill_s, 3),

@@ -77,6 +77,10 @@ typedef struct {
   int32_t no_steering;               /* 0: SD^2 (Eq. 2 biases in every drafter MLP). 1: the pretrained
                                         drafter alone, the baseline the paper compares with: no steering
                                         stage and no bias (the steering weights may then be null) */
+  int32_t steering_site;             /* 0: Eq. 2, the bias added to W_u a before the gating (SD^2);
+                                        W_s is [L_D * F_D, d_g]. 1: the "Inv. Bias after MLP" ablation
+                                        of Sec. 5, the bias added to each drafter layer's output;
+                                        W_s is [L_D * d_D, d_g] */
 } sd2_config;
 
 typedef struct {
@@ -92,7 +96,8 @@ typedef struct {
   const void* w_hml;                 /* [d_g, 3*d_v] bf16, columns ordered [h | m | l] (Sec. 3.1) */
   const void* steer_ln_gamma;        /* [d_g] bf16 layer-norm gain (App. A.2) */
   const void* steer_ln_beta;         /* [d_g] bf16 layer-norm shift */
-  const void* w_s;                   /* [L_D*F_D, d_g] bf16: rows l*F_D.. give W_s^(l) of Eq. 2 */
+  const void* w_s;                   /* [L_D*F_D, d_g] bf16: rows l*F_D.. give W_s^(l) of Eq. 2
+                                        ([L_D*d_D, d_g] with steering_site 1) */
 } sd2_weights;
 
 typedef struct sd2_ctx sd2_ctx;
@@ -141,7 +146,7 @@ sd2_status sd2_set_graphs(sd2_ctx* ctx, int32_t enable);
 /* Read-only views of the context's device buffers, for tests and measurement. `which`:
  *   0 target logits  [B, k+1, V] f32     1 draft logits [B, k, V] f32     2 drafts x^ [B, k] i32
  *   3 verifier taps  [B, k+1, 3, d_v] f32 (order h, m, l)   4 steering vector g [B, d_g] f32
- *   5 steering biases [B, L_D*F_D] f32   6 committed tokens [B, max_ctx] i32
+ *   5 steering biases [B, L_D*F_D] f32 ([B, L_D*d_D] with steering_site 1)   6 committed tokens [B, max_ctx] i32
  *   7 per-sequence state [B, 4] i32: committed length n, drafter cached length, j, stopped
  *   8 iteration counter [1] i32 (the `step` of the Philox counters; 0 = prefill)
  * *d_ptr, *n_elems and *dtype (SD2_DTYPE_*) describe the buffer; B is the prefilled batch. */
@@ -201,7 +206,8 @@ sd2_status sd2_steer(const float* d_taps, int32_t B, int32_t d_v, const void* w_
 
 /* Weight-streaming GEMM of the decoder on caller buffers, Y[m, n] = sum_k X[m, k] W[n, k]:
  *   d_x [M, ldx] bf16 (first K columns used), d_w [N, K] bf16 (nn.Linear layout).
- *   epilogue 0: d_out[m*ldo + n] = Y (f32); 1: d_out[m*ldo + n] += Y (the residual add);
+ *   epilogue 0: d_out[m*ldo + n] = Y (f32); 1: d_out[m*ldo + n] += Y (the residual add), plus
+ *      d_bias[seq[m]*ld_bias + n] when d_bias is given (the after-MLP steering site);
  *   2: the steered SwiGLU of Eq. 2 with d_w = W_gate, d_w_up = W_up (both [N, K]):
  *      d_h[m*N + f] = bf16((up + d_bias[seq[m]*ld_bias + f]) * SiLU(gate)), d_bias/d_seq optional.
  *   impl 0: tensor cores (tcgen05, TMA) where the shape allows (K % 64 == 0; N % 128 == 0, or

@@ -243,6 +243,9 @@ GemmArgs& tc(sd2_ctx* c, GemmArgs& g) {
   return g;
 }
 
+// Steering bias entries per drafter layer: F_D for Eq. 2 (inside the MLP), d_D after the MLP.
+int bias_width(const sd2_ctx* c) { return c->cfg.steering_site ? c->D.c.d_model : c->D.c.d_ffn; }
+
 double gemm_bytes(int M, int N, int K, int out_bytes) {
   return 2.0 * N * K + 2.0 * M * K + static_cast<double>(out_bytes) * M * N;
 }
@@ -274,7 +277,7 @@ sd2_status head(sd2_ctx* c, const Model& m, const Plan& p, const FwdOut& o) {
 // The drafter's layers over plan p in one persistent launch (chain.cu), then the head. Used for
 // the drafter steps when the chain takes their shape; forward() otherwise.
 bool chain_takes(sd2_ctx* c, const Plan& p) {
-  if (!c->chain_ok || !c->use_chain || c->gemm_impl != 0) return false;
+  if (!c->chain_ok || !c->use_chain || c->gemm_impl != 0 || c->cfg.steering_site != 0) return false;
   ChainRun r;
   r.M = p.M; r.n_splits = p.n_splits; r.chunk = p.chunk; r.max_rows = p.max_rows;
   return chain_supported(c->chain, r);
@@ -336,14 +339,22 @@ sd2_status forward(sd2_ctx* c, const Model& m, const Plan& p, const FwdOut& o) {
     g.x = c->a; g.ldx = d; g.M = M; g.K = d;
     g.seg[0] = {m.W(l, SD2_W_GATE), F}; g.seg[1] = {m.W(l, SD2_W_UP), F}; g.nseg = 2;
     g.epi = EPI_SWIGLU; g.out_bf = c->h; g.ldh = F;
-    g.bias = o.bias ? o.bias + static_cast<size_t>(l) * F : nullptr;
-    g.ld_bias = L * F; g.row_seq = p.seq;
+    if (c->cfg.steering_site == 0) {     // Eq. 2: added to W_u a before the gating
+      g.bias = o.bias ? o.bias + static_cast<size_t>(l) * F : nullptr;
+      g.ld_bias = L * F;
+    }
+    g.row_seq = p.seq;
     return g;
   };
   auto down_args = [&](int l) {
     GemmArgs g{};
     g.x = c->h; g.ldx = F; g.M = M; g.K = F;
     g.seg[0] = {m.W(l, SD2_W_DOWN), d}; g.nseg = 1; g.epi = EPI_ADD; g.out = c->x; g.ldo = d;
+    if (c->cfg.steering_site == 1 && o.bias) {   // after the MLP: added to the layer's output
+      g.bias = o.bias + static_cast<size_t>(l) * d;
+      g.ld_bias = L * d;
+      g.row_seq = p.seq;
+    }
     return g;
   };
   // producer / consumer halves of a fused RMSNorm with gamma
@@ -416,7 +427,7 @@ sd2_status forward(sd2_ctx* c, const Model& m, const Plan& p, const FwdOut& o) {
 // a1: g = LN(W_hml [h; m; l]) at each sequence's steering row, biases = W_s g.
 sd2_status steer(sd2_ctx* c, const int* row_idx) {
   const int B = c->B, dv = c->V.c.d_model, dg = c->cfg.d_steer, k = c->cfg.k;
-  const int nb = c->D.c.n_layers * c->D.c.d_ffn;
+  const int nb = c->D.c.n_layers * bias_width(c);
   CK(timed(c, PC_OTHER, 0, [&] {
     return gather_rows_bf16(c->taps, (k + 1) * 3 * dv, row_idx, 3 * dv, B, c->hml_in, c->st);
   }));
@@ -580,6 +591,7 @@ sd2_status sd2_init(const sd2_config* cfg, const sd2_weights* w, void* stream, s
   if (cfg->max_ctx < cfg->k + 3) return fail(nullptr, SD2_EINVAL, "max_ctx too small for one block");
   if (cfg->d_steer <= 0 || cfg->d_steer % 8) return fail(nullptr, SD2_EINVAL, "d_steer must be a positive multiple of 8");
   if (cfg->max_prefill_tokens < 1) return fail(nullptr, SD2_EINVAL, "max_prefill_tokens must be positive");
+  if (cfg->steering_site != 0 && cfg->steering_site != 1) return fail(nullptr, SD2_EINVAL, "steering_site must be 0 or 1");
   for (int t = 0; t < 3; ++t)
     if (cfg->tap_layers[t] < 1 || cfg->tap_layers[t] > cfg->verifier.n_layers)
       return fail(nullptr, SD2_EINVAL, "tap_layers must be 1-based verifier layers");
@@ -630,7 +642,8 @@ sd2_status sd2_init(const sd2_config* cfg, const sd2_weights* w, void* stream, s
     ALLOC(c->g_pre, static_cast<size_t>(maxB) * cfg->d_steer);
     ALLOC(c->g, static_cast<size_t>(maxB) * cfg->d_steer);
     ALLOC(c->g_bf, static_cast<size_t>(maxB) * cfg->d_steer * 2);
-    ALLOC(c->bias, static_cast<size_t>(maxB) * cfg->drafter.n_layers * cfg->drafter.d_ffn);
+    ALLOC(c->bias, static_cast<size_t>(maxB) * cfg->drafter.n_layers *
+                       std::max(cfg->drafter.d_ffn, cfg->drafter.d_model));
     ALLOC(c->samp_slot, maxB);
     ALLOC(c->samp_counter, maxB);
     void* acc;
@@ -864,7 +877,7 @@ sd2_status sd2_debug_buffer(const sd2_ctx* c, int32_t which, void** d_ptr, int64
     case 2: *d_ptr = c->xhat; *n_elems = B * k; *dtype = -1; break;
     case 3: *d_ptr = c->taps; *n_elems = B * (k + 1) * 3 * c->V.c.d_model; *dtype = SD2_DTYPE_F32; break;
     case 4: *d_ptr = c->g; *n_elems = B * c->cfg.d_steer; *dtype = SD2_DTYPE_F32; break;
-    case 5: *d_ptr = c->bias; *n_elems = B * c->D.c.n_layers * c->D.c.d_ffn; *dtype = SD2_DTYPE_F32; break;
+    case 5: *d_ptr = c->bias; *n_elems = B * c->D.c.n_layers * bias_width(c); *dtype = SD2_DTYPE_F32; break;
     case 6: *d_ptr = c->committed; *n_elems = B * c->cfg.max_ctx; *dtype = -1; break;
     case 7: *d_ptr = c->state; *n_elems = 4 * static_cast<int64_t>(c->maxB); *dtype = -1; break;
     case 8: *d_ptr = c->iter; *n_elems = 1; *dtype = -1; break;

@@ -91,6 +91,11 @@ __global__ void __launch_bounds__(kThreads) gemm_simt_kernel(const GemmArgs a, i
           a.out[static_cast<size_t>(m) * a.ldo + n0] = v0;
           if (n1 >= 0) a.out[static_cast<size_t>(m) * a.ldo + n1] = v1;
         } else if (EPI == EPI_ADD) {
+          if (a.bias) {   // a bias of the row's sequence added with the output (after-MLP steering)
+            const float* bs = a.bias + static_cast<size_t>(a.row_seq ? a.row_seq[m] : 0) * a.ld_bias;
+            v0 += bs[n0];
+            if (n1 >= 0) v1 += bs[n1];
+          }
           a.out[static_cast<size_t>(m) * a.ldo + n0] += v0;
           if (n1 >= 0) a.out[static_cast<size_t>(m) * a.ldo + n1] += v1;
         } else {

@@ -87,9 +87,12 @@ constexpr int kXS = 17;   // padded row of the epilogue exchange buffer (128 row
 
 // ------------------------------------------------------------------------------ epilogue stores
 // One output value of weight row `row` of tile (wt, tt) for token m (m < M).
+__device__ __forceinline__ float add_bias_of(const TcArgs& a, int n, int m) {
+  return a.bias ? a.bias[static_cast<size_t>(a.row_seq ? a.row_seq[m] : 0) * a.ld_bias + n] : 0.f;
+}
 __device__ __forceinline__ void emit_plain(const TcArgs& a, int wt, int row, int m, float v) {
   float* o = a.out + static_cast<size_t>(m) * a.ldo + wt * kWRows + row;
-  if (a.epi == EPI_ADD) *o += v;
+  if (a.epi == EPI_ADD) *o += v + add_bias_of(a, wt * kWRows + row, m);
   else *o = v;
 }
 // Eq. 2 for feature f of the tile (gate row f, up row f + 64).
@@ -193,7 +196,7 @@ __device__ __forceinline__ void finish_chunk(const TcArgs& a, int wt, int tt, in
       float sq = 0.f;
       if (m0 + j < a.M) {
         float* o = a.out + static_cast<size_t>(m0 + j) * a.ldo + n;
-        const float xn = *o + v[j];
+        const float xn = *o + (v[j] + add_bias_of(a, n, m0 + j));
         *o = xn;
         norm_produce(a, m0 + j, n, xn, g);
         sq = xn * xn;
@@ -239,12 +242,12 @@ __device__ __forceinline__ int pairs_max(int sp) { return (64 + sp - 1) / sp; }
 // are known: residuals (EPI_ADD), steering bias (SwiGLU), or position, rotary factors and KV
 // block (QKV; blk = -1 when the pair is a q head or the row writes no KV).
 struct PairOps {
-  float r0, r1, bias, g0, g1;
+  float r0, r1, bias, bias1, g0, g1;   // bias: SwiGLU's, or EPI_ADD's for member 0 (bias1: member 1)
   float2 cs;
   int pos, blk;
 };
 __device__ __forceinline__ PairOps pair_ops(const TcArgs& a, int wt, int p, int m) {
-  PairOps o{0.f, 0.f, 0.f, 0.f, 0.f, make_float2(1.f, 0.f), 0, -1};
+  PairOps o{0.f, 0.f, 0.f, 0.f, 0.f, 0.f, make_float2(1.f, 0.f), 0, -1};
   if (a.swiglu) {
     if (a.bias) o.bias = a.bias[static_cast<size_t>(a.row_seq ? a.row_seq[m] : 0) * a.ld_bias + wt * 64 + p];
   } else if (a.epi == EPI_QKV) {
@@ -260,6 +263,8 @@ __device__ __forceinline__ PairOps pair_ops(const TcArgs& a, int wt, int p, int 
     const float* x = a.out + static_cast<size_t>(m) * a.ldo + wt * kWRows;
     o.r0 = x[pair_row(a, p, 0)];
     o.r1 = x[pair_row(a, p, 1)];
+    o.bias = add_bias_of(a, wt * kWRows + pair_row(a, p, 0), m);
+    o.bias1 = add_bias_of(a, wt * kWRows + pair_row(a, p, 1), m);
     if (a.norm_out) {
       o.g0 = __bfloat162float(a.norm_gamma[wt * kWRows + pair_row(a, p, 0)]);
       o.g1 = __bfloat162float(a.norm_gamma[wt * kWRows + pair_row(a, p, 1)]);
@@ -298,7 +303,7 @@ __device__ __forceinline__ float pair_emit(const TcArgs& a, int wt, int p, int m
   } else {
     float* x = a.out + static_cast<size_t>(m) * a.ldo + wt * kWRows;
     const bool add = a.epi == EPI_ADD;
-    const float x0 = add ? o.r0 + s0 : s0, x1 = add ? o.r1 + s1 : s1;
+    const float x0 = add ? o.r0 + (s0 + o.bias) : s0, x1 = add ? o.r1 + (s1 + o.bias1) : s1;
     x[pair_row(a, p, 0)] = x0;
     x[pair_row(a, p, 1)] = x1;
     if (a.norm_out) {

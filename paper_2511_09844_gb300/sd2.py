@@ -40,7 +40,8 @@ class LMConfig(ctypes.Structure):
 class Config(ctypes.Structure):
     _fields_ = [("verifier", LMConfig), ("drafter", LMConfig), ("d_steer", c_int32), ("tap_layers", c_int32 * 3),
                 ("steer_ln_eps", c_float), ("k", c_int32), ("max_batch", c_int32), ("max_ctx", c_int32),
-                ("max_prefill_tokens", c_int32), ("kv_block", c_int32), ("no_steering", c_int32)]
+                ("max_prefill_tokens", c_int32), ("kv_block", c_int32), ("no_steering", c_int32),
+                ("steering_site", c_int32)]
 
 
 class LMWeights(ctypes.Structure):
@@ -153,6 +154,7 @@ class SD2Engine:
         cfg.max_prefill_tokens = max_prefill_tokens
         cfg.kv_block = work.kv_block
         cfg.no_steering = 0 if steering else 1     # False: the pretrained drafter, no steering stage
+        cfg.steering_site = {"mlp_up": 0, "after_mlp": 1}[work.steering_site]
         self.cfg = cfg
         w = Weights()
         w.verifier = self._lm_weights(verifier_w)

@@ -83,6 +83,18 @@ def test_pretrained_drafter_mode(temp):
     assert rep.blocks == 6
 
 
+@pytest.mark.parametrize("gemm_impl", [0, 1])
+def test_after_mlp_steering_site(gemm_impl):
+    """The "Inv. Bias after MLP" ablation (Sec. 5): W_s g (d_D wide) added to each drafter layer's
+    output, through the residual-adding GEMM epilogue; parity with the oracle's same site."""
+    work = parity.tiny_work(steering_site="after_mlp")
+    vw, dw, st = parity.tiny_weights(work, seed=9)
+    assert st["w_s"].shape[0] == work.drafter.n_layers * work.drafter.d_model
+    prompts = W.make_prompts(work.verifier.vocab, 2, (20, 33), seed=13)
+    rep = parity.run(work, vw, dw, st, prompts, [1.0, 0.0], seed=17, n_steps=5, gemm_impl=gemm_impl)
+    assert rep.blocks == 10
+
+
 def test_stage_timing_keeps_results():
     """Stage event nodes in the captured step change no output; the stage times are positive."""
     work = parity.tiny_work()

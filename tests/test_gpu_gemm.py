@@ -54,6 +54,22 @@ def test_residual_add_and_strided_rows(impl):
 
 
 @pytest.mark.parametrize("impl", [1, 2])
+@pytest.mark.parametrize("M,N,K", [(5, 640, 448), (2, 2048, 8192), (144, 256, 1024)])
+def test_residual_add_with_sequence_bias(impl, M, N, K):
+    """Residual add plus a per-sequence bias (the after-MLP steering site): out += Y + bias[seq[m]]."""
+    x, w = _operands(M, N, K, 5 + M)
+    g = torch.Generator().manual_seed(6)
+    out0 = torch.randn(M, N, generator=g)
+    bias = torch.randn(3, N, generator=g)
+    seq = torch.randint(0, 3, (M,), generator=g).to(torch.int32)
+    out = out0.clone().cuda()
+    sd2.gemm(x.cuda(), w.cuda(), epilogue=1, out=out, bias=bias.cuda(), seq=seq.cuda(), impl=impl)
+    torch.cuda.synchronize()
+    ref = out0 + x.float() @ w.float().T + bias[seq.long()]
+    assert parity.row_rel_err(out.cpu(), ref) < TOL
+
+
+@pytest.mark.parametrize("impl", [1, 2])
 @pytest.mark.parametrize("M,F,K", [(6, 256, 512), (18, 192, 2048), (1, 64, 4864)])
 def test_steered_swiglu_epilogue(impl, M, F, K):
     g = torch.Generator().manual_seed(M + F)
