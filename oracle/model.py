@@ -88,14 +88,27 @@ def steered_swiglu(a: torch.Tensor, w_gate, w_up, w_down, bias: Optional[torch.T
     return (up * silu(a @ w_gate.float().T)) @ w_down.float().T
 
 
+def cond_bias(f: torch.Tensor, g: torch.Tensor, st: Dict, layer: int) -> torch.Tensor:
+    """The "Cond. Bias in MLP" variant (Sec. 5): b = W_c2 SiLU(W_c1 [f; g]) per position, with f the
+    layer's input f^(l-1) [T, d_D] and g [T, d_g]; W_c1 = [W_c1x | W_c1g] split by input block."""
+    dg = st["w_c1g"].shape[1]
+    F = st["w_c2"].shape[0] // (st["w_c1x"].shape[0] // dg)
+    w1x = st["w_c1x"][layer * dg:(layer + 1) * dg].float()
+    w1g = st["w_c1g"][layer * dg:(layer + 1) * dg].float()
+    w2 = st["w_c2"][layer * F:(layer + 1) * F].float()
+    return silu(f @ w1x.T + g @ w1g.T) @ w2.T
+
+
 def forward(shape, w: Dict, tokens: Sequence[int], bias: Optional[torch.Tensor] = None,
             tap_layers: Optional[Sequence[int]] = None, logit_rows: Optional[Sequence[int]] = None,
-            bias_site: str = "mlp_up"):
+            bias_site: str = "mlp_up", cond: Optional[tuple] = None):
     """Run the decoder over `tokens` (positions 0..T-1).
 
     bias: None, or [T, L, w] fp32 steering biases b^(l) per position. bias_site "mlp_up": w = d_ffn,
       added to W_u a before the gating (Eq. 2); "after_mlp": w = d_model, added to the layer's output
       f^(l) = x + MLP(...) (the "Inv. Bias after MLP" variant of Sec. 5).
+    cond: with bias_site "cond_mlp", (g [T, d_g] per position, steering weights): the bias of layer l
+      at each position is cond_bias(f^(l-1), g) and enters as in Eq. 2 ("Cond. Bias in MLP", Sec. 5).
     tap_layers: 1-based layers whose output residual stream is returned (App. A.2 order h, m, l).
     logit_rows: positions whose logits are computed (default: all).
     Returns (logits [R, V] fp32, taps [T, len(tap_layers), d] fp32 or None).
@@ -107,6 +120,7 @@ def forward(shape, w: Dict, tokens: Sequence[int], bias: Optional[torch.Tensor] 
     taps = {}
     H, Hkv, hd = shape.n_heads, shape.n_kv_heads, shape.head_dim
     for li, lw in enumerate(w["layers"]):
+        f_in = x                                             # f^(l-1): this layer's input
         a = rms_norm(x, lw["attn_norm"], shape.norm_eps)
         q = (a @ lw["wq"].float().T).view(T, H, hd)
         k = (a @ lw["wk"].float().T).view(T, Hkv, hd)
@@ -117,7 +131,9 @@ def forward(shape, w: Dict, tokens: Sequence[int], bias: Optional[torch.Tensor] 
         x = x + o @ lw["wo"].float().T
         a = rms_norm(x, lw["mlp_norm"], shape.norm_eps)
         b = None if bias is None else bias[:, li, :]
-        if bias_site == "mlp_up":
+        if bias_site == "cond_mlp" and cond is not None:
+            b = cond_bias(f_in, cond[0], cond[1], li)
+        if bias_site in ("mlp_up", "cond_mlp"):
             x = x + steered_swiglu(a, lw["w_gate"], lw["w_up"], lw["w_down"], b)
         else:
             x = x + steered_swiglu(a, lw["w_gate"], lw["w_up"], lw["w_down"], None)

@@ -79,7 +79,13 @@ class OracleSD:
         return z, tp[first:last + 1]
 
     def drafter_last(self, tokens: Sequence[int], bias_ids: Sequence[int]) -> torch.Tensor:
-        """Drafter logits at the last position; position t computed under biases[bias_ids[t]]."""
+        """Drafter logits at the last position; position t computed under the steering of stage
+        bias_ids[t] (its biases, or for "cond_mlp" its g)."""
+        if self.work.steering_site == "cond_mlp":
+            g_rows = torch.stack([self.gs[i] for i in bias_ids])
+            z, _ = model.forward(self.ds, self.dw, tokens, logit_rows=[len(tokens) - 1], bias_site="cond_mlp",
+                                 cond=(g_rows, self.st))
+            return z[0]
         bias = torch.stack([self.biases[i] for i in bias_ids])
         z, _ = model.forward(self.ds, self.dw, tokens, bias=bias, logit_rows=[len(tokens) - 1],
                              bias_site=self.work.steering_site)
@@ -88,7 +94,10 @@ class OracleSD:
     def _new_bias(self, taps_hml: torch.Tensor) -> int:
         g = steering.steering_vector(taps_hml, self.st, self.work.steer_ln_eps)
         self.gs.append(g)
-        self.biases.append(steering.steering_bias(g, self.st, self.ds.n_layers, self.work.bias_width))
+        if self.work.steering_site == "cond_mlp":     # the biases depend on each position's input
+            self.biases.append(torch.zeros(0))
+        else:
+            self.biases.append(steering.steering_bias(g, self.st, self.ds.n_layers, self.work.bias_width))
         return len(self.biases) - 1
 
     # -- the loop -------------------------------------------------------------------------------

@@ -87,7 +87,9 @@ class PairWorkload:
     description: str = ""
     # where the steering bias enters the drafter: "mlp_up" is Eq. 2 (added to W_u a before the
     # gating, F_D wide per layer); "after_mlp" is the "Inv. Bias after MLP" ablation of Sec. 5
-    # (added to each layer's output, d_D wide per layer)
+    # (added to each layer's output, d_D wide per layer); "cond_mlp" is its "Cond. Bias in MLP"
+    # ablation (per position, a 2-layer MLP of the layer input f^(l-1) and g gives the bias used
+    # as in Eq. 2)
     steering_site: str = "mlp_up"
 
     @property
@@ -97,7 +99,7 @@ class PairWorkload:
     @property
     def bias_width(self) -> int:
         """Steering bias entries per drafter layer."""
-        return self.drafter.d_ffn if self.steering_site == "mlp_up" else self.drafter.d_model
+        return self.drafter.d_model if self.steering_site == "after_mlp" else self.drafter.d_ffn
 
 
 TINY_V = LMShape(4, 256, 4, 4, 64, 1024, 4096, 10000.0, 1e-5)
@@ -202,6 +204,15 @@ def make_steering_weights(work: PairWorkload, seed: int, device: str = "cpu", st
     else:
         st["ln_gamma"] = _norm_weight(dg, ln_jitter, seed * 1000 + 902, device)
         st["ln_beta"] = _normal((dg,), ln_jitter, seed * 1000 + 903, device)
+    if work.steering_site == "cond_mlp":
+        # the conditional bias MLP of every drafter layer: hidden width d_g, input [f^(l-1); g]
+        # split into its two column blocks W_c1 = [W_c1x | W_c1g]; W_c2 maps back to F_D
+        L, dd = work.drafter.n_layers, work.drafter.d_model
+        st["w_c1x"] = _normal((L * dg, dd), std, seed * 1000 + 905, device)
+        st["w_c1g"] = _normal((L * dg, dg), std, seed * 1000 + 906, device)
+        st["w_c2"] = (torch.zeros((n_out, dg), dtype=torch.bfloat16, device=device) if zero_ws
+                      else _normal((n_out, dg), std, seed * 1000 + 907, device))
+        return st
     if zero_ws:
         st["w_s"] = torch.zeros((n_out, dg), dtype=torch.bfloat16, device=device)
     else:

@@ -201,3 +201,37 @@ def test_after_mlp_bias_site():
     assert torch.allclose(taps_1[:, 0] - taps0[:, 0], b1[:, 0], atol=1e-5, rtol=0)
     assert (taps_1[:, 1] - taps0[:, 1] - b1[:, 0]).abs().max() > 1e-4   # layer 2 saw the shifted input
     assert vs.d_model != vs.d_ffn
+
+
+def test_cond_bias_site():
+    """The "Cond. Bias in MLP" variant (Sec. 5): b = W_c2 SiLU(W_c1 [f^(l-1); g]) per position,
+    used as in Eq. 2. W_c2 = 0 leaves the drafter unsteered; with W_c1x = 0 the bias no longer
+    depends on the position's input and the pass equals Eq. 2 with the stage bias
+    W_c2 SiLU(W_c1g g); the bias reads this layer's input (a change of f changes it)."""
+    vs = _small_pair()
+    dg = 8
+    w = W.make_lm_weights(vs, seed=10, norm_jitter=0.1)
+    toks = [3, 1, 4, 1, 5, 9]
+    T, L = len(toks), vs.n_layers
+    g = torch.Generator().manual_seed(11)
+    st = {"w_c1x": torch.randn(L * dg, vs.d_model, generator=g) * 0.1,
+          "w_c1g": torch.randn(L * dg, dg, generator=g) * 0.1,
+          "w_c2": torch.zeros(L * vs.d_ffn, dg)}
+    g_rows = torch.randn(T, dg, generator=g)
+    base, _ = model.forward(vs, w, toks)
+    zero, _ = model.forward(vs, w, toks, bias_site="cond_mlp", cond=(g_rows, st))
+    assert torch.equal(base, zero)
+    st["w_c2"] = torch.randn(L * vs.d_ffn, dg, generator=g) * 0.1
+    st_nox = dict(st, w_c1x=torch.zeros_like(st["w_c1x"]))
+    cond, _ = model.forward(vs, w, toks, bias_site="cond_mlp", cond=(g_rows, st_nox))
+    stage = torch.stack([model.silu(g_rows @ st["w_c1g"][l * dg:(l + 1) * dg].T) @
+                         st["w_c2"][l * vs.d_ffn:(l + 1) * vs.d_ffn].T for l in range(L)], dim=1)
+    eq2, _ = model.forward(vs, w, toks, bias=stage)
+    assert torch.allclose(cond, eq2, atol=1e-5, rtol=1e-4)
+    full, _ = model.forward(vs, w, toks, bias_site="cond_mlp", cond=(g_rows, st))
+    assert (full - cond).abs().max() > 1e-4
+    # the hand-evaluated bias of layer 0 at one position (f^(-1) = the embedding row)
+    f0 = w["embed"][toks[2]].float()
+    b0 = model.cond_bias(f0[None], g_rows[2:3], st, 0)[0]
+    ref = model.silu(f0 @ st["w_c1x"][:dg].T + g_rows[2] @ st["w_c1g"][:dg].T) @ st["w_c2"][:vs.d_ffn].T
+    assert torch.allclose(b0, ref)
