@@ -45,9 +45,9 @@ def parse():
                     help="profiling aid: 'LV,LD' keeps the first LV verifier and LD drafter layers of the "
                          "workload (same widths, context and batch) so that an ncu capture holds a few GB; the "
                          "JSON line's config names the depth")
-    ap.add_argument("--steer-site", default="mlp_up", choices=["mlp_up", "after_mlp"],
+    ap.add_argument("--steer-site", default="mlp_up", choices=["mlp_up", "after_mlp", "cond_mlp"],
                     help="where the steering bias enters the drafter: mlp_up = Eq. 2 (SD^2), after_mlp = the "
-                         "'Inv. Bias after MLP' ablation of Sec. 5")
+                         "'Inv. Bias after MLP' ablation of Sec. 5, cond_mlp = its 'Cond. Bias in MLP' ablation")
     ap.add_argument("--pretrained", action="store_true",
                     help="the unsteered pretrained drafter (no steering stage, no bias): the baseline SD^2 "
                          "is compared with")
@@ -325,7 +325,9 @@ def run_ours(args, rank, world, local_rank):
                                                        if args.depth else {}),
                                                     **({"drafter": "pretrained, unsteered (no steering stage)"}
                                                        if args.pretrained else {}),
-                                                    **({"steering_site": "after the MLP (Sec. 5 ablation)"}
+                                                    **({"steering_site": {"after_mlp": "after the MLP (Sec. 5 ablation)",
+                                                                          "cond_mlp": "conditional bias MLP (Sec. 5 ablation)"}
+                                                        [work.steering_site]}
                                                        if work.steering_site != "mlp_up" else {}))),
         "tau": round(tau, 4),
         "tokens_per_s_at_paper_tau": {"tau": 5.00, "value": round(5.00 / (ms_max / args.steps / 1e3), 2)},

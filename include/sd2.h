@@ -80,7 +80,9 @@ typedef struct {
   int32_t steering_site;             /* 0: Eq. 2, the bias added to W_u a before the gating (SD^2);
                                         W_s is [L_D * F_D, d_g]. 1: the "Inv. Bias after MLP" ablation
                                         of Sec. 5, the bias added to each drafter layer's output;
-                                        W_s is [L_D * d_D, d_g] */
+                                        W_s is [L_D * d_D, d_g]. 2: its "Cond. Bias in MLP" ablation,
+                                        a per-position bias from a 2-layer MLP of the layer input and
+                                        g, used as in Eq. 2 (weights w_c1x, w_c1g, w_c2) */
 } sd2_config;
 
 typedef struct {
@@ -97,7 +99,12 @@ typedef struct {
   const void* steer_ln_gamma;        /* [d_g] bf16 layer-norm gain (App. A.2) */
   const void* steer_ln_beta;         /* [d_g] bf16 layer-norm shift */
   const void* w_s;                   /* [L_D*F_D, d_g] bf16: rows l*F_D.. give W_s^(l) of Eq. 2
-                                        ([L_D*d_D, d_g] with steering_site 1) */
+                                        ([L_D*d_D, d_g] with steering_site 1; unused with 2) */
+  /* steering_site 2 only: the conditional bias MLP of every drafter layer l,
+   * b = W_c2^(l) SiLU(W_c1x^(l) f^(l-1) + W_c1g^(l) g), hidden width d_g (null otherwise) */
+  const void* w_c1x;                 /* [L_D*d_g, d_D] bf16 */
+  const void* w_c1g;                 /* [L_D*d_g, d_g] bf16 */
+  const void* w_c2;                  /* [L_D*F_D, d_g] bf16 */
 } sd2_weights;
 
 typedef struct sd2_ctx sd2_ctx;
@@ -209,7 +216,9 @@ sd2_status sd2_steer(const float* d_taps, int32_t B, int32_t d_v, const void* w_
  *   epilogue 0: d_out[m*ldo + n] = Y (f32); 1: d_out[m*ldo + n] += Y (the residual add), plus
  *      d_bias[seq[m]*ld_bias + n] when d_bias is given (the after-MLP steering site);
  *   2: the steered SwiGLU of Eq. 2 with d_w = W_gate, d_w_up = W_up (both [N, K]):
- *      d_h[m*N + f] = bf16((up + d_bias[seq[m]*ld_bias + f]) * SiLU(gate)), d_bias/d_seq optional.
+ *      d_h[m*N + f] = bf16((up + d_bias[seq[m]*ld_bias + f]) * SiLU(gate)), d_bias/d_seq optional;
+ *   4: d_h[m*N + n] = bf16(SiLU(Y + d_bias[seq[m]*ld_bias + n])), d_bias/d_seq optional (the hidden
+ *      layer of the conditional bias MLP).
  *   impl 0: tensor cores (tcgen05, TMA) where the shape allows (K % 64 == 0; N % 128 == 0, or
  *   N % 64 == 0 for epilogue 2), else CUDA cores; 1: CUDA cores; 2: tensor cores or SD2_EINVAL.
  *   No device memory is allocated except, once, a 4-byte error word. */

@@ -75,6 +75,7 @@ struct sd2_ctx {
   sd2_config cfg{};
   Model V, D;
   const void *w_hml = nullptr, *ln_g = nullptr, *ln_b = nullptr, *w_s = nullptr;
+  const void *w_c1x = nullptr, *w_c1g = nullptr, *w_c2 = nullptr;   // steering_site 2
   cudaStream_t st = nullptr, cap_st = nullptr;
   int B = 0, phase = 0, maxB = 0, max_rows = 0;
   unsigned long long seed = 0;
@@ -91,6 +92,13 @@ struct sd2_ctx {
   float *x = nullptr, *qkv = nullptr, *q = nullptr, *logits_t = nullptr, *logits_d = nullptr;
   float *taps = nullptr, *g_pre = nullptr, *g = nullptr, *bias = nullptr;
   float* ssq = nullptr;          // fused RMSNorm: [slices][max_rows] sums of squares of the residual stream
+  // steering_site 2: per-stage W_c1g g [B, L_D*d_g], per-layer f^(l-1) in bf16 [R, d_D], the bias
+  // MLP's hidden layer [R, d_g] and its per-row output [R, F_D]; row index table [R]
+  float* cg = nullptr;
+  void* fb = nullptr;
+  void* cu_h = nullptr;
+  float* rowbias = nullptr;
+  int* row_ident = nullptr;
   ChainPlan chain{};             // the drafter's persistent layer chain (chain.cu), when its shape allows
   bool chain_ok = false;
   bool use_chain = false;        // measured slower than the per-kernel path on GB300 (off by default)
@@ -388,6 +396,23 @@ sd2_status forward(sd2_ctx* c, const Model& m, const Plan& p, const FwdOut& o) {
         return rmsnorm(c->x, nullptr, m.W(l, SD2_W_ATTN_NORM), mc.norm_eps, M, d, c->a, o.taps, o.tap_row, tap_mask(l),
                        c->st);
       }));
+    if (c->cfg.steering_site == 2 && o.bias) {
+      // "Cond. Bias in MLP" (Sec. 5): b = W_c2 SiLU(W_c1x f^(l-1) + W_c1g g) per row, from this
+      // layer's input f^(l-1) = x (before the attention) and the stage's W_c1g g
+      const int dg = c->cfg.d_steer;
+      CK(timed(c, PC_OTHER, 0, [&] { return rows_to_bf16(c->x, d, M, d, c->fb, c->st); }));
+      GemmArgs c1{};
+      c1.x = c->fb; c1.ldx = d; c1.M = M; c1.K = d;
+      c1.seg[0] = {static_cast<const char*>(c->w_c1x) + static_cast<size_t>(l) * dg * d * 2, dg}; c1.nseg = 1;
+      c1.epi = EPI_SILU; c1.out_bf = c->cu_h; c1.ldh = dg;
+      c1.bias = c->cg + static_cast<size_t>(l) * dg; c1.ld_bias = L * dg; c1.row_seq = p.seq;
+      CK(timed(c, PC_GEMM, gemm_bytes(M, dg, d, 2), [&] { return gemm(tc(c, c1), c->st); }));
+      GemmArgs c2{};
+      c2.x = c->cu_h; c2.ldx = dg; c2.M = M; c2.K = dg;
+      c2.seg[0] = {static_cast<const char*>(c->w_c2) + static_cast<size_t>(l) * F * dg * 2, F}; c2.nseg = 1;
+      c2.epi = EPI_STORE; c2.out = c->rowbias; c2.ldo = F;
+      CK(timed(c, PC_GEMM, gemm_bytes(M, F, dg, 4), [&] { return gemm(tc(c, c2), c->st); }));
+    }
     GemmArgs g = qkv_args(l);
     if (fused) consume(g, parts);
     CK(timed(c, PC_GEMM, gemm_bytes(M, m.qkv_width(), d, 4), [&] { return gemm(tc(c, g), c->st); }));
@@ -412,6 +437,9 @@ sd2_status forward(sd2_ctx* c, const Model& m, const Plan& p, const FwdOut& o) {
       }));
     GemmArgs gu = gu_args(l);
     if (fused) consume(gu, parts);
+    if (c->cfg.steering_site == 2 && o.bias) {   // per-row biases of the conditional MLP (below)
+      gu.bias = c->rowbias; gu.ld_bias = F; gu.row_seq = c->row_ident;
+    }
     CK(timed(c, PC_GEMM, gemm_bytes(M, 2 * F, d, 1), [&] { return gemm(tc(c, gu), c->st); }));
     GemmArgs gd = down_args(l);
     if (fused && l + 1 < L) {
@@ -440,6 +468,12 @@ sd2_status steer(sd2_ctx* c, const int* row_idx) {
   }));
   GemmArgs gs{};
   gs.x = c->g_bf; gs.ldx = dg; gs.M = B; gs.K = dg;
+  if (c->cfg.steering_site == 2) {        // the g half of the conditional bias MLP's first layer
+    const int ncg = c->D.c.n_layers * dg;
+    gs.seg[0] = {c->w_c1g, ncg}; gs.nseg = 1; gs.epi = EPI_STORE; gs.out = c->cg; gs.ldo = ncg;
+    CK(timed(c, PC_GEMM, gemm_bytes(B, ncg, dg, 4), [&] { return gemm(tc(c, gs), c->st); }));
+    return SD2_OK;
+  }
   gs.seg[0] = {c->w_s, nb}; gs.nseg = 1; gs.epi = EPI_STORE; gs.out = c->bias; gs.ldo = nb;
   CK(timed(c, PC_GEMM, gemm_bytes(B, nb, dg, 4), [&] { return gemm(tc(c, gs), c->st); }));
   return SD2_OK;
@@ -591,11 +625,13 @@ sd2_status sd2_init(const sd2_config* cfg, const sd2_weights* w, void* stream, s
   if (cfg->max_ctx < cfg->k + 3) return fail(nullptr, SD2_EINVAL, "max_ctx too small for one block");
   if (cfg->d_steer <= 0 || cfg->d_steer % 8) return fail(nullptr, SD2_EINVAL, "d_steer must be a positive multiple of 8");
   if (cfg->max_prefill_tokens < 1) return fail(nullptr, SD2_EINVAL, "max_prefill_tokens must be positive");
-  if (cfg->steering_site != 0 && cfg->steering_site != 1) return fail(nullptr, SD2_EINVAL, "steering_site must be 0 or 1");
+  if (cfg->steering_site < 0 || cfg->steering_site > 2) return fail(nullptr, SD2_EINVAL, "steering_site must be 0, 1 or 2");
   for (int t = 0; t < 3; ++t)
     if (cfg->tap_layers[t] < 1 || cfg->tap_layers[t] > cfg->verifier.n_layers)
       return fail(nullptr, SD2_EINVAL, "tap_layers must be 1-based verifier layers");
-  if (!cfg->no_steering && (!aligned16(w->w_hml) || !aligned16(w->w_s) || !w->steer_ln_gamma || !w->steer_ln_beta))
+  if (!cfg->no_steering && (!aligned16(w->w_hml) || !w->steer_ln_gamma || !w->steer_ln_beta ||
+                            (cfg->steering_site == 2 ? !aligned16(w->w_c1x) || !aligned16(w->w_c1g) || !aligned16(w->w_c2)
+                                                     : !aligned16(w->w_s))))
     return fail(nullptr, SD2_EINVAL, "steering weights null or not 16-byte aligned");
 
   c = new sd2_ctx();
@@ -603,6 +639,7 @@ sd2_status sd2_init(const sd2_config* cfg, const sd2_weights* w, void* stream, s
   c->st = static_cast<cudaStream_t>(stream);
   c->maxB = cfg->max_batch;
   c->w_hml = w->w_hml; c->ln_g = w->steer_ln_gamma; c->ln_b = w->steer_ln_beta; c->w_s = w->w_s;
+  c->w_c1x = w->w_c1x; c->w_c1g = w->w_c1g; c->w_c2 = w->w_c2;
   sd2_status s;
   if ((s = load_model(c, c->V, cfg->verifier, w->verifier, "verifier")) != SD2_OK ||
       (s = load_model(c, c->D, cfg->drafter, w->drafter, "drafter")) != SD2_OK) {
@@ -635,6 +672,17 @@ sd2_status sd2_init(const sd2_config* cfg, const sd2_weights* w, void* stream, s
     ALLOC(c->attn, static_cast<size_t>(R) * hmax * 2);
     ALLOC(c->h, static_cast<size_t>(R) * fmax * 2);
     ALLOC(c->ssq, static_cast<size_t>(R) * (dmax / 128 + 1) * 8);
+    if (cfg->steering_site == 2) {
+      const int Ld = cfg->drafter.n_layers, dd = cfg->drafter.d_model, dg = cfg->d_steer;
+      ALLOC(c->cg, static_cast<size_t>(maxB) * Ld * dg);
+      ALLOC(c->fb, static_cast<size_t>(R) * dd * 2);      // bf16 (void buffers are sized in bytes)
+      ALLOC(c->cu_h, static_cast<size_t>(R) * dg * 2);
+      ALLOC(c->rowbias, static_cast<size_t>(R) * cfg->drafter.d_ffn);
+      ALLOC(c->row_ident, R);
+      std::vector<int> ident(R);
+      for (int i = 0; i < R; ++i) ident[i] = i;
+      CK(cudaMemcpy(c->row_ident, ident.data(), sizeof(int) * R, cudaMemcpyHostToDevice));
+    }
     ALLOC(c->logits_t, static_cast<size_t>(maxB) * (k + 1) * Vv);
     ALLOC(c->logits_d, static_cast<size_t>(maxB) * k * Vv);
     ALLOC(c->taps, static_cast<size_t>(maxB) * (k + 1) * 3 * cfg->verifier.d_model);
@@ -1009,8 +1057,9 @@ sd2_status sd2_gemm(const void* d_x, int32_t ldx, int32_t M, int32_t K, const vo
   sd2_ctx* c = nullptr;
   if (!d_x || !d_w || M < 1 || K < 8 || K % 8 || ldx < K || ldx % 8 || N < 1)
     return fail(nullptr, SD2_EINVAL, "bad GEMM shape or null input");
-  if (epilogue < EPI_STORE || epilogue > EPI_SWIGLU) return fail(nullptr, SD2_EINVAL, "unknown epilogue");
-  if (epilogue == EPI_SWIGLU ? (!d_w_up || !d_h) : (!d_out || ldo < N))
+  if (epilogue < EPI_STORE || epilogue > EPI_SILU || epilogue == EPI_QKV)
+    return fail(nullptr, SD2_EINVAL, "unknown epilogue");
+  if (epilogue == EPI_SWIGLU ? (!d_w_up || !d_h) : epilogue == EPI_SILU ? !d_h : (!d_out || ldo < N))
     return fail(nullptr, SD2_EINVAL, "missing output for the epilogue");
   if (impl < 0 || impl > 2) return fail(nullptr, SD2_EINVAL, "impl must be 0, 1 or 2");
   GemmArgs g{};

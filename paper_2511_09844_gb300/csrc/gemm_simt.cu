@@ -98,6 +98,15 @@ __global__ void __launch_bounds__(kThreads) gemm_simt_kernel(const GemmArgs a, i
           }
           a.out[static_cast<size_t>(m) * a.ldo + n0] += v0;
           if (n1 >= 0) a.out[static_cast<size_t>(m) * a.ldo + n1] += v1;
+        } else if (EPI == EPI_SILU) {
+          bf16* hb = static_cast<bf16*>(a.out_bf) + static_cast<size_t>(m) * a.ldh;
+          const float* bs = a.bias ? a.bias + static_cast<size_t>(a.row_seq ? a.row_seq[m] : 0) * a.ld_bias : nullptr;
+          const float y0 = v0 + (bs ? bs[n0] : 0.f);
+          hb[n0] = __float2bfloat16_rn(y0 / (1.f + __expf(-y0)));
+          if (n1 >= 0) {
+            const float y1 = v1 + (bs ? bs[n1] : 0.f);
+            hb[n1] = __float2bfloat16_rn(y1 / (1.f + __expf(-y1)));
+          }
         } else {
           float up = v1;
           if (a.bias) {
@@ -142,6 +151,7 @@ cudaError_t gemm_simt(const GemmArgs& a, cudaStream_t st) {
     case EPI_QKV:
     case EPI_STORE: { const cudaError_t e_ = launch_pdl(gemm_simt_kernel<EPI_STORE>, dim3(blocks), dim3(kThreads), 0, st, a, n_units, n_total); if (e_ != cudaSuccess) return e_; } break;
     case EPI_ADD: { const cudaError_t e_ = launch_pdl(gemm_simt_kernel<EPI_ADD>, dim3(blocks), dim3(kThreads), 0, st, a, n_units, n_total); if (e_ != cudaSuccess) return e_; } break;
+    case EPI_SILU: { const cudaError_t e_ = launch_pdl(gemm_simt_kernel<EPI_SILU>, dim3(blocks), dim3(kThreads), 0, st, a, n_units, n_total); if (e_ != cudaSuccess) return e_; } break;
     default: { const cudaError_t e_ = launch_pdl(gemm_simt_kernel<EPI_SWIGLU>, dim3(blocks), dim3(kThreads), 0, st, a, n_units, n_total); if (e_ != cudaSuccess) return e_; } break;
   }
   return cudaGetLastError();

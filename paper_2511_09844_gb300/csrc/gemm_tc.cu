@@ -90,9 +90,15 @@ constexpr int kXS = 17;   // padded row of the epilogue exchange buffer (128 row
 __device__ __forceinline__ float add_bias_of(const TcArgs& a, int n, int m) {
   return a.bias ? a.bias[static_cast<size_t>(a.row_seq ? a.row_seq[m] : 0) * a.ld_bias + n] : 0.f;
 }
+__device__ __forceinline__ float silu_f(float y) { return y / (1.f + __expf(-y)); }
 __device__ __forceinline__ void emit_plain(const TcArgs& a, int wt, int row, int m, float v) {
-  float* o = a.out + static_cast<size_t>(m) * a.ldo + wt * kWRows + row;
-  if (a.epi == EPI_ADD) *o += v + add_bias_of(a, wt * kWRows + row, m);
+  const int n = wt * kWRows + row;
+  if (a.epi == EPI_SILU) {
+    a.out_bf[static_cast<size_t>(m) * a.ldh + n] = __float2bfloat16_rn(silu_f(v + add_bias_of(a, n, m)));
+    return;
+  }
+  float* o = a.out + static_cast<size_t>(m) * a.ldo + n;
+  if (a.epi == EPI_ADD) *o += v + add_bias_of(a, n, m);
   else *o = v;
 }
 // Eq. 2 for feature f of the tile (gate row f, up row f + 64).
@@ -259,6 +265,9 @@ __device__ __forceinline__ PairOps pair_ops(const TcArgs& a, int wt, int p, int 
       o.cs = reinterpret_cast<const float2*>(a.rope_cs)[static_cast<size_t>(o.pos) * half + i];
     if (head >= a.n_heads && a.row_valid[m])
       o.blk = a.kv_table[static_cast<size_t>(a.row_seq[m]) * a.kv_bt_stride + (o.pos >> 4)];
+  } else if (a.epi == EPI_SILU) {
+    o.bias = add_bias_of(a, wt * kWRows + pair_row(a, p, 0), m);
+    o.bias1 = add_bias_of(a, wt * kWRows + pair_row(a, p, 1), m);
   } else if (a.epi == EPI_ADD) {
     const float* x = a.out + static_cast<size_t>(m) * a.ldo + wt * kWRows;
     o.r0 = x[pair_row(a, p, 0)];
@@ -300,6 +309,10 @@ __device__ __forceinline__ float pair_emit(const TcArgs& a, int wt, int p, int m
       dst[i] = __float2bfloat16_rn(o0);
       dst[i + half] = __float2bfloat16_rn(o1);
     }
+  } else if (a.epi == EPI_SILU) {
+    bf16* hb = a.out_bf + static_cast<size_t>(m) * a.ldh + wt * kWRows;
+    hb[pair_row(a, p, 0)] = __float2bfloat16_rn(silu_f(s0 + o.bias));
+    hb[pair_row(a, p, 1)] = __float2bfloat16_rn(silu_f(s1 + o.bias1));
   } else {
     float* x = a.out + static_cast<size_t>(m) * a.ldo + wt * kWRows;
     const bool add = a.epi == EPI_ADD;

@@ -62,6 +62,7 @@ enum GemmEpilogue {
                     //   segments: seg0 = W_gate [F, K], seg1 = W_up [F, K]
   EPI_QKV = 3,      // segments W_q | W_k | W_v: rotary embedding on q and k, q -> q_out [M, H, hd] f32,
                     //   k and v of valid rows -> the paged KV cache of `layer` at (row_seq, row_pos)
+  EPI_SILU = 4,     // out_bf[m*ldh + n] = bf16(SiLU(y + bias[seq[m]*ld_bias + n])) (bias optional)
 };
 struct GemmSeg {
   const void* w;
@@ -127,6 +128,8 @@ bool encode_weight_map(void* map, const void* w, int rows, int K, int box_rows);
 int sm_count_cached();
 
 // ---------------------------------------------------------------- decoder elementwise
+// out[m, :w] = bf16(x[m * ld + 0 .. w-1]) for m < M.
+cudaError_t rows_to_bf16(const float* x, int ld, int M, int w, void* out, cudaStream_t st);
 // x[m] = embed[tok[m]] (f32), a[m] = bf16(RMSNorm(x[m]) * gamma); ids are clamped to [0, vocab).
 cudaError_t embed_rmsnorm(const int* tok, const void* embed, const void* gamma, float eps, int M, int d, int vocab,
                           float* x, void* a, cudaStream_t st);

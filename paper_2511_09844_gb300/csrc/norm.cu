@@ -75,6 +75,14 @@ __global__ void __launch_bounds__(kNormThreads) embed_scaled_kernel(const int* t
   if (threadIdx.x == 0) ssq[m] = ss;
 }
 
+__global__ void rows_to_bf16_kernel(const float* x, int ld, int w, bf16* out) {
+  pdl_trigger();
+  pdl_wait();
+  const int m = blockIdx.x;
+  for (int j = threadIdx.x; j < w; j += blockDim.x)
+    out[static_cast<size_t>(m) * w + j] = __float2bfloat16_rn(x[static_cast<size_t>(m) * ld + j]);
+}
+
 __global__ void __launch_bounds__(kNormThreads) rmsnorm_kernel(const float* x, const int* rows, const bf16* gamma,
                                                                 float eps, int d, bf16* a, float* tap,
                                                                 const int* tap_row, int tap_mask) {
@@ -204,6 +212,11 @@ cudaError_t embed_scaled(const int* tok, const void* embed, const void* gamma, i
   if (M <= 0) return cudaSuccess;
   return launch_pdl(embed_scaled_kernel, dim3(M), dim3(kNormThreads), 0, st, tok, static_cast<const bf16*>(embed),
                     static_cast<const bf16*>(gamma), d, vocab, x, static_cast<bf16*>(a), ssq);
+}
+
+cudaError_t rows_to_bf16(const float* x, int ld, int M, int w, void* out, cudaStream_t st) {
+  if (M <= 0) return cudaSuccess;
+  return launch_pdl(rows_to_bf16_kernel, dim3(M), dim3(256), 0, st, x, ld, w, static_cast<bf16*>(out));
 }
 
 cudaError_t rmsnorm(const float* x, const int* rows, const void* gamma, float eps, int M, int d, void* a, float* tap,

@@ -50,7 +50,8 @@ class LMWeights(ctypes.Structure):
 
 class Weights(ctypes.Structure):
     _fields_ = [("verifier", LMWeights), ("drafter", LMWeights), ("w_hml", c_void_p), ("steer_ln_gamma", c_void_p),
-                ("steer_ln_beta", c_void_p), ("w_s", c_void_p)]
+                ("steer_ln_beta", c_void_p), ("w_s", c_void_p), ("w_c1x", c_void_p), ("w_c1g", c_void_p),
+                ("w_c2", c_void_p)]
 
 
 _LIB = None
@@ -154,7 +155,7 @@ class SD2Engine:
         cfg.max_prefill_tokens = max_prefill_tokens
         cfg.kv_block = work.kv_block
         cfg.no_steering = 0 if steering else 1     # False: the pretrained drafter, no steering stage
-        cfg.steering_site = {"mlp_up": 0, "after_mlp": 1}[work.steering_site]
+        cfg.steering_site = {"mlp_up": 0, "after_mlp": 1, "cond_mlp": 2}[work.steering_site]
         self.cfg = cfg
         w = Weights()
         w.verifier = self._lm_weights(verifier_w)
@@ -163,7 +164,10 @@ class SD2Engine:
             w.w_hml = _ptr(steer_w["w_hml"])
             w.steer_ln_gamma = _ptr(steer_w["ln_gamma"])
             w.steer_ln_beta = _ptr(steer_w["ln_beta"])
-            w.w_s = _ptr(steer_w["w_s"])
+            w.w_s = _ptr(steer_w.get("w_s"))
+            w.w_c1x = _ptr(steer_w.get("w_c1x"))
+            w.w_c1g = _ptr(steer_w.get("w_c1g"))
+            w.w_c2 = _ptr(steer_w.get("w_c2"))
         self.stream = stream if stream is not None else torch.cuda.current_stream()
         ctx = c_void_p()
         _check(self.lib, self.lib.sd2_init(ctypes.byref(cfg), ctypes.byref(w), _stream(self.stream), ctypes.byref(ctx)))
@@ -307,16 +311,17 @@ def gemm(x: torch.Tensor, w: torch.Tensor, epilogue: int = 0, out: Optional[torc
          w_up: Optional[torch.Tensor] = None, bias: Optional[torch.Tensor] = None,
          seq: Optional[torch.Tensor] = None, impl: int = 0, stream=None):
     """Standalone weight-streaming GEMM (sd2_gemm). epilogue 0: returns X W^T (f32); 1: adds it into
-    `out`; 2: steered SwiGLU with w = W_gate, w_up = W_up, returns bf16 [M, N]."""
+    `out` (plus bias[seq] if given); 2: steered SwiGLU with w = W_gate, w_up = W_up, returns bf16
+    [M, N]; 4: returns bf16(SiLU(X W^T + bias[seq]))."""
     lib = load_library()
     M, K = x.shape
     N = w.shape[0]
     h = None
     if epilogue == 0 and out is None:
         out = torch.empty((M, N), dtype=torch.float32, device=x.device)
-    if epilogue == 2:
+    if epilogue in (2, 4):
         h = torch.empty((M, N), dtype=torch.bfloat16, device=x.device)
     _check(lib, lib.sd2_gemm(_ptr(x), x.stride(0), M, K, _ptr(w), _ptr(w_up), N, epilogue, _ptr(out),
                              0 if out is None else out.stride(0), _ptr(h), _ptr(bias), _ptr(seq),
                              0 if bias is None else bias.stride(0), impl, _stream(stream)))
-    return h if epilogue == 2 else out
+    return h if epilogue in (2, 4) else out

@@ -83,9 +83,11 @@ def run(work, vw, dw, st, prompts, temps, seed, n_steps, max_ctx=None, graphs=Tr
             rep.decisions += 1
         g0 = eng.buffer(sd2.BUF_G).view(B, -1)
         b0 = eng.buffer(sd2.BUF_BIAS).view(B, -1)
+        stage_biases = work.steering_site != "cond_mlp"    # cond: per-row biases, checked via the logits
         for b in range(B if steering else 0):
             rep.note("g", row_rel_err(g0[b], ora.gs[ora.seqs[b].cur_bias]))
-            rep.note("bias", row_rel_err(b0[b], ora.biases[ora.seqs[b].cur_bias].reshape(-1)))
+            if stage_biases:
+                rep.note("bias", row_rel_err(b0[b], ora.biases[ora.seqs[b].cur_bias].reshape(-1)))
         for step in range(1, n_steps + 1):
             state_before = eng.buffer(sd2.BUF_STATE).view(4, -1)[:, :B].cpu()
             eng.step()
@@ -107,7 +109,8 @@ def run(work, vw, dw, st, prompts, temps, seed, n_steps, max_ctx=None, graphs=Tr
                 assert int(state_before[0, b]) == len(s.tokens)
                 if steering:
                     rep.note("g", row_rel_err(gg[b], ora.gs[s.cur_bias]))
-                    rep.note("bias", row_rel_err(bb[b], ora.biases[s.cur_bias].reshape(-1)))
+                    if stage_biases:
+                        rep.note("bias", row_rel_err(bb[b], ora.biases[s.cur_bias].reshape(-1)))
                 xb = [int(x) for x in xh[b]]
                 out = ora.stage(b, step, forced_xhat=xb)
                 rep.note("draft_logits", row_rel_err(drf[b], out["draft"]))

@@ -95,6 +95,18 @@ def test_after_mlp_steering_site(gemm_impl):
     assert rep.blocks == 10
 
 
+@pytest.mark.parametrize("gemm_impl", [0, 1])
+def test_cond_bias_steering_site(gemm_impl):
+    """The "Cond. Bias in MLP" ablation (Sec. 5): per row and layer b = W_c2 SiLU(W_c1x f^(l-1) +
+    W_c1g g), added as in Eq. 2; parity with the oracle's same site."""
+    work = parity.tiny_work(steering_site="cond_mlp")
+    vw, dw, st = parity.tiny_weights(work, seed=12)
+    assert "w_s" not in st and st["w_c2"].shape[0] == work.drafter.n_layers * work.drafter.d_ffn
+    prompts = W.make_prompts(work.verifier.vocab, 2, (18, 30), seed=14)
+    rep = parity.run(work, vw, dw, st, prompts, [1.0, 0.0], seed=19, n_steps=5, gemm_impl=gemm_impl)
+    assert rep.blocks == 10
+
+
 def test_stage_timing_keeps_results():
     """Stage event nodes in the captured step change no output; the stage times are positive."""
     work = parity.tiny_work()

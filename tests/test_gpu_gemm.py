@@ -70,6 +70,21 @@ def test_residual_add_with_sequence_bias(impl, M, N, K):
 
 
 @pytest.mark.parametrize("impl", [1, 2])
+@pytest.mark.parametrize("M,N,K", [(3, 128, 256), (16, 2048, 2048), (150, 384, 512)])
+def test_silu_bias_epilogue(impl, M, N, K):
+    """Epilogue 4: bf16(SiLU(Y + bias[seq[m]])) (the conditional bias MLP's hidden layer)."""
+    x, w = _operands(M, N, K, 9 + M)
+    g = torch.Generator().manual_seed(10)
+    bias = torch.randn(2, N, generator=g)
+    seq = torch.randint(0, 2, (M,), generator=g).to(torch.int32)
+    h = sd2.gemm(x.cuda(), w.cuda(), epilogue=4, bias=bias.cuda(), seq=seq.cuda(), impl=impl)
+    torch.cuda.synchronize()
+    y = x.float() @ w.float().T + bias[seq.long()]
+    ref = omodel.silu(y)
+    assert parity.row_rel_err(h.float().cpu(), ref) < 1e-2   # bf16 output
+
+
+@pytest.mark.parametrize("impl", [1, 2])
 @pytest.mark.parametrize("M,F,K", [(6, 256, 512), (18, 192, 2048), (1, 64, 4864)])
 def test_steered_swiglu_epilogue(impl, M, F, K):
     g = torch.Generator().manual_seed(M + F)
