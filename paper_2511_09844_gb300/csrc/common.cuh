@@ -185,6 +185,12 @@ __device__ __forceinline__ uint32_t cluster_rank() {
 __device__ __forceinline__ void cluster_sync_all() {
   asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
+// The two halves of a cluster barrier: every thread of the cluster arrives once (relaxed: after
+// the mbarrier initialisation fence) and waits once, later.
+__device__ __forceinline__ void cluster_arrive_relaxed() {
+  asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_wait() { asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory"); }
 __device__ __forceinline__ uint32_t dsmem_addr(uint32_t saddr, uint32_t rank) {
   uint32_t remote;
   asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(saddr), "r"(rank));
@@ -210,6 +216,14 @@ __device__ __forceinline__ float4 ld_dsmem_v4(uint32_t saddr, uint32_t rank) {
 __device__ __forceinline__ void st_dsmem_v4(uint32_t saddr, uint32_t rank, float x, float y, float z, float w) {
   asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(dsmem_addr(saddr, rank)), "f"(x), "f"(y),
                "f"(z), "f"(w)
+               : "memory");
+}
+
+// four fp32 stored asynchronously to `raddr` (a shared::cluster address, 16-byte aligned); the
+// store's 16 bytes complete a transaction on the mbarrier at `rbar` (shared::cluster, same CTA)
+__device__ __forceinline__ void st_async_v4(uint32_t raddr, uint32_t rbar, float x, float y, float z, float w) {
+  asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.v4.f32 [%0], {%1, %2, %3, %4}, [%5];" ::"r"(raddr),
+               "f"(x), "f"(y), "f"(z), "f"(w), "r"(rbar)
                : "memory");
 }
 

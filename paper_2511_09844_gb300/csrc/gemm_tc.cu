@@ -340,16 +340,17 @@ __global__ void __launch_bounds__(kThreads, 2) gemm_tc_kernel(const __grid_const
   const uint32_t recv_bytes = sp > 1 ? static_cast<uint32_t>(sp * npmax * 2 * NT * 4) : 0u;
   float* recv = reinterpret_cast<float*>(smem + static_cast<size_t>(S) * stage_bytes);  // split-K partials in
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + static_cast<size_t>(S) * stage_bytes + recv_bytes);
-  // bars: full[S], empty[S], tfull[2], tempty[2], drain
+  // bars: full[S], empty[S], tfull[2], tempty[2], drain, recv (split-K partials of this rank's pairs)
   float* xbuf = reinterpret_cast<float*>(bars + 2 * S + 6);
   volatile int* flags = reinterpret_cast<volatile int*>(xbuf + kWRows * kXS);
-  // flags: [0] abort, [1] TMEM base, [3] stages consumed, [4] go
+  // flags: [0] abort, [1] TMEM base, [3] stages consumed, [4] go, [5] partials received
   float* rs = const_cast<float*>(reinterpret_cast<volatile float*>(flags + 16));   // [kMaxNT] fused-norm scales
   const uint32_t full0 = smem_u32(bars), empty0 = full0 + 8 * S, tfull0 = empty0 + 8 * S, tempty0 = tfull0 + 16,
-                 drain = tempty0 + 16;
+                 drain = tempty0 + 16, rbar = drain + 8;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   uint32_t ncols = 32;
   while (ncols < static_cast<uint32_t>((sp == 1 ? 2 : 1) * NT)) ncols <<= 1;
+  const int rank = sp > 1 ? static_cast<int>(cluster_rank()) : 0;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
@@ -361,7 +362,16 @@ __global__ void __launch_bounds__(kThreads, 2) gemm_tc_kernel(const __grid_const
     mbar_init(tempty0, 4);
     mbar_init(tempty0 + 8, 4);
     mbar_init(drain, 1);
-    flags[0] = 0; flags[3] = 0; flags[4] = 0;
+    if (sp > 1) {
+      // Split-K: every rank pushes its partial of each row to the rank owning the row's pair;
+      // the owner's receive barrier completes when all sp partials of its pairs have landed:
+      // sp x (2 rows x its pairs) x 64 bytes per 16 token columns.
+      const int np = (rank + 1) * 64 / sp - rank * 64 / sp;
+      const int cols = min(NT, a.M - (static_cast<int>(blockIdx.x) / sp / a.n_wtiles) * NT);
+      mbar_init(rbar, 1);
+      mbar_expect_tx(rbar, static_cast<uint32_t>(sp * 2 * np * ((cols + 15) / 16) * 64));
+    }
+    flags[0] = 0; flags[3] = 0; flags[4] = 0; flags[5] = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   if (warp == 1) {
@@ -371,12 +381,12 @@ __global__ void __launch_bounds__(kThreads, 2) gemm_tc_kernel(const __grid_const
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  if (sp > 1) cluster_arrive_relaxed();      // waited for before the first push into another rank
   const uint32_t tmem = static_cast<uint32_t>(flags[1]);
   volatile int* abort_flag = flags;
 
   // This CTA's segments: sp > 1 -> one K-slice of tile blockIdx.x / sp; sp == 1 -> whole tiles
   // blockIdx.x, blockIdx.x + gridDim.x, ...
-  const int rank = sp > 1 ? static_cast<int>(cluster_rank()) : 0;
   const int first_tile = sp > 1 ? static_cast<int>(blockIdx.x) / sp : static_cast<int>(blockIdx.x);
   const int tile_step = sp > 1 ? a.tiles : static_cast<int>(gridDim.x);
   const int kb_lo = rank * a.KB / sp, kb_hi = (rank + 1) * a.KB / sp;
@@ -477,17 +487,76 @@ __global__ void __launch_bounds__(kThreads, 2) gemm_tc_kernel(const __grid_const
       mma_commit(drain);                      // all MMAs issued by this thread have completed
       wait_bar_budget(drain, 0, kDrainCycles);
     }
+  } else if (sp > 1) {
+    // Split-K epilogue of the CTA's single tile. Everything but the sums (this thread's
+    // destination in the owner's receive buffer, the operands of its first owned output, the
+    // RMSNorm scales) is prepared while the MMAs run.
+    const int q = warp & 3, r = q * 32 + lane, tid = threadIdx.x - 64;
+    const bool leader = (warp == 2 && lane == 0);
+    pdl_wait();                              // outputs, residuals and biases come from earlier kernels
+    const int wt = first_tile % a.n_wtiles, tt = first_tile / a.n_wtiles;
+    const int cols = min(NT, a.M - tt * NT);
+    const int p_lo = rank * 64 / sp, np = (rank + 1) * 64 / sp - p_lo;
+    if (tid < np * cols) pf = pair_ops(a, wt, p_lo + tid % np, tt * NT + tid / np);
+    const int p = pair_of(a, r), owner = pair_owner(p, sp);
+    const int slot = ((rank * npmax + p - owner * 64 / sp) * 2 + member_of(a, r)) * NT;
+    const uint32_t dst = dsmem_addr(smem_u32(recv + slot), static_cast<uint32_t>(owner));
+    const uint32_t dst_bar = dsmem_addr(rbar, static_cast<uint32_t>(owner));
+    if (a.norm_ssq_in) tile_rstd(a, tt, rs, tid);
+    if (leader) flags[4] = wait_bar(tfull0, 0, abort_flag, a.err) ? 1 : 0;
+    named_bar_epi();                         // the accumulator is complete (or the wait gave up); rs is set
+    tc_fence_after();
+    cluster_wait();                          // every rank's receive barrier is armed
+    if (flags[4] != 0) {
+      const uint32_t tbase = tmem + (static_cast<uint32_t>(q * 32) << 16);
+      for (int ch = 0; ch * 16 < cols; ++ch) {
+        float v[16];
+        tmem_ld16(tbase + ch * 16, v);
+#pragma unroll
+        for (int k4 = 0; k4 < 4; ++k4)
+          st_async_v4(dst + static_cast<uint32_t>((ch * 16 + 4 * k4) * 4), dst_bar, v[4 * k4], v[4 * k4 + 1],
+                      v[4 * k4 + 2], v[4 * k4 + 3]);
+      }
+      if (leader) flags[5] = wait_bar(rbar, 0, abort_flag, a.err) ? 1 : 0;
+      named_bar_epi();
+      if (flags[5] != 0) {
+        // every rank's partial of this rank's pairs is in the receive buffer: sums in rank order
+        float* sq = reinterpret_cast<float*>(smem);   // [cols][np] fused-norm sums of squares (drained ring)
+        for (int e = tid; e < np * cols; e += 128) {
+          const int lp = e % np, col = e / np;
+          const float* rv = recv + lp * 2 * NT + col;
+          float s0 = 0.f, s1 = 0.f;
+#pragma unroll
+          for (int k = 0; k < 8; ++k)
+            if (k < sp) {
+              s0 += rv[k * npmax * 2 * NT];
+              s1 += rv[k * npmax * 2 * NT + NT];
+            }
+          if (a.norm_ssq_in) {
+            s0 *= rs[col];
+            s1 *= rs[col];
+          }
+          const int m = tt * NT + col;
+          const float q2 = pair_emit(a, wt, p_lo + lp, m, s0, s1, e == tid ? pf : pair_ops(a, wt, p_lo + lp, m));
+          if (a.norm_out) sq[col * np + lp] = q2;
+        }
+        if (a.norm_out) {   // this rank's slice of the tile: sums of squares per token, in pair order
+          named_bar_epi();
+          for (int c = tid; c < cols; c += 128) {
+            float ssum = 0.f;
+            for (int lp = 0; lp < np; ++lp) ssum += sq[c * np + lp];
+            a.norm_ssq_out[static_cast<size_t>(wt * sp + rank) * a.ld_ssq + tt * NT + c] = ssum;
+          }
+        }
+      } else if (leader) {
+        wait_bar_budget(rbar, 0, kDrainCycles);   // let partials still in flight land before leaving
+      }
+    }
   } else {
     const int q = warp & 3;                   // TMEM lane quarter of this warp
     const int r = q * 32 + lane;              // weight row within the tile
     const bool leader = (warp == 2 && lane == 0);
     pdl_wait();                              // outputs, residuals and biases come from earlier kernels
-    if (sp > 1) {                            // fetched while the main loop runs
-      const int wt = first_tile % a.n_wtiles, tt = first_tile / a.n_wtiles;
-      const int np = (rank + 1) * 64 / sp - rank * 64 / sp;
-      const int tid = threadIdx.x - 64;
-      if (tid < np * min(NT, a.M - tt * NT)) pf = pair_ops(a, wt, rank * 64 / sp + tid % np, tt * NT + tid / np);
-    }
     uint32_t segi = 0;
     int rs_tt = -1;
     for (int t = first_tile; t < a.tiles; t += tile_step, ++segi) {
@@ -504,30 +573,11 @@ __global__ void __launch_bounds__(kThreads, 2) gemm_tc_kernel(const __grid_const
       tc_fence_after();
       if (!go) break;
       const uint32_t tbase = tmem + (static_cast<uint32_t>(q * 32) << 16) + acc * NT;
-      const int nchunk = NT / 16;
       const int cols = min(NT, a.M - tt * NT);   // token columns of this tile that exist
-      if (sp == 1) {
-        for (int ch = 0; ch < nchunk; ++ch) {
-          if (ch * 16 >= cols) break;
-          float v[16];
-          tmem_ld16(tbase + ch * 16, v);
-          finish_chunk(a, wt, tt, r, ch * 16, v, xbuf, rs);
-        }
-      } else {
-        // this CTA's K-slice partial of row r -> the receive buffer of the rank owning its pair
-        const int p = pair_of(a, r), mem = member_of(a, r);
-        const int owner = pair_owner(p, sp);
-        const int lp = p - owner * 64 / sp;
-        const uint32_t dst = smem_u32(recv) + static_cast<uint32_t>((((rank * npmax + lp) * 2 + mem) * NT) * 4);
-        for (int ch = 0; ch < nchunk; ++ch) {
-          if (ch * 16 >= cols) break;
-          float v[16];
-          tmem_ld16(tbase + ch * 16, v);
-#pragma unroll
-          for (int k4 = 0; k4 < 4; ++k4)
-            st_dsmem_v4(dst + static_cast<uint32_t>((ch * 16 + 4 * k4) * 4), static_cast<uint32_t>(owner), v[4 * k4],
-                        v[4 * k4 + 1], v[4 * k4 + 2], v[4 * k4 + 3]);
-        }
+      for (int ch = 0; ch * 16 < cols; ++ch) {
+        float v[16];
+        tmem_ld16(tbase + ch * 16, v);
+        finish_chunk(a, wt, tt, r, ch * 16, v, xbuf, rs);
       }
       tc_fence_before();
       __syncwarp();
@@ -535,46 +585,10 @@ __global__ void __launch_bounds__(kThreads, 2) gemm_tc_kernel(const __grid_const
     }
   }
 
-  if (sp > 1) {
-    // Split-K reduction: after the barrier every partial of this rank's pairs is in its own
-    // receive buffer; sum them in rank order and run the epilogue. Nothing remote is read, so no
-    // second barrier is needed before the CTA leaves.
+  if (sp > 1 && warp < 2) {                  // the producer and MMA warps take their half of the cluster barrier
     __syncwarp();
-    cluster_sync_all();
-    if (warp >= 2 && flags[0] == 0) {
-      const int tid = threadIdx.x - 64;
-      const int t = first_tile;
-      const int wt = t % a.n_wtiles, tt = t / a.n_wtiles;
-      const int cols = min(NT, a.M - tt * NT);
-      const int p_lo = rank * 64 / sp, np = (rank + 1) * 64 / sp - p_lo;
-      float* sq = reinterpret_cast<float*>(smem);   // [cols][np] fused-norm sums of squares (drained ring)
-      for (int e = tid; e < np * cols; e += 128) {
-        const int lp = e % np, col = e / np;
-        const float* rv = recv + lp * 2 * NT + col;
-        float s0 = 0.f, s1 = 0.f;
-        for (int q = 0; q < sp; ++q) {
-          s0 += rv[q * npmax * 2 * NT];
-          s1 += rv[q * npmax * 2 * NT + NT];
-        }
-        if (a.norm_ssq_in) {
-          s0 *= rs[col];
-          s1 *= rs[col];
-        }
-        const int p = p_lo + lp, m = tt * NT + col;
-        const float q2 = pair_emit(a, wt, p, m, s0, s1, e == tid ? pf : pair_ops(a, wt, p, m));
-        if (a.norm_out) sq[col * np + lp] = q2;
-      }
-      if (a.norm_out) {   // this rank's slice of the tile: sums of squares per token, in pair order
-        named_bar_epi();
-        for (int c = tid; c < cols; c += 128) {
-          float ssum = 0.f;
-          for (int lp = 0; lp < np; ++lp) ssum += sq[c * np + lp];
-          a.norm_ssq_out[static_cast<size_t>(wt * sp + rank) * a.ld_ssq + tt * NT + c] = ssum;
-        }
-      }
-    }
+    cluster_wait();
   }
-
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
