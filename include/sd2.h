@@ -135,8 +135,9 @@ sd2_status sd2_step(sd2_ctx* ctx);
  * Errors: SD2_ESTATE (no step to accept). */
 sd2_status sd2_accept(sd2_ctx* ctx, int32_t* d_tokens, int32_t* d_n_emitted);
 
-/* Wait for the context's stream and report the device error word (SD2_OK, SD2_ENUMERIC or
- * SD2_ETIMEOUT), clearing it. */
+/* Wait for the context's stream and report the device error word (SD2_OK, SD2_ENUMERIC,
+ * SD2_ETIMEOUT, or SD2_ECAPACITY when an attention row of a step lay beyond the cache positions
+ * that step was planned to write), clearing it. */
 sd2_status sd2_check(sd2_ctx* ctx);
 
 /* Release everything the context owns (waits for its stream first). Null is allowed. */

@@ -7,20 +7,27 @@
 //   scores S = Q K^T      warp w owns positions 8w .. 8w+7 of the tile, every query tile
 //   online softmax        4 threads per query row: running max/sum, P = e^{S - m} in bf16
 //   O = O * corr + P V    warp w owns 8 (hd 64) or 16 (hd 128) output dimensions
-// The contractions are tiny (M <= 64); the kernel is bound by the latency of its loads. The block
-// ids of the split are read before the programmatic wait (they are fixed before the step starts),
-// the row positions and queries are fetched together after it, and K/V tiles are staged with
-// cp.async (zero-filled past the last position), two tiles in flight. Every K/V byte of the split
-// is read from HBM once per CTA.
+// The contractions are tiny (M <= 64); the kernel is bound by the latency of its loads, so they
+// are ordered by when their data is final. The block ids of the split are read before the
+// programmatic wait (they are fixed before the step starts). In a decode step the cache positions
+// below the sequence's pre-step length were also written before the step: their K/V rows are
+// requested before the wait, and the few rows the step itself may have written are requested
+// right after it, together with the queries and row positions. K/V tiles are staged with
+// cp.async (zero-filled where no row exists), two tiles in flight; every K/V byte of the split is
+// read from HBM once per CTA.
 //
-// The splits of one (row group, KV head) form a thread-block cluster (at most 8). Each CTA leaves
-// its partial (accumulator, max, sum) in shared memory; after a cluster barrier, rank r merges
-// the r-th share of the group's outputs, reading every split's partial through distributed shared
-// memory, so no partial goes through global memory and the merge is spread over the cluster.
+// The splits of one (row group, KV head) form a thread-block cluster. Split merge: the (query
+// vector, 4 dimensions) elements of the group are shared out over the splits; every split pushes
+// its running max and sum of each query vector to every split, and each accumulator pair to the
+// split owning its element, with asynchronous stores that complete on the owner's receive
+// mbarrier. The owner waits only for its own share, merges it and writes the output; no partial
+// goes through global memory and no cluster barrier is held while the partials travel.
+#include <limits.h>
 #include <math.h>
 
 #include "common.cuh"
 #include "kernels.h"
+#include "tc.cuh"
 
 namespace sd2 {
 namespace {
@@ -37,9 +44,7 @@ struct AttnCfg {
   static constexpr int KS = HD + 8;                     // Q/K/V row stride, bf16 (conflict-free fragments)
   static constexpr int SS = kTile + 8;                  // score row stride, f32
   static constexpr int PS = kTile + 8;                  // probability row stride, bf16
-  static constexpr int REC = HD + 4;                    // partial accumulator row, f32
-  // per query vector: position, correction, max, sum; per (query vector, split): max, sum / weight
-  static constexpr int ROW_BYTES = 4 * kMaxQV * 4 + 2 * kMaxQV * kMaxSplits * 4;
+  static constexpr int ROW_BYTES = 4 * kMaxQV * 4;      // per query vector: position, correction, max, sum
   static constexpr int KV_TILE = 2 * kTile * KS * 2;    // K and V of one tile
   __host__ __device__ static int qrows(int max_rows, int G) {
     const int r = ((max_rows * G + 15) / 16) * 16;
@@ -53,11 +58,19 @@ struct AttnCfg {
   __host__ __device__ static size_t blk_off(int qr, int chunk) {
     return kv_off(qr) + static_cast<size_t>(nbuf(chunk)) * KV_TILE;
   }
-  static size_t bytes(int qr, int chunk) {
+  // split merge (ns > 1): receive barrier; every split's (max, sum) per query vector [ns][qr];
+  // every split's accumulators of this rank's share of elements [ns][share] (float4 each)
+  __host__ __device__ static int share(int qr, int ns) { return (qr * (HD / 4) + ns - 1) / ns; }
+  __host__ __device__ static size_t rcv_off(int qr, int chunk) {
     return blk_off(qr, chunk) + ((static_cast<size_t>(chunk / 16) * 4 + 15) & ~static_cast<size_t>(15));
   }
-  // the partial accumulators [qr][REC] overlay Q, S and P once the tiles are done
-  static_assert(2 * KS + SS * 4 + PS * 2 >= REC * 4, "partials fit over the tile working set");
+  __host__ __device__ static size_t ml_off(int qr, int chunk) { return rcv_off(qr, chunk) + 16; }
+  __host__ __device__ static size_t acc_off(int qr, int chunk, int ns) {
+    return ml_off(qr, chunk) + static_cast<size_t>(ns) * qr * 8;
+  }
+  static size_t bytes(int qr, int chunk, int ns) {
+    return ns > 1 ? acc_off(qr, chunk, ns) + static_cast<size_t>(ns) * share(qr, ns) * 16 : rcv_off(qr, chunk);
+  }
 };
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
@@ -75,6 +88,13 @@ __device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, bool v
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
 template <int N>
 __device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
+// two fp32 stored asynchronously to `raddr` (shared::cluster, 8-byte aligned), completing 8 bytes
+// of a transaction on the mbarrier at `rbar` (shared::cluster, same CTA)
+__device__ __forceinline__ void st_async_v2(uint32_t raddr, uint32_t rbar, float x, float y) {
+  asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.v2.f32 [%0], {%1, %2}, [%3];" ::"r"(raddr),
+               "f"(x), "f"(y), "r"(rbar)
+               : "memory");
+}
 
 // D(16x8, f32) += A(16x16, bf16, row-major) * B(16x8, bf16, column-major)
 __device__ __forceinline__ void mma_bf16(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
@@ -100,11 +120,12 @@ __device__ __forceinline__ void ldsm_x2_t(uint32_t addr, uint32_t& r0, uint32_t&
 template <int HD>
 __global__ void __launch_bounds__(kThreads, 2) attn_kernel(const AttnArgs a) {
   using C = AttnCfg<HD>;
-  constexpr int KS = C::KS, SS = C::SS, PS = C::PS, REC = C::REC;
+  constexpr int KS = C::KS, SS = C::SS, PS = C::PS;
   constexpr int NT = HD / 64;  // n8 tiles of output dimensions per warp
   pdl_trigger();
   extern __shared__ __align__(16) unsigned char smem[];
   __shared__ int sPmax[2];
+  __shared__ int sRecv;
 
   const int split = blockIdx.x, g = blockIdx.y, kvh = blockIdx.z;
   const int NS = a.n_splits;
@@ -114,27 +135,76 @@ __global__ void __launch_bounds__(kThreads, 2) attn_kernel(const AttnArgs a) {
   const int QR = C::qrows(a.max_rows, G);
   int* sPos = reinterpret_cast<int*>(smem);
   float* sCorr = reinterpret_cast<float*>(smem) + kMaxQV;
-  float* sM = sCorr + kMaxQV;
-  float* sL = sM + kMaxQV;
-  float* sWm = sL + kMaxQV;                 // [kMaxQV][kMaxSplits] split maxima, then weights
-  float* sWl = sWm + kMaxQV * kMaxSplits;   // [kMaxQV][kMaxSplits] split sums
+  float* sL = sCorr + 2 * kMaxQV;
   bf16* sQ = reinterpret_cast<bf16*>(smem + C::q_off());
   float* sS = reinterpret_cast<float*>(smem + C::s_off(QR));
   bf16* sP = reinterpret_cast<bf16*>(smem + C::p_off(QR));
   unsigned char* sKV = smem + C::kv_off(QR);
   int* sBlk = reinterpret_cast<int*>(smem + C::blk_off(QR, a.chunk));
+  const uint32_t rbar = smem_u32(smem + C::rcv_off(QR, a.chunk));
+  const float2* rML = reinterpret_cast<const float2*>(smem + C::ml_off(QR, a.chunk));
+  const float4* rAcc = reinterpret_cast<const float4*>(smem + C::acc_off(QR, a.chunk, NS));
+  const int share = C::share(QR, NS);
 
-  // The plan tables and the block table are written before the step's first kernel, so they are
-  // read before the wait; everything the preceding kernels write is read after it.
+  // Before the wait: the plan tables and the block table (written before the step's first
+  // kernel) and, in a decode step, the sequence's pre-step length.
   const int r0 = a.grp_row0[g], nr = a.grp_nrows[g], seq = a.grp_seq[g];
   const int nqv = nr * G;
   const int lo = split * a.chunk;
+  const int nblk = min(a.chunk >> 4, a.kv.bt_stride - (lo >> 4));
+  const int row_end = lo + nblk * 16;               // positions the split's block ids cover
   {
     const int* table = a.kv.table + static_cast<size_t>(seq) * a.kv.bt_stride + (lo >> 4);
-    const int nblk = min(a.chunk >> 4, a.kv.bt_stride - (lo >> 4));
     for (int i = tid; i < nblk; i += kThreads) sBlk[i] = table[i];
   }
+  const bool early = a.pre_len != nullptr;
+  int pre_hi = lo, fresh_hi = lo;                   // rows [lo, pre_hi) early, [pre_hi, fresh_hi) after the wait
+  if (early) {
+    const int len = a.pre_len[seq];
+    pre_hi = min(max(lo, len + a.pre_stable), row_end);
+    fresh_hi = min(max(pre_hi, len + a.pre_stable + a.pre_fresh), row_end);
+  }
+  const int E4 = nqv * (HD / 4);                    // merge elements: (query vector, 4 dimensions)
+  const int e_lo = split * E4 / NS, e_hi = (split + 1) * E4 / NS;
+  if (NS > 1 && tid == 0) {
+    tc::mbar_init(rbar, 1);
+    tc::mbar_expect_tx(rbar, static_cast<uint32_t>(NS * ((e_hi - e_lo) * 16 + nqv * 8)));
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  __syncthreads();                                  // block ids and the receive barrier
+  if (NS > 1) cluster_arrive_relaxed();             // waited for before the first push
+
+  const bf16* pool = static_cast<const bf16*>(a.kv.pool);
+  const size_t head_stride = static_cast<size_t>(16) * HD;
+  const size_t blk_stride = static_cast<size_t>(2) * Hkv * head_stride;
+  const bf16* layer_base = pool + static_cast<size_t>(a.layer) * a.kv.n_blocks * blk_stride + kvh * head_stride;
+  // rows p in [p_from, p_to) of tile i (positions lo + 64 i ..) -> buffer i & 1: loaded below
+  // `valid_end`, zero-filled from it on
+  auto issue_rows = [&](int i, int p_from, int p_to, int valid_end) {
+    bf16* dK = reinterpret_cast<bf16*>(sKV + (i & 1) * C::KV_TILE);
+    bf16* dV = dK + kTile * KS;
+    const int t0 = lo + i * kTile;
+#pragma unroll
+    for (int u = 0; u < kTile * (HD / 8) / kThreads; ++u) {
+      const int idx = tid + u * kThreads, t = idx / (HD / 8), c = idx % (HD / 8);
+      const int p = t0 + t;
+      if (p < p_from || p >= p_to) continue;
+      const bool ok = p < valid_end;
+      const bf16* src = layer_base;
+      if (ok) src += static_cast<size_t>(sBlk[(p - lo) >> 4]) * blk_stride + static_cast<size_t>(p & 15) * HD + c * 8;
+      cp_async16(smem_u32(dK + t * KS + c * 8), src, ok);
+      cp_async16(smem_u32(dV + t * KS + c * 8), ok ? src + Hkv * head_stride : layer_base, ok);
+    }
+  };
+  const int nb = C::nbuf(a.chunk);
+  if (early)
+    for (int i = 0; i < nb; ++i) issue_rows(i, lo, pre_hi, pre_hi);
   pdl_wait();
+  if (early)   // the rows this step may have written, beside the queries
+    for (int i = 0; i < nb; ++i) {
+      issue_rows(i, pre_hi, INT_MAX, fresh_hi);
+      cp_async_commit();
+    }
   int pq = -1;
   if (tid < nqv) pq = __ldcg(a.row_pos + r0 + tid / G);
   constexpr int QC = HD / 4;                        // float4 per query vector
@@ -161,32 +231,17 @@ __global__ void __launch_bounds__(kThreads, 2) attn_kernel(const AttnArgs a) {
   __syncthreads();
   const int pmax = max(sPmax[0], sPmax[1]);
   // A split that starts after every row of the group has no tiles; it still takes part in the
-  // cluster's merge with an empty partial.
+  // merge with an empty partial.
   const int hi = min(lo + a.chunk, pmax + 1);
   const int ntiles = hi > lo ? (hi - lo + kTile - 1) / kTile : 0;
   const int nmt = (nqv + 15) >> 4;
-
-  const bf16* pool = static_cast<const bf16*>(a.kv.pool);
-  const size_t head_stride = static_cast<size_t>(16) * HD;
-  const size_t blk_stride = static_cast<size_t>(2) * Hkv * head_stride;
-  const bf16* layer_base = pool + static_cast<size_t>(a.layer) * a.kv.n_blocks * blk_stride + kvh * head_stride;
-  // positions t0 .. t0+63 of tile i -> buffer i & 1 (zero-filled at and beyond hi)
-  auto issue_tile = [&](int i) {
-    bf16* dK = reinterpret_cast<bf16*>(sKV + (i & 1) * C::KV_TILE);
-    bf16* dV = dK + kTile * KS;
-    const int t0 = lo + i * kTile;
-#pragma unroll
-    for (int u = 0; u < kTile * (HD / 8) / kThreads; ++u) {
-      const int idx = tid + u * kThreads, t = idx / (HD / 8), c = idx % (HD / 8);
-      const int p = t0 + t;
-      const bool ok = p < hi;
-      const bf16* src = layer_base;
-      if (ok) src += static_cast<size_t>(sBlk[(p - lo) >> 4]) * blk_stride + static_cast<size_t>(p & 15) * HD + c * 8;
-      cp_async16(smem_u32(dK + t * KS + c * 8), src, ok);
-      cp_async16(smem_u32(dV + t * KS + c * 8), ok ? src + Hkv * head_stride : layer_base, ok);
-    }
-    cp_async_commit();
-  };
+  if (early) {
+    // every row the queries can see in the early tiles must have been loaded
+    if (tid == 0 && min(hi, lo + nb * kTile) > fresh_hi && a.err) atomicOr(a.err, static_cast<unsigned>(ERR_RANGE));
+  } else {
+    if (ntiles > 0) { issue_rows(0, lo, INT_MAX, hi); cp_async_commit(); }
+    if (ntiles > 1) { issue_rows(1, lo, INT_MAX, hi); cp_async_commit(); }
+  }
 
   const float scale = rsqrtf(static_cast<float>(HD));
   const int srow = tid >> 2, squart = tid & 3;  // softmax: query row, quarter of the tile
@@ -200,13 +255,11 @@ __global__ void __launch_bounds__(kThreads, 2) attn_kernel(const AttnArgs a) {
       for (int e = 0; e < 4; ++e) acc[mt][nt][e] = 0.f;
 
   // two tiles in flight: tiles 0 and 1 now, tile i+1 at the top of iteration i >= 1
-  if (ntiles > 0) issue_tile(0);
-  if (ntiles > 1) issue_tile(1);
   for (int i = 0; i < ntiles; ++i) {
     if (i == 0 && ntiles > 1) cp_async_wait<1>();
     else cp_async_wait<0>();
     __syncthreads();  // tile i visible to all; every warp is past tile i-1, so its buffer is free
-    if (i >= 1 && i + 1 < ntiles) issue_tile(i + 1);
+    if (i >= 1 && i + 1 < ntiles) { issue_rows(i + 1, lo, INT_MAX, hi); cp_async_commit(); }
     const int t0 = lo + i * kTile;
     const bf16* sK = reinterpret_cast<const bf16*>(sKV + (i & 1) * C::KV_TILE);
     const bf16* sV = sK + kTile * KS;
@@ -314,11 +367,12 @@ __global__ void __launch_bounds__(kThreads, 2) attn_kernel(const AttnArgs a) {
       }
     }
   }
+  cp_async_wait<0>();  // early tiles the row positions turned out not to need
 
-  if (srow < nmt * 16 && squart == 0) { sM[srow] = m_run; sL[srow] = l_run; }
-  __syncthreads();  // also: every warp is done with the tile working set that the partials overlay
   const int d0 = warp * 8 * NT;
   if (NS == 1) {
+    if (srow < nmt * 16 && squart == 0) sL[srow] = l_run;
+    __syncthreads();
 #pragma unroll
     for (int mt = 0; mt < 4; ++mt) {
       if (mt >= nmt) break;
@@ -337,73 +391,73 @@ __global__ void __launch_bounds__(kThreads, 2) attn_kernel(const AttnArgs a) {
     return;
   }
 
-  // Split merge across the cluster (rank = split): out = sum_s acc_s e^{m_s - M} / sum_s l_s e^{m_s - M}.
-  // Each CTA publishes its partial in shared memory; rank r then finishes the r-th share of the
-  // group's (query vector, 4 dimensions) elements, reading the partials of every split.
-  float* sAcc = reinterpret_cast<float*>(smem + C::q_off());  // [QR][REC]
+  // Split merge: out = sum_s acc_s e^{m_s - M} / sum_s l_s e^{m_s - M}, M = max_s m_s. Element e
+  // of the group (query vector e / (hd/4), dimensions 4 (e % (hd/4)) ..) belongs to the split r
+  // with r E4 / NS <= e < (r+1) E4 / NS. Splits that hold no position a row can see contribute
+  // m = -inf, l = 0, acc = 0, hence weight 0.
+  cluster_wait();                                   // every split's receive barrier is armed
+  if (srow < nqv && squart == 0) {                  // (max, sum) of the query vector to every split
+    const uint32_t src = smem_u32(rML + split * QR + srow);
+    for (int s2 = 0; s2 < NS; ++s2)
+      st_async_v2(dsmem_addr(src, static_cast<uint32_t>(s2)), dsmem_addr(rbar, static_cast<uint32_t>(s2)), m_run,
+                  l_run);
+  }
 #pragma unroll
   for (int mt = 0; mt < 4; ++mt) {
     if (mt >= nmt) break;
 #pragma unroll
     for (int half = 0; half < 2; ++half) {
       const int qv = mt * 16 + g8 + 8 * half;
+      if (qv >= nqv) continue;
 #pragma unroll
-      for (int nt = 0; nt < NT; ++nt)
-        *reinterpret_cast<float2*>(sAcc + qv * REC + d0 + nt * 8 + 2 * t4) =
-            make_float2(acc[mt][nt][2 * half], acc[mt][nt][2 * half + 1]);
+      for (int nt = 0; nt < NT; ++nt) {
+        const int d = d0 + nt * 8 + 2 * t4;
+        const int e = qv * (HD / 4) + (d >> 2);
+        const int owner = ((e + 1) * NS - 1) / E4;
+        const uint32_t dst = smem_u32(rAcc + split * share + (e - owner * E4 / NS)) + static_cast<uint32_t>((d & 3) * 4);
+        st_async_v2(dsmem_addr(dst, static_cast<uint32_t>(owner)), dsmem_addr(rbar, static_cast<uint32_t>(owner)),
+                    acc[mt][nt][2 * half], acc[mt][nt][2 * half + 1]);
+      }
     }
   }
-  cluster_sync_all();  // every split's partial is in its shared memory
-  for (int t = tid; t < nqv * NS; t += kThreads) {
-    const int qv = t / NS, s2 = t % NS;
-    const int ns = min(NS, sPos[qv] / a.chunk + 1);  // splits that start at or before this row
-    float m = -INFINITY, l = 0.f;
-    if (s2 < ns) {
-      m = ld_dsmem(smem_u32(sM + qv), s2);
-      l = ld_dsmem(smem_u32(sL + qv), s2);
+  if (tid == 0) {
+    sRecv = tc::wait_bar_budget(rbar, 0, tc::kWaitCycles) ? 1 : 0;
+    if (!sRecv) {
+      if (a.err) atomicOr(a.err, static_cast<unsigned>(ERR_TIMEOUT));
+      tc::wait_bar_budget(rbar, 0, tc::kDrainCycles);   // let partials still in flight land before leaving
     }
-    sWm[qv * kMaxSplits + s2] = m;
-    sWl[qv * kMaxSplits + s2] = l;
   }
   __syncthreads();
-  if (tid < nqv) {
-    float* wm = sWm + tid * kMaxSplits;
-    const float* wl = sWl + tid * kMaxSplits;
-    float M = -INFINITY;
-    for (int s2 = 0; s2 < NS; ++s2) M = fmaxf(M, wm[s2]);
-    float Lsum = 0.f;
-    for (int s2 = 0; s2 < NS; ++s2) {
-      const float w = __expf(wm[s2] - M);  // absent splits: e^{-inf} = 0
-      wm[s2] = w;
-      Lsum += wl[s2] * w;
-    }
-    const float inv = 1.f / Lsum;
-    for (int s2 = 0; s2 < NS; ++s2) wm[s2] *= inv;
-  }
-  __syncthreads();
-  const int E4 = nqv * (HD / 4);
-  const int e_hi = (split + 1) * E4 / NS;
-  const uint32_t acc_base = smem_u32(sAcc);
-  for (int e = split * E4 / NS + tid; e < e_hi; e += kThreads) {
+  if (!sRecv) return;
+  for (int e = e_lo + tid; e < e_hi; e += kThreads) {
     const int qv = e / (HD / 4), d4 = e % (HD / 4);
-    const int ns = min(NS, sPos[qv] / a.chunk + 1);
-    const uint32_t addr = acc_base + static_cast<uint32_t>((qv * REC + d4 * 4) * 4);
-    float4 v[kMaxSplits];
+    float w[kMaxSplits];
+    float M = -INFINITY;
 #pragma unroll
     for (int s2 = 0; s2 < kMaxSplits; ++s2)
-      v[s2] = s2 < ns ? ld_dsmem_v4(addr, s2) : make_float4(0.f, 0.f, 0.f, 0.f);
+      if (s2 < NS) M = fmaxf(M, rML[s2 * QR + qv].x);
+    float Lsum = 0.f;
+#pragma unroll
+    for (int s2 = 0; s2 < kMaxSplits; ++s2)
+      if (s2 < NS) {
+        const float2 ml = rML[s2 * QR + qv];
+        w[s2] = __expf(ml.x - M);
+        Lsum += ml.y * w[s2];
+      }
+    const float inv = 1.f / Lsum;
     float4 o = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
-    for (int s2 = 0; s2 < kMaxSplits; ++s2) {
-      const float w = s2 < ns ? sWm[qv * kMaxSplits + s2] : 0.f;
-      o.x = fmaf(w, v[s2].x, o.x); o.y = fmaf(w, v[s2].y, o.y);
-      o.z = fmaf(w, v[s2].z, o.z); o.w = fmaf(w, v[s2].w, o.w);
-    }
+    for (int s2 = 0; s2 < kMaxSplits; ++s2)
+      if (s2 < NS) {
+        const float ws = w[s2] * inv;
+        const float4 v = rAcc[s2 * share + (e - e_lo)];
+        o.x = fmaf(ws, v.x, o.x); o.y = fmaf(ws, v.y, o.y);
+        o.z = fmaf(ws, v.z, o.z); o.w = fmaf(ws, v.w, o.w);
+      }
     const size_t rh = static_cast<size_t>(r0 + qv / G) * a.H + kvh * G + qv % G;
     *reinterpret_cast<uint2*>(static_cast<bf16*>(a.out) + rh * HD + d4 * 4) =
         make_uint2(pack_bf2(o.x, o.y), pack_bf2(o.z, o.w));
   }
-  cluster_sync_all();  // no CTA leaves while another still reads its shared memory
 }
 
 template <int HD>
@@ -423,7 +477,7 @@ bool clusters_fit(int n) {
   cudaLaunchConfig_t cfg{};
   cfg.gridDim = dim3(n, 1, 1);
   cfg.blockDim = dim3(kThreads);
-  cfg.dynamicSmemBytes = AttnCfg<HD>::bytes(kMaxQV, 2 * kTile);
+  cfg.dynamicSmemBytes = AttnCfg<HD>::bytes(kMaxQV, 2 * kTile, n);
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = static_cast<unsigned>(n);
@@ -440,7 +494,7 @@ cudaError_t launch(const AttnArgs& a, cudaStream_t st) {
   const cudaError_t e = configure<HD>();
   if (e != cudaSuccess) return e;
   const int qr = AttnCfg<HD>::qrows(a.max_rows, a.H / a.kv.Hkv);
-  const size_t smem = AttnCfg<HD>::bytes(qr, a.chunk);
+  const size_t smem = AttnCfg<HD>::bytes(qr, a.chunk, a.n_splits);
   if (smem > static_cast<size_t>(kMaxSmem)) return cudaErrorInvalidValue;
   return launch_pdl_cluster(attn_kernel<HD>, dim3(a.n_splits, a.n_groups, a.kv.Hkv), dim3(kThreads), smem, st,
                             a.n_splits, a);

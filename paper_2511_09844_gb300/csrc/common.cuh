@@ -228,6 +228,6 @@ __device__ __forceinline__ void st_async_v4(uint32_t raddr, uint32_t rbar, float
 }
 
 // Device error word bits (latched; read and cleared by the host).
-enum { ERR_NONFINITE = 1, ERR_TIMEOUT = 2 };
+enum { ERR_NONFINITE = 1, ERR_TIMEOUT = 2, ERR_RANGE = 4 };
 
 }  // namespace sd2

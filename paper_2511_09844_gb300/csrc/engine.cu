@@ -61,6 +61,9 @@ struct Plan {
   const int* g_seq = nullptr;
   int n_splits = 1, chunk = 64;
   int max_rows = 1;  // rows of the largest attention group
+  // decode steps: the pre-step lengths attention may read before its programmatic wait (AttnArgs)
+  const int* pre_len = nullptr;
+  int pre_stable = 0, pre_fresh = 0;
 };
 
 struct ProfRec {
@@ -420,6 +423,7 @@ sd2_status forward(sd2_ctx* c, const Model& m, const Plan& p, const FwdOut& o) {
     at.q = c->q; at.kv = m.cache(); at.layer = l; at.row_pos = p.pos;
     at.grp_row0 = p.g_row0; at.grp_nrows = p.g_nrows; at.grp_seq = p.g_seq; at.n_groups = p.n_groups;
     at.M = M; at.H = H; at.hd = hd; at.n_splits = p.n_splits; at.chunk = p.chunk; at.max_rows = p.max_rows; at.out = c->attn;
+    at.pre_len = p.pre_len; at.pre_stable = p.pre_stable; at.pre_fresh = p.pre_fresh; at.err = c->errw;
     double kvb = 0;
     if (c->prof && !c->h_n.empty()) {
       for (int b = 0; b < c->B; ++b) kvb += 2.0 * 2.0 * Hkv * hd * (c->h_n[b] + 16);
@@ -806,6 +810,14 @@ sd2_status sd2_prefill(sd2_ctx* c, int32_t batch, const int32_t* d_tokens, const
   c->p_d1 = step_plan(2 * batch, (int)d1r0.size(), o_d1r0, o_d1nr, o_d1sq, std::min(2, c->D.group_rows()));
   c->p_dn = step_plan(batch, (int)dnr0.size(), o_dnr0, o_dnnr, o_dnsq, 1);
   c->p_v = step_plan(batch * (k + 1), (int)sr0.size(), o_sr0, o_snr, o_ssq, std::min(k + 1, c->V.group_rows()));
+  // State rows written before each step (by the previous commit or the prefill): the drafter cache
+  // holds positions [0, D), the verifier cache [0, n - 1). A drafter step's rows lie in [D, D + k + 1)
+  // (at most 2 pending tokens, then the drafts), the verify rows in [n - 1, n + k).
+  c->p_d1.pre_len = c->p_dn.pre_len = c->state + c->maxB;
+  c->p_d1.pre_fresh = c->p_dn.pre_fresh = k + 1;
+  c->p_v.pre_len = c->state;
+  c->p_v.pre_stable = -1;
+  c->p_v.pre_fresh = k + 1;
   c->logit_rows_d1 = S + o_lr1;
 
   // verifier over the prompts: logits of each last row -> row b*(k+1) of the target buffer
@@ -877,6 +889,7 @@ sd2_status sd2_check(sd2_ctx* c) {
   CK(cudaMemset(c->errw, 0, sizeof(unsigned)));
   if (w & ERR_NONFINITE) return fail(c, SD2_ENUMERIC, "non-finite logits seen on the device");
   if (w & ERR_TIMEOUT) return fail(c, SD2_ETIMEOUT, "a device-side wait timed out");
+  if (w & ERR_RANGE) return fail(c, SD2_ECAPACITY, "an attention row lay outside the positions planned for the step");
   return SD2_OK;
 }
 

@@ -180,6 +180,13 @@ struct AttnArgs {
   int n_splits, chunk;   // context splits (<= attention_max_splits(), one cluster) of `chunk` positions (a multiple of 64)
   int max_rows;          // upper bound of grp_nrows (max_rows x heads per KV head <= 64)
   void* out;             // [M, H * hd] bf16
+  // Decode steps: per sequence, cache positions [0, pre_len[seq] + pre_stable) were written before
+  // the step's first kernel (their K/V rows are loaded before the programmatic wait), and the rows
+  // of the step lie below pre_len[seq] + pre_stable + pre_fresh; the cache rows in between must
+  // hold finite values (the pool starts zeroed). nullptr: every row is loaded after the wait.
+  const int* pre_len;
+  int pre_stable, pre_fresh;
+  unsigned* err;         // ERR_TIMEOUT (split merge), ERR_RANGE (a row outside the planned range); may be null
 };
 cudaError_t attention(const AttnArgs& a, cudaStream_t st);
 // Most context splits (= CTAs of one cluster) attention takes on this device: 16 where clusters of
