@@ -431,29 +431,32 @@ __global__ void __launch_bounds__(kThreads, 2) attn_kernel(const AttnArgs a) {
   if (!sRecv) return;
   for (int e = e_lo + tid; e < e_hi; e += kThreads) {
     const int qv = e / (HD / 4), d4 = e % (HD / 4);
-    float w[kMaxSplits];
+    // every split's values are loaded first (indices clamped, so no load waits behind a branch),
+    // then combined in split order; splits past NS are selected away
+    float2 ml[kMaxSplits];
+#pragma unroll
+    for (int s2 = 0; s2 < kMaxSplits; ++s2) ml[s2] = rML[min(s2, NS - 1) * QR + qv];
     float M = -INFINITY;
 #pragma unroll
-    for (int s2 = 0; s2 < kMaxSplits; ++s2)
-      if (s2 < NS) M = fmaxf(M, rML[s2 * QR + qv].x);
+    for (int s2 = 0; s2 < kMaxSplits; ++s2) M = s2 < NS ? fmaxf(M, ml[s2].x) : M;
+    float w[kMaxSplits];
     float Lsum = 0.f;
 #pragma unroll
-    for (int s2 = 0; s2 < kMaxSplits; ++s2)
-      if (s2 < NS) {
-        const float2 ml = rML[s2 * QR + qv];
-        w[s2] = __expf(ml.x - M);
-        Lsum += ml.y * w[s2];
-      }
+    for (int s2 = 0; s2 < kMaxSplits; ++s2) {
+      w[s2] = __expf(ml[s2].x - M);
+      Lsum = s2 < NS ? Lsum + ml[s2].y * w[s2] : Lsum;
+    }
     const float inv = 1.f / Lsum;
     float4 o = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
-    for (int s2 = 0; s2 < kMaxSplits; ++s2)
+    for (int s2 = 0; s2 < kMaxSplits; ++s2) {
+      const float ws = w[s2] * inv;
+      const float4 v = rAcc[min(s2, NS - 1) * share + (e - e_lo)];
       if (s2 < NS) {
-        const float ws = w[s2] * inv;
-        const float4 v = rAcc[s2 * share + (e - e_lo)];
         o.x = fmaf(ws, v.x, o.x); o.y = fmaf(ws, v.y, o.y);
         o.z = fmaf(ws, v.z, o.z); o.w = fmaf(ws, v.w, o.w);
       }
+    }
     const size_t rh = static_cast<size_t>(r0 + qv / G) * a.H + kvh * G + qv % G;
     *reinterpret_cast<uint2*>(static_cast<bf16*>(a.out) + rh * HD + d4 * 4) =
         make_uint2(pack_bf2(o.x, o.y), pack_bf2(o.z, o.w));

@@ -148,7 +148,8 @@ __device__ __forceinline__ void norm_produce(const TcArgs& a, int m, int n, floa
 }
 // Fused RMSNorm, consumer side: rs[c] = rsqrt(mean of x_new^2 + eps) of the token tile's columns,
 // from the producer's slices summed in a fixed order (8 strided partial sums, then a butterfly
-// over the 8 lanes). Called by the 128 epilogue threads (tid = 0..127).
+// over the 8 lanes). Called by the 128 epilogue threads (tid = 0..127). Each lane requests its
+// slices in blocks of 32 before adding any (indices clamped), so a block costs one L2 round trip.
 __device__ __forceinline__ void tile_rstd(const TcArgs& a, int tt, float* rs, int tid) {
   const int cols = min(a.NT, a.M - tt * a.NT);
   const int j = tid & 7;
@@ -157,8 +158,13 @@ __device__ __forceinline__ void tile_rstd(const TcArgs& a, int tt, float* rs, in
     float s = 0.f;
     if (c < cols) {
       const float* src = a.norm_ssq_in + tt * a.NT + c;
-#pragma unroll 4
-      for (int p = j; p < a.norm_parts; p += 8) s += src[static_cast<size_t>(p) * a.ld_ssq];
+      for (int p0 = j; p0 < a.norm_parts; p0 += 8 * 32) {
+        float v[32];
+#pragma unroll
+        for (int u = 0; u < 32; ++u) v[u] = src[static_cast<size_t>(min(p0 + 8 * u, a.norm_parts - 1)) * a.ld_ssq];
+#pragma unroll
+        for (int u = 0; u < 32; ++u) s = p0 + 8 * u < a.norm_parts ? s + v[u] : s;
+      }
     }
     s += __shfl_xor_sync(0xffffffffu, s, 1);
     s += __shfl_xor_sync(0xffffffffu, s, 2);
@@ -525,13 +531,19 @@ __global__ void __launch_bounds__(kThreads, 2) gemm_tc_kernel(const __grid_const
         for (int e = tid; e < np * cols; e += 128) {
           const int lp = e % np, col = e / np;
           const float* rv = recv + lp * 2 * NT + col;
+          float v0[8], v1[8];                // every rank's partial loaded first (clamped rank index)
+#pragma unroll
+          for (int k = 0; k < 8; ++k) {
+            const int kk = min(k, sp - 1);
+            v0[k] = rv[kk * npmax * 2 * NT];
+            v1[k] = rv[kk * npmax * 2 * NT + NT];
+          }
           float s0 = 0.f, s1 = 0.f;
 #pragma unroll
-          for (int k = 0; k < 8; ++k)
-            if (k < sp) {
-              s0 += rv[k * npmax * 2 * NT];
-              s1 += rv[k * npmax * 2 * NT + NT];
-            }
+          for (int k = 0; k < 8; ++k) {
+            s0 = k < sp ? s0 + v0[k] : s0;
+            s1 = k < sp ? s1 + v1[k] : s1;
+          }
           if (a.norm_ssq_in) {
             s0 *= rs[col];
             s1 *= rs[col];
