@@ -227,6 +227,29 @@ sd2_status sd2_gemm(const void* d_x, int32_t ldx, int32_t M, int32_t K, const vo
                     int32_t N, int32_t epilogue, float* d_out, int32_t ldo, void* d_h, const float* d_bias,
                     const int32_t* d_seq, int32_t ld_bias, int32_t impl, void* stream);
 
+/* Causal grouped-query attention of the decoder layers (Sec. 3.2, the SwiGLU decoders of drafter and
+ * verifier) over a paged KV cache, on caller buffers (the kernel of the engine's steps).
+ *   d_q [M, H, hd] f32: rotated queries of M rows; hd 64 or 128; H a multiple of Hkv.
+ *   d_pool bf16 [L][n_blocks][2 (K, V)][Hkv][16][hd]; d_table int32 [n_seq, bt_stride]: the block
+ *   holding positions 16 i .. 16 i + 15 of sequence s (ids in [0, n_blocks)); `layer` selects L.
+ *   Groups g < n_groups: rows d_grp_row0[g] .. d_grp_row0[g] + d_grp_nrows[g] - 1 belong to sequence
+ *   d_grp_seq[g]; row m (position d_row_pos[m]) attends to its sequence's positions 0 .. d_row_pos[m].
+ *   max_rows >= every d_grp_nrows, max_rows * H / Hkv <= 64. The context is cut into n_splits chunks
+ *   of `chunk` positions (a multiple of 64; 1 <= n_splits <= 16 where the device schedules clusters
+ *   of 16 CTAs, else 8); positions at or beyond n_splits * chunk or 16 * bt_stride are not read.
+ *   d_pre_len (may be null): per sequence, positions below d_pre_len[s] + pre_stable are read before
+ *   the programmatic wait (they must not be written by the kernel launched just before on the
+ *   stream), and every row lies below d_pre_len[s] + pre_stable + pre_fresh; cache rows between
+ *   the two bounds must hold finite values.
+ *   d_out [M, H * hd] bf16. d_err (may be null): a device word or-ed with 2 (a merge wait timed out)
+ *   or 4 (a row lay beyond the d_pre_len bound). No device memory is allocated. */
+sd2_status sd2_attention(const float* d_q, int32_t M, int32_t H, int32_t Hkv, int32_t hd, const void* d_pool,
+                         int32_t n_blocks, const int32_t* d_table, int32_t bt_stride, int32_t layer,
+                         const int32_t* d_row_pos, const int32_t* d_grp_row0, const int32_t* d_grp_nrows,
+                         const int32_t* d_grp_seq, int32_t n_groups, int32_t max_rows, int32_t n_splits, int32_t chunk,
+                         const int32_t* d_pre_len, int32_t pre_stable, int32_t pre_fresh, void* d_out,
+                         uint32_t* d_err, void* stream);
+
 /* Choose the GEMM of a context: 0 tensor cores where the shape allows (default), 1 CUDA cores.
  * Drops captured graphs. */
 sd2_status sd2_set_gemm_impl(sd2_ctx* ctx, int32_t impl);

@@ -189,7 +189,7 @@ __global__ void __launch_bounds__(kThreads, 2) attn_kernel(const AttnArgs a) {
       const int idx = tid + u * kThreads, t = idx / (HD / 8), c = idx % (HD / 8);
       const int p = t0 + t;
       if (p < p_from || p >= p_to) continue;
-      const bool ok = p < valid_end;
+      const bool ok = p < valid_end && p < row_end;   // block ids exist only below row_end
       const bf16* src = layer_base;
       if (ok) src += static_cast<size_t>(sBlk[(p - lo) >> 4]) * blk_stride + static_cast<size_t>(p & 15) * HD + c * 8;
       cp_async16(smem_u32(dK + t * KS + c * 8), src, ok);
@@ -237,7 +237,8 @@ __global__ void __launch_bounds__(kThreads, 2) attn_kernel(const AttnArgs a) {
   const int nmt = (nqv + 15) >> 4;
   if (early) {
     // every row the queries can see in the early tiles must have been loaded
-    if (tid == 0 && min(hi, lo + nb * kTile) > fresh_hi && a.err) atomicOr(a.err, static_cast<unsigned>(ERR_RANGE));
+    if (tid == 0 && ntiles > 0 && min(hi, lo + nb * kTile) > fresh_hi && a.err)
+      atomicOr(a.err, static_cast<unsigned>(ERR_RANGE));
   } else {
     if (ntiles > 0) { issue_rows(0, lo, INT_MAX, hi); cp_async_commit(); }
     if (ntiles > 1) { issue_rows(1, lo, INT_MAX, hi); cp_async_commit(); }

@@ -28,7 +28,7 @@ EXPORTS = ["sd2_init", "sd2_prefill", "sd2_step", "sd2_accept", "sd2_check", "sd
            "sd2_set_graphs", "sd2_debug_buffer", "sd2_profile", "sd2_profile_read", "sd2_accept_workspace_bytes",
            "sd2_accept_logits", "sd2_steer_workspace_bytes", "sd2_steer", "sd2_swiglu_steered",
            "sd2_accept_logits_noalloc", "sd2_gemm", "sd2_set_gemm_impl", "sd2_stage_timing", "sd2_stage_read",
-           "sd2_set_drafter_chain"]
+           "sd2_set_drafter_chain", "sd2_attention"]
 
 
 class LMConfig(ctypes.Structure):
@@ -91,6 +91,9 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
     lib.sd2_gemm.argtypes = [c_void_p, c_int32, c_int32, c_int32, c_void_p, c_void_p, c_int32, c_int32, c_void_p,
                              c_int32, c_void_p, c_void_p, c_void_p, c_int32, c_int32, c_void_p]
     lib.sd2_set_gemm_impl.argtypes = [c_void_p, c_int32]
+    lib.sd2_attention.argtypes = [c_void_p, c_int32, c_int32, c_int32, c_int32, c_void_p, c_int32, c_void_p, c_int32,
+                                  c_int32, c_void_p, c_void_p, c_void_p, c_void_p, c_int32, c_int32, c_int32, c_int32,
+                                  c_void_p, c_int32, c_int32, c_void_p, c_void_p, c_void_p]
     lib.sd2_set_drafter_chain.argtypes = [c_void_p, c_int32]
     lib.sd2_accept_logits_noalloc.argtypes = [c_void_p, c_void_p, c_int32, c_void_p, c_void_p, c_int32, c_int32,
                                               c_int32, c_uint64, c_uint32, c_void_p, c_void_p, c_void_p]
@@ -305,6 +308,24 @@ def swiglu_steered(gate: torch.Tensor, up: torch.Tensor, bias: Optional[torch.Te
     h = torch.empty((M, F), dtype=torch.bfloat16, device=gate.device)
     _check(lib, lib.sd2_swiglu_steered(_ptr(gate), _ptr(up), _ptr(bias), _ptr(seq), M, F, _ptr(h), _stream(stream)))
     return h
+
+
+def attention(q: torch.Tensor, pool: torch.Tensor, table: torch.Tensor, layer: int, row_pos: torch.Tensor,
+              grp_row0: torch.Tensor, grp_nrows: torch.Tensor, grp_seq: torch.Tensor, max_rows: int,
+              n_splits: int, chunk: int, pre_len: Optional[torch.Tensor] = None, pre_stable: int = 0,
+              pre_fresh: int = 0, err: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
+    """Standalone paged causal attention (sd2_attention). q [M, H, hd] f32; pool bf16
+    [L, n_blocks, 2, Hkv, 16, hd]; table int32 [n_seq, bt_stride]; returns bf16 [M, H * hd]. `err`, a
+    one-element int32 device tensor, collects the device error bits."""
+    lib = load_library()
+    M, H, hd = q.shape
+    Hkv, n_blocks = pool.shape[3], pool.shape[1]
+    out = torch.empty((M, H * hd), dtype=torch.bfloat16, device=q.device)
+    _check(lib, lib.sd2_attention(_ptr(q), M, H, Hkv, hd, _ptr(pool), n_blocks, _ptr(table), table.shape[1], layer,
+                                  _ptr(row_pos), _ptr(grp_row0), _ptr(grp_nrows), _ptr(grp_seq), grp_row0.numel(),
+                                  max_rows, n_splits, chunk, _ptr(pre_len), pre_stable, pre_fresh, _ptr(out),
+                                  _ptr(err), _stream(stream)))
+    return out
 
 
 def gemm(x: torch.Tensor, w: torch.Tensor, epilogue: int = 0, out: Optional[torch.Tensor] = None,
