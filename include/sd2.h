@@ -260,6 +260,13 @@ sd2_status sd2_set_gemm_impl(sd2_ctx* ctx, int32_t impl);
  * arithmetic of a2. Only with the tensor-core GEMM (sd2_set_gemm_impl 0). Drops captured graphs. */
 sd2_status sd2_set_drafter_chain(sd2_ctx* ctx, int32_t enable);
 
+/* Decode steps of one sequence (batch 1): run each layer's attention inside its O projection
+ * (1, where the model allows it: head dim 64, 2..8 KV heads, rows x heads per KV head <= 16,
+ * context <= 4096, the projection's tiles x KV heads <= the SM count) or as a kernel of its own
+ * (0, the default: faster on GB300, where the fused kernel's shared memory keeps the neighbouring
+ * kernels from overlapping it). Either way the same arithmetic. Drops captured graphs. */
+sd2_status sd2_set_fused_attention(sd2_ctx* ctx, int32_t enable);
+
 /* Steered SwiGLU activation of Eq. 2 on caller buffers (the injection step of a2):
  *   h[m, f] = (up[m, f] + bias[seq[m], f]) * SiLU(gate[m, f]) as bf16, with gate/up [M, F] f32,
  *   bias [*, F] f32 (row seq[m]; d_seq may be null for bias row 0), h [M, F] bf16. */

@@ -105,6 +105,7 @@ struct sd2_ctx {
   ChainPlan chain{};             // the drafter's persistent layer chain (chain.cu), when its shape allows
   bool chain_ok = false;
   bool use_chain = false;        // measured slower than the per-kernel path on GB300 (off by default)
+  bool attn_in_o = false;        // decode attention inside the O projection: measured slower on GB300 (off by default)
   void *a = nullptr, *attn = nullptr, *h = nullptr, *g_bf = nullptr, *hml_in = nullptr;
   int gemm_impl = 0;            // 0 tensor cores where the shape allows, 1 CUDA cores
   unsigned long long* samp_slot = nullptr;
@@ -419,6 +420,22 @@ sd2_status forward(sd2_ctx* c, const Model& m, const Plan& p, const FwdOut& o) {
     GemmArgs g = qkv_args(l);
     if (fused) consume(g, parts);
     CK(timed(c, PC_GEMM, gemm_bytes(M, m.qkv_width(), d, 4), [&] { return gemm(tc(c, g), c->st); }));
+    // A decode step of one sequence may run its attention inside the O projection (gemm_tc.cu).
+    GemmArgs go = o_args(l);
+    if (fused) produce(go, m.W(l, SD2_W_MLP_NORM));
+    bool in_o = false;
+    if (c->attn_in_o && p.pre_len && p.n_groups == 1 && c->gemm_impl == 0) {
+      GemmArgs ga = go;
+      ga.attn_q = c->q; ga.attn_seq = p.g_seq; ga.attn_pre_len = p.pre_len;
+      ga.attn_pre_stable = p.pre_stable; ga.attn_pre_fresh = p.pre_fresh;
+      ga.kv_pool = m.kv_pool; ga.kv_table = m.table; ga.kv_bt_stride = m.bt_stride; ga.kv_n_blocks = m.n_blocks;
+      ga.n_heads = H; ga.n_kv_heads = Hkv; ga.head_dim = hd; ga.layer = l; ga.row_pos = p.pos;
+      if (gemm_attn_supported(tc(c, ga))) {
+        go = ga;
+        in_o = true;
+      }
+    }
+    if (fused) parts = gemm_norm_parts(go);
     AttnArgs at{};
     at.q = c->q; at.kv = m.cache(); at.layer = l; at.row_pos = p.pos;
     at.grp_row0 = p.g_row0; at.grp_nrows = p.g_nrows; at.grp_seq = p.g_seq; at.n_groups = p.n_groups;
@@ -428,13 +445,12 @@ sd2_status forward(sd2_ctx* c, const Model& m, const Plan& p, const FwdOut& o) {
     if (c->prof && !c->h_n.empty()) {
       for (int b = 0; b < c->B; ++b) kvb += 2.0 * 2.0 * Hkv * hd * (c->h_n[b] + 16);
     }
-    CK(timed(c, PC_ATTN, kvb, [&] { return attention(at, c->st); }));
-    GemmArgs go = o_args(l);
-    if (fused) {
-      produce(go, m.W(l, SD2_W_MLP_NORM));
-      parts = gemm_norm_parts(go);
+    if (in_o)
+      CK(timed(c, PC_GEMM, gemm_bytes(M, d, H * hd, 8) + kvb, [&] { return gemm(tc(c, go), c->st); }));
+    else {
+      CK(timed(c, PC_ATTN, kvb, [&] { return attention(at, c->st); }));
+      CK(timed(c, PC_GEMM, gemm_bytes(M, d, H * hd, 8), [&] { return gemm(tc(c, go), c->st); }));
     }
-    CK(timed(c, PC_GEMM, gemm_bytes(M, d, H * hd, 8), [&] { return gemm(tc(c, go), c->st); }));
     if (!fused)
       CK(timed(c, PC_OTHER, 0, [&] {
         return rmsnorm(c->x, nullptr, m.W(l, SD2_W_MLP_NORM), mc.norm_eps, M, d, c->a, nullptr, nullptr, 0, c->st);
@@ -904,6 +920,13 @@ sd2_status sd2_set_gemm_impl(sd2_ctx* c, int32_t impl) {
   if (!c) return fail(nullptr, SD2_EINVAL, "null context");
   if (impl != 0 && impl != 1) return fail(c, SD2_EINVAL, "impl must be 0 (tensor cores) or 1 (CUDA cores)");
   c->gemm_impl = impl;
+  drop_graphs(c);
+  return SD2_OK;
+}
+
+sd2_status sd2_set_fused_attention(sd2_ctx* c, int32_t enable) {
+  if (!c) return fail(nullptr, SD2_EINVAL, "null context");
+  c->attn_in_o = enable != 0;
   drop_graphs(c);
   return SD2_OK;
 }

@@ -124,6 +124,7 @@ __global__ void __launch_bounds__(kThreads) gemm_simt_kernel(const GemmArgs a, i
 }  // namespace
 
 cudaError_t gemm(const GemmArgs& a, cudaStream_t st) {
+  if (a.attn_q) return a.impl != 1 && a.err && gemm_attn_supported(a) ? gemm_tc(a, a.err, st) : cudaErrorNotSupported;
   if (a.impl != 1 && a.err && gemm_tc_supported(a)) return gemm_tc(a, a.err, st);
   if (a.norm_out || a.norm_ssq_in) return cudaErrorNotSupported;  // the fused RMSNorm is tensor-core only
   if (a.epi != EPI_QKV) return gemm_simt(a, st);

@@ -23,6 +23,7 @@
 // (each warp its 32-lane quarter) and run the epilogue. Every wait is bounded by a clock budget;
 // on expiry the kernel records ERR_TIMEOUT, drains what it issued and returns.
 #include <cuda.h>
+#include <limits.h>
 
 #include <mutex>
 #include <unordered_map>
@@ -79,6 +80,11 @@ struct TcArgs {
   int norm_parts, norm_d;
   float norm_eps;
   int ld_ssq;
+  // fused decode attention (see GemmArgs)
+  const float* attn_q;
+  const int* attn_seq;
+  const int* attn_pre_len;
+  int attn_pre_stable, attn_pre_fresh;
 };
 
 
@@ -334,6 +340,101 @@ __device__ __forceinline__ float pair_emit(const TcArgs& a, int wt, int p, int m
   return 0.f;
 }
 
+
+// Shared memory and launch facts the split-K epilogue needs.
+struct SplitK {
+  unsigned char* smem;                       // the drained ring: fused-norm scratch
+  float* recv;                               // [sp][npmax][2][NT] partials of this rank's pairs
+  float* rs;                                 // RMSNorm row scales (consumers)
+  volatile int* flags;
+  uint32_t tfull0, rbar, tmem;
+  int rank, sp, npmax, NT, first_tile;
+};
+// The global operands of the first output this epilogue thread (tid 0..127) owns, fetched early.
+__device__ __forceinline__ PairOps first_pair_ops(const TcArgs& a, int rank, int sp, int NT, int first_tile, int tid) {
+  const int wt = first_tile % a.n_wtiles, tt = first_tile / a.n_wtiles;
+  const int cols = min(NT, a.M - tt * NT);
+  const int p_lo = rank * 64 / sp, np = (rank + 1) * 64 / sp - p_lo;
+  return tid < np * cols ? pair_ops(a, wt, p_lo + tid % np, tt * NT + tid / np) : PairOps{};
+}
+// Split-K epilogue of the CTA's single tile (sp > 1), run by the four epilogue warps (warp % 4 =
+// the TMEM lane quarter): this rank's partial of every row goes to the rank owning the row's pair
+// (st.async onto the owner's receive barrier); the owner waits for its own pairs only, sums the
+// partials in rank order and runs the epilogue. Everything but the sums is prepared while the
+// MMAs run. pf: the operands of the thread's first owned output (first_pair_ops).
+__device__ __forceinline__ void splitk_epilogue(const TcArgs& a, const SplitK& sk, int warp, int lane, const PairOps& pf) {
+  const int q = warp & 3, r = q * 32 + lane, tid = threadIdx.x - 64;
+  const bool leader = (warp == 2 && lane == 0);
+  const int sp = sk.sp, npmax = sk.npmax, NT = sk.NT, rank = sk.rank;
+  volatile int* flags = sk.flags;
+  volatile int* abort_flag = sk.flags;
+  float* recv = sk.recv;
+  float* rs = sk.rs;
+  const int wt = sk.first_tile % a.n_wtiles, tt = sk.first_tile / a.n_wtiles;
+  const int cols = min(NT, a.M - tt * NT);
+  const int p_lo = rank * 64 / sp, np = (rank + 1) * 64 / sp - p_lo;
+  const int p = pair_of(a, r), owner = pair_owner(p, sp);
+  const int slot = ((rank * npmax + p - owner * 64 / sp) * 2 + member_of(a, r)) * NT;
+  const uint32_t dst = dsmem_addr(smem_u32(recv + slot), static_cast<uint32_t>(owner));
+  const uint32_t dst_bar = dsmem_addr(sk.rbar, static_cast<uint32_t>(owner));
+  if (a.norm_ssq_in) tile_rstd(a, tt, rs, tid);
+  if (leader) flags[4] = wait_bar(sk.tfull0, 0, abort_flag, a.err) ? 1 : 0;
+  named_bar_epi();                         // the accumulator is complete (or the wait gave up); rs is set
+  tc_fence_after();
+  cluster_wait();                          // every rank's receive barrier is armed
+  if (flags[4] != 0) {
+    const uint32_t tbase = sk.tmem + (static_cast<uint32_t>(q * 32) << 16);
+    for (int ch = 0; ch * 16 < cols; ++ch) {
+      float v[16];
+      tmem_ld16(tbase + ch * 16, v);
+#pragma unroll
+      for (int k4 = 0; k4 < 4; ++k4)
+        st_async_v4(dst + static_cast<uint32_t>((ch * 16 + 4 * k4) * 4), dst_bar, v[4 * k4], v[4 * k4 + 1],
+                    v[4 * k4 + 2], v[4 * k4 + 3]);
+    }
+    if (leader) flags[5] = wait_bar(sk.rbar, 0, abort_flag, a.err) ? 1 : 0;
+    named_bar_epi();
+    if (flags[5] != 0) {
+      // every rank's partial of this rank's pairs is in the receive buffer: sums in rank order
+      float* sq = reinterpret_cast<float*>(sk.smem);   // [cols][np] fused-norm sums of squares (drained ring)
+      for (int e = tid; e < np * cols; e += 128) {
+        const int lp = e % np, col = e / np;
+        const float* rv = recv + lp * 2 * NT + col;
+        float v0[8], v1[8];                // every rank's partial loaded first (clamped rank index)
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          const int kk = min(j, sp - 1);
+          v0[j] = rv[kk * npmax * 2 * NT];
+          v1[j] = rv[kk * npmax * 2 * NT + NT];
+        }
+        float s0 = 0.f, s1 = 0.f;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          s0 = j < sp ? s0 + v0[j] : s0;
+          s1 = j < sp ? s1 + v1[j] : s1;
+        }
+        if (a.norm_ssq_in) {
+          s0 *= rs[col];
+          s1 *= rs[col];
+        }
+        const int m = tt * NT + col;
+        const float q2 = pair_emit(a, wt, p_lo + lp, m, s0, s1, e == tid ? pf : pair_ops(a, wt, p_lo + lp, m));
+        if (a.norm_out) sq[col * np + lp] = q2;
+      }
+      if (a.norm_out) {   // this rank's slice of the tile: sums of squares per token, in pair order
+        named_bar_epi();
+        for (int c = tid; c < cols; c += 128) {
+          float ssum = 0.f;
+          for (int lp = 0; lp < np; ++lp) ssum += sq[c * np + lp];
+          a.norm_ssq_out[static_cast<size_t>(wt * sp + rank) * a.ld_ssq + tt * NT + c] = ssum;
+        }
+      }
+    } else if (leader) {
+      wait_bar_budget(sk.rbar, 0, kDrainCycles);   // let partials still in flight land before leaving
+    }
+  }
+}
+
 __global__ void __launch_bounds__(kThreads, 2) gemm_tc_kernel(const __grid_constant__ TcArgs a) {
   extern __shared__ unsigned char smem_raw[];
   unsigned char* smem =
@@ -497,73 +598,9 @@ __global__ void __launch_bounds__(kThreads, 2) gemm_tc_kernel(const __grid_const
     // Split-K epilogue of the CTA's single tile. Everything but the sums (this thread's
     // destination in the owner's receive buffer, the operands of its first owned output, the
     // RMSNorm scales) is prepared while the MMAs run.
-    const int q = warp & 3, r = q * 32 + lane, tid = threadIdx.x - 64;
-    const bool leader = (warp == 2 && lane == 0);
     pdl_wait();                              // outputs, residuals and biases come from earlier kernels
-    const int wt = first_tile % a.n_wtiles, tt = first_tile / a.n_wtiles;
-    const int cols = min(NT, a.M - tt * NT);
-    const int p_lo = rank * 64 / sp, np = (rank + 1) * 64 / sp - p_lo;
-    if (tid < np * cols) pf = pair_ops(a, wt, p_lo + tid % np, tt * NT + tid / np);
-    const int p = pair_of(a, r), owner = pair_owner(p, sp);
-    const int slot = ((rank * npmax + p - owner * 64 / sp) * 2 + member_of(a, r)) * NT;
-    const uint32_t dst = dsmem_addr(smem_u32(recv + slot), static_cast<uint32_t>(owner));
-    const uint32_t dst_bar = dsmem_addr(rbar, static_cast<uint32_t>(owner));
-    if (a.norm_ssq_in) tile_rstd(a, tt, rs, tid);
-    if (leader) flags[4] = wait_bar(tfull0, 0, abort_flag, a.err) ? 1 : 0;
-    named_bar_epi();                         // the accumulator is complete (or the wait gave up); rs is set
-    tc_fence_after();
-    cluster_wait();                          // every rank's receive barrier is armed
-    if (flags[4] != 0) {
-      const uint32_t tbase = tmem + (static_cast<uint32_t>(q * 32) << 16);
-      for (int ch = 0; ch * 16 < cols; ++ch) {
-        float v[16];
-        tmem_ld16(tbase + ch * 16, v);
-#pragma unroll
-        for (int k4 = 0; k4 < 4; ++k4)
-          st_async_v4(dst + static_cast<uint32_t>((ch * 16 + 4 * k4) * 4), dst_bar, v[4 * k4], v[4 * k4 + 1],
-                      v[4 * k4 + 2], v[4 * k4 + 3]);
-      }
-      if (leader) flags[5] = wait_bar(rbar, 0, abort_flag, a.err) ? 1 : 0;
-      named_bar_epi();
-      if (flags[5] != 0) {
-        // every rank's partial of this rank's pairs is in the receive buffer: sums in rank order
-        float* sq = reinterpret_cast<float*>(smem);   // [cols][np] fused-norm sums of squares (drained ring)
-        for (int e = tid; e < np * cols; e += 128) {
-          const int lp = e % np, col = e / np;
-          const float* rv = recv + lp * 2 * NT + col;
-          float v0[8], v1[8];                // every rank's partial loaded first (clamped rank index)
-#pragma unroll
-          for (int k = 0; k < 8; ++k) {
-            const int kk = min(k, sp - 1);
-            v0[k] = rv[kk * npmax * 2 * NT];
-            v1[k] = rv[kk * npmax * 2 * NT + NT];
-          }
-          float s0 = 0.f, s1 = 0.f;
-#pragma unroll
-          for (int k = 0; k < 8; ++k) {
-            s0 = k < sp ? s0 + v0[k] : s0;
-            s1 = k < sp ? s1 + v1[k] : s1;
-          }
-          if (a.norm_ssq_in) {
-            s0 *= rs[col];
-            s1 *= rs[col];
-          }
-          const int m = tt * NT + col;
-          const float q2 = pair_emit(a, wt, p_lo + lp, m, s0, s1, e == tid ? pf : pair_ops(a, wt, p_lo + lp, m));
-          if (a.norm_out) sq[col * np + lp] = q2;
-        }
-        if (a.norm_out) {   // this rank's slice of the tile: sums of squares per token, in pair order
-          named_bar_epi();
-          for (int c = tid; c < cols; c += 128) {
-            float ssum = 0.f;
-            for (int lp = 0; lp < np; ++lp) ssum += sq[c * np + lp];
-            a.norm_ssq_out[static_cast<size_t>(wt * sp + rank) * a.ld_ssq + tt * NT + c] = ssum;
-          }
-        }
-      } else if (leader) {
-        wait_bar_budget(rbar, 0, kDrainCycles);   // let partials still in flight land before leaving
-      }
-    }
+    pf = first_pair_ops(a, rank, sp, NT, first_tile, threadIdx.x - 64);
+    splitk_epilogue(a, SplitK{smem, recv, rs, flags, tfull0, rbar, tmem, rank, sp, npmax, NT, first_tile}, warp, lane, pf);
   } else {
     const int q = warp & 3;                   // TMEM lane quarter of this warp
     const int r = q * 32 + lane;              // weight row within the tile
@@ -605,6 +642,337 @@ __global__ void __launch_bounds__(kThreads, 2) gemm_tc_kernel(const __grid_const
   __syncthreads();
   tc_fence_after();
   if (warp == 1) tmem_dealloc(tmem, ncols);
+}
+
+
+// ------------------------------------------------------------------------------ fused decode attention
+// The O projection of a decode step of one sequence with its attention folded in. With sp = H_kv
+// ranks per tile, rank r's K-slice of W_O is exactly the G = H / H_kv query heads of KV head r
+// (hd 64: one k-block per head), so CTA (tile, r) computes the causal attention of KV head r for
+// the step's rows over the whole context and writes it, in bf16 and in the 128-byte-swizzled
+// K-major layout a TMA load would give, as the token operand of its stages; the MMA and the
+// split-K epilogue are those of gemm_tc_kernel. The attention is split over 8 warps by position
+// ranges (each a flash-decoding pass with its own running max and sum, K/V staged by cp.async
+// three 16-position sub-tiles ahead, no CTA barrier per sub-tile), then merged across the warps.
+// The 16 O tiles that share a KV head each recompute it (from L2); what this saves is the
+// attention kernel, its cluster merge and one kernel boundary per layer.
+constexpr int kAoWarps = 10;                 // 0 TMA, 1 MMA, 2-9 attention (2-5 also the epilogue)
+constexpr int kAoThreads = kAoWarps * 32;
+constexpr int kAoSub = 16;                   // positions per sub-tile
+constexpr int kAoBuf = 3;                    // sub-tiles in flight per warp
+constexpr int kAoKS = 64 + 8;                // K/V/Q row stride (bf16), hd 64
+constexpr int kAoAS = 64 + 4;                // per-warp partial accumulator row stride (f32)
+constexpr int kAoMaxBlk = 32;                // cache blocks (of 16 positions) per warp: context <= 4096
+constexpr int kAoWarpBytes = kAoBuf * 2 * kAoSub * kAoKS * 2;   // one warp's K/V buffers
+
+__device__ __forceinline__ void named_bar_attn() { asm volatile("bar.sync 2, 256;" ::: "memory"); }
+__device__ __forceinline__ uint32_t ao_ld_u32(const bf16* p) { return *reinterpret_cast<const uint32_t*>(p); }
+__device__ __forceinline__ uint32_t ao_pack(float x, float y) {
+  const __nv_bfloat162 h = __floats2bfloat162_rn(x, y);
+  return *reinterpret_cast<const uint32_t*>(&h);
+}
+__device__ __forceinline__ void ao_cp16(uint32_t dst, const void* src, bool valid) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(valid ? 16 : 0) : "memory");
+}
+__device__ __forceinline__ void ao_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void ao_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
+__device__ __forceinline__ void ao_mma(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3, uint32_t b0,
+                                       uint32_t b1) {
+  asm("mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+__device__ __forceinline__ void ao_ldsm_x2_t(uint32_t addr, uint32_t& r0, uint32_t& r1) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x2.trans.shared.b16 {%0,%1}, [%2];" : "=r"(r0), "=r"(r1) : "r"(addr) : "memory");
+}
+
+// Shared memory of the fused kernel after the GEMM part (ring, receive buffer, barriers, flags):
+// Q [16][kAoKS] bf16, row positions [16], per-warp (max, sum) [8][16][2], per-warp block ids
+// [8][kAoMaxBlk], per-warp K/V buffers [8][kAoWarpBytes] (then each warp's partial accumulators).
+constexpr int kAoQBytes = 16 * kAoKS * 2;
+constexpr int kAoAttnBytes = kAoQBytes + 16 * 4 + 8 * 16 * 8 + 8 * kAoMaxBlk * 4 + 8 * kAoWarpBytes;
+
+__global__ void __launch_bounds__(kAoThreads, 1) gemm_attn_kernel(const __grid_constant__ TcArgs a) {
+  extern __shared__ unsigned char smem_raw[];
+  unsigned char* smem =
+      reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  const int S = a.stages, NT = a.NT, sp = a.sp;   // S = k-blocks of the slice = G
+  const uint32_t a_bytes = kWRows * kBK * 2;
+  const uint32_t b_bytes = static_cast<uint32_t>(NT) * kBK * 2;
+  const uint32_t stage_bytes = a_bytes + b_bytes;
+  const int npmax = pairs_max(sp);
+  const uint32_t recv_bytes = static_cast<uint32_t>(sp * npmax * 2 * NT * 4);
+  float* recv = reinterpret_cast<float*>(smem + static_cast<size_t>(S) * stage_bytes);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + static_cast<size_t>(S) * stage_bytes + recv_bytes);
+  volatile int* flags = reinterpret_cast<volatile int*>(bars + 2 * S + 6);
+  float* rs = const_cast<float*>(reinterpret_cast<volatile float*>(flags + 16));
+  unsigned char* attn = reinterpret_cast<unsigned char*>(rs + 16);
+  bf16* sQ = reinterpret_cast<bf16*>(attn);
+  int* sPos = reinterpret_cast<int*>(attn + kAoQBytes);
+  float* sML = reinterpret_cast<float*>(sPos + 16);                 // [8 warps][16 rows][max, sum]
+  int* sBlk = reinterpret_cast<int*>(sML + 8 * 16 * 2);               // [8 warps][kAoMaxBlk]
+  unsigned char* sKV = reinterpret_cast<unsigned char*>(sBlk + 8 * kAoMaxBlk);
+  const uint32_t full0 = smem_u32(bars), empty0 = full0 + 8 * S, tfull0 = empty0 + 8 * S, tempty0 = tfull0 + 16,
+                 drain = tempty0 + 16, rbar = drain + 8;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int rank = static_cast<int>(cluster_rank());
+  const int first_tile = static_cast<int>(blockIdx.x) / sp;
+  const int wt = first_tile % a.n_wtiles;
+  const int M = a.M, G = a.n_heads / a.n_kv_heads, nqv = M * G;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < S; ++s) {
+      mbar_init(full0 + 8 * s, 2);           // the weight tile's bytes + the attention's token operand
+      mbar_init(empty0 + 8 * s, 1);
+    }
+    mbar_init(tfull0, 1);
+    mbar_init(tfull0 + 8, 1);
+    mbar_init(tempty0, 4);
+    mbar_init(tempty0 + 8, 4);
+    mbar_init(drain, 1);
+    const int np = (rank + 1) * 64 / sp - rank * 64 / sp;
+    mbar_init(rbar, 1);
+    mbar_expect_tx(rbar, static_cast<uint32_t>(sp * 2 * np * ((M + 15) / 16) * 64));
+    flags[0] = 0; flags[3] = 0; flags[4] = 0; flags[5] = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(const_cast<int*>(flags) + 1), 32);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  cluster_arrive_relaxed();
+  const uint32_t tmem = static_cast<uint32_t>(flags[1]);
+  volatile int* abort_flag = flags;
+  pdl_trigger();
+
+  PairOps pf{};
+  if (warp == 0) {
+    if (lane == 0) {   // the K-slice of W_O: S weight tiles, requested before the wait (weights are static)
+      const uint64_t wpol = l2_evict_first();
+      for (int j = 0; j < S; ++j) {
+        mbar_expect_tx(full0 + 8 * j, a_bytes);
+        tma_load_2d_stream(smem_u32(smem + static_cast<size_t>(j) * stage_bytes), &a.mapA[0], (rank * S + j) * kBK,
+                           wt * kWRows, full0 + 8 * j, wpol);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      const uint32_t idesc = idesc_bf16(kWRows, NT);
+      bool ok = true;
+      for (int j = 0; j < S && ok; ++j) {
+        if (!wait_bar(full0 + 8 * j, 0, abort_flag, a.err)) { ok = false; break; }
+        tc_fence_after();
+        const uint32_t abase = smem_u32(smem + static_cast<size_t>(j) * stage_bytes);
+        const uint64_t ad = sw128_desc(abase), bd = sw128_desc(abase + a_bytes);
+#pragma unroll
+        for (int kk = 0; kk < kBK / 16; ++kk) mma_bf16(tmem, ad + 2 * kk, bd + 2 * kk, idesc, (j > 0 || kk > 0) ? 1u : 0u);
+        mma_commit(empty0 + 8 * j);
+      }
+      if (ok) mma_commit(tfull0);
+      mma_commit(drain);
+      wait_bar_budget(drain, 0, kDrainCycles);
+    }
+  } else {
+    // ---- attention of KV head `rank` for the M rows (warps 2-9) ----
+    const int aw = warp - 2, at = threadIdx.x - 64;   // attention warp 0..7, thread 0..255
+    const int g8 = lane >> 2, t4 = lane & 3;
+    const int Hkv = a.n_kv_heads, kvh = rank;
+    const int seq = *a.attn_seq;
+    const int len = a.attn_pre_len[seq];
+    const int row_end = a.kv_bt_stride * 16;
+    const int stable = min(max(0, len + a.attn_pre_stable), row_end);
+    const int ctx_hi = min(max(stable, len + a.attn_pre_stable + a.attn_pre_fresh), row_end);
+    const int P = ((ctx_hi + 8 * kAoSub - 1) / (8 * kAoSub)) * kAoSub;      // positions per warp
+    const int w_lo = aw * P, w_hi = min(w_lo + P, ctx_hi);
+    const int nsub_all = w_hi > w_lo ? (w_hi - w_lo + kAoSub - 1) / kAoSub : 0;
+    int* blk = sBlk + aw * kAoMaxBlk;
+    for (int i = lane; i < (P >> 4) && i < kAoMaxBlk; i += 32) {
+      const int b16 = (w_lo >> 4) + i;
+      blk[i] = b16 < a.kv_bt_stride ? a.kv_table[static_cast<size_t>(seq) * a.kv_bt_stride + b16] : 0;
+    }
+    __syncwarp();
+    const bf16* layer_base = a.kv_pool + static_cast<size_t>(a.layer) * a.kv_n_blocks * 2 * Hkv * 16 * 64 +
+                             static_cast<size_t>(kvh) * 16 * 64;
+    const size_t blk_stride = static_cast<size_t>(2) * Hkv * 16 * 64;
+    unsigned char* wkv = sKV + static_cast<size_t>(aw) * kAoWarpBytes;
+    // rows p in [p_from, p_to) of sub-tile j -> slot j % kAoBuf: loaded below `valid_end`, else zero
+    auto issue = [&](int j, int p_from, int p_to, int valid_end) {
+      bf16* dK = reinterpret_cast<bf16*>(wkv + (j % kAoBuf) * 2 * kAoSub * kAoKS * 2);
+      bf16* dV = dK + kAoSub * kAoKS;
+      const int t0 = w_lo + j * kAoSub;
+#pragma unroll
+      for (int u = 0; u < kAoSub * 8 / 32; ++u) {
+        const int idx = lane + 32 * u, t = idx >> 3, c = idx & 7;
+        const int p = t0 + t;
+        if (p < p_from || p >= p_to) continue;
+        const bool ok = p < valid_end;
+        const bf16* src = layer_base;
+        if (ok) src += static_cast<size_t>(blk[(p - w_lo) >> 4]) * blk_stride + static_cast<size_t>(p & 15) * 64 + c * 8;
+        ao_cp16(smem_u32(dK + t * kAoKS + c * 8), src, ok);
+        ao_cp16(smem_u32(dV + t * kAoKS + c * 8), ok ? src + Hkv * 16 * 64 : layer_base, ok);
+      }
+    };
+    const int pre_hi = max(w_lo, min(stable, w_hi));
+    for (int j = 0; j < kAoBuf && j < nsub_all; ++j) issue(j, w_lo, pre_hi, pre_hi);   // rows written before the step
+    pdl_wait();
+    for (int j = 0; j < kAoBuf; ++j) {                // the step's own rows, then one group per sub-tile
+      if (j < nsub_all) issue(j, pre_hi, INT_MAX, w_hi);
+      ao_commit();
+    }
+    if (at < 128) pf = first_pair_ops(a, rank, sp, NT, first_tile, at);
+    {  // queries of the group's rows on this KV head -> bf16, row positions
+      const int qv = at >> 4, c4 = at & 15;
+      float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (qv < nqv)
+        v = __ldcg(reinterpret_cast<const float4*>(a.attn_q + (static_cast<size_t>(qv / G) * a.n_heads + kvh * G + qv % G) * 64) + c4);
+      *reinterpret_cast<uint2*>(sQ + qv * kAoKS + c4 * 4) = make_uint2(ao_pack(v.x, v.y), ao_pack(v.z, v.w));
+      if (at < 16) sPos[at] = at < nqv ? __ldcg(a.row_pos + at / G) : -1;
+    }
+    named_bar_attn();
+    int pmax = -1;
+#pragma unroll
+    for (int i = 0; i < 16; ++i) pmax = max(pmax, sPos[i]);
+    if (at == 0 && pmax + 1 > ctx_hi && a.err) atomicOr(a.err, static_cast<unsigned>(ERR_RANGE));
+    const int hi = min(pmax + 1, w_hi);
+    const int nsub = hi > w_lo ? (hi - w_lo + kAoSub - 1) / kAoSub : 0;
+    const int pa = sPos[g8], pb = sPos[g8 + 8];
+    uint32_t qa[4][4];
+#pragma unroll
+    for (int kk = 0; kk < 4; ++kk) {
+      const bf16* q0 = sQ + g8 * kAoKS + kk * 16 + 2 * t4;
+      qa[kk][0] = ao_ld_u32(q0);
+      qa[kk][1] = ao_ld_u32(q0 + 8 * kAoKS);
+      qa[kk][2] = ao_ld_u32(q0 + 8);
+      qa[kk][3] = ao_ld_u32(q0 + 8 * kAoKS + 8);
+    }
+    float m_a = -INFINITY, m_b = -INFINITY, l_a = 0.f, l_b = 0.f;
+    float acc[8][4];
+#pragma unroll
+    for (int dt = 0; dt < 8; ++dt) acc[dt][0] = acc[dt][1] = acc[dt][2] = acc[dt][3] = 0.f;
+    for (int j = 0; j < nsub; ++j) {
+      ao_wait<kAoBuf - 1>();
+      __syncwarp();
+      const bf16* sK = reinterpret_cast<const bf16*>(wkv + (j % kAoBuf) * 2 * kAoSub * kAoKS * 2);
+      const bf16* sV = sK + kAoSub * kAoKS;
+      float sc[2][4];
+#pragma unroll
+      for (int nt = 0; nt < 2; ++nt) {
+        float c[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int kk = 0; kk < 4; ++kk) {
+          const bf16* kp = sK + (nt * 8 + g8) * kAoKS + kk * 16 + 2 * t4;
+          ao_mma(c, qa[kk][0], qa[kk][1], qa[kk][2], qa[kk][3], ao_ld_u32(kp), ao_ld_u32(kp + 8));
+        }
+        const int pc = w_lo + j * kAoSub + nt * 8 + 2 * t4;
+        sc[nt][0] = pc <= pa ? c[0] * 0.125f : -INFINITY;
+        sc[nt][1] = pc + 1 <= pa ? c[1] * 0.125f : -INFINITY;
+        sc[nt][2] = pc <= pb ? c[2] * 0.125f : -INFINITY;
+        sc[nt][3] = pc + 1 <= pb ? c[3] * 0.125f : -INFINITY;
+      }
+      float mx_a = fmaxf(fmaxf(sc[0][0], sc[0][1]), fmaxf(sc[1][0], sc[1][1]));
+      float mx_b = fmaxf(fmaxf(sc[0][2], sc[0][3]), fmaxf(sc[1][2], sc[1][3]));
+      mx_a = fmaxf(mx_a, __shfl_xor_sync(0xffffffffu, mx_a, 1));
+      mx_a = fmaxf(mx_a, __shfl_xor_sync(0xffffffffu, mx_a, 2));
+      mx_b = fmaxf(mx_b, __shfl_xor_sync(0xffffffffu, mx_b, 1));
+      mx_b = fmaxf(mx_b, __shfl_xor_sync(0xffffffffu, mx_b, 2));
+      const float mn_a = fmaxf(m_a, mx_a), mn_b = fmaxf(m_b, mx_b);
+      const float mu_a = mn_a == -INFINITY ? 0.f : mn_a, mu_b = mn_b == -INFINITY ? 0.f : mn_b;
+      const float cr_a = __expf(m_a - mu_a), cr_b = __expf(m_b - mu_b);
+      m_a = mn_a;
+      m_b = mn_b;
+      uint32_t pk[4];
+      float ps_a = 0.f, ps_b = 0.f;
+#pragma unroll
+      for (int nt = 0; nt < 2; ++nt) {
+        const __nv_bfloat162 ha = __floats2bfloat162_rn(__expf(sc[nt][0] - mu_a), __expf(sc[nt][1] - mu_a));
+        const __nv_bfloat162 hb = __floats2bfloat162_rn(__expf(sc[nt][2] - mu_b), __expf(sc[nt][3] - mu_b));
+        ps_a += __low2float(ha) + __high2float(ha);
+        ps_b += __low2float(hb) + __high2float(hb);
+        pk[2 * nt] = *reinterpret_cast<const uint32_t*>(&ha);
+        pk[2 * nt + 1] = *reinterpret_cast<const uint32_t*>(&hb);
+      }
+      l_a = l_a * cr_a + ps_a;
+      l_b = l_b * cr_b + ps_b;
+      const int vrow = (lane & 7) + ((lane >> 3) & 1) * 8;
+#pragma unroll
+      for (int dt = 0; dt < 8; ++dt) {
+        acc[dt][0] *= cr_a; acc[dt][1] *= cr_a;
+        acc[dt][2] *= cr_b; acc[dt][3] *= cr_b;
+        uint32_t v0, v1;
+        ao_ldsm_x2_t(smem_u32(sV + vrow * kAoKS + dt * 8), v0, v1);
+        ao_mma(acc[dt], pk[0], pk[1], pk[2], pk[3], v0, v1);
+      }
+      __syncwarp();                                    // every lane is done with this slot
+      if (j + kAoBuf < nsub) issue(j + kAoBuf, w_lo, INT_MAX, w_hi);
+      ao_commit();
+    }
+    ao_wait<0>();
+    __syncwarp();
+    l_a += __shfl_xor_sync(0xffffffffu, l_a, 1);
+    l_a += __shfl_xor_sync(0xffffffffu, l_a, 2);
+    l_b += __shfl_xor_sync(0xffffffffu, l_b, 1);
+    l_b += __shfl_xor_sync(0xffffffffu, l_b, 2);
+    // this warp's partial over its positions, over its own K/V buffers
+    float* pacc = reinterpret_cast<float*>(wkv);        // [16 rows][kAoAS]
+#pragma unroll
+    for (int dt = 0; dt < 8; ++dt) {
+      *reinterpret_cast<float2*>(pacc + g8 * kAoAS + dt * 8 + 2 * t4) = make_float2(acc[dt][0], acc[dt][1]);
+      *reinterpret_cast<float2*>(pacc + (g8 + 8) * kAoAS + dt * 8 + 2 * t4) = make_float2(acc[dt][2], acc[dt][3]);
+    }
+    if (t4 == 0) {
+      sML[(aw * 16 + g8) * 2] = m_a;
+      sML[(aw * 16 + g8) * 2 + 1] = l_a;
+      sML[(aw * 16 + g8 + 8) * 2] = m_b;
+      sML[(aw * 16 + g8 + 8) * 2 + 1] = l_b;
+    }
+    named_bar_attn();
+    // merge over the 8 warps (in warp order) -> the token operand: stage s holds head s of the KV
+    // head, token row t at byte t * 128 of the stage's operand, 16-byte chunk ch at (ch ^ (t & 7))
+    for (int e = at; e < NT * S * 8; e += 256) {
+      const int ch = e & 7, sgi = (e >> 3) % S, t = (e >> 3) / S;
+      uint4 pkd = make_uint4(0u, 0u, 0u, 0u);
+      if (t < M) {
+        const int qv = t * G + sgi;
+        float mw[8], M_ = -INFINITY;
+#pragma unroll
+        for (int w = 0; w < 8; ++w) {
+          mw[w] = sML[(w * 16 + qv) * 2];
+          M_ = fmaxf(M_, mw[w]);
+        }
+        float L = 0.f, o[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int w = 0; w < 8; ++w) {
+          const float ww = __expf(mw[w] - M_);
+          L += sML[(w * 16 + qv) * 2 + 1] * ww;
+          const float* src = reinterpret_cast<const float*>(sKV + static_cast<size_t>(w) * kAoWarpBytes) + qv * kAoAS + ch * 8;
+#pragma unroll
+          for (int d = 0; d < 8; ++d) o[d] = fmaf(ww, src[d], o[d]);
+        }
+        const float inv = L > 0.f ? 1.f / L : 0.f;
+        pkd = make_uint4(ao_pack(o[0] * inv, o[1] * inv), ao_pack(o[2] * inv, o[3] * inv), ao_pack(o[4] * inv, o[5] * inv),
+                         ao_pack(o[6] * inv, o[7] * inv));
+      }
+      *reinterpret_cast<uint4*>(smem + static_cast<size_t>(sgi) * stage_bytes + a_bytes + t * 128 + ((ch ^ (t & 7)) << 4)) = pkd;
+    }
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");   // the operand is read by the tensor cores
+    named_bar_attn();
+    if (at == 0)
+      for (int j = 0; j < S; ++j) mbar_arrive(full0 + 8 * j);
+    if (warp < 6)                                       // warps 2-5: the split-K epilogue
+      splitk_epilogue(a, SplitK{smem, recv, rs, flags, tfull0, rbar, tmem, rank, sp, npmax, NT, first_tile}, warp, lane, pf);
+  }
+  if (warp < 2 || warp >= 6) {                          // everyone but the epilogue takes its half of the cluster barrier
+    __syncwarp();
+    cluster_wait();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 1) tmem_dealloc(tmem, 32);
 }
 
 // ------------------------------------------------------------------------------ host side
@@ -706,6 +1074,7 @@ bool encode_weight_map(void* map, const void* w, int rows, int K, int box_rows) 
 int sm_count_cached() { return sm_count(); }
 
 int gemm_norm_parts(const GemmArgs& g) {
+  if (g.attn_q) return (g.seg[0].rows / kWRows) * g.n_kv_heads;   // fused attention: sp = H_kv
   const int NT = gemm_tc_token_tile(g.M);
   const int n_wtiles = n_out_rows(g) / kWRows;
   const int tiles = n_wtiles * ((g.M + NT - 1) / NT);
@@ -731,7 +1100,63 @@ bool gemm_tc_supported(const GemmArgs& g) {
   return true;
 }
 
+// Shared memory of the fused attention kernel for S k-blocks per rank and token tile NT.
+size_t gemm_attn_smem(int S, int NT, int sp) {
+  const size_t stage_bytes = static_cast<size_t>(kWRows + NT) * kBK * 2;
+  const size_t recv = static_cast<size_t>(sp) * ((64 + sp - 1) / sp) * 2 * NT * 4;
+  return 1024 + S * stage_bytes + recv + 8 * (2 * S + 6) + 16 * 4 + 16 * 4 + kAoAttnBytes;
+}
+
+bool gemm_attn_supported(const GemmArgs& g) {
+  if (!g.attn_q || !g.attn_seq || !g.attn_pre_len || !g.kv_pool || !g.kv_table || !g.row_pos) return false;
+  if (g.epi != EPI_ADD || g.nseg != 1 || g.norm_ssq_in || g.head_dim != 64) return false;
+  if (g.n_kv_heads < 2 || g.n_kv_heads > 8 || g.n_heads % g.n_kv_heads || g.K != g.n_heads * 64) return false;
+  if (g.norm_out && (!g.norm_gamma || !g.norm_ssq_out)) return false;
+  if (g.tap_mask && (!g.norm_out || !g.tap)) return false;
+  const int G = g.n_heads / g.n_kv_heads;
+  if (g.M < 1 || g.M * G > 16 || g.seg[0].rows % kWRows != 0) return false;
+  if (g.kv_bt_stride < 1 || g.kv_bt_stride * 16 > 8 * kAoMaxBlk * 16) return false;   // context <= 4096
+  const int tiles = g.seg[0].rows / kWRows;
+  if (tiles * g.n_kv_heads > sm_count()) return false;   // one CTA per SM, one wave
+  return gemm_attn_smem(G, gemm_tc_token_tile(g.M), g.n_kv_heads) <= static_cast<size_t>(kSmemBudget);
+}
+
+cudaError_t gemm_attn(const GemmArgs& g, unsigned* err, cudaStream_t st) {
+  TcArgs a{};
+  a.nseg = 1;
+  a.seg_rows[0] = g.seg[0].rows;
+  if (!weight_map(&a.mapA[0], g.seg[0].w, g.seg[0].rows, g.K, kWRows)) return cudaErrorInvalidValue;
+  a.NT = gemm_tc_token_tile(g.M);
+  a.M = g.M; a.K = g.K; a.KB = g.K / kBK;
+  a.n_wtiles = g.seg[0].rows / kWRows;
+  a.n_ttiles = 1;
+  a.tiles = a.n_wtiles;
+  a.epi = EPI_ADD; a.out = g.out; a.ldo = g.ldo;
+  a.bias = g.bias; a.ld_bias = g.ld_bias; a.row_seq = g.row_seq;
+  a.err = err;
+  a.kv_pool = static_cast<bf16*>(g.kv_pool); a.kv_table = g.kv_table;
+  a.kv_bt_stride = g.kv_bt_stride; a.kv_n_blocks = g.kv_n_blocks; a.n_heads = g.n_heads;
+  a.n_kv_heads = g.n_kv_heads; a.head_dim = 64; a.layer = g.layer; a.row_pos = g.row_pos;
+  a.norm_gamma = static_cast<const bf16*>(g.norm_gamma); a.norm_out = static_cast<bf16*>(g.norm_out);
+  a.norm_ssq_out = g.norm_ssq_out; a.tap = g.tap; a.tap_row = g.tap_row; a.tap_mask = g.tap_mask;
+  a.ld_ssq = g.ld_ssq;
+  a.attn_q = g.attn_q; a.attn_seq = g.attn_seq; a.attn_pre_len = g.attn_pre_len;
+  a.attn_pre_stable = g.attn_pre_stable; a.attn_pre_fresh = g.attn_pre_fresh;
+  a.sp = g.n_kv_heads;
+  a.stages = g.n_heads / g.n_kv_heads;
+  const size_t smem = gemm_attn_smem(a.stages, a.NT, a.sp);
+  static bool configured = false;
+  if (!configured) {
+    cudaError_t e = cudaFuncSetAttribute(gemm_attn_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBudget);
+    if (e != cudaSuccess) return e;
+    configured = true;
+  }
+  return launch_pdl_cluster(gemm_attn_kernel, dim3(static_cast<unsigned>(a.tiles * a.sp)), dim3(kAoThreads), smem, st,
+                            a.sp, a);
+}
+
 cudaError_t gemm_tc(const GemmArgs& g, unsigned* err, cudaStream_t st) {
+  if (g.attn_q) return gemm_attn(g, err, st);
   TcArgs a{};  // built on the host; passed by value as the kernel parameter
   a.nseg = g.nseg;
   a.swiglu = (g.epi == EPI_SWIGLU) ? 1 : 0;

@@ -111,6 +111,16 @@ struct GemmArgs {
   int norm_parts, norm_d;
   float norm_eps;
   int ld_ssq;
+  // Fused decode attention (tensor-core path, gemm_attn_supported): with attn_q set, the token
+  // operand x is not read; it is the causal attention output of the M rows, all of sequence
+  // *attn_seq (a plan table written before the step), computed in the kernel from attn_q
+  // [M, n_heads, 64] f32 and the paged cache (kv_* fields, layer, row_pos). Cache positions below
+  // attn_pre_len[seq] + attn_pre_stable were written before the step; every row lies below that
+  // + attn_pre_fresh, and the cache rows up to there hold finite values.
+  const float* attn_q;
+  const int* attn_seq;
+  const int* attn_pre_len;
+  int attn_pre_stable, attn_pre_fresh;
 };
 // Number of sums-of-squares slices a producer launch with these arguments writes.
 int gemm_norm_parts(const GemmArgs& a);
@@ -118,6 +128,8 @@ int gemm_norm_parts(const GemmArgs& a);
 // to the CUDA-core kernel (gemm_simt.cu).
 cudaError_t gemm(const GemmArgs& a, cudaStream_t st);
 bool gemm_tc_supported(const GemmArgs& a);
+// Whether the fused decode attention (attn_q) can run for these arguments on this device.
+bool gemm_attn_supported(const GemmArgs& a);
 cudaError_t gemm_tc(const GemmArgs& a, unsigned* err, cudaStream_t st);
 int gemm_tc_token_tile(int M);
 cudaError_t gemm_simt(const GemmArgs& a, cudaStream_t st);

@@ -28,7 +28,7 @@ EXPORTS = ["sd2_init", "sd2_prefill", "sd2_step", "sd2_accept", "sd2_check", "sd
            "sd2_set_graphs", "sd2_debug_buffer", "sd2_profile", "sd2_profile_read", "sd2_accept_workspace_bytes",
            "sd2_accept_logits", "sd2_steer_workspace_bytes", "sd2_steer", "sd2_swiglu_steered",
            "sd2_accept_logits_noalloc", "sd2_gemm", "sd2_set_gemm_impl", "sd2_stage_timing", "sd2_stage_read",
-           "sd2_set_drafter_chain", "sd2_attention"]
+           "sd2_set_drafter_chain", "sd2_attention", "sd2_set_fused_attention"]
 
 
 class LMConfig(ctypes.Structure):
@@ -95,6 +95,7 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
                                   c_int32, c_void_p, c_void_p, c_void_p, c_void_p, c_int32, c_int32, c_int32, c_int32,
                                   c_void_p, c_int32, c_int32, c_void_p, c_void_p, c_void_p]
     lib.sd2_set_drafter_chain.argtypes = [c_void_p, c_int32]
+    lib.sd2_set_fused_attention.argtypes = [c_void_p, c_int32]
     lib.sd2_accept_logits_noalloc.argtypes = [c_void_p, c_void_p, c_int32, c_void_p, c_void_p, c_int32, c_int32,
                                               c_int32, c_uint64, c_uint32, c_void_p, c_void_p, c_void_p]
     for name in EXPORTS:
@@ -245,6 +246,10 @@ class SD2Engine:
     def set_drafter_chain(self, enable: bool):
         """Drafter steps as one persistent kernel, or one kernel per projection (the default)."""
         self._call(self.lib.sd2_set_drafter_chain(self.ctx, 1 if enable else 0))
+
+    def set_fused_attention(self, enable: bool):
+        """Batch-1 decode: attention inside the O projection, or its own kernel (the default)."""
+        self._call(self.lib.sd2_set_fused_attention(self.ctx, 1 if enable else 0))
 
     def stage_timing(self, enable: bool):
         """Record stage events inside the captured step (steering, k drafter steps, verify)."""

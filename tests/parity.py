@@ -53,7 +53,7 @@ class ParityReport:
 
 
 def run(work, vw, dw, st, prompts, temps, seed, n_steps, max_ctx=None, graphs=True, tol=TOL,
-        check_taps=True, gemm_impl=0, steering=True, chain=False) -> ParityReport:
+        check_taps=True, gemm_impl=0, steering=True, chain=False, fused_attention=False) -> ParityReport:
     """Run prefill + n_steps iterations on the GPU and check each against the oracle.
 
     steering=False runs the engine's pretrained-drafter mode (no steering stage, no bias); the
@@ -67,6 +67,7 @@ def run(work, vw, dw, st, prompts, temps, seed, n_steps, max_ctx=None, graphs=Tr
     eng.set_graphs(graphs)
     eng.set_gemm_impl(gemm_impl)
     eng.set_drafter_chain(chain)
+    eng.set_fused_attention(fused_attention)
     rep = ParityReport()
     try:
         first = eng.prefill(prompts, temps, seed).cpu().tolist()

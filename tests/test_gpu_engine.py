@@ -13,15 +13,17 @@ from paper_2511_09844_gb300 import workloads as W
 pytestmark = pytest.mark.gpu
 
 
-@pytest.mark.parametrize("gemm_impl,chain", [(0, True), (0, False), (1, False)])
+@pytest.mark.parametrize("gemm_impl,chain,fused", [(0, True, False), (0, False, False), (0, False, True), (1, False, False)])
 @pytest.mark.parametrize("temp", [0.0, 1.0])
-def test_tiny_single_sequence(temp, gemm_impl, chain):
+def test_tiny_single_sequence(temp, gemm_impl, chain, fused):
     """gemm_impl 0: tensor-core GEMM with fused epilogues, the drafter steps as one persistent
-    kernel (chain) or one kernel per projection; 1: CUDA-core GEMM + separate kernels."""
+    kernel (chain) or one kernel per projection, the decode attention in its own kernel or inside
+    the O projection (fused: both tiny models take it, hd 64); 1: CUDA-core GEMM + separate kernels."""
     work = parity.tiny_work()
     vw, dw, st = parity.tiny_weights(work)
     prompts = W.make_prompts(work.verifier.vocab, 1, (32, 32), seed=7)
-    rep = parity.run(work, vw, dw, st, prompts, [temp], seed=1234, n_steps=8, gemm_impl=gemm_impl, chain=chain)
+    rep = parity.run(work, vw, dw, st, prompts, [temp], seed=1234, n_steps=8, gemm_impl=gemm_impl, chain=chain,
+                     fused_attention=fused)
     assert rep.blocks == 8 and rep.decisions > 8 * work.k
 
 

@@ -65,6 +65,17 @@ def test_full_width_slice_drafter_chain():
     assert rep.blocks == 2
 
 
+def test_full_width_slice_attention_in_o_projection():
+    """The 1B drafter's decode attention inside its O projection (16 tiles x 8 KV heads) at the 8B/1B
+    pair's widths; the 8B verifier (hd 128) keeps the attention kernel."""
+    work = _one_layer(W.WORKLOADS["llama8b_1b"])
+    work = dataclasses.replace(work, drafter=dataclasses.replace(W.WORKLOADS["llama8b_1b"].drafter, n_layers=2))
+    vw, dw, st = _weights(work, 29)
+    prompts = W.make_prompts(work.verifier.vocab, work.batch, work.prompt_len, seed=20)
+    rep = parity.run(work, vw, dw, st, prompts, _temps(work), seed=8, n_steps=2, fused_attention=True)
+    assert rep.blocks == 2
+
+
 def test_long_context_verify_16k():
     """8B-shaped verify at a 16384-token context, batch 1 (one-layer slice, k = 1)."""
     work = _one_layer(W.WORKLOADS["llama8b_1b"], k=1, prompt_len=(16384, 16384))
