@@ -367,11 +367,14 @@ def barrier(world):
 
 
 def reduce_max_sum(ms, count, world):
+    """(max of ms over the ranks, sum of count over the ranks): the job's time is its slowest
+    replica's, its work every replica's."""
     if world == 1:
         return ms, count
     import torch.distributed as dist
-    t = torch.tensor([ms], dtype=torch.float64, device="cuda")
-    c = torch.tensor([count], dtype=torch.float64, device="cuda")
+    device = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([ms], dtype=torch.float64, device=device)
+    c = torch.tensor([count], dtype=torch.float64, device=device)
     dist.all_reduce(t, op=dist.ReduceOp.MAX)
     dist.all_reduce(c, op=dist.ReduceOp.SUM)
     return float(t.item()), int(c.item())
