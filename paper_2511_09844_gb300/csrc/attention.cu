@@ -150,17 +150,25 @@ __global__ void __launch_bounds__(kThreads, 2) attn_kernel(const AttnArgs a) {
   // kernel) and, in a decode step, the sequence's pre-step length.
   const int r0 = a.grp_row0[g], nr = a.grp_nrows[g], seq = a.grp_seq[g];
   const int nqv = nr * G;
-  const int lo = split * a.chunk;
-  const int nblk = min(a.chunk >> 4, a.kv.bt_stride - (lo >> 4));
+  // A decode step knows, before the wait, that its rows lie below len + pre_stable + pre_fresh: the
+  // splits share that range (whole tiles, at most a.chunk each) instead of the planned maximum, so
+  // no split is empty while another holds several tiles.
+  const bool early = a.pre_len != nullptr;
+  const int len = early ? a.pre_len[seq] : 0;
+  int chunk = a.chunk;
+  if (early) {
+    const int per = (len + a.pre_stable + a.pre_fresh + NS - 1) / NS;
+    chunk = min(a.chunk, max(kTile, ((per + kTile - 1) / kTile) * kTile));
+  }
+  const int lo = split * chunk;
+  const int nblk = min(chunk >> 4, a.kv.bt_stride - (lo >> 4));
   const int row_end = lo + nblk * 16;               // positions the split's block ids cover
   {
     const int* table = a.kv.table + static_cast<size_t>(seq) * a.kv.bt_stride + (lo >> 4);
     for (int i = tid; i < nblk; i += kThreads) sBlk[i] = table[i];
   }
-  const bool early = a.pre_len != nullptr;
   int pre_hi = lo, fresh_hi = lo;                   // rows [lo, pre_hi) early, [pre_hi, fresh_hi) after the wait
   if (early) {
-    const int len = a.pre_len[seq];
     pre_hi = min(max(lo, len + a.pre_stable), row_end);
     fresh_hi = min(max(pre_hi, len + a.pre_stable + a.pre_fresh), row_end);
   }
@@ -196,7 +204,7 @@ __global__ void __launch_bounds__(kThreads, 2) attn_kernel(const AttnArgs a) {
       cp_async16(smem_u32(dV + t * KS + c * 8), ok ? src + Hkv * head_stride : layer_base, ok);
     }
   };
-  const int nb = C::nbuf(a.chunk);
+  const int nb = C::nbuf(chunk);
   if (early)
     for (int i = 0; i < nb; ++i) issue_rows(i, lo, pre_hi, pre_hi);
   pdl_wait();
@@ -232,7 +240,7 @@ __global__ void __launch_bounds__(kThreads, 2) attn_kernel(const AttnArgs a) {
   const int pmax = max(sPmax[0], sPmax[1]);
   // A split that starts after every row of the group has no tiles; it still takes part in the
   // merge with an empty partial.
-  const int hi = min(lo + a.chunk, pmax + 1);
+  const int hi = min(lo + chunk, pmax + 1);
   const int ntiles = hi > lo ? (hi - lo + kTile - 1) / kTile : 0;
   const int nmt = (nqv + 15) >> 4;
   if (early) {
