@@ -104,7 +104,11 @@ __device__ __forceinline__ float bits_to_u01(uint32_t x) {
 
 __device__ __forceinline__ float exp_cw(float t) {
   if (t < -80.0f) return 0.0f;
-  const float n = rintf(__fmul_rn(t, 0x1.715476p+0f));
+  // n = rint(t / ln2) by adding and subtracting 1.5 * 2^23 (exact round-half-even for |t / ln2| <
+  // 2^22; here t <= 0 and t / ln2 >= -116); the integer n sits in the low mantissa bits of the sum.
+  const float nm = __fadd_rn(__fmul_rn(t, 0x1.715476p+0f), 0x1.8p+23f);
+  const float n = __fsub_rn(nm, 0x1.8p+23f);
+  const int ni = __float_as_int(nm) - 0x4B400000;
   float r = __fsub_rn(t, __fmul_rn(n, 0x1.62e400p-1f));
   r = __fsub_rn(r, __fmul_rn(n, 0x1.7f7d1cp-20f));
   float p = 0x1.a01a02p-13f;
@@ -116,7 +120,7 @@ __device__ __forceinline__ float exp_cw(float t) {
   p = __fadd_rn(__fmul_rn(p, r), 1.0f);
   p = __fadd_rn(__fmul_rn(p, r), 1.0f);
   // p in [0.7, 1.5] and n >= -116: adding n to the exponent field is the exact scaling by 2^n.
-  return __int_as_float(__float_as_int(p) + static_cast<int>(n) * (1 << 23));
+  return __int_as_float(__float_as_int(p) + ni * (1 << 23));
 }
 
 __device__ __forceinline__ float log_at(float x) {
@@ -137,9 +141,27 @@ __device__ __forceinline__ float log_at(float x) {
   return __fadd_rn(__fmul_rn(ef, 0x1.62e400p-1f), __fadd_rn(__fmul_rn(ef, 0x1.7f7d1cp-20f), ln_m));
 }
 
-// e in (0, ~1] to the fixed point floor(e * 2^45) used by the exact softmax normaliser.
+// e in [0, 1] to the fixed point floor(e * 2^45) used by the exact softmax normaliser, from the
+// bits of e: with e = m 2^(x - 150) (24-bit significand m), e 2^45 = m 2^(x - 105), so the floor is
+// m shifted left by x - 105 or right by 105 - x (integer shifts only: a 64-bit conversion would
+// run on the FP64 pipe).
+// The same value as two exact 32-bit parts, floor(e 2^45) = hi 2^23 + lo with hi = floor(e 2^22)
+// (<= 2^22) and lo = floor(e 2^45 - hi 2^23) (< 2^23), in fp32 operations that are all exact: the
+// floors are round-toward-zero additions of 2^23 (the integer is read from the sum's bits), and
+// e 2^45 - hi 2^23 is a multiple of the ulp of e 2^45 below 2^23. Sums of up to 2^9 parts fit.
+__device__ __forceinline__ void fixed45_parts(float e, uint32_t& hi, uint32_t& lo) {
+  const float h = __fadd_rz(__fmul_rn(e, 0x1p22f), 0x1p23f);
+  hi = __float_as_uint(h) - 0x4B000000u;
+  const float r = __fmaf_rn(-__fsub_rn(h, 0x1p23f), 0x1p23f, __fmul_rn(e, 0x1p45f));
+  lo = __float_as_uint(__fadd_rz(r, 0x1p23f)) - 0x4B000000u;
+}
 __device__ __forceinline__ unsigned long long fixed45(float e) {
-  return __float2ull_rz(__fmul_rn(e, 0x1p45f));
+  const uint32_t b = __float_as_uint(e);
+  const int x = static_cast<int>(b >> 23);                       // biased exponent (e >= 0)
+  const unsigned long long m = static_cast<unsigned long long>((b & 0x7FFFFFu) | 0x800000u);
+  const unsigned long long up = m << min(max(x - 105, 0), 40);
+  const unsigned long long dn = m >> min(max(105 - x, 0), 63);
+  return x == 0 ? 0ull : (x >= 105 ? up : dn);
 }
 
 // ------------------------------------------------------------------------------------------

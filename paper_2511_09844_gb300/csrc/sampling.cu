@@ -128,22 +128,43 @@ __global__ void __launch_bounds__(kThreads) rowmax_kernel(const T* target, const
   const float invT = greedy ? 1.f : inv_temp(t);
   const T* row = (rr.is_draft ? draft : target) + rr.offset;
   const int lo = blockIdx.y * kStatsPerCta, hi = min(V, lo + kStatsPerCta);
-  unsigned long long best = 0;
-  bool bad = false;
+  // this thread's (max, first index of it) in 32 bits: its entries come in increasing index order,
+  // so a strictly greater value is the only update (+0 and -0 compare equal, as the packed key
+  // folds them); packed once for the exact cross-thread maximum
+  // Each group of 8 is reduced with fmaxf first; only a group that beats the running maximum is
+  // searched for the first index of its maximum. Non-finite entries show as a NaN in sum(z - z).
+  float best_s = -INFINITY;
+  int best_i = -1;
+  float nf = 0.f;
 #pragma unroll 2
   for (int v = lo + threadIdx.x * 8; v < hi; v += kThreads * 8) {
     float z[8];
     const int n = min(8, hi - v);
     load8<T>(row, v, n, z);
+    float s[8];
+    if (n == 8) {
 #pragma unroll
-    for (int j = 0; j < 8; ++j) {
-      if (j >= n) break;
-      bad |= !isfinite(z[j]);
-      const float s = greedy ? z[j] : __fmul_rn(z[j], invT);
-      const unsigned long long key = pack_key(s, v + j);
-      best = key > best ? key : best;
+      for (int j = 0; j < 8; ++j) {
+        nf += __fsub_rn(z[j], z[j]);
+        s[j] = greedy ? z[j] : __fmul_rn(z[j], invT);
+      }
+    } else {
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        nf += j < n ? __fsub_rn(z[j], z[j]) : 0.f;
+        s[j] = j < n ? (greedy ? z[j] : __fmul_rn(z[j], invT)) : -INFINITY;
+      }
+    }
+    const float g = fmaxf(fmaxf(fmaxf(s[0], s[1]), fmaxf(s[2], s[3])), fmaxf(fmaxf(s[4], s[5]), fmaxf(s[6], s[7])));
+    if (g > best_s || best_i < 0) {
+      int jj = 7;
+#pragma unroll
+      for (int j = 7; j >= 0; --j) jj = (j < n && s[j] == g) ? j : jj;
+      if (g > best_s || best_i < 0) { best_s = g; best_i = v + jj; }
     }
   }
+  const bool bad = !(nf == 0.f);
+  unsigned long long best = best_i < 0 ? 0ull : pack_key(best_s, static_cast<uint32_t>(best_i));
   best = block_max_u64(best, red);
   if (threadIdx.x == 0) atomicMax(&rowkey[blockIdx.x], best);
   if (bad) atomicOr(err, static_cast<unsigned>(ERR_NONFINITE));
@@ -166,7 +187,7 @@ __global__ void __launch_bounds__(kThreads) rowsum_kernel(const T* target, const
   const float m = packed_key(rowkey[blockIdx.x]);
   const T* row = (rr.is_draft ? draft : target) + rr.offset;
   const int lo = blockIdx.y * kStatsPerCta, hi = min(V, lo + kStatsPerCta);
-  unsigned long long acc = 0;
+  uint32_t acc_hi = 0, acc_lo = 0;        // at most 64 entries per thread: no overflow
 #pragma unroll 2
   for (int v = lo + threadIdx.x * 8; v < hi; v += kThreads * 8) {
     float z[8];
@@ -174,8 +195,14 @@ __global__ void __launch_bounds__(kThreads) rowsum_kernel(const T* target, const
     load8<T>(row, v, n, z);
 #pragma unroll
     for (int j = 0; j < 8; ++j)
-      if (j < n) acc += fixed45(exp_cw(__fsub_rn(__fmul_rn(z[j], invT), m)));
+      if (j < n) {
+        uint32_t ph, pl;
+        fixed45_parts(exp_cw(__fsub_rn(__fmul_rn(z[j], invT), m)), ph, pl);
+        acc_hi += ph;
+        acc_lo += pl;
+      }
   }
+  unsigned long long acc = (static_cast<unsigned long long>(acc_hi) << 23) + acc_lo;
   acc = block_sum_u64(acc, red);
   if (threadIdx.x == 0 && acc) atomicAdd(&rowsum[blockIdx.x], acc);
 }
