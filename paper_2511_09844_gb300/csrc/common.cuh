@@ -141,27 +141,18 @@ __device__ __forceinline__ float log_at(float x) {
   return __fadd_rn(__fmul_rn(ef, 0x1.62e400p-1f), __fadd_rn(__fmul_rn(ef, 0x1.7f7d1cp-20f), ln_m));
 }
 
-// e in [0, 1] to the fixed point floor(e * 2^45) used by the exact softmax normaliser, from the
-// bits of e: with e = m 2^(x - 150) (24-bit significand m), e 2^45 = m 2^(x - 105), so the floor is
-// m shifted left by x - 105 or right by 105 - x (integer shifts only: a 64-bit conversion would
-// run on the FP64 pipe).
-// The same value as two exact 32-bit parts, floor(e 2^45) = hi 2^23 + lo with hi = floor(e 2^22)
-// (<= 2^22) and lo = floor(e 2^45 - hi 2^23) (< 2^23), in fp32 operations that are all exact: the
-// floors are round-toward-zero additions of 2^23 (the integer is read from the sum's bits), and
-// e 2^45 - hi 2^23 is a multiple of the ulp of e 2^45 below 2^23. Sums of up to 2^9 parts fit.
+// e in [0, 1] to the fixed point floor(e * 2^45) of the exact softmax normaliser (the sum over the
+// vocabulary of floor(e_v 2^45) is an integer, so its value does not depend on the summation
+// order), as two exact 32-bit parts: floor(e 2^45) = hi 2^23 + lo with hi = floor(e 2^22) (<= 2^22)
+// and lo = floor(e 2^45 - hi 2^23) (< 2^23). Every fp32 operation here is exact: the floors are
+// round-toward-zero additions of 2^23 whose integer is read from the sum's bits, and
+// e 2^45 - hi 2^23 is a multiple of the ulp of e 2^45 below 2^23. Sums of up to 2^9 parts fit in
+// 32 bits. (A float-to-64-bit conversion would run on the FP64 pipe.)
 __device__ __forceinline__ void fixed45_parts(float e, uint32_t& hi, uint32_t& lo) {
   const float h = __fadd_rz(__fmul_rn(e, 0x1p22f), 0x1p23f);
   hi = __float_as_uint(h) - 0x4B000000u;
   const float r = __fmaf_rn(-__fsub_rn(h, 0x1p23f), 0x1p23f, __fmul_rn(e, 0x1p45f));
   lo = __float_as_uint(__fadd_rz(r, 0x1p23f)) - 0x4B000000u;
-}
-__device__ __forceinline__ unsigned long long fixed45(float e) {
-  const uint32_t b = __float_as_uint(e);
-  const int x = static_cast<int>(b >> 23);                       // biased exponent (e >= 0)
-  const unsigned long long m = static_cast<unsigned long long>((b & 0x7FFFFFu) | 0x800000u);
-  const unsigned long long up = m << min(max(x - 105, 0), 40);
-  const unsigned long long dn = m >> min(max(105 - x, 0), 63);
-  return x == 0 ? 0ull : (x >= 105 ? up : dn);
 }
 
 // ------------------------------------------------------------------------------------------
