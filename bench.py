@@ -256,7 +256,12 @@ def run_ours(args, rank, world, local_rank):
     tau = emitted / (args.steps * B)
 
     # end to end through the public API: step, accept, read the emitted tokens back into pinned
-    # host memory every step (the per-step work of a serving loop; no per-step host input exists)
+    # host memory every step (the per-step work of a serving loop; no per-step host input exists).
+    # The context restarts from the same prompts and seed and repeats the warm-up, so the timed
+    # steps emit the same tokens as above (the engine is deterministic) and only the host loop differs.
+    eng.prefill(prompts, [temp] * B, seed=args.seed + rank)
+    for i in range(args.warmup):
+        one_step(i % args.steps)
     h_tok = torch.empty((B, k + 1), dtype=torch.int32, pin_memory=True)
     h_n = torch.empty(B, dtype=torch.int32, pin_memory=True)
     e2e_emitted = 0
@@ -333,7 +338,8 @@ def run_ours(args, rank, world, local_rank):
         "tokens_per_s_at_paper_tau": {"tau": 5.00, "value": round(5.00 / (ms_max / args.steps / 1e3), 2)},
         "prefill_s": round(prefill_s, 3),
         "e2e": {"value": round(e2e_value, 3), "unit": "tokens/s/sequence", "h2d_bytes_per_step": 0,
-                "d2h_bytes_per_step": int(h_tok.numel() * 4 + h_n.numel() * 4)},
+                "d2h_bytes_per_step": int(h_tok.numel() * 4 + h_n.numel() * 4),
+                "same_tokens_as_timed_steps": e2e_emitted == emitted},
         "roofline": {"bound": "hbm", "kernel": "weight-streaming GEMM (all projections + lm_head)",
                      "achieved": round(gemm_gbs, 1), "peak": hbm, "unit": "GB/s",
                      "frac": round(gemm_gbs / hbm, 4),
