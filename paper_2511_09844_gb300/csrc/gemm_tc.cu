@@ -1043,20 +1043,51 @@ int sm_count() {
 constexpr int kSmemBudget = 227 * 1024;
 constexpr int kSmemShared = 110 * 1024;
 
-// CTAs per tile: split each tile's K over up to 8 CTAs of a cluster when there are fewer tiles
-// than SMs (and the token tile is at most 128 wide), aiming at about 1.5 CTAs per SM: two CTAs
-// share an SM's shared memory, so more weight bytes are in flight per SM, while part of the SMs
-// stay free for the next kernel's CTAs to start and prefetch.
-int split_factor(int tiles, int NT, int KB) {
+// Launch shape of a grid of `tiles` weight tiles x token tiles: split factor sp (CTAs per tile, one
+// cluster), ring stages, dynamic shared memory and grid. Two CTAs share an SM when the ring (at
+// least 3 stages) and the split-K receive buffer fit in half its shared memory: more weight bytes in
+// flight per SM, and room for the next kernel's CTAs to start early. With fewer tiles than resident
+// CTAs the K range is split, aiming at 1.5 CTAs per SM (two-per-SM plans) or one (one-per-SM plans),
+// never past one wave. Of the two, the plan with more CTAs streaming at once wins (ties: two per SM).
+struct TcPlan {
+  int sp = 0, stages = 0, smem = 0, grid = 0;
+};
+TcPlan plan_tc(int tiles, int NT, int KB) {
   const int sms = sm_count();
-  int sp = 1;
-  if (tiles < sms && NT <= 128) {
-    sp = (3 * sms / 2 + tiles / 2) / tiles;
-    if (sp > 8) sp = 8;
-    if (sp > KB) sp = KB;
-    if (sp < 1) sp = 1;
+  const int stage_bytes = (kWRows + NT) * kBK * 2;
+  auto fixed_of = [&](int sp) {
+    const int recv = sp > 1 ? sp * ((64 + sp - 1) / sp) * 2 * NT * 4 : 0;   // split-K receive buffer
+    return 1024 + recv + kWRows * kXS * 4 + 64 + kMaxNT * 4 + 8 * (2 * 16 + 6);
+  };
+  TcPlan best;
+  int best_active = 0;
+  for (int occ = 2; occ >= 1; --occ) {
+    const int budget = occ == 2 ? kSmemShared : kSmemBudget;
+    const int min_stages = occ == 2 ? 3 : 2;
+    if (occ == 2 && NT > 128) continue;                  // the accumulators would not fit twice in TMEM
+    int sp = 1;
+    if (tiles < sms * occ) {                             // split-K tiles keep one NT-column accumulator
+      sp = ((occ == 2 ? 3 * sms / 2 : sms) + tiles / 2) / tiles;
+      sp = std::max(1, std::min(sp, std::min(8, KB)));
+      while (sp > 1 && tiles * sp > sms * occ) --sp;
+    }
+    for (; sp >= 1; --sp) {
+      const int S = std::min(8, (budget - fixed_of(sp)) / stage_bytes);
+      if (S < min_stages) continue;
+      TcPlan pl;
+      pl.sp = sp;
+      pl.stages = S;
+      pl.smem = fixed_of(sp) + S * stage_bytes;
+      pl.grid = sp > 1 ? tiles * sp : std::min(tiles, occ * sms);
+      const int active = std::min(pl.grid, occ * sms);
+      if (active > best_active) {
+        best = pl;
+        best_active = active;
+      }
+      break;
+    }
   }
-  return sp;
+  return best;
 }
 
 int n_out_rows(const GemmArgs& g) {
@@ -1078,7 +1109,7 @@ int gemm_norm_parts(const GemmArgs& g) {
   const int NT = gemm_tc_token_tile(g.M);
   const int n_wtiles = n_out_rows(g) / kWRows;
   const int tiles = n_wtiles * ((g.M + NT - 1) / NT);
-  return n_wtiles * split_factor(tiles, NT, g.K / kBK);
+  return n_wtiles * std::max(1, plan_tc(tiles, NT, g.K / kBK).sp);
 }
 
 int gemm_tc_token_tile(int M) {
@@ -1184,26 +1215,19 @@ cudaError_t gemm_tc(const GemmArgs& g, unsigned* err, cudaStream_t st) {
   a.norm_ssq_out = g.norm_ssq_out; a.tap = g.tap; a.tap_row = g.tap_row; a.tap_mask = g.tap_mask;
   a.norm_ssq_in = g.norm_ssq_in; a.norm_parts = g.norm_parts; a.norm_d = g.norm_d; a.norm_eps = g.norm_eps;
   a.ld_ssq = g.ld_ssq;
-  const int sp = split_factor(a.tiles, a.NT, a.KB);
+  const TcPlan pl = plan_tc(a.tiles, a.NT, a.KB);
+  if (pl.sp < 1) return cudaErrorInvalidValue;
+  const int sp = pl.sp;
   a.sp = sp;
-  const int stage_bytes = (kWRows + a.NT) * kBK * 2;
-  const int recv = sp > 1 ? sp * ((64 + sp - 1) / sp) * 2 * a.NT * 4 : 0;   // split-K receive buffer
-  const int fixed = 1024 + recv + kWRows * kXS * 4 + 64 + kMaxNT * 4 + 8 * (2 * 16 + 6);
-  // Up to NT = 128 the ring fits in half an SM's shared memory (and the accumulators in half of
-  // TMEM), so the next GEMM's CTA can start on the same SM while this one drains.
-  int S = (kSmemShared - fixed) / stage_bytes;
-  if (a.NT > 128 || S < 3) S = (kSmemBudget - fixed) / stage_bytes;
-  if (S > 8) S = 8;
-  if (S < 2) return cudaErrorInvalidValue;
-  a.stages = S;
-  const int smem = fixed + S * stage_bytes;
+  a.stages = pl.stages;
+  const int smem = pl.smem;
   static bool configured = false;
   if (!configured) {
     cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBudget);
     if (e != cudaSuccess) return e;
     configured = true;
   }
-  const int grid = sp > 1 ? a.tiles * sp : std::min(a.tiles, 2 * sm_count());
+  const int grid = pl.grid;
   return launch_pdl_cluster(gemm_tc_kernel, dim3(static_cast<unsigned>(grid)), dim3(kThreads),
                             static_cast<size_t>(smem), st, sp, a);
 }
