@@ -15,6 +15,8 @@
 //                        everywhere, argmax_v (s_v - ln E_v) on row j
 //   bonus / draft       argmax_v (s_v - ln E_v)   (exponential race in log form)
 //   T = 0               accept iff x_i = argmax z_{i-1}; emit argmax of the row
+#include <algorithm>
+
 #include "common.cuh"
 #include "kernels.h"
 
@@ -22,9 +24,19 @@ namespace sd2 {
 namespace {
 
 constexpr int kThreads = 256;
-constexpr int kPerCta = kThreads * 4 * 8;   // vocabulary entries per CTA (8 iterations of 4)
-constexpr int kStatsPerCta = kThreads * 8 * 8;   // the row-statistics passes: 8 iterations of 8
+constexpr int kPerCta = kThreads * 4 * 8;   // most vocabulary entries per CTA (8 passes of 4 per thread)
+constexpr int kStatsPerCta = kThreads * 8 * 8;   // the row-statistics passes: at most 8 passes of 8
 enum { MODE_NONE = 0, MODE_DONE = 1, MODE_RESIDUAL = 2, MODE_BONUS = 3 };
+
+// Vocabulary entries per CTA for `rows` rows: enough CTAs per row to fill the GPU about twice over,
+// in whole passes of `gran` entries per thread, at most max_span (few rows: more, shorter CTAs; a
+// large batch keeps long ones). Every decision is independent of how the vocabulary is split.
+int vocab_span(int V, int rows, int gran, int max_span) {
+  const int pass = kThreads * gran;
+  const int want = std::max(1, (2 * sm_count_cached() + rows - 1) / std::max(1, rows));
+  const int span = (((V + want - 1) / want + pass - 1) / pass) * pass;
+  return std::min(max_span, std::max(pass, span));
+}
 
 template <typename T>
 __device__ __forceinline__ void load4(const T* row, int v, float z[4]);
@@ -116,7 +128,7 @@ __device__ __forceinline__ unsigned step_value(const int* step_ptr, unsigned ste
 template <typename T>
 __global__ void __launch_bounds__(kThreads) rowmax_kernel(const T* target, const T* draft, int B, int k, int V,
                                                           const float* temp, const int* stopped,
-                                                          unsigned long long* rowkey, unsigned* err) {
+                                                          unsigned long long* rowkey, unsigned* err, int span) {
   pdl_trigger();
   pdl_wait();
   __shared__ unsigned long long red[32];
@@ -127,7 +139,7 @@ __global__ void __launch_bounds__(kThreads) rowmax_kernel(const T* target, const
   if (greedy && rr.is_draft) return;
   const float invT = greedy ? 1.f : inv_temp(t);
   const T* row = (rr.is_draft ? draft : target) + rr.offset;
-  const int lo = blockIdx.y * kStatsPerCta, hi = min(V, lo + kStatsPerCta);
+  const int lo = blockIdx.y * span, hi = min(V, lo + span);
   // this thread's (max, first index of it) in 32 bits: its entries come in increasing index order,
   // so a strictly greater value is the only update (+0 and -0 compare equal, as the packed key
   // folds them); packed once for the exact cross-thread maximum
@@ -175,7 +187,7 @@ template <typename T>
 __global__ void __launch_bounds__(kThreads) rowsum_kernel(const T* target, const T* draft, int B, int k, int V,
                                                           const float* temp, const int* stopped,
                                                           const unsigned long long* rowkey,
-                                                          unsigned long long* rowsum) {
+                                                          unsigned long long* rowsum, int span) {
   pdl_trigger();
   pdl_wait();
   __shared__ unsigned long long red[32];
@@ -186,7 +198,7 @@ __global__ void __launch_bounds__(kThreads) rowsum_kernel(const T* target, const
   const float invT = inv_temp(t);
   const float m = packed_key(rowkey[blockIdx.x]);
   const T* row = (rr.is_draft ? draft : target) + rr.offset;
-  const int lo = blockIdx.y * kStatsPerCta, hi = min(V, lo + kStatsPerCta);
+  const int lo = blockIdx.y * span, hi = min(V, lo + span);
   uint32_t acc_hi = 0, acc_lo = 0;        // at most 64 entries per thread: no overflow
 #pragma unroll 2
   for (int v = lo + threadIdx.x * 8; v < hi; v += kThreads * 8) {
@@ -281,7 +293,7 @@ __global__ void __launch_bounds__(kThreads) resample_kernel(const T* target, con
                                                             int k, int V, unsigned long long seed, const int* step_ptr,
                                                             unsigned step, const unsigned long long* rowkey,
                                                             const unsigned long long* rowsum, int* tokens, int* n,
-                                                            AcceptScratch s) {
+                                                            AcceptScratch s, int span) {
   pdl_trigger();
   pdl_wait();
   __shared__ unsigned long long red[32];
@@ -305,7 +317,7 @@ __global__ void __launch_bounds__(kThreads) resample_kernel(const T* target, con
     dq = row_dist(rowkey, rowsum, rd);
     drow = draft + static_cast<size_t>(rd - nt) * V;
   }
-  const int lo = blockIdx.y * kPerCta, hi = min(V, lo + kPerCta);
+  const int lo = blockIdx.y * span, hi = min(V, lo + span);
   unsigned long long best_r = 0, best_l = 0;
   for (int v = lo + threadIdx.x * 4; v < hi; v += kThreads * 4) {
     const uint4 c = philox4x32_10(make_uint4(static_cast<uint32_t>(v >> 2), (RNG_RESAMPLE << 16) | j,
@@ -353,7 +365,7 @@ __global__ void __launch_bounds__(kThreads) sample_kernel(const float* logits, l
                                                           unsigned long long seed, int purpose, int i,
                                                           const int* step_ptr, unsigned step, int* out, int ld_out,
                                                           int* out2, int ld_out2, unsigned long long* slot,
-                                                          int* counter, unsigned* err) {
+                                                          int* counter, unsigned* err, int span) {
   pdl_trigger();
   pdl_wait();
   __shared__ unsigned long long red[32];
@@ -365,7 +377,7 @@ __global__ void __launch_bounds__(kThreads) sample_kernel(const float* logits, l
   const float invT = greedy ? 1.f : inv_temp(t);
   const unsigned stp = step_value(step_ptr, step);
   const uint32_t k0 = static_cast<uint32_t>(seed), k1 = static_cast<uint32_t>(seed >> 32);
-  const int lo = blockIdx.y * kPerCta, hi = min(V, lo + kPerCta);
+  const int lo = blockIdx.y * span, hi = min(V, lo + span);
   unsigned long long best = 0;
   bool bad = false;
   for (int v = lo + threadIdx.x * 4; v < hi; v += kThreads * 4) {
@@ -411,16 +423,16 @@ cudaError_t accept_typed(const T* target, const T* draft, const int* xhat, const
                          unsigned long long seed, unsigned step, const int* step_ptr, const int* stopped, int* tokens,
                          int* n, const AcceptScratch& s, unsigned* err, cudaStream_t st) {
   const int R = B * (2 * k + 1);
-  const int S = (V + kPerCta - 1) / kPerCta;
-  const int SS = (V + kStatsPerCta - 1) / kStatsPerCta;
+  const int span = vocab_span(V, B, 4, kPerCta), S = (V + span - 1) / span;
+  const int sspan = vocab_span(V, R, 8, kStatsPerCta), SS = (V + sspan - 1) / sspan;
   cudaError_t e = cudaMemsetAsync(s.rowkey, 0, sizeof(unsigned long long) * 2 * R, st);  // rowkey + rowsum
   if (e != cudaSuccess) return e;
-  { const cudaError_t e_ = launch_pdl(rowmax_kernel<T>, dim3(dim3(R, SS)), dim3(kThreads), 0, st, target, draft, B, k, V, temp, stopped, s.rowkey, err); if (e_ != cudaSuccess) return e_; }
-  { const cudaError_t e_ = launch_pdl(rowsum_kernel<T>, dim3(dim3(R, SS)), dim3(kThreads), 0, st, target, draft, B, k, V, temp, stopped, s.rowkey, s.rowsum); if (e_ != cudaSuccess) return e_; }
+  { const cudaError_t e_ = launch_pdl(rowmax_kernel<T>, dim3(dim3(R, SS)), dim3(kThreads), 0, st, target, draft, B, k, V, temp, stopped, s.rowkey, err, sspan); if (e_ != cudaSuccess) return e_; }
+  { const cudaError_t e_ = launch_pdl(rowsum_kernel<T>, dim3(dim3(R, SS)), dim3(kThreads), 0, st, target, draft, B, k, V, temp, stopped, s.rowkey, s.rowsum, sspan); if (e_ != cudaSuccess) return e_; }
   { const cudaError_t e_ = launch_pdl(decide_kernel<T>, dim3((B + 127) / 128), dim3(128), 0, st, target, draft, xhat, temp, B, k, V, seed, step_ptr, step, stopped,
                                                     s.rowkey, s.rowsum, tokens, n, s); if (e_ != cudaSuccess) return e_; }
   { const cudaError_t e_ = launch_pdl(resample_kernel<T>, dim3(dim3(B, S)), dim3(kThreads), 0, st, target, draft, temp, B, k, V, seed, step_ptr, step, s.rowkey,
-                                                      s.rowsum, tokens, n, s); if (e_ != cudaSuccess) return e_; }
+                                                      s.rowsum, tokens, n, s, span); if (e_ != cudaSuccess) return e_; }
   return cudaGetLastError();
 }
 
@@ -458,9 +470,9 @@ cudaError_t sample_rows(const float* logits, long long ld, int B, int V, const f
                         int purpose, int i, const int* step_ptr, unsigned step, int* out, int ld_out, int* out2,
                         int ld_out2, unsigned long long* slot, int* counter, unsigned* err, cudaStream_t st) {
   if (B <= 0) return cudaSuccess;
-  const int S = (V + kPerCta - 1) / kPerCta;
+  const int span = vocab_span(V, B, 4, kPerCta), S = (V + span - 1) / span;
   { const cudaError_t e_ = launch_pdl(sample_kernel, dim3(dim3(B, S)), dim3(kThreads), 0, st, logits, ld, V, temp, seed, purpose, i, step_ptr, step, out, ld_out,
-                                                 out2, ld_out2, slot, counter, err); if (e_ != cudaSuccess) return e_; }
+                                                 out2, ld_out2, slot, counter, err, span); if (e_ != cudaSuccess) return e_; }
   return cudaGetLastError();
 }
 
