@@ -263,14 +263,17 @@ double gemm_bytes(int M, int N, int K, int out_bytes) {
 }
 
 // Final RMSNorm (with the last tap) and lm_head over the logit rows, from the residual stream c->x.
-sd2_status head(sd2_ctx* c, const Model& m, const Plan& p, const FwdOut& o) {
+// Final RMSNorm and lm_head. final_parts > 0: the last layer's down projection already produced
+// bf16(x * gamma_final), the last taps and final_parts slices of the sums of squares (every row
+// takes logits), so the lm_head applies the norm's row scale itself.
+sd2_status head(sd2_ctx* c, const Model& m, const Plan& p, const FwdOut& o, int final_parts = 0) {
   const sd2_lm_config& mc = m.c;
   const int M = p.M, d = mc.d_model, L = mc.n_layers;
   int mask = 0;
   if (o.taps)
     for (int s = 0; s < 3; ++s)
       if (o.tap_layers[s] == L) mask |= 1 << s;
-  if (o.n_logit_rows > 0 || mask) {
+  if (final_parts == 0 && (o.n_logit_rows > 0 || mask)) {
     const int nr = o.n_logit_rows > 0 ? o.n_logit_rows : M;
     CK(timed(c, PC_OTHER, 0, [&] {
       return rmsnorm(c->x, o.logit_rows, m.final_norm, mc.norm_eps, nr, d, c->a, o.taps, o.tap_row, mask, c->st);
@@ -281,6 +284,10 @@ sd2_status head(sd2_ctx* c, const Model& m, const Plan& p, const FwdOut& o) {
     gl.x = c->a; gl.ldx = d; gl.M = o.n_logit_rows; gl.K = d;
     gl.seg[0] = {m.lm_head, mc.vocab}; gl.nseg = 1; gl.epi = EPI_STORE; gl.out = o.logits;
     gl.ldo = static_cast<int>(o.ld_logits);
+    if (final_parts > 0) {
+      gl.norm_ssq_in = c->ssq; gl.norm_parts = final_parts; gl.norm_d = d; gl.norm_eps = mc.norm_eps;
+      gl.ld_ssq = c->max_rows;
+    }
     CK(timed(c, PC_GEMM, gemm_bytes(o.n_logit_rows, mc.vocab, d, 4), [&] { return gemm(tc(c, gl), c->st); }));
   }
   return SD2_OK;
@@ -385,6 +392,8 @@ sd2_status forward(sd2_ctx* c, const Model& m, const Plan& p, const FwdOut& o) {
             gemm_norm_parts(g1) <= (d / 128 + 1) * 8 && gemm_norm_parts(g3) <= (d / 128 + 1) * 8;
   }
   int parts = 1;   // slices of the sums of squares the last producer wrote
+  // every row of the plan takes logits: the last down projection can produce the final norm too
+  const bool final_in_down = o.n_logit_rows == M && o.logit_rows == nullptr && !o.tap_row;
   if (fused) {
     CK(timed(c, PC_OTHER, 0, [&] {
       return embed_scaled(p.tok, m.embed, m.W(0, SD2_W_ATTN_NORM), M, d, mc.vocab, c->x, c->a, c->ssq, c->st);
@@ -473,10 +482,14 @@ sd2_status forward(sd2_ctx* c, const Model& m, const Plan& p, const FwdOut& o) {
       produce(gd, m.W(l + 1, SD2_W_ATTN_NORM));
       gd.tap = o.taps; gd.tap_row = o.tap_row; gd.tap_mask = tap_mask(l + 1);
       parts = gemm_norm_parts(gd);
+    } else if (fused && final_in_down) {   // the final RMSNorm of a head that takes every row
+      produce(gd, m.final_norm);
+      gd.tap = o.taps; gd.tap_row = o.tap_row; gd.tap_mask = tap_mask(L);
+      parts = gemm_norm_parts(gd);
     }
     CK(timed(c, PC_GEMM, gemm_bytes(M, d, F, 8), [&] { return gemm(tc(c, gd), c->st); }));
   }
-  return head(c, m, p, o);
+  return head(c, m, p, o, fused && final_in_down ? parts : 0);
 }
 
 // a1: g = LN(W_hml [h; m; l]) at each sequence's steering row, biases = W_s g.
