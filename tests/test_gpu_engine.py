@@ -39,6 +39,18 @@ def test_tiny_ragged_batch_mixed_temperatures_gqa():
     assert rep.blocks == 18
 
 
+def test_tiny_longest_draft_and_wider_batch():
+    """k = 16 (the largest draft length: 17 verify rows per sequence) over 8 ragged sequences with
+    mixed temperatures: wide token tiles, many attention groups, long acceptance blocks."""
+    base = parity.tiny_work()
+    work = dataclasses.replace(base, k=16, batch=8)
+    vw, dw, st = parity.tiny_weights(work, seed=5)
+    prompts = W.make_prompts(base.verifier.vocab, 8, (9, 70), seed=11)
+    temps = [0.0, 1.0, 0.7, 1.0, 0.0, 0.5, 1.0, 0.9]
+    rep = parity.run(work, vw, dw, st, prompts, temps, seed=91, n_steps=3)
+    assert rep.blocks == 24
+
+
 def test_high_acceptance_with_self_drafting():
     """Drafter = verifier with W_s = 0 at T = 0: every block is fully accepted (tau = k + 1)."""
     base = parity.tiny_work()
