@@ -252,9 +252,18 @@ __device__ __forceinline__ int pair_row(const TcArgs& a, int p, int m) {
   return pairs_of_32(a) ? (p >> 5) * 64 + m * 32 + (p & 31) : p + 64 * m;
 }
 // Rank r of sp owns pairs [64 r / sp, 64 (r + 1) / sp); its receive buffer holds, per source
-// rank q and owned pair lp, both members' NT columns: [q][lp][member][NT] floats.
+// rank q and owned pair lp, both members' NT columns: [q][lp][member][NT] floats. Within a row
+// the 16-byte chunks of four columns are rotated by lp mod 8 (recv_chunk), so the owner's reads
+// of one column across consecutive pairs fall in different bank groups: unrotated, every row
+// starts at the same bank (2 NT is a multiple of 32 words) and such a read is np-way conflicted.
 __device__ __forceinline__ int pair_owner(int p, int sp) { return ((p + 1) * sp - 1) / 64; }
 __device__ __forceinline__ int pairs_max(int sp) { return (64 + sp - 1) / sp; }
+__device__ __forceinline__ int recv_chunk(int c4, int lp, int nch) {   // nch = NT / 4, a multiple of 4
+  int rot = lp & 7;
+  rot = rot >= nch ? rot - nch : rot;
+  const int x = c4 + rot;
+  return x >= nch ? x - nch : x;
+}
 
 // The global operands of one output pair (pair p of tile wt, token m), loaded before its sums
 // are known: residuals (EPI_ADD), steering bias (SwiGLU), or position, rotary factors and KV
@@ -355,7 +364,36 @@ __device__ __forceinline__ PairOps first_pair_ops(const TcArgs& a, int rank, int
   const int wt = first_tile % a.n_wtiles, tt = first_tile / a.n_wtiles;
   const int cols = min(NT, a.M - tt * NT);
   const int p_lo = rank * 64 / sp, np = (rank + 1) * 64 / sp - p_lo;
-  return tid < np * cols ? pair_ops(a, wt, p_lo + tid % np, tt * NT + tid / np) : PairOps{};
+  return tid < np * cols && np * cols <= 128 ? pair_ops(a, wt, p_lo + tid % np, tt * NT + tid / np) : PairOps{};
+}
+// Sum in rank order of the sp partials of one receive-buffer word (T = float) or four adjacent
+// ones (T = float4); rv points at rank 0's member-0 value, member 1 is NT floats on, rank q at q
+// rstride floats. C >= sp loads per member are issued before any add (rank index clamped).
+__device__ __forceinline__ void add_part(float& s, float v) { s += v; }
+__device__ __forceinline__ void add_part(float4& s, float4 v) { s.x += v.x; s.y += v.y; s.z += v.z; s.w += v.w; }
+template <int C, typename T>
+__device__ __forceinline__ void sum_parts(const float* rv, int rstride, int NT, int sp, T& s0, T& s1) {
+  T v0[C], v1[C];
+#pragma unroll
+  for (int j = 0; j < C; ++j) {
+    const int kk = min(j, sp - 1);
+    v0[j] = *reinterpret_cast<const T*>(rv + kk * rstride);
+    v1[j] = *reinterpret_cast<const T*>(rv + kk * rstride + NT);
+  }
+  s0 = v0[0];
+  s1 = v1[0];
+#pragma unroll
+  for (int j = 1; j < C; ++j)
+    if (j < sp) {
+      add_part(s0, v0[j]);
+      add_part(s1, v1[j]);
+    }
+}
+template <typename T>
+__device__ __forceinline__ void sum_parts_any(const float* rv, int rstride, int NT, int sp, T& s0, T& s1) {
+  if (sp <= 2) sum_parts<2>(rv, rstride, NT, sp, s0, s1);
+  else if (sp <= 4) sum_parts<4>(rv, rstride, NT, sp, s0, s1);
+  else sum_parts<8>(rv, rstride, NT, sp, s0, s1);
 }
 // Split-K epilogue of the CTA's single tile (sp > 1), run by the four epilogue warps (warp % 4 =
 // the TMEM lane quarter): this rank's partial of every row goes to the rank owning the row's pair
@@ -373,8 +411,8 @@ __device__ __forceinline__ void splitk_epilogue(const TcArgs& a, const SplitK& s
   const int wt = sk.first_tile % a.n_wtiles, tt = sk.first_tile / a.n_wtiles;
   const int cols = min(NT, a.M - tt * NT);
   const int p_lo = rank * 64 / sp, np = (rank + 1) * 64 / sp - p_lo;
-  const int p = pair_of(a, r), owner = pair_owner(p, sp);
-  const int slot = ((rank * npmax + p - owner * 64 / sp) * 2 + member_of(a, r)) * NT;
+  const int p = pair_of(a, r), owner = pair_owner(p, sp), lpd = p - owner * 64 / sp, nch = NT >> 2;
+  const int slot = ((rank * npmax + lpd) * 2 + member_of(a, r)) * NT;
   const uint32_t dst = dsmem_addr(smem_u32(recv + slot), static_cast<uint32_t>(owner));
   const uint32_t dst_bar = dsmem_addr(sk.rbar, static_cast<uint32_t>(owner));
   if (a.norm_ssq_in) tile_rstd(a, tt, rs, tid);
@@ -389,37 +427,53 @@ __device__ __forceinline__ void splitk_epilogue(const TcArgs& a, const SplitK& s
       tmem_ld16(tbase + ch * 16, v);
 #pragma unroll
       for (int k4 = 0; k4 < 4; ++k4)
-        st_async_v4(dst + static_cast<uint32_t>((ch * 16 + 4 * k4) * 4), dst_bar, v[4 * k4], v[4 * k4 + 1],
-                    v[4 * k4 + 2], v[4 * k4 + 3]);
+        st_async_v4(dst + static_cast<uint32_t>(recv_chunk(ch * 4 + k4, lpd, nch) * 16), dst_bar, v[4 * k4],
+                    v[4 * k4 + 1], v[4 * k4 + 2], v[4 * k4 + 3]);
     }
     if (leader) flags[5] = wait_bar(sk.rbar, 0, abort_flag, a.err) ? 1 : 0;
     named_bar_epi();
     if (flags[5] != 0) {
       // every rank's partial of this rank's pairs is in the receive buffer: sums in rank order
       float* sq = reinterpret_cast<float*>(sk.smem);   // [cols][np] fused-norm sums of squares (drained ring)
-      for (int e = tid; e < np * cols; e += 128) {
-        const int lp = e % np, col = e / np;
-        const float* rv = recv + lp * 2 * NT + col;
-        float v0[8], v1[8];                // every rank's partial loaded first (clamped rank index)
+      const int rstride = npmax * 2 * NT, n_own = np * cols;
+      if (n_own <= 128) {
+        // one output per thread, whose operands were fetched while the MMAs ran
+        const int e = tid;
+        if (e < n_own) {
+          const int lp = e % np, col = e / np;
+          float s0, s1;
+          sum_parts_any(recv + lp * 2 * NT + recv_chunk(col >> 2, lp, nch) * 4 + (col & 3), rstride, NT, sp, s0, s1);
+          if (a.norm_ssq_in) {
+            s0 *= rs[col];
+            s1 *= rs[col];
+          }
+          const float q2 = pair_emit(a, wt, p_lo + lp, tt * NT + col, s0, s1, pf);
+          if (a.norm_out) sq[col * np + lp] = q2;
+        }
+      } else {
+        // wide token tiles: a thread takes pair lp over four adjacent columns, reads their
+        // partials as 16-byte words (one rotated chunk) and requests all four outputs' global
+        // operands before it stores any, so each pass costs one memory round trip, not four
+        const int nq = np * ((cols + 3) >> 2);
+        for (int e = tid; e < nq; e += 128) {
+          const int lp = e % np, c4 = e / np;
+          PairOps o[4];
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {
-          const int kk = min(j, sp - 1);
-          v0[j] = rv[kk * npmax * 2 * NT];
-          v1[j] = rv[kk * npmax * 2 * NT + NT];
-        }
-        float s0 = 0.f, s1 = 0.f;
+          for (int u = 0; u < 4; ++u) o[u] = pair_ops(a, wt, p_lo + lp, tt * NT + min(4 * c4 + u, cols - 1));
+          float4 s0, s1;
+          sum_parts_any(recv + lp * 2 * NT + recv_chunk(c4, lp, nch) * 4, rstride, NT, sp, s0, s1);
+          const float v0[4] = {s0.x, s0.y, s0.z, s0.w}, v1[4] = {s1.x, s1.y, s1.z, s1.w};
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {
-          s0 = j < sp ? s0 + v0[j] : s0;
-          s1 = j < sp ? s1 + v1[j] : s1;
+          for (int u = 0; u < 4; ++u) {
+            const int col = 4 * c4 + u;
+            if (col < cols) {
+              const float sc = a.norm_ssq_in ? rs[col] : 1.f;
+              const float q2 = pair_emit(a, wt, p_lo + lp, tt * NT + col, a.norm_ssq_in ? v0[u] * sc : v0[u],
+                                         a.norm_ssq_in ? v1[u] * sc : v1[u], o[u]);
+              if (a.norm_out) sq[col * np + lp] = q2;
+            }
+          }
         }
-        if (a.norm_ssq_in) {
-          s0 *= rs[col];
-          s1 *= rs[col];
-        }
-        const int m = tt * NT + col;
-        const float q2 = pair_emit(a, wt, p_lo + lp, m, s0, s1, e == tid ? pf : pair_ops(a, wt, p_lo + lp, m));
-        if (a.norm_out) sq[col * np + lp] = q2;
       }
       if (a.norm_out) {   // this rank's slice of the tile: sums of squares per token, in pair order
         named_bar_epi();
