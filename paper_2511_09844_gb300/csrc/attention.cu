@@ -13,15 +13,18 @@
 // below the sequence's pre-step length were also written before the step: their K/V rows are
 // requested before the wait, and the few rows the step itself may have written are requested
 // right after it, together with the queries and row positions. K/V tiles are staged with
-// cp.async (zero-filled where no row exists), two tiles in flight; every K/V byte of the split is
-// read from HBM once per CTA.
+// cp.async (zero-filled where no row exists) through a ring of 2 to 4 tiles (the launcher takes
+// the deepest ring that keeps the grid resident); every K/V byte of the split is read from HBM
+// once per CTA.
 //
 // The splits of one (row group, KV head) form a thread-block cluster. Split merge: the (query
 // vector, 4 dimensions) elements of the group are shared out over the splits; every split pushes
 // its running max and sum of each query vector to every split, and each accumulator pair to the
 // split owning its element, with asynchronous stores that complete on the owner's receive
 // mbarrier. The owner waits only for its own share, merges it and writes the output; no partial
-// goes through global memory and no cluster barrier is held while the partials travel.
+// goes through global memory and no cluster barrier is held while the partials travel. Where
+// two CTAs per SM fit only that way, the receive buffers lie over the K/V ring: each split then
+// arrives on the cluster barrier after its last tile, so no partial lands in a ring still read.
 #include <limits.h>
 #include <math.h>
 
@@ -38,6 +41,8 @@ constexpr int kThreads = kWarps * 32;
 constexpr int kMaxQV = 64;              // query vectors per CTA
 constexpr int kMaxSplits = 16;          // context splits = CTAs of one cluster (16: non-portable size)
 constexpr int kMaxSmem = 200 * 1024;   // dynamic shared memory opt-in (static arrays come on top)
+constexpr int kTwoPerSm = 112 * 1024;  // dynamic shared memory of a CTA that leaves room for a second
+constexpr int kMaxBuf = 4;             // K/V tiles of the ring
 
 template <int HD>
 struct AttnCfg {
@@ -50,26 +55,31 @@ struct AttnCfg {
     const int r = ((max_rows * G + 15) / 16) * 16;
     return r < kMaxQV ? r : kMaxQV;
   }
-  __host__ __device__ static int nbuf(int chunk) { return chunk > kTile ? 2 : 1; }
+  // layout: row data, Q, S, P, a ring of nb K/V tiles, the split's block ids; split merge (ns > 1):
+  // receive barrier, every split's (max, sum) per query vector [ns][qr] and every split's
+  // accumulators of this rank's share of elements [ns][share] (float4 each), after the block ids
+  // or, with `ring`, over the K/V ring
   __host__ __device__ static size_t q_off() { return ROW_BYTES; }
   __host__ __device__ static size_t s_off(int qr) { return q_off() + static_cast<size_t>(qr) * KS * 2; }
   __host__ __device__ static size_t p_off(int qr) { return s_off(qr) + static_cast<size_t>(qr) * SS * 4; }
   __host__ __device__ static size_t kv_off(int qr) { return p_off(qr) + static_cast<size_t>(qr) * PS * 2; }
-  __host__ __device__ static size_t blk_off(int qr, int chunk) {
-    return kv_off(qr) + static_cast<size_t>(nbuf(chunk)) * KV_TILE;
-  }
-  // split merge (ns > 1): receive barrier; every split's (max, sum) per query vector [ns][qr];
-  // every split's accumulators of this rank's share of elements [ns][share] (float4 each)
+  __host__ __device__ static size_t blk_off(int qr, int nb) { return kv_off(qr) + static_cast<size_t>(nb) * KV_TILE; }
   __host__ __device__ static int share(int qr, int ns) { return (qr * (HD / 4) + ns - 1) / ns; }
-  __host__ __device__ static size_t rcv_off(int qr, int chunk) {
-    return blk_off(qr, chunk) + ((static_cast<size_t>(chunk / 16) * 4 + 15) & ~static_cast<size_t>(15));
+  __host__ __device__ static size_t rcv_off(int qr, int chunk, int nb) {
+    return blk_off(qr, nb) + ((static_cast<size_t>(chunk / 16) * 4 + 15) & ~static_cast<size_t>(15));
   }
-  __host__ __device__ static size_t ml_off(int qr, int chunk) { return rcv_off(qr, chunk) + 16; }
-  __host__ __device__ static size_t acc_off(int qr, int chunk, int ns) {
-    return ml_off(qr, chunk) + static_cast<size_t>(ns) * qr * 8;
+  __host__ __device__ static size_t ml_off(int qr, int chunk, int nb, int ring) {
+    return ring ? kv_off(qr) : rcv_off(qr, chunk, nb) + 16;
   }
-  static size_t bytes(int qr, int chunk, int ns) {
-    return ns > 1 ? acc_off(qr, chunk, ns) + static_cast<size_t>(ns) * share(qr, ns) * 16 : rcv_off(qr, chunk);
+  __host__ __device__ static size_t acc_off(int qr, int chunk, int nb, int ring, int ns) {
+    return ml_off(qr, chunk, nb, ring) + static_cast<size_t>(ns) * qr * 8;
+  }
+  static size_t merge_bytes(int qr, int ns) {
+    return static_cast<size_t>(ns) * qr * 8 + static_cast<size_t>(ns) * share(qr, ns) * 16;
+  }
+  static size_t bytes(int qr, int chunk, int ns, int nb, int ring) {
+    if (ns == 1) return rcv_off(qr, chunk, nb);
+    return ring ? rcv_off(qr, chunk, nb) + 16 : acc_off(qr, chunk, nb, 0, ns) + static_cast<size_t>(ns) * share(qr, ns) * 16;
   }
 };
 
@@ -88,6 +98,13 @@ __device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, bool v
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
 template <int N>
 __device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
+// wait until at most n (0..3) of this thread's most recent cp.async groups are pending
+__device__ __forceinline__ void cp_async_wait_n(int n) {
+  if (n <= 0) cp_async_wait<0>();
+  else if (n == 1) cp_async_wait<1>();
+  else if (n == 2) cp_async_wait<2>();
+  else cp_async_wait<3>();
+}
 // two fp32 stored asynchronously to `raddr` (shared::cluster, 8-byte aligned), completing 8 bytes
 // of a transaction on the mbarrier at `rbar` (shared::cluster, same CTA)
 __device__ __forceinline__ void st_async_v2(uint32_t raddr, uint32_t rbar, float x, float y) {
@@ -117,8 +134,10 @@ __device__ __forceinline__ void ldsm_x2_t(uint32_t addr, uint32_t& r0, uint32_t&
                : "memory");
 }
 
+// NB: K/V tiles of the shared-memory layout (>= 2 when a.chunk > 64); ring: the split-merge
+// receive buffers lie over the K/V ring (n_splits > 1).
 template <int HD>
-__global__ void __launch_bounds__(kThreads, 2) attn_kernel(const AttnArgs a) {
+__global__ void __launch_bounds__(kThreads, 2) attn_kernel(const AttnArgs a, int NB, int ring) {
   using C = AttnCfg<HD>;
   constexpr int KS = C::KS, SS = C::SS, PS = C::PS;
   constexpr int NT = HD / 64;  // n8 tiles of output dimensions per warp
@@ -140,10 +159,10 @@ __global__ void __launch_bounds__(kThreads, 2) attn_kernel(const AttnArgs a) {
   float* sS = reinterpret_cast<float*>(smem + C::s_off(QR));
   bf16* sP = reinterpret_cast<bf16*>(smem + C::p_off(QR));
   unsigned char* sKV = smem + C::kv_off(QR);
-  int* sBlk = reinterpret_cast<int*>(smem + C::blk_off(QR, a.chunk));
-  const uint32_t rbar = smem_u32(smem + C::rcv_off(QR, a.chunk));
-  const float2* rML = reinterpret_cast<const float2*>(smem + C::ml_off(QR, a.chunk));
-  const float4* rAcc = reinterpret_cast<const float4*>(smem + C::acc_off(QR, a.chunk, NS));
+  int* sBlk = reinterpret_cast<int*>(smem + C::blk_off(QR, NB));
+  const uint32_t rbar = smem_u32(smem + C::rcv_off(QR, a.chunk, NB));
+  const float2* rML = reinterpret_cast<const float2*>(smem + C::ml_off(QR, a.chunk, NB, ring));
+  const float4* rAcc = reinterpret_cast<const float4*>(smem + C::acc_off(QR, a.chunk, NB, ring, NS));
   const int share = C::share(QR, NS);
 
   // Before the wait: the plan tables and the block table (written before the step's first
@@ -180,16 +199,18 @@ __global__ void __launch_bounds__(kThreads, 2) attn_kernel(const AttnArgs a) {
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   __syncthreads();                                  // block ids and the receive barrier
-  if (NS > 1) cluster_arrive_relaxed();             // waited for before the first push
+  if (NS > 1 && !ring) cluster_arrive_relaxed();    // waited for before the first push
 
   const bf16* pool = static_cast<const bf16*>(a.kv.pool);
   const size_t head_stride = static_cast<size_t>(16) * HD;
   const size_t blk_stride = static_cast<size_t>(2) * Hkv * head_stride;
   const bf16* layer_base = pool + static_cast<size_t>(a.layer) * a.kv.n_blocks * blk_stride + kvh * head_stride;
-  // rows p in [p_from, p_to) of tile i (positions lo + 64 i ..) -> buffer i & 1: loaded below
+  // ring slots used (the dynamic chunk may hold fewer tiles than the layout)
+  const int nb = chunk > kTile ? max(2, min(NB, chunk / kTile)) : 1;
+  // rows p in [p_from, p_to) of tile i (positions lo + 64 i ..) -> ring slot i % nb: loaded below
   // `valid_end`, zero-filled from it on
   auto issue_rows = [&](int i, int p_from, int p_to, int valid_end) {
-    bf16* dK = reinterpret_cast<bf16*>(sKV + (i & 1) * C::KV_TILE);
+    bf16* dK = reinterpret_cast<bf16*>(sKV + (i % nb) * C::KV_TILE);
     bf16* dV = dK + kTile * KS;
     const int t0 = lo + i * kTile;
 #pragma unroll
@@ -204,7 +225,6 @@ __global__ void __launch_bounds__(kThreads, 2) attn_kernel(const AttnArgs a) {
       cp_async16(smem_u32(dV + t * KS + c * 8), ok ? src + Hkv * head_stride : layer_base, ok);
     }
   };
-  const int nb = C::nbuf(chunk);
   if (early)
     for (int i = 0; i < nb; ++i) issue_rows(i, lo, pre_hi, pre_hi);
   pdl_wait();
@@ -243,13 +263,17 @@ __global__ void __launch_bounds__(kThreads, 2) attn_kernel(const AttnArgs a) {
   const int hi = min(lo + chunk, pmax + 1);
   const int ntiles = hi > lo ? (hi - lo + kTile - 1) / kTile : 0;
   const int nmt = (nqv + 15) >> 4;
+  int committed = 0;                                // cp.async groups so far: one per tile, in tile order
   if (early) {
+    committed = nb;
     // every row the queries can see in the early tiles must have been loaded
     if (tid == 0 && ntiles > 0 && min(hi, lo + nb * kTile) > fresh_hi && a.err)
       atomicOr(a.err, static_cast<unsigned>(ERR_RANGE));
   } else {
-    if (ntiles > 0) { issue_rows(0, lo, INT_MAX, hi); cp_async_commit(); }
-    if (ntiles > 1) { issue_rows(1, lo, INT_MAX, hi); cp_async_commit(); }
+    for (; committed < min(nb, ntiles); ++committed) {
+      issue_rows(committed, lo, INT_MAX, hi);
+      cp_async_commit();
+    }
   }
 
   const float scale = rsqrtf(static_cast<float>(HD));
@@ -263,14 +287,18 @@ __global__ void __launch_bounds__(kThreads, 2) attn_kernel(const AttnArgs a) {
 #pragma unroll
       for (int e = 0; e < 4; ++e) acc[mt][nt][e] = 0.f;
 
-  // two tiles in flight: tiles 0 and 1 now, tile i+1 at the top of iteration i >= 1
+  // nb tiles in flight: tiles 0 .. nb-1 now, tile i+nb-1 at the top of iteration i >= 1 (into the
+  // slot of tile i-1)
   for (int i = 0; i < ntiles; ++i) {
-    if (i == 0 && ntiles > 1) cp_async_wait<1>();
-    else cp_async_wait<0>();
-    __syncthreads();  // tile i visible to all; every warp is past tile i-1, so its buffer is free
-    if (i >= 1 && i + 1 < ntiles) { issue_rows(i + 1, lo, INT_MAX, hi); cp_async_commit(); }
+    cp_async_wait_n(committed - (i + 1));
+    __syncthreads();  // tile i visible to all; every warp is past tile i-1, so its slot is free
+    if (i >= 1 && i + nb - 1 < ntiles) {
+      issue_rows(i + nb - 1, lo, INT_MAX, hi);
+      cp_async_commit();
+      ++committed;
+    }
     const int t0 = lo + i * kTile;
-    const bf16* sK = reinterpret_cast<const bf16*>(sKV + (i & 1) * C::KV_TILE);
+    const bf16* sK = reinterpret_cast<const bf16*>(sKV + (i % nb) * C::KV_TILE);
     const bf16* sV = sK + kTile * KS;
 
     // (1) S = Q K^T * scale, causal and range masks
@@ -404,7 +432,11 @@ __global__ void __launch_bounds__(kThreads, 2) attn_kernel(const AttnArgs a) {
   // of the group (query vector e / (hd/4), dimensions 4 (e % (hd/4)) ..) belongs to the split r
   // with r E4 / NS <= e < (r+1) E4 / NS. Splits that hold no position a row can see contribute
   // m = -inf, l = 0, acc = 0, hence weight 0.
-  cluster_wait();                                   // every split's receive barrier is armed
+  if (ring) {                                       // the receive buffers lie over this CTA's ring
+    __syncthreads();                                // every warp is past its last K/V read
+    cluster_arrive_release();
+  }
+  cluster_wait();                                   // every split's receive barrier is armed (and ring free)
   if (srow < nqv && squart == 0) {                  // (max, sum) of the query vector to every split
     const uint32_t src = smem_u32(rML + split * QR + srow);
     for (int s2 = 0; s2 < NS; ++s2)
@@ -489,7 +521,7 @@ bool clusters_fit(int n) {
   cudaLaunchConfig_t cfg{};
   cfg.gridDim = dim3(n, 1, 1);
   cfg.blockDim = dim3(kThreads);
-  cfg.dynamicSmemBytes = AttnCfg<HD>::bytes(kMaxQV, 2 * kTile, n);
+  cfg.dynamicSmemBytes = AttnCfg<HD>::bytes(kMaxQV, 2 * kTile, n, 2, 0);
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = static_cast<unsigned>(n);
@@ -505,11 +537,29 @@ template <int HD>
 cudaError_t launch(const AttnArgs& a, cudaStream_t st) {
   const cudaError_t e = configure<HD>();
   if (e != cudaSuccess) return e;
-  const int qr = AttnCfg<HD>::qrows(a.max_rows, a.H / a.kv.Hkv);
-  const size_t smem = AttnCfg<HD>::bytes(qr, a.chunk, a.n_splits);
+  using C = AttnCfg<HD>;
+  const int qr = C::qrows(a.max_rows, a.H / a.kv.Hkv), ns = a.n_splits;
+  // The deepest K/V ring (2 to 4 tiles, at most the chunk's) within the shared memory a CTA may
+  // take: room for a second CTA per SM when the grid is larger than the SM count, the opt-in
+  // maximum otherwise. The merge buffers go over the ring only where that is what makes it fit.
+  const int max_nb = a.chunk > kTile ? std::min(kMaxBuf, a.chunk / kTile) : 1;
+  const size_t cap = static_cast<size_t>(ns) * a.n_groups * a.kv.Hkv > static_cast<size_t>(sm_count_cached())
+                         ? static_cast<size_t>(kTwoPerSm) : static_cast<size_t>(kMaxSmem);
+  int nb = std::min(2, max_nb), ring = 0;
+  bool found = false;
+  for (int n = max_nb; n >= std::min(2, max_nb) && !found; --n)
+    for (int r = 0; r <= 1 && !found; ++r) {
+      if (r && (ns == 1 || C::merge_bytes(qr, ns) > static_cast<size_t>(n) * C::KV_TILE)) continue;
+      if (C::bytes(qr, a.chunk, ns, n, r) <= cap) {
+        nb = n;
+        ring = r;
+        found = true;
+      }
+    }
+  const size_t smem = C::bytes(qr, a.chunk, ns, nb, ring);
   if (smem > static_cast<size_t>(kMaxSmem)) return cudaErrorInvalidValue;
-  return launch_pdl_cluster(attn_kernel<HD>, dim3(a.n_splits, a.n_groups, a.kv.Hkv), dim3(kThreads), smem, st,
-                            a.n_splits, a);
+  return launch_pdl_cluster(attn_kernel<HD>, dim3(ns, a.n_groups, a.kv.Hkv), dim3(kThreads), smem, st, ns, a, nb,
+                            ring);
 }
 
 }  // namespace

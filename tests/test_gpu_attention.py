@@ -7,8 +7,9 @@ and probabilities in bf16). Covered: 1 to 16 context splits with empty splits, c
 several tiles, verifier-, drafter- and prompt-shaped groups, GQA ratios 1, 4 and 8, head dims 64 and
 128, and the decode-step path whose cache rows below a pre-step length are read before the
 programmatic wait (boundaries inside a tile, on a tile edge, on a split edge, at zero), with finite
-stale rows between the last row and the planned bound. A row beyond the planned bound must raise the
-range bit of the error word, not fault.
+stale rows between the last row and the planned bound; K/V rings of 2 to 4 tiles and split-merge
+buffers laid over the ring. A row beyond the planned bound must raise the range bit of the error
+word, not fault.
 """
 import pytest
 import torch
@@ -149,3 +150,19 @@ def test_bad_arguments_are_rejected_on_the_host():
         _run(c, 2, 96)                  # chunk not a multiple of 64
     with pytest.raises(sd2.SD2Error):
         _run(c, 2, 64, max_rows=17)     # 17 rows x 4 heads per KV head > 64 query vectors
+
+
+@pytest.mark.parametrize("hd,k1,n_splits,chunk", [(128, 9, 2, 768), (128, 9, 16, 128), (64, 2, 2, 768), (64, 1, 9, 256)])
+def test_ring_depths_and_merge_over_the_ring(hd, k1, n_splits, chunk):
+    """K/V rings of 2 to 4 tiles and, where two CTAs per SM fit only that way (48 query vectors at
+    16 splits), the split-merge buffers laid over the ring; decode steps and plain launches."""
+    lens = [1030, 517, 70]
+    c = _case(7, seq_lens=lens, rows_per_group=[k1] * 3, H=32, Hkv=8, hd=hd)
+    ref = _reference(c)
+    pre_len = [max(0, L - k1 + 1) for L in lens]
+    out, err = _run(c, n_splits, chunk, pre_len=pre_len, pre_stable=-1, pre_fresh=k1 + 1)
+    assert err == 0
+    _check(out, ref)
+    out, err = _run(c, n_splits, chunk)
+    assert err == 0
+    _check(out, ref)
