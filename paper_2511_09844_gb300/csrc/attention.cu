@@ -41,8 +41,11 @@ constexpr int kThreads = kWarps * 32;
 constexpr int kMaxQV = 64;              // query vectors per CTA
 constexpr int kMaxSplits = 16;          // context splits = CTAs of one cluster (16: non-portable size)
 constexpr int kMaxSmem = 200 * 1024;   // dynamic shared memory opt-in (static arrays come on top)
-constexpr int kTwoPerSm = 112 * 1024;  // dynamic shared memory of a CTA that leaves room for a second
 constexpr int kMaxBuf = 4;             // K/V tiles of the ring
+// Resident CTAs per SM the register budget allows: hd = 64 fits 64 registers a thread, so four
+// CTAs; hd = 128 keeps two.
+template <int HD>
+constexpr int kCtasPerSm = HD == 64 ? 4 : 2;
 
 template <int HD>
 struct AttnCfg {
@@ -137,7 +140,7 @@ __device__ __forceinline__ void ldsm_x2_t(uint32_t addr, uint32_t& r0, uint32_t&
 // NB: K/V tiles of the shared-memory layout (>= 2 when a.chunk > 64); ring: the split-merge
 // receive buffers lie over the K/V ring (n_splits > 1).
 template <int HD>
-__global__ void __launch_bounds__(kThreads, 2) attn_kernel(const AttnArgs a, int NB, int ring) {
+__global__ void __launch_bounds__(kThreads, kCtasPerSm<HD>) attn_kernel(const AttnArgs a, int NB, int ring) {
   using C = AttnCfg<HD>;
   constexpr int KS = C::KS, SS = C::SS, PS = C::PS;
   constexpr int NT = HD / 64;  // n8 tiles of output dimensions per warp
@@ -504,6 +507,23 @@ __global__ void __launch_bounds__(kThreads, 2) attn_kernel(const AttnArgs a, int
   }
 }
 
+// Dynamic shared memory each of n resident CTAs can take: the SM's capacity split n ways, less the
+// per-block reservation and the kernel's static arrays (with a little room).
+size_t smem_share(int n) {
+  static const int sm_bytes = [] {
+    int dev = 0, v = 0;
+    cudaGetDevice(&dev);
+    return cudaDeviceGetAttribute(&v, cudaDevAttrMaxSharedMemoryPerMultiprocessor, dev) == cudaSuccess ? v : 0;
+  }();
+  static const int reserved = [] {
+    int dev = 0, v = 0;
+    cudaGetDevice(&dev);
+    return cudaDeviceGetAttribute(&v, cudaDevAttrReservedSharedMemoryPerBlock, dev) == cudaSuccess ? v : 1024;
+  }();
+  const long share = static_cast<long>(sm_bytes) / n - reserved - 256;
+  return share > 0 ? static_cast<size_t>(share) : 0;
+}
+
 template <int HD>
 cudaError_t configure() {
   static cudaError_t e = [] {
@@ -540,11 +560,13 @@ cudaError_t launch(const AttnArgs& a, cudaStream_t st) {
   using C = AttnCfg<HD>;
   const int qr = C::qrows(a.max_rows, a.H / a.kv.Hkv), ns = a.n_splits;
   // The deepest K/V ring (2 to 4 tiles, at most the chunk's) within the shared memory a CTA may
-  // take: room for a second CTA per SM when the grid is larger than the SM count, the opt-in
-  // maximum otherwise. The merge buffers go over the ring only where that is what makes it fit.
+  // take: its share of the SM when the grid needs several CTAs per SM resident (up to the register
+  // bound), the opt-in maximum otherwise. The merge buffers go over the ring only where that is
+  // what makes it fit.
   const int max_nb = a.chunk > kTile ? std::min(kMaxBuf, a.chunk / kTile) : 1;
-  const size_t cap = static_cast<size_t>(ns) * a.n_groups * a.kv.Hkv > static_cast<size_t>(sm_count_cached())
-                         ? static_cast<size_t>(kTwoPerSm) : static_cast<size_t>(kMaxSmem);
+  const long ctas = static_cast<long>(ns) * a.n_groups * a.kv.Hkv, sms = sm_count_cached();
+  const int per_sm = static_cast<int>(std::min<long>(kCtasPerSm<HD>, (ctas + sms - 1) / sms));
+  const size_t cap = per_sm <= 1 ? static_cast<size_t>(kMaxSmem) : smem_share(per_sm);
   int nb = std::min(2, max_nb), ring = 0;
   bool found = false;
   for (int n = max_nb; n >= std::min(2, max_nb) && !found; --n)
@@ -563,6 +585,8 @@ cudaError_t launch(const AttnArgs& a, cudaStream_t st) {
 }
 
 }  // namespace
+
+int attention_ctas_per_sm(int hd) { return hd == 64 ? kCtasPerSm<64> : kCtasPerSm<128>; }
 
 int attention_max_splits() {
   static const int n = (clusters_fit<128>(kMaxSplits) && clusters_fit<64>(kMaxSplits)) ? kMaxSplits : 8;

@@ -449,8 +449,8 @@ sd2_status forward(sd2_ctx* c, const Model& m, const Plan& p, const FwdOut& o) {
     at.q = c->q; at.kv = m.cache(); at.layer = l; at.row_pos = p.pos;
     at.grp_row0 = p.g_row0; at.grp_nrows = p.g_nrows; at.grp_seq = p.g_seq; at.n_groups = p.n_groups;
     at.M = M; at.H = H; at.hd = hd; at.n_splits = p.n_splits; at.chunk = p.chunk; at.max_rows = p.max_rows; at.out = c->attn;
-    if (p.pre_len) {   // decode step: as many context splits as fill the GPU about twice over, no more
-      const int want = std::max(1, 2 * sm_count_cached() / std::max(1, p.n_groups * Hkv));
+    if (p.pre_len) {   // decode step: as many context splits as the GPU holds resident at once, no more
+      const int want = std::max(1, attention_ctas_per_sm(hd) * sm_count_cached() / std::max(1, p.n_groups * Hkv));
       if (want < at.n_splits) {
         at.n_splits = want;
         at.chunk = 64 * ((c->cfg.max_ctx + 64 * want - 1) / (64 * want));

@@ -204,6 +204,8 @@ cudaError_t attention(const AttnArgs& a, cudaStream_t st);
 // Most context splits (= CTAs of one cluster) attention takes on this device: 16 where clusters of
 // 16 CTAs can be scheduled, else 8.
 int attention_max_splits();
+// CTAs of one attention launch an SM can hold at once for head dim hd (4 for 64, 2 for 128).
+int attention_ctas_per_sm(int hd);
 
 // ---------------------------------------------------------------- persistent layer chain
 // Every decoder layer of one forward pass over at most 16 token rows in one cooperative launch
