@@ -166,3 +166,18 @@ def test_ring_depths_and_merge_over_the_ring(hd, k1, n_splits, chunk):
     out, err = _run(c, n_splits, chunk)
     assert err == 0
     _check(out, ref)
+
+
+def test_many_sequences_four_ctas_per_sm():
+    """16 drafter-shaped groups x 8 KV heads x 4 splits = 512 CTAs: the hd = 64 launch sized for four
+    resident CTAs per SM (its shared-memory share), in a decode step and a plain launch."""
+    lens = [70 + 61 * i for i in range(16)]
+    c = _case(8, seq_lens=lens, rows_per_group=[1] * 16, H=32, Hkv=8, hd=64)
+    ref = _reference(c)
+    pre_len = [L - 1 for L in lens]
+    out, err = _run(c, 4, 320, pre_len=pre_len, pre_stable=0, pre_fresh=1)
+    assert err == 0
+    _check(out, ref)
+    out, err = _run(c, 4, 320)
+    assert err == 0
+    _check(out, ref)
