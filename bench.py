@@ -5,6 +5,7 @@ Default workload: a Llama-3-8B-shaped verifier with a Llama-3.2-1B-shaped drafte
 prompt 512 uniform-random ids, k = 5, T = 1.0 (random-init bf16 weights N(0, 0.02^2)).
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference] [--workload NAME]
+  python bench.py --sweep      # the kernel sweep: acceptance grid, steering, 16K-context verify
 
 Prints one JSON line. `value` is emitted tokens per second per sequence (N > 1: summed over the
 N independent replicas). The reference arm times the CPU oracle on a bounded slice of the same
@@ -51,6 +52,10 @@ def parse():
     ap.add_argument("--pretrained", action="store_true",
                     help="the unsteered pretrained drafter (no steering stage, no bias): the baseline SD^2 "
                          "is compared with")
+    ap.add_argument("--sweep", action="store_true",
+                    help="instead of the iteration benchmark, the kernel sweep (one JSON line): acceptance "
+                         "over vocab x batch x k, the steering step and Eq. 2 activation at both drafter widths "
+                         "and four batch sizes, and the 8B-shaped verify at a 16384-token context")
     return ap.parse_args()
 
 
@@ -165,6 +170,118 @@ def accept_sweep(sd2, dev, hbm, B=256, k=16, V=152064, reps=10):
             "alu_note": "about 32 fp32/integer operations per logit over the two passes (exact fixed-sequence exp "
                         "and 2^-45 fixed-point normaliser); peak = SMs x 128 lanes x 2.07 GHz",
             "timing": f"CUDA events around {reps} calls of sd2_accept_logits, inputs larger than L2"}
+
+
+def timed_ms(fn, reps, flush):
+    """Median device time of fn() over reps calls (CUDA events on the current stream), L2 flushed
+    before each call outside the timed region, after two untimed calls."""
+    for _ in range(2):
+        fn()
+    evs = []
+    for _ in range(reps):
+        flush.zero_()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        fn()
+        e1.record()
+        evs.append((e0, e1))
+    torch.cuda.synchronize()
+    return statistics.median(a.elapsed_time(b) for a, b in evs)
+
+
+def run_sweep(args):
+    """The kernel sweep on one GPU: acceptance (a4) over vocab {32000, 128256, 152064} x batch
+    {1, 16, 64, 256} x k {1, 4, 8, 16} on bf16 logits N(0, 3^2) with a boosted token per row; the
+    steering step (a1: g = LN(W_hml [h; m; l]), biases W_s g) and the Eq. 2 activation for the 2048-
+    and 896-wide drafters at batch {1, 16, 64, 256} on random hidden states; the 8B-shaped verify
+    stage at a 16384-token context, batch 1, k = 5, inside the captured iteration."""
+    from paper_2511_09844_gb300 import build as _build
+    from paper_2511_09844_gb300 import sd2
+    _build.build()
+    dev = "cuda:0"
+    torch.cuda.set_device(0)
+    peaks, _ = measured_peaks()
+    hbm = float(peaks.get("hbm_gbs", 6800.0)) if peaks else 6800.0
+    flush = torch.empty(64 * 1024 * 1024, dtype=torch.float32, device=dev)   # 256 MB > L2
+    lib = sd2.load_library()
+    out = {"mode": "kernel sweep", "timing": "median of CUDA-event times per call, L2 flushed before each call",
+           "peak_hbm_gbs": hbm}
+
+    acc = []
+    for V in (32000, 128256, 152064):
+        for B in (1, 16, 64, 256):
+            for k in (1, 4, 8, 16):
+                target, draft, xhat = W.make_sweep_logits(B, k, V, seed=11, device=dev)
+                temp = torch.ones(B, dtype=torch.float32, device=dev)
+                ws = torch.empty(lib.sd2_accept_workspace_bytes(B, k), dtype=torch.uint8, device=dev)
+                step = [0]
+
+                def call():
+                    step[0] += 1
+                    sd2.accept_logits(target, draft, xhat, temp, seed=5, step=step[0], workspace=ws)
+                ms = timed_ms(call, 10, flush)
+                nbytes = (target.numel() + draft.numel()) * 2      # every logit read once: (2k+1) V B bf16
+                acc.append({"V": V, "B": B, "k": k, "ms": round(ms, 4), "logit_bytes": nbytes,
+                            "gbs": round(nbytes / (ms / 1e3) / 1e9, 1)})
+                del target, draft, xhat, ws
+    out["accept"] = acc
+
+    steer = []
+    for name in ("llama8b_1b", "qwen32b_05b"):
+        work = W.WORKLOADS[name]
+        st = W.make_steering_weights(work, 21, device=dev)
+        dv, dg, F = work.verifier.d_model, work.d_steer, work.bias_width
+        n_bias = work.drafter.n_layers * F
+        wbytes = (st["w_hml"].numel() + st["w_s"].numel()) * 2
+        for B in (1, 16, 64, 256):
+            g = torch.Generator(device=dev).manual_seed(B)
+            taps = torch.randn(B, 3, dv, generator=g, device=dev)
+            ms = timed_ms(lambda: sd2.steer(taps, st, work.steer_ln_eps, n_bias), 10, flush)
+            nbytes = wbytes + taps.numel() * 4 + B * (dg + n_bias) * 4
+            gate = torch.randn(B, F, generator=g, device=dev)
+            up = torch.randn(B, F, generator=g, device=dev)
+            bias = torch.randn(B, F, generator=g, device=dev)
+            seq = torch.arange(B, dtype=torch.int32, device=dev)
+            ms2 = timed_ms(lambda: sd2.swiglu_steered(gate, up, bias, seq), 10, flush)
+            steer.append({"pair": name, "d_v": dv, "d_g": dg, "d_d": work.drafter.d_model, "F_D": F, "B": B,
+                          "steer_ms": round(ms, 4), "steer_bytes": nbytes,
+                          "steer_gbs": round(nbytes / (ms / 1e3) / 1e9, 1),
+                          "eq2_ms": round(ms2, 4), "eq2_bytes": B * F * 14})
+        del st
+    out["steering"] = steer
+
+    # the verify stage at a 16384-token context (batch 1, k = 5) inside the captured iteration
+    work = W.WORKLOADS["llama8b_1b"]
+    prompts = W.make_prompts(work.verifier.vocab, 1, (16384, 16384), seed=7)
+    vw, dw, st = make_device_weights(work, args.seed, dev)
+    eng = sd2.SD2Engine(work, vw, dw, st, max_batch=1, max_ctx=16384 + 40 * (work.k + 1),
+                        max_prefill_tokens=16384, stream=torch.cuda.current_stream())
+    eng.prefill(prompts, [1.0], seed=args.seed)
+    for _ in range(4):
+        eng.step()
+        eng.accept()
+    eng.stage_timing(True)
+    st_ms = {"steer": 0.0, "draft": 0.0, "verify": 0.0}
+    for _ in range(8):
+        eng.step()
+        eng.accept()
+        for key, v in eng.stage_read().items():
+            st_ms[key] += v / 8
+    eng.stage_timing(False)
+    v = work.verifier
+    ctx = 16384 + 8 * (work.k + 1) // 2             # about the mean context of the timed steps
+    kv = ctx * v.n_layers * 2 * v.n_kv_heads * v.head_dim * 2
+    per_layer = v.d_model * (v.n_heads + 2 * v.n_kv_heads) * v.head_dim + v.n_heads * v.head_dim * v.d_model \
+        + 3 * v.d_ffn * v.d_model
+    wts = (v.n_layers * per_layer + v.vocab * v.d_model) * 2   # every non-embedding weight incl. lm_head, bf16
+    ms = st_ms["verify"]
+    out["verify_16k"] = {"context": 16384, "B": 1, "k": work.k, "verify_ms": round(ms, 4),
+                         "weight_bytes": wts, "kv_read_bytes": kv,
+                         "gbs": round((wts + kv) / (ms / 1e3) / 1e9, 1),
+                         "frac_of_measured_hbm": round((wts + kv) / (ms / 1e3) / 1e9 / hbm, 4),
+                         "draft_step_ms": round(st_ms["draft"] / work.k, 4),
+                         "timing": "CUDA event nodes between the stages of the captured iteration, mean of 8"}
+    return out
 
 
 def sm_count_of(dev):
@@ -514,7 +631,9 @@ def main():
         if backend == "nccl":
             torch.cuda.set_device(local_rank)
         dist.init_process_group(backend)
-    if args.impl == "reference":
+    if args.sweep:
+        line = run_sweep(args) if rank == 0 else None
+    elif args.impl == "reference":
         line = run_reference(args, rank, world)
     else:
         line, work, tau, keep = run_ours(args, rank, world, local_rank)

@@ -1075,7 +1075,8 @@ sd2_status sd2_accept_logits(const void* d_target, const void* d_draft, int32_t 
 size_t sd2_steer_workspace_bytes(int32_t B, int32_t d_v, int32_t d_g) {
   if (B < 1 || d_v < 1 || d_g < 1) return 0;
   const size_t b = static_cast<size_t>(B);
-  return ((b * 3 * d_v * 2 + 255) / 256 + (b * d_g * 4 + 255) / 256 + (b * d_g * 2 + 255) / 256) * 256;
+  // bf16 taps, f32 pre-norm g, bf16 g, and the wait flag of the tensor-core GEMMs
+  return ((b * 3 * d_v * 2 + 255) / 256 + (b * d_g * 4 + 255) / 256 + (b * d_g * 2 + 255) / 256 + 1) * 256;
 }
 
 sd2_status sd2_steer(const float* d_taps, int32_t B, int32_t d_v, const void* w_hml, const void* ln_gamma,
@@ -1094,14 +1095,16 @@ sd2_status sd2_steer(const float* d_taps, int32_t B, int32_t d_v, const void* w_
   void* x_bf = ws;
   float* g_pre = reinterpret_cast<float*>(ws + (b * 3 * d_v * 2 + 255) / 256 * 256);
   void* g_bf = ws + (b * 3 * d_v * 2 + 255) / 256 * 256 + (b * d_g * 4 + 255) / 256 * 256;
+  unsigned* err = reinterpret_cast<unsigned*>(static_cast<char*>(g_bf) + (b * d_g * 2 + 255) / 256 * 256);
+  CK(cudaMemsetAsync(err, 0, sizeof(unsigned), st));   // the tensor-core GEMMs' wait flag
   CK(gather_rows_bf16(d_taps, 3 * d_v, nullptr, 3 * d_v, B, x_bf, st));
   GemmArgs g{};
-  g.x = x_bf; g.ldx = 3 * d_v; g.M = B; g.K = 3 * d_v;
+  g.x = x_bf; g.ldx = 3 * d_v; g.M = B; g.K = 3 * d_v; g.err = err;
   g.seg[0] = {w_hml, d_g}; g.nseg = 1; g.epi = EPI_STORE; g.out = g_pre; g.ldo = d_g;
   CK(gemm(g, st));
   CK(layernorm(g_pre, ln_gamma, ln_beta, ln_eps, B, d_g, d_g_out, g_bf, st));
   GemmArgs gs{};
-  gs.x = g_bf; gs.ldx = d_g; gs.M = B; gs.K = d_g;
+  gs.x = g_bf; gs.ldx = d_g; gs.M = B; gs.K = d_g; gs.err = err;
   gs.seg[0] = {w_s, n_bias}; gs.nseg = 1; gs.epi = EPI_STORE; gs.out = d_bias; gs.ldo = n_bias;
   CK(gemm(gs, st));
   return SD2_OK;

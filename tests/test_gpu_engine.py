@@ -197,3 +197,18 @@ def test_standalone_steering_and_swiglu():
     h = sd2.swiglu_steered(gate.cuda(), up.cuda(), bb.cuda(), seq.cuda())
     ref = (up + bb[seq.long()]) * omodel.silu(gate)
     assert parity.row_rel_err(h, ref) < 1e-2
+
+
+@pytest.mark.parametrize("B", [37, 256])
+def test_standalone_steering_full_width(B):
+    """The steering step at the Qwen pair's widths (d_v 5120 -> d_g 896, 24 x 4864 biases) for 37 and
+    256 sequences: both projections on the tensor cores, with ragged and full-width token tiles."""
+    work = W.WORKLOADS["qwen32b_05b"]
+    st = W.make_steering_weights(work, 5)
+    taps = W.make_taps(B, work.verifier.d_model, seed=6)
+    nb = work.drafter.n_layers * work.drafter.d_ffn
+    g, bias = sd2.steer(taps.cuda(), parity.to_device(st), work.steer_ln_eps, nb)
+    g_ref = steering.steering_vector(taps, st, work.steer_ln_eps)
+    b_ref = steering.steering_bias(g_ref, st, work.drafter.n_layers, work.drafter.d_ffn).reshape(B, -1)
+    assert parity.row_rel_err(g, g_ref) < parity.TOL
+    assert parity.row_rel_err(bias, b_ref) < parity.TOL
