@@ -66,3 +66,54 @@ def test_product_path_fails_loudly_without_library(monkeypatch, tmp_path):
     monkeypatch.setattr(sd2, "_LIB", None)
     with pytest.raises(RuntimeError, match="missing"):
         sd2.load_library(str(tmp_path / "nope.so"))
+
+
+def test_standalone_entry_points_check_arguments_on_the_host(lib):
+    """Each standalone kernel entry rejects bad arguments with SD2_EINVAL before any device work
+    (the pointers below are never dereferenced: every call fails a host check first)."""
+    L = sd2.load_library()
+    P = ctypes.c_void_p(1 << 20)                      # a 256-byte-aligned stand-in address
+    U = ctypes.c_void_p((1 << 20) + 4)                # a misaligned one
+
+    def err_is(st, word):
+        return st == sd2.SD2_EINVAL and word in L.sd2_last_error(None)
+
+    # steering (a1): workspace size, then argument checks in order
+    assert L.sd2_steer_workspace_bytes(0, 4096, 2048) == 0
+    sizes = [L.sd2_steer_workspace_bytes(B, 4096, 2048) for B in (1, 16, 256)]
+    for B, n in zip((1, 16, 256), sizes):
+        assert n % 256 == 0 and n >= B * (3 * 4096 * 2 + 2048 * 4 + 2048 * 2) + 4
+    assert sizes == sorted(sizes)
+    ws = L.sd2_steer_workspace_bytes(2, 64, 32)
+
+    def steer(taps=P, B=2, dv=64, w_hml=P, dg=32, w_s=P, work=P, nbytes=ws):
+        return L.sd2_steer(taps, B, dv, w_hml, P, P, 1e-5, dg, w_s, 96, P, P, work, nbytes, None)
+    assert err_is(steer(taps=None), b"null")
+    assert err_is(steer(w_hml=U), b"unaligned")
+    assert err_is(steer(dv=60), b"multiples of 8")
+    assert err_is(steer(B=0), b"B >= 1")
+    assert err_is(steer(nbytes=ws - 1), b"workspace too small")
+    assert err_is(steer(work=U), b"256-byte")
+
+    # GEMM on caller buffers
+    def gemm(x=P, ldx=64, M=2, K=64, w=P, w_up=None, N=128, epi=0, out=P, ldo=128, h=None, impl=0):
+        return L.sd2_gemm(x, ldx, M, K, w, w_up, N, epi, out, ldo, h, None, None, 0, impl, None)
+    assert err_is(gemm(K=60, ldx=60), b"bad GEMM shape")
+    assert err_is(gemm(x=None), b"bad GEMM shape")
+    assert err_is(gemm(epi=99), b"unknown epilogue")
+    assert err_is(gemm(epi=2), b"missing output")           # SwiGLU without W_up and h
+    assert err_is(gemm(ldo=64), b"missing output")          # f32 output narrower than N
+    assert err_is(gemm(impl=3), b"impl")
+
+    # Eq. 2 activation alone
+    assert err_is(L.sd2_swiglu_steered(None, P, None, None, 2, 64, P, None), b"bad argument")
+    assert err_is(L.sd2_swiglu_steered(P, P, None, None, 2, 0, P, None), b"bad argument")
+
+    # paged attention
+    def attn(q=P, M=6, H=32, Hkv=8, hd=128, max_rows=6):
+        return L.sd2_attention(q, M, H, Hkv, hd, P, 64, P, 8, 0, P, P, P, P, 1, max_rows, 2, 128,
+                               None, 0, 0, P, None, None)
+    assert err_is(attn(q=None), b"null")
+    assert err_is(attn(hd=96), b"bad attention shape")
+    assert err_is(attn(H=30), b"bad attention shape")       # H not a multiple of Hkv
+    assert err_is(attn(max_rows=17), b"bad attention shape")  # 17 rows x 4 heads > 64 query vectors
