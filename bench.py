@@ -56,6 +56,9 @@ def parse():
                     help="instead of the iteration benchmark, the kernel sweep (one JSON line): acceptance "
                          "over vocab x batch x k, the steering step and Eq. 2 activation at both drafter widths "
                          "and four batch sizes, and the 8B-shaped verify at a 16384-token context")
+    ap.add_argument("--sweep-parts", default="accept,steering,verify16k",
+                    help="comma-separated parts of the kernel sweep to run (with --depth the 16K verify keeps "
+                         "only the first layers: a profiling aid)")
     return ap.parse_args()
 
 
@@ -206,9 +209,10 @@ def run_sweep(args):
     lib = sd2.load_library()
     out = {"mode": "kernel sweep", "timing": "median of CUDA-event times per call, L2 flushed before each call",
            "peak_hbm_gbs": hbm}
+    parts = set(args.sweep_parts.split(","))
 
     acc = []
-    for V in (32000, 128256, 152064):
+    for V in ((32000, 128256, 152064) if "accept" in parts else ()):
         for B in (1, 16, 64, 256):
             for k in (1, 4, 8, 16):
                 target, draft, xhat = W.make_sweep_logits(B, k, V, seed=11, device=dev)
@@ -224,10 +228,11 @@ def run_sweep(args):
                 acc.append({"V": V, "B": B, "k": k, "ms": round(ms, 4), "logit_bytes": nbytes,
                             "gbs": round(nbytes / (ms / 1e3) / 1e9, 1)})
                 del target, draft, xhat, ws
-    out["accept"] = acc
+    if acc:
+        out["accept"] = acc
 
     steer = []
-    for name in ("llama8b_1b", "qwen32b_05b"):
+    for name in (("llama8b_1b", "qwen32b_05b") if "steering" in parts else ()):
         work = W.WORKLOADS[name]
         st = W.make_steering_weights(work, 21, device=dev)
         dv, dg, F = work.verifier.d_model, work.d_steer, work.bias_width
@@ -248,10 +253,13 @@ def run_sweep(args):
                           "steer_gbs": round(nbytes / (ms / 1e3) / 1e9, 1),
                           "eq2_ms": round(ms2, 4), "eq2_bytes": B * F * 14})
         del st
-    out["steering"] = steer
+    if steer:
+        out["steering"] = steer
+    if "verify16k" not in parts:
+        return out
 
     # the verify stage at a 16384-token context (batch 1, k = 5) inside the captured iteration
-    work = W.WORKLOADS["llama8b_1b"]
+    work = bench_workload(argparse.Namespace(workload="llama8b_1b", steer_site="mlp_up", depth=args.depth))
     prompts = W.make_prompts(work.verifier.vocab, 1, (16384, 16384), seed=7)
     vw, dw, st = make_device_weights(work, args.seed, dev)
     eng = sd2.SD2Engine(work, vw, dw, st, max_batch=1, max_ctx=16384 + 40 * (work.k + 1),
@@ -275,7 +283,8 @@ def run_sweep(args):
         + 3 * v.d_ffn * v.d_model
     wts = (v.n_layers * per_layer + v.vocab * v.d_model) * 2   # every non-embedding weight incl. lm_head, bf16
     ms = st_ms["verify"]
-    out["verify_16k"] = {"context": 16384, "B": 1, "k": work.k, "verify_ms": round(ms, 4),
+    out["verify_16k"] = {"context": 16384, "B": 1, "k": work.k, "verify_layers": v.n_layers,
+                         "verify_ms": round(ms, 4),
                          "weight_bytes": wts, "kv_read_bytes": kv,
                          "gbs": round((wts + kv) / (ms / 1e3) / 1e9, 1),
                          "frac_of_measured_hbm": round((wts + kv) / (ms / 1e3) / 1e9 / hbm, 4),
