@@ -917,12 +917,9 @@ cudaError_t chain_forward(const ChainPlan& p, const ChainRun& r, cudaStream_t st
   if (S < 2) return cudaErrorInvalidValue;
   a.stages = S;
   const int smem = fixed + S * kAStage;
-  static bool configured = false;
-  if (!configured) {
-    const cudaError_t e = cudaFuncSetAttribute(chain_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmem);
-    if (e != cudaSuccess) return e;
-    configured = true;
-  }
+  static const cudaError_t configured =   // once per process (thread-safe initialisation)
+      cudaFuncSetAttribute(chain_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmem);
+  if (configured != cudaSuccess) return configured;
   cudaError_t e = cudaMemsetAsync(p.sync, 0, sizeof(unsigned), st);
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg{};

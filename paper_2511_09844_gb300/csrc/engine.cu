@@ -1129,11 +1129,17 @@ sd2_status sd2_gemm(const void* d_x, int32_t ldx, int32_t M, int32_t K, const vo
   g.epi = epilogue; g.out = d_out; g.ldo = ldo; g.out_bf = d_h; g.ldh = N;
   g.bias = d_bias; g.ld_bias = ld_bias; g.row_seq = d_seq;
   g.impl = impl == 1 ? 1 : 0;
-  static unsigned* err_word = nullptr;  // timeout flag of context-free tensor-core launches
-  if (!err_word) {
-    CK(cudaMalloc(&err_word, sizeof(unsigned)));
-    CK(cudaMemset(err_word, 0, sizeof(unsigned)));
-  }
+  // timeout flag of context-free tensor-core launches, allocated once per process (thread-safe)
+  static unsigned* const err_word = [] {
+    unsigned* w = nullptr;
+    if (cudaMalloc(&w, sizeof(unsigned)) != cudaSuccess) return static_cast<unsigned*>(nullptr);
+    if (cudaMemset(w, 0, sizeof(unsigned)) != cudaSuccess) {
+      cudaFree(w);
+      return static_cast<unsigned*>(nullptr);
+    }
+    return w;
+  }();
+  if (!err_word) return fail(nullptr, SD2_ENOMEM, "could not allocate the GEMM wait flag");
   g.err = err_word;
   if (impl == 2 && !gemm_tc_supported(g))
     return fail(nullptr, SD2_EINVAL, "shape not supported by the tensor-core GEMM (K % 64, rows % 128)");
