@@ -206,7 +206,12 @@ sd2_status sd2_accept_logits(const void* d_target, const void* d_draft, int32_t 
  * W_s g for B sequences (Sec. 3.1, Eq. 2, App. A.2).
  *   d_taps [B, 3, d_v] f32 in the order (h, m, l); weights bf16 as in sd2_weights;
  *   outputs d_g [B, d_g] f32 and d_bias [B, n_bias] f32, n_bias = L_D * F_D.
- *   d_workspace: scratch of sd2_steer_workspace_bytes(B, d_v, d_g) bytes. */
+ *   Both projections run on the tensor-core GEMM where the shapes allow it (d_g and n_bias
+ *   multiples of 128, 3 d_v and d_g multiples of 64), else on CUDA cores.
+ *   d_workspace: device scratch of sd2_steer_workspace_bytes(B, d_v, d_g) bytes, 256-byte aligned;
+ *   contents need not be initialised (it also holds the GEMM's wait flag, reset by each call), so
+ *   calls whose GPU work overlaps must not share it. Errors: SD2_EINVAL (null, unaligned, sizes,
+ *   workspace too small), SD2_ECUDA. No device memory is allocated. */
 size_t sd2_steer_workspace_bytes(int32_t B, int32_t d_v, int32_t d_g);
 sd2_status sd2_steer(const float* d_taps, int32_t B, int32_t d_v, const void* w_hml, const void* ln_gamma,
                      const void* ln_beta, float ln_eps, int32_t d_g, const void* w_s, int32_t n_bias,
