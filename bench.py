@@ -42,6 +42,8 @@ def parse():
     ap.add_argument("--workload", default="llama8b_1b", choices=sorted(W.WORKLOADS))
     ap.add_argument("--seed", type=int, default=1234)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-extras", action="store_true",
+                    help="leave out the other configurations' blocks (batch 16, Qwen pair, sweep corners, 16K verify)")
     ap.add_argument("--depth", default=None,
                     help="profiling aid: 'LV,LD' keeps the first LV verifier and LD drafter layers of the "
                          "workload (same widths, context and batch) so that an ncu capture holds a few GB; the "
@@ -75,7 +77,9 @@ def workload_config(work, n_gpus, extra=None):
            "prompt_len": list(work.prompt_len), "k": work.k, "temperature": work.temperatures[-1],
            "gen_tokens": work.gen_tokens, "parallelism": f"replicas x{n_gpus}",
            "l2": "no flush: the weights streamed every step (%.1f GB) exceed the 126 MB L2" % (
-               2e-9 * (work.verifier.param_count() + work.drafter.param_count()))}
+               2e-9 * (work.verifier.param_count() + work.drafter.param_count()))
+           if 2 * (work.verifier.param_count() + work.drafter.param_count()) > 126e6 else
+           "weights fit in L2 (a parity-sized workload)"}
     if extra:
         cfg.update(extra)
     return cfg
@@ -141,40 +145,6 @@ class ClockSampler:
 # ---------------------------------------------------------------------------------------------
 # our arm
 # ---------------------------------------------------------------------------------------------
-def accept_sweep(sd2, dev, hbm, B=256, k=16, V=152064, reps=10):
-    """The acceptance kernels (a4) alone at the sweep's largest point: bf16 logits N(0, 3^2) with a
-    boosted token per row, B = 256, k = 16, V = 152064 (2.57 GB of logits, larger than L2)."""
-    target, draft, xhat = W.make_sweep_logits(B, k, V, seed=11, device=dev)
-    temp = torch.ones(B, dtype=torch.float32, device=dev)
-    ws = torch.empty(sd2.load_library().sd2_accept_workspace_bytes(B, k), dtype=torch.uint8, device=dev)
-    for i in range(3):
-        sd2.accept_logits(target, draft, xhat, temp, seed=5, step=i + 1, workspace=ws)
-    torch.cuda.synchronize()
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record()
-    for i in range(reps):
-        sd2.accept_logits(target, draft, xhat, temp, seed=5, step=i + 4, workspace=ws)
-    e1.record()
-    torch.cuda.synchronize()
-    ms = e0.elapsed_time(e1) / reps
-    logit_bytes = (target.numel() + draft.numel()) * 2
-    gbs = 2 * logit_bytes / (ms / 1e3) / 1e9          # two passes over every row: max, exact normaliser
-    del target, draft
-    # the normaliser pass evaluates the fixed-sequence exp (about 24 fp32 operations) and the
-    # 2^-45 fixed-point sum for every logit, the max pass about 8 operations: ALU-bound, not HBM
-    elems = B * (2 * k + 1) * V
-    ops = 32.0 * elems
-    alu_peak = sm_count_of(dev) * 128 * 2.07e9 / 1e12      # fp32 lanes x max SM clock, Tops/s
-    return {"B": B, "k": k, "V": V, "dtype": "bf16", "ms_per_call": round(ms, 4),
-            "logit_bytes": logit_bytes, "algorithmic_bytes": 2 * logit_bytes, "achieved_gbs": round(gbs, 1),
-            "frac_of_measured_hbm": round(gbs / hbm, 4),
-            "bound": "alu", "alu_tops": round(ops / (ms / 1e3) / 1e12, 2), "alu_peak_tops": round(alu_peak, 1),
-            "alu_frac": round(ops / (ms / 1e3) / 1e12 / alu_peak, 4),
-            "alu_note": "about 32 fp32/integer operations per logit over the two passes (exact fixed-sequence exp "
-                        "and 2^-45 fixed-point normaliser); peak = SMs x 128 lanes x 2.07 GHz",
-            "timing": f"CUDA events around {reps} calls of sd2_accept_logits, inputs larger than L2"}
-
-
 def timed_ms(fn, reps, flush):
     """Median device time of fn() over reps calls (CUDA events on the current stream), L2 flushed
     before each call outside the timed region, after two untimed calls."""
@@ -331,6 +301,96 @@ def make_device_weights(work, seed, device):
     return vw, dw, st
 
 
+def gemm_stamp_summary(steps, hbm):
+    """The weight-streaming GEMM's roofline from the in-graph globaltimer stamps of several steps.
+
+    Each launch's time is its exposed duration: from the later of its programmatic wait returning
+    (the kernel before it has completed) and the previous GEMM's exit, to its own exit. These
+    intervals do not overlap and lie inside the step, so their sum is at most the step's time;
+    weight bytes a kernel prefetched before its wait count for it, the wait itself does not."""
+    tot_ns, tot_bytes, n = 0, 0.0, 0
+    by_stage = {"steer": [0, 0.0], "draft": [0, 0.0], "verify": [0, 0.0]}
+    span = 0
+    for launches in steps:
+        prev_exit = None
+        k1 = max(l["stage"] for l in launches)
+        for l in launches:
+            start = l["wait"] if prev_exit is None else max(l["wait"], prev_exit)
+            dur = max(0, l["exit"] - start)
+            prev_exit = l["exit"] if prev_exit is None else max(prev_exit, l["exit"])
+            tot_ns += dur
+            tot_bytes += l["bytes"]
+            n += 1
+            key = "steer" if l["stage"] == 0 else ("verify" if l["stage"] == k1 else "draft")
+            by_stage[key][0] += dur
+            by_stage[key][1] += l["bytes"]
+        span += launches[-1]["exit"] - min(l["entry"] for l in launches)
+    ns = len(steps)
+    gbs = tot_bytes / (tot_ns * 1e-9) / 1e9 if tot_ns else 0.0
+    out = {"achieved": round(gbs, 1), "frac": round(gbs / hbm, 4), "gemm_ms_per_step": round(tot_ns / ns / 1e6, 4),
+           "launches_per_step": n // ns, "bytes_per_launch": round(tot_bytes / n),
+           "avg_launch_us": round(tot_ns / n / 1e3, 3), "gemm_span_ms_per_step": round(span / ns / 1e6, 4)}
+    for key, (t, b) in by_stage.items():
+        if t:
+            out[f"{key}_gbs"] = round(b / (t * 1e-9) / 1e9, 1)
+            out[f"{key}_frac"] = round(b / (t * 1e-9) / 1e9 / hbm, 4)
+    return out
+
+
+def committed_len(eng):
+    """Committed length of each sequence (host read of the device state; outside timed regions)."""
+    st = eng.buffer(7)
+    return st[:eng.batch].tolist()
+
+
+def timed_steps(eng, steps, stream):
+    """K graph-replayed iterations bracketed by CUDA events on the engine's stream: (ms, emitted)."""
+    B, k = eng.batch, eng.k
+    n_all = torch.zeros((steps, B), dtype=torch.int32, device="cuda")
+    tok_all = torch.zeros((steps, B, k + 1), dtype=torch.int32, device="cuda")
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    ev0.record(stream)
+    for i in range(steps):
+        eng.step()
+        eng.accept(tok_all[i], n_all[i])
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    return ev0.elapsed_time(ev1), int(n_all.sum().item())
+
+
+def stage_times(eng, steps):
+    eng.stage_timing(True)
+    acc = {"steer": 0.0, "draft": 0.0, "verify": 0.0}
+    for _ in range(steps):
+        eng.step()
+        eng.accept()
+        for key, v in eng.stage_read().items():
+            acc[key] += v / steps
+    eng.stage_timing(False)
+    return acc
+
+
+def stage_bytes(work):
+    """Weights streamed by one verify (a3) and by one drafter step (a2): every layer + lm_head."""
+    def model(m):
+        per = m.d_model * (m.n_heads + 2 * m.n_kv_heads) * m.head_dim + m.n_heads * m.head_dim * m.d_model \
+            + 3 * m.d_ffn * m.d_model
+        return 2.0 * (m.n_layers * per + m.vocab * m.d_model)
+    return model(work.verifier), model(work.drafter)
+
+
+def advance_to(eng, target):
+    """Untimed iterations until every sequence's committed length reaches `target`: the timed
+    steps then sit in the middle of the configuration's generation instead of right after the prompt."""
+    steps = 0
+    while min(committed_len(eng)) < target and steps < 10000:
+        eng.step()
+        eng.accept()
+        steps += 1
+    return steps
+
+
 def run_ours(args, rank, world, local_rank):
     from paper_2511_09844_gb300 import build as _build
     from paper_2511_09844_gb300 import sd2
@@ -341,10 +401,15 @@ def run_ours(args, rank, world, local_rank):
     B, k, V = work.batch, work.k, work.verifier.vocab
     temp = work.temperatures[-1]
     prompts = W.make_prompts(V, B, work.prompt_len, seed=7 + rank)
-    steps_total = args.warmup + 2 * args.steps + 2 * min(args.steps, 8) + 2
-    max_ctx = max(len(p) for p in prompts) + steps_total * (k + 1) + k + 8
+    plen = max(len(p) for p in prompts)
+    # the timed steps start at about prompt + gen/2 - steps tokens, i.e. around the middle of the
+    # configuration's generation (tau ~ 2 tokens per step)
+    start_ctx = plen + work.gen_tokens // 2 - args.steps
+    max_ctx = plen + work.gen_tokens + (args.warmup + args.steps + 16) * (k + 1) + k + 8
     vw, dw, st = make_device_weights(work, args.seed, dev)
     stream = torch.cuda.current_stream()
+    peaks, peak_src = measured_peaks()
+    hbm = float(peaks["hbm_gbs"])
     eng = sd2.SD2Engine(work, vw, dw, st, max_batch=B, max_ctx=max_ctx,
                         max_prefill_tokens=sum(len(p) for p in prompts), stream=stream,
                         steering=not args.pretrained)
@@ -353,129 +418,113 @@ def run_ours(args, rank, world, local_rank):
     eng.prefill(prompts, [temp] * B, seed=args.seed + rank)
     torch.cuda.synchronize()
     prefill_s = time.perf_counter() - t0
-
-    tok_all = torch.zeros((args.steps, B, k + 1), dtype=torch.int32, device=dev)
-    n_all = torch.zeros((args.steps, B), dtype=torch.int32, device=dev)
-
-    def one_step(i):
+    advance = advance_to(eng, start_ctx)
+    for _ in range(args.warmup):
         eng.step()
-        eng.accept(tok_all[i], n_all[i])
-
-    for i in range(args.warmup):
-        one_step(i % args.steps)
+        eng.accept()
     torch.cuda.synchronize()
-    n_all.zero_()
+    ctx0 = committed_len(eng)
     barrier(world)
-    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     with ClockSampler(local_rank) as clocks:
-        torch.cuda.synchronize()
-        ev0.record(stream)
-        for i in range(args.steps):
-            one_step(i)
-        ev1.record(stream)
-        torch.cuda.synchronize()
+        ms, emitted = timed_steps(eng, args.steps, stream)
     barrier(world)
-    ms = ev0.elapsed_time(ev1)
-    emitted = int(n_all.sum().item())
+    ctx1 = committed_len(eng)
     ms_max, emitted_all = reduce_max_sum(ms, emitted, world)
     value = emitted_all / B / (ms_max / 1e3)
     tau = emitted / (args.steps * B)
 
-    # end to end through the public API: step, accept, read the emitted tokens back into pinned
-    # host memory every step (the per-step work of a serving loop; no per-step host input exists).
-    # The context restarts from the same prompts and seed and repeats the warm-up, so the timed
-    # steps emit the same tokens as above (the engine is deterministic) and only the host loop differs.
-    eng.prefill(prompts, [temp] * B, seed=args.seed + rank)
-    for i in range(args.warmup):
-        one_step(i % args.steps)
-    h_tok = torch.empty((B, k + 1), dtype=torch.int32, pin_memory=True)
-    h_n = torch.empty(B, dtype=torch.int32, pin_memory=True)
-    e2e_emitted = 0
-    torch.cuda.synchronize()
-    barrier(world)
-    t0 = time.perf_counter()
-    for _ in range(args.steps):
-        eng.step()
-        tok, n = eng.accept()
-        h_tok.copy_(tok, non_blocking=True)
-        h_n.copy_(n, non_blocking=True)
-        stream.synchronize()
-        e2e_emitted += int(h_n.sum())
-    e2e_s = time.perf_counter() - t0
-    e2e_s_max, e2e_all = reduce_max_sum(e2e_s * 1e3, e2e_emitted, world)
-    e2e_value = e2e_all / B / (e2e_s_max / 1e3)
-
-    # stage times inside the captured step (event nodes between the stages, graph replay as above)
+    # stage times inside the captured step (event nodes between the stages)
     stage_steps = min(args.steps, 8)
-    eng.stage_timing(True)
-    st_ms = {"steer": 0.0, "draft": 0.0, "verify": 0.0}
+    st_ms = stage_times(eng, stage_steps)
+    verify_bytes, draft_bytes = stage_bytes(work)
+    verify_gbs = verify_bytes / (st_ms["verify"] / 1e3) / 1e9 if st_ms["verify"] else 0.0
+    draft_gbs = draft_bytes / (st_ms["draft"] / k / 1e3) / 1e9 if st_ms["draft"] else 0.0
+
+    # the GEMM's roofline from globaltimer stamps inside the captured step
+    eng.gemm_timing(True)
+    stamped = []
     for _ in range(stage_steps):
         eng.step()
         eng.accept()
-        for key, v in eng.stage_read().items():
-            st_ms[key] += v / stage_steps
-    eng.stage_timing(False)
+        stamped.append(eng.gemm_timing_read())
+    eng.gemm_timing(False)
+    gemm = gemm_stamp_summary(stamped, hbm)
 
-    # one more pass with per-launch CUDA events on the engine's stream (no graphs) for the
-    # roofline of the dominant kernel
-    prof_steps = min(args.steps, 8)
+    # kernel launches per iteration: one pass with the per-launch profile (no graphs, not timed)
     eng.profile(True)
-    for _ in range(prof_steps):
+    for _ in range(2):
         eng.step()
         eng.accept()
     prof = eng.profile_read()
     eng.profile(False)
-    eng.check()
-    peaks, peak_src = measured_peaks()
-    hbm = float(peaks["hbm_gbs"])
-    g = prof["gemm"]
-    gemm_gbs = g["bytes"] / (g["ms"] / 1e3) / 1e9 if g["ms"] else 0.0
-    ver, dra = prof["verify"], prof["draft"]
-    verify_bytes = ver["bytes"] / max(1, ver["launches"])      # weights streamed by one verify (a3)
-    draft_bytes = dra["bytes"] / max(1, dra["launches"])       # weights streamed by one drafter step (a2)
-    verify_gbs = verify_bytes / (st_ms["verify"] / 1e3) / 1e9 if st_ms["verify"] else 0.0
-    draft_gbs = draft_bytes / (st_ms["draft"] / k / 1e3) / 1e9 if st_ms["draft"] else 0.0
     launches_per_step = sum(v["launches"] for name, v in prof.items()
-                            if name in ("gemm", "attention", "accept", "sample", "other")) / prof_steps
-    step_ms_prof = sum(v["ms"] for name, v in prof.items() if name in ("verify", "draft", "steer")) / prof_steps
-    gemm_share = g["ms"] / max(1e-9, sum(prof[c]["ms"] for c in ("gemm", "attention", "accept", "sample", "other")))
+                            if name in ("gemm", "attention", "accept", "sample", "other")) / 2
+    eng.check()
+
+    # end to end through the public API on host buffers: one whole request of the configuration
+    # (prompt upload, prefill, decode until gen_tokens new tokens per sequence, every step's
+    # tokens copied back to host memory), host wall clock
+    e2e_runs = []
+    for r in range(2):
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        out = eng.generate(prompts, [temp] * B, seed=args.seed + rank + 100 * r, max_new=work.gen_tokens)
+        e2e_runs.append((time.perf_counter() - t0, sum(len(o) for o in out)))
+    e2e_s = statistics.median(t for t, _ in e2e_runs)
+    e2e_tokens = e2e_runs[0][1]
+    e2e_s_max, e2e_all = reduce_max_sum(e2e_s * 1e3, e2e_tokens, world)
+    e2e_value = e2e_all / B / (e2e_s_max / 1e3)
+    e2e_steps = max(1, round((e2e_tokens / B - 1) / max(tau, 1e-9)))
+    h2d_req = 4 * sum(len(p) for p in prompts) + 4 * B
     eng.close()
     keep = (vw, dw, st) if (rank == 0 and world == 1 and not args.no_cpu_baseline) else None
+    extras = None
+    if not args.depth and not args.no_extras and rank == 0:
+        extras = other_workloads(sd2, dev, args, hbm, vw, dw, st)
     del vw, dw, st
-    sweep = accept_sweep(sd2, dev, hbm) if not args.depth else None
 
     line = {
         "metric": METRIC, "value": round(value, 3), "unit": "tokens/s/sequence", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_max / args.steps, 4),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic: random-init bf16 weights N(0, 0.02^2), uniform-random prompt ids",
-        "config": workload_config(work, world, dict({"max_ctx": max_ctx},
-                                                    **({"depth": f"{work.verifier.n_layers} verifier + "
-                                                                 f"{work.drafter.n_layers} drafter layers "
-                                                                 "(profiling aid, not the workload)"}
-                                                       if args.depth else {}),
+        "config": workload_config(work, world, dict(**({"depth": f"{work.verifier.n_layers} verifier + "
+                                                                  f"{work.drafter.n_layers} drafter layers "
+                                                                  "(profiling aid, not the workload)"}
+                                                        if args.depth else {}),
                                                     **({"drafter": "pretrained, unsteered (no steering stage)"}
                                                        if args.pretrained else {}),
                                                     **({"steering_site": {"after_mlp": "after the MLP (Sec. 5 ablation)",
                                                                           "cond_mlp": "conditional bias MLP (Sec. 5 ablation)"}
                                                         [work.steering_site]}
                                                        if work.steering_site != "mlp_up" else {}))),
+        "timed_context": {"start": ctx0, "end": ctx1, "untimed_steps_before": advance + args.warmup,
+                          "note": "the timed steps sit around the middle of the configuration's generation "
+                                  "(prompt + gen_tokens/2); e2e runs whole requests of gen_tokens"},
+        "max_ctx": max_ctx,
         "tau": round(tau, 4),
         "tokens_per_s_at_paper_tau": {"tau": 5.00, "value": round(5.00 / (ms_max / args.steps / 1e3), 2)},
         "prefill_s": round(prefill_s, 3),
-        "e2e": {"value": round(e2e_value, 3), "unit": "tokens/s/sequence", "h2d_bytes_per_step": 0,
-                "d2h_bytes_per_step": int(h_tok.numel() * 4 + h_n.numel() * 4),
-                "same_tokens_as_timed_steps": e2e_emitted == emitted},
-        "roofline": {"bound": "hbm", "kernel": "weight-streaming GEMM (all projections + lm_head)",
-                     "achieved": round(gemm_gbs, 1), "peak": hbm, "unit": "GB/s",
-                     "frac": round(gemm_gbs / hbm, 4),
-                     "traffic": gemm_traffic(g["bytes"] / max(1, g["launches"])),
-                     "traffic_note": "bytes per launch (mean over the GEMM launches): algorithmic bytes x the "
-                                     "DRAM/algorithmic ratio ncu measured on this kernel source "
-                                     "(profiles/gemm_tc_traffic.json); null if the source changed since",
-                     "peak_source": f"{peak_src} hbm_gbs (MEASURED_PEAKS.json)" if peak_src == "measured" else
-                     "fallback 6800 GB/s", "time_share": round(gemm_share, 4),
-                     "timing": f"CUDA events per launch on the engine stream over {prof_steps} profiled steps"},
+        "e2e": {"value": round(e2e_value, 3), "unit": "tokens/s/sequence",
+                "h2d_bytes_per_step": int(round(h2d_req / e2e_steps)),
+                "d2h_bytes_per_step": 4 * B * (k + 2),
+                "h2d_bytes_per_request": h2d_req, "new_tokens_per_sequence": work.gen_tokens,
+                "seconds_per_request": [round(t, 4) for t, _ in e2e_runs],
+                "how": "sd2_generate (C ABI, host buffers): prompt upload, prefill, sd2_step + sd2_accept until "
+                       f"{work.gen_tokens} new tokens per sequence, each step's tokens copied to host and waited "
+                       "for; host wall clock, median of 2 requests (graphs re-captured after each prefill)"},
+        "roofline": dict({"bound": "hbm", "kernel": "weight-streaming GEMM (gemm_tc_kernel: all projections + lm_head)",
+                          "peak": hbm, "unit": "GB/s",
+                          "traffic": gemm_traffic(gemm["bytes_per_launch"]),
+                          "traffic_note": "DRAM bytes per launch: the algorithmic bytes per launch x the "
+                                          "DRAM/algorithmic ratio ncu measured on this kernel source "
+                                          "(profiles/gemm_tc_traffic.json); null if the source changed since",
+                          "peak_source": f"{peak_src} hbm_gbs (MEASURED_PEAKS.json)" if peak_src == "measured" else
+                          "fallback 6800 GB/s",
+                          "timing": f"globaltimer stamps of every GEMM launch inside the captured step, {stage_steps} "
+                                    "steps: per launch from its programmatic wait returning (or the previous GEMM's "
+                                    "exit, if later) to its last CTA's exit; achieved = algorithmic bytes / that time"},
+                         **gemm),
         "stages": {"timing": f"CUDA event nodes between the stages of the captured step, mean of {stage_steps} steps",
                    "bytes": "weights streamed per stage (verify: all layers + lm_head; draft step: all layers + lm_head)",
                    "verify_ms": round(st_ms["verify"], 4), "verify_gb": round(verify_bytes / 1e9, 3),
@@ -483,13 +532,113 @@ def run_ours(args, rank, world, local_rank):
                    "verify_frac_of_measured": round(verify_gbs / hbm, 4),
                    "draft_step_ms": round(st_ms["draft"] / k, 4), "draft_step_gb": round(draft_bytes / 1e9, 3),
                    "draft_step_gbs": round(draft_gbs, 1), "draft_step_frac_of_measured": round(draft_gbs / hbm, 4),
-                   "steer_ms": round(st_ms["steer"], 4),
-                   "profiled_step_ms": round(step_ms_prof, 4)},
-        "accept_sweep": sweep,
+                   "steer_ms": round(st_ms["steer"], 4)},
         "gpu_launches": int(round(launches_per_step * args.steps)),
         "clocks": clocks.summary(),
     }
+    if extras:
+        line["other_configs"] = extras
     return line, work, tau, keep
+
+
+def run_pair(sd2, work, vw, dw, st, hbm, steps=10, warmup=3, max_ctx=None, temps=None, seed=1234):
+    """One workload's iteration in the captured graph: ms, tau, emitted tokens/s/seq, stage fractions."""
+    B, k, V = work.batch, work.k, work.verifier.vocab
+    prompts = W.make_prompts(V, B, work.prompt_len, seed=7)
+    temps = temps or [work.temperatures[b % len(work.temperatures)] for b in range(B)]
+    plen = max(len(p) for p in prompts)
+    max_ctx = max_ctx or plen + (warmup + steps + 8 + 8) * (k + 1) + k + 8
+    eng = sd2.SD2Engine(work, vw, dw, st, max_batch=B, max_ctx=max_ctx, max_prefill_tokens=sum(len(p) for p in prompts),
+                        stream=torch.cuda.current_stream())
+    eng.prefill(prompts, temps, seed=seed)
+    for _ in range(warmup):
+        eng.step()
+        eng.accept()
+    ms, emitted = timed_steps(eng, steps, torch.cuda.current_stream())
+    sms = stage_times(eng, 4)
+    eng.check()
+    eng.close()
+    vb, db = stage_bytes(work)
+    it = ms / steps
+    return {"ms_per_iteration": round(it, 4), "tau": round(emitted / (steps * B), 4),
+            "tokens_per_s_per_sequence": round(emitted / B / (ms / 1e3), 2),
+            "verify_ms": round(sms["verify"], 4), "verify_frac_of_measured": round(vb / (sms["verify"] / 1e3) / 1e9 / hbm, 4),
+            "draft_step_ms": round(sms["draft"] / k, 4),
+            "draft_step_frac_of_measured": round(db / (sms["draft"] / k / 1e3) / 1e9 / hbm, 4),
+            "steer_ms": round(sms["steer"], 4)}
+
+
+def other_workloads(sd2, dev, args, hbm, vw8, dw1, st8):
+    """The other configurations, each timed in the captured graph on its own workload: the 8B/1B pair
+    at batch 16 (ragged prompts, k = 8, T in {0, 0.7, 1}), the Qwen-32B/0.5B pair (batch 4, prompt
+    2048, k = 6), and the kernel sweep's corners (acceptance, steering) and its 16K-context verify."""
+    out = {}
+    flush = torch.empty(64 * 1024 * 1024, dtype=torch.float32, device=dev)   # 256 MB > L2
+    b16 = W.WORKLOADS["llama8b_1b_b16"]
+    out["llama8b_1b_b16"] = dict({"config": b16.description}, **run_pair(sd2, b16, vw8, dw1, st8, hbm))
+    # the 16K-context verify of the kernel sweep (8B-shaped, batch 1, k = 5)
+    w8 = W.WORKLOADS["llama8b_1b"]
+    prompts = W.make_prompts(w8.verifier.vocab, 1, (16384, 16384), seed=7)
+    eng = sd2.SD2Engine(w8, vw8, dw1, st8, max_batch=1, max_ctx=16384 + 40 * (w8.k + 1), max_prefill_tokens=16384,
+                        stream=torch.cuda.current_stream())
+    eng.prefill(prompts, [1.0], seed=args.seed)
+    for _ in range(4):
+        eng.step()
+        eng.accept()
+    sms = stage_times(eng, 8)
+    eng.check()
+    eng.close()
+    v = w8.verifier
+    kv = (16384 + 8) * v.n_layers * 2 * v.n_kv_heads * v.head_dim * 2
+    vb, _ = stage_bytes(w8)
+    out["verify_16k"] = {"config": "8B-shaped verify at context 16384, batch 1, k = 5 (kernel sweep)",
+                         "verify_ms": round(sms["verify"], 4), "weight_bytes": vb, "kv_read_bytes": kv,
+                         "frac_of_measured": round((vb + kv) / (sms["verify"] / 1e3) / 1e9 / hbm, 4),
+                         "draft_step_ms": round(sms["draft"] / w8.k, 4)}
+    # acceptance corners (bf16 logits N(0, 3^2) with a boosted token per row, V = 152064)
+    lib = sd2.load_library()
+    acc = []
+    for B, k in ((1, 1), (1, 16), (256, 1), (256, 16)):
+        V = 152064
+        target, draft, xhat = W.make_sweep_logits(B, k, V, seed=11, device=dev)
+        temp = torch.ones(B, dtype=torch.float32, device=dev)
+        ws = torch.empty(lib.sd2_accept_workspace_bytes(B, k), dtype=torch.uint8, device=dev)
+        step = [0]
+
+        def call():
+            step[0] += 1
+            sd2.accept_logits(target, draft, xhat, temp, seed=5, step=step[0], workspace=ws)
+        ms = timed_ms(call, 10, flush)
+        nbytes = (target.numel() + draft.numel()) * 2
+        acc.append({"V": V, "B": B, "k": k, "ms": round(ms, 4), "logit_bytes": nbytes,
+                    "frac_of_measured_hbm_one_read": round(nbytes / (ms / 1e3) / 1e9 / hbm, 4)})
+        del target, draft, xhat, ws
+    out["accept_corners"] = {"config": "sd2_accept_logits, bf16 logits N(0, 3^2) + one boosted token per row, "
+                                       "L2 flushed before each call, median of 10", "points": acc}
+    # steering step at both drafter widths
+    steer = []
+    for name in ("llama8b_1b", "qwen32b_05b"):
+        wk = W.WORKLOADS[name]
+        stw = W.make_steering_weights(wk, 21, device=dev)
+        dv, dg, F = wk.verifier.d_model, wk.d_steer, wk.bias_width
+        n_bias = wk.drafter.n_layers * F
+        wbytes = (stw["w_hml"].numel() + stw["w_s"].numel()) * 2
+        for B in (1, 256):
+            taps = torch.randn(B, 3, dv, generator=torch.Generator(device=dev).manual_seed(B), device=dev)
+            ms = timed_ms(lambda: sd2.steer(taps, stw, wk.steer_ln_eps, n_bias), 10, flush)
+            nbytes = wbytes + taps.numel() * 4 + B * (dg + n_bias) * 4
+            steer.append({"pair": name, "d_d": wk.drafter.d_model, "B": B, "ms": round(ms, 4),
+                          "frac_of_measured_hbm": round(nbytes / (ms / 1e3) / 1e9 / hbm, 4)})
+        del stw
+    out["steering"] = {"config": "sd2_steer on random hidden states N(0,1), L2 flushed, median of 10", "points": steer}
+    del flush
+    # the Qwen-32B / 0.5B pair
+    q = W.WORKLOADS["qwen32b_05b"]
+    qv, qd, qs = make_device_weights(q, args.seed, dev)
+    out["qwen32b_05b"] = dict({"config": q.description}, **run_pair(sd2, q, qv, qd, qs, hbm))
+    del qv, qd, qs
+    torch.cuda.empty_cache()
+    return out
 
 
 def barrier(world):
@@ -518,12 +667,15 @@ def reduce_max_sum(ms, count, world):
 class OracleSlices:
     """The oracle on two slices of the workload (1 and 2 decoder layers per model, same widths,
     same context); the difference prices one layer, which scales the slice to the full depth.
-    Weights: the first layers of the given models (copied to the host), or freshly generated."""
+    Weights: the first layers of the given models (copied to the host), or freshly generated.
+    The context is the prompt plus half the configuration's generation, where the GPU arm's
+    timed steps sit. Each repeat draws its random numbers from its own seed, so the accepted
+    drafts of the repeats sample the oracle's own block efficiency tau on the slices."""
 
     def __init__(self, work, seed, weights=None):
         import dataclasses
         self.work = work
-        self.context = work.prompt_len[0]
+        self.context = work.prompt_len[0] + work.gen_tokens // 2
         two_v = dataclasses.replace(work.verifier, n_layers=2)
         two_d = dataclasses.replace(work.drafter, n_layers=2)
         if weights is None:
@@ -551,22 +703,24 @@ class OracleSlices:
             self.slices.append((sw, v_n, d_n, st_n))
         self.prompt = W.make_prompts(work.verifier.vocab, 1, (self.context, self.context), seed=7)[0]
         self.seed = seed
+        self.blocks = []          # tokens emitted per oracle iteration (j + 1)
 
-    def _iteration(self, sl):
+    def _iteration(self, sl, rep):
         from oracle.sd import OracleSD
         sw, vw, dw, st = sl
-        ora = OracleSD(sw, vw, dw, st, self.seed)
+        ora = OracleSD(sw, vw, dw, st, self.seed + rep)
         ora.prefill([self.prompt], [self.work.temperatures[-1]], forced_first=[1])
         t0 = time.perf_counter()
         out = ora.stage(0, 1)
         emitted, j = ora.accept(0, 1, out)
         ora.commit(0, emitted, j, out["taps"])
+        self.blocks.append(j + 1)
         return time.perf_counter() - t0
 
-    def estimate(self):
+    def estimate(self, rep=0):
         """(seconds per iteration scaled to full depth, seconds of CPU work measured)."""
-        t1 = self._iteration(self.slices[0])
-        t2 = self._iteration(self.slices[1])
+        t1 = self._iteration(self.slices[0], rep)
+        t2 = self._iteration(self.slices[1], rep)
         per_pair = max(0.0, t2 - t1)                       # one verifier layer + one drafter layer (x k)
         fixed = max(0.0, t1 - per_pair)
         work = self.work
@@ -576,11 +730,16 @@ class OracleSlices:
         full = fixed + per_pair * (v_share * work.verifier.n_layers + (1 - v_share) * work.drafter.n_layers)
         return full, t1 + t2
 
-    def sample_text(self, measured, tau):
+    def tau(self):
+        return statistics.mean(self.blocks) if self.blocks else 1.0
+
+    def sample_text(self, measured):
         w = self.work
         return (f"oracle iterations (fp32, full recompute, no KV cache) on 1- and 2-layer slices of the "
                 f"same shapes at context {self.context}, scaled to {w.verifier.n_layers} verifier + "
-                f"{w.drafter.n_layers} drafter layers; {round(measured, 1)} s of CPU work; tau {round(tau, 3)}")
+                f"{w.drafter.n_layers} drafter layers (per-iteration seconds extrapolated from the two "
+                f"slices, not a full-depth run); {round(measured, 1)} s of CPU work; tau {round(self.tau(), 3)} "
+                f"= the oracle's own mean emitted tokens per iteration over {len(self.blocks)} iterations")
 
 
 def run_reference(args, rank, world):
@@ -588,45 +747,58 @@ def run_reference(args, rank, world):
         return None
     work = W.WORKLOADS[args.workload]
     sl = OracleSlices(work, args.seed)
-    tau = float(os.environ.get("SD2_REFERENCE_TAU", "1.0"))
-    for _ in range(args.warmup):
-        sl.estimate()
+    for r in range(args.warmup):
+        sl.estimate(rep=r)
+    sl.blocks.clear()
     per_step, cpu_s = [], 0.0
     t_start = time.perf_counter()
-    for _ in range(args.steps):
-        est, measured = sl.estimate()
+    for r in range(args.steps):
+        est, measured = sl.estimate(rep=args.warmup + r)
         per_step.append(est)
         cpu_s += measured
         if time.perf_counter() - t_start > 150:      # keep the arm within a few minutes
             break
     t_iter = statistics.median(per_step)
+    tau = sl.tau()
     value = tau / t_iter
     return {
         "impl": "reference", "metric": METRIC, "value": round(value, 6), "unit": "tokens/s/sequence",
         "n_gpus": world, "steps": len(per_step), "warmup": args.warmup, "ms_per_step": round(t_iter * 1e3, 2),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
-        "data": "synthetic: random-init weights N(0, 0.02^2), uniform-random prompt ids",
+        "data": "synthetic: random-init bf16 weights N(0, 0.02^2), uniform-random prompt ids",
         "config": workload_config(work, 1),
+        "tau": round(tau, 4), "seconds_per_iteration": round(t_iter, 3),
         "cpu_baseline": {"value": round(value, 6), "unit": "tokens/s/sequence", "cores": torch.get_num_threads(),
-                         "kind": "oracle", "sample": sl.sample_text(cpu_s, tau)},
+                         "kind": "oracle", "sample": sl.sample_text(cpu_s)},
         "e2e": {"value": round(value, 6), "unit": "tokens/s/sequence", "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
     }
 
 
-def cpu_baseline(work, seed, tau, weights=None, min_cpu_s=10.0, max_repeats=8):
-    """The oracle's sliced iteration, repeated until about min_cpu_s of CPU work is measured;
-    the median of the scaled estimates."""
+def cpu_baseline(work, seed, weights=None, min_cpu_s=10.0, max_repeats=8):
+    """The oracle's sliced iteration, repeated (each with its own seed) until about min_cpu_s of
+    CPU work is measured; the median of the scaled estimates, at the oracle's own tau. Then one
+    more estimate on a single thread."""
     sl = OracleSlices(work, seed, weights)
     ests, measured = [], 0.0
     while measured < min_cpu_s and len(ests) < max_repeats:
-        est, m = sl.estimate()
+        est, m = sl.estimate(rep=len(ests))
         ests.append(est)
         measured += m
     est = statistics.median(ests)
-    return {"value": round(tau / est, 6), "unit": "tokens/s/sequence", "cores": torch.get_num_threads(),
-            "kind": "oracle", "seconds_per_iteration": round(est, 3), "repeats": len(ests),
-            "sample": sl.sample_text(measured, tau) + f"; median of {len(ests)} repeats"}
+    tau = sl.tau()
+    out = {"value": round(tau / est, 6), "unit": "tokens/s/sequence", "cores": torch.get_num_threads(),
+           "kind": "oracle", "seconds_per_iteration": round(est, 3), "repeats": len(ests), "tau": round(tau, 4),
+           "sample": sl.sample_text(measured) + f"; median of {len(ests)} repeats"}
+    threads = torch.get_num_threads()
+    torch.set_num_threads(1)
+    try:
+        est1, m1 = sl.estimate(rep=len(ests))
+    finally:
+        torch.set_num_threads(threads)
+    out["single_thread"] = {"value": round(tau / est1, 6), "seconds_per_iteration": round(est1, 3), "cores": 1,
+                            "cpu_seconds": round(m1, 1)}
+    return out
 
 
 def main():
@@ -647,7 +819,7 @@ def main():
     else:
         line, work, tau, keep = run_ours(args, rank, world, local_rank)
         if keep is not None:
-            line["cpu_baseline"] = cpu_baseline(work, args.seed, tau, keep)
+            line["cpu_baseline"] = cpu_baseline(work, args.seed, keep)
     if rank == 0 and line is not None:
         print(json.dumps(line), flush=True)
     if world > 1:

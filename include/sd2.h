@@ -135,6 +135,17 @@ sd2_status sd2_step(sd2_ctx* ctx);
  * Errors: SD2_ESTATE (no step to accept). */
 sd2_status sd2_accept(sd2_ctx* ctx, int32_t* d_tokens, int32_t* d_n_emitted);
 
+/* One whole generation request on host buffers (the serving loop built from the calls above):
+ * copies the prompts h_tokens (back to back, h_cu_lens[batch+1] host prefix offsets) to the device,
+ * runs sd2_prefill (h_temperature, seed as there) and then sd2_step + sd2_accept until every
+ * sequence has max_new tokens or has stopped at the context's capacity, copying each step's
+ * emitted tokens back to host memory and waiting for them. Writes h_out[b * max_new + t] for
+ * t < h_n_out[b] (the first token from the prefill, then the emitted blocks, cut at max_new).
+ * Blocks the calling thread until done. Errors: those of sd2_prefill, sd2_step and sd2_accept. */
+sd2_status sd2_generate(sd2_ctx* ctx, int32_t batch, const int32_t* h_tokens, const int32_t* h_cu_lens,
+                        const float* h_temperature, uint64_t seed, int32_t max_new, int32_t* h_out,
+                        int32_t* h_n_out);
+
 /* Wait for the context's stream and report the device error word (SD2_OK, SD2_ENUMERIC,
  * SD2_ETIMEOUT, or SD2_ECAPACITY when an attention row of a step lay beyond the cache positions
  * that step was planned to write), clearing it. */
@@ -177,6 +188,31 @@ sd2_status sd2_profile_read(sd2_ctx* ctx, int64_t* launches, double* ms, double*
  * ms[2] verifier forward. SD2_ESTATE when no timed step has run. */
 sd2_status sd2_stage_timing(sd2_ctx* ctx, int32_t enable);
 sd2_status sd2_stage_read(sd2_ctx* ctx, double* ms);
+
+/* Failure-detection hooks for tests (the paper has no counterpart).
+ * sd2_debug_fail_alloc(after): process-wide; the device allocation of a context (sd2_init) that
+ * comes `after` allocations from now fails as if cudaMalloc had, once: the call that makes it
+ * returns SD2_ENOMEM and releases what it had allocated. A negative value disarms the hook.
+ * sd2_debug_expire_wait(ctx, cycles): enqueue on the context's stream one bounded device wait of
+ * the kind every kernel wait is (an mbarrier wait with a clock budget), on a barrier nothing
+ * arrives on, with a budget of `cycles` (1 .. the kernels' own budget of about 2 s): it gives up,
+ * latches the time-out in the context's error word and returns, so the next sd2_check reports
+ * SD2_ETIMEOUT and the context stays usable. */
+sd2_status sd2_debug_fail_alloc(int32_t after);
+sd2_status sd2_debug_expire_wait(sd2_ctx* ctx, int64_t cycles);
+
+/* In-graph timing of the weight-streaming GEMM: with it enabled, every following sd2_step (graph
+ * replayed as usual, re-captured when this is toggled) has each tensor-core GEMM launch record
+ * three %globaltimer stamps (ns) into a slot of its own: the earliest entry of any of its CTAs,
+ * the earliest return from the programmatic wait (the kernel before it has completed) and the
+ * latest CTA exit. The launches are otherwise exactly those of an untimed step.
+ * sd2_gemm_timing_read waits for the ctx stream and gives, for the last timed step, *n launches
+ * in stream order and, for the first min(*n, cap): stamps[3 i .. 3 i + 2], the launch's
+ * algorithmic bytes (weights + activations in + outputs) and its stage (0 steering, 1..k drafter
+ * step i, k + 1 verify). SD2_ESTATE when no timed step has run. */
+sd2_status sd2_gemm_timing(sd2_ctx* ctx, int32_t enable);
+sd2_status sd2_gemm_timing_read(sd2_ctx* ctx, int32_t cap, int32_t* n, uint64_t* stamps, double* bytes,
+                                int32_t* stage);
 
 /* ---------------------------------------------------------------------------------------------
  * Standalone kernels (no context): the acceptance and steering steps on caller buffers.
@@ -284,18 +320,29 @@ sd2_status sd2_swiglu_steered(const float* d_gate, const float* d_up, const floa
  * another component's allocator, or a loop that must not risk the device-wide synchronisation a
  * cudaMalloc/cudaFree can cause. Arguments and outputs are those of sd2_accept_logits, minus the
  * workspace: the scratch is a fixed 256 KiB device array inside the library, held on every GPU
- * that loads it until the process exits. The tables take 16*B*(2k+1) + 28*B + 68 bytes; requests
- * above 262144 bytes (256 KiB) return SD2_ECAPACITY (B = 256 with k = 16 needs 142404 bytes).
- *   - The first call on each device looks up the array's device address (cudaGetSymbolAddress)
- *     with that device current; make that first call before any stream capture.
+ * that loads it until the process exits. Its acceptance tables take 16*B*(2k+1) + 28*B + 64
+ * bytes of it and the error word sits in its last 256 bytes, so requests above 261888 bytes of
+ * tables return SD2_ECAPACITY (B = 256 with k = 16 needs 142400 bytes; k = 16 allows B <= 470).
+ *   - The array's device address belongs to a CUDA context: the first call in each context (the
+ *     device's primary context, or one the caller made current) looks it up with
+ *     cudaGetSymbolAddress, and later calls in that context reuse it. Make that first call before
+ *     any stream capture.
  *   - Every call on a device shares the one array and leaves its contents behind; the call
  *     clears what must start at zero. Calls whose GPU work overlaps (other streams, other host
  *     threads) race on the array: order them on one stream.
- *   - Errors: the status, with the text in sd2_last_error(NULL). */
+ *   - Errors: the status, with the text in sd2_last_error(NULL). Non-finite logits are found on
+ *     the GPU after the call has returned: sd2_accept_logits_noalloc_check reports them. */
 sd2_status sd2_accept_logits_noalloc(const void* d_target, const void* d_draft, int32_t dtype,
                                      const int32_t* d_xhat, const float* d_temperature, int32_t B,
                                      int32_t k, int32_t V, uint64_t seed, uint32_t step,
                                      int32_t* d_tokens, int32_t* d_n, void* stream);
+
+/* Error word of the last sd2_accept_logits_noalloc call in the current context: waits for
+ * `stream` (the stream that call was given), reads the word from the fixed array, clears it and
+ * returns SD2_ENUMERIC if that call saw a non-finite logit, else SD2_OK (SD2_ECUDA if a CUDA call
+ * fails). Allocates nothing. Each acceptance call clears the word when it starts, so the check
+ * reports the last call only. */
+sd2_status sd2_accept_logits_noalloc_check(void* stream);
 
 #ifdef __cplusplus
 }

@@ -137,6 +137,68 @@ __device__ __forceinline__ void ldsm_x2_t(uint32_t addr, uint32_t& r0, uint32_t&
                : "memory");
 }
 
+// Context clusters (R > 1): the cluster's owner of an element share writes its unnormalised partial
+// (sum over its splits of e^{m_s - M_r} acc_s, with M_r and L_r = sum e^{m_s - M_r} l_s) to global
+// scratch, then counts itself in with a self-resetting atomicInc; the last of the R owners of the
+// share combines the R partials (max, weights e^{M_r - M}, normaliser, in cluster order) and writes
+// the output. No CTA waits for another.
+template <int HD>
+__device__ void ctx_cluster_merge(const AttnArgs& a, const float2* rML, const float4* rAcc, int QR, int share,
+                                  int e_lo, int e_hi, int g, int kvh, int rank, int cr, int R, int r0, int G,
+                                  int* sLast) {
+  const int NS = a.n_splits, Hkv = a.kv.Hkv, tid = threadIdx.x;
+  constexpr int E4MAX = kMaxQV * (HD / 4);                          // partial slots per (group, KV head, cluster)
+  float4* pacc = static_cast<float4*>(a.part_acc);
+  float2* pml = static_cast<float2*>(a.part_ml);
+  const size_t base = (static_cast<size_t>(g) * Hkv + kvh) * R * E4MAX;
+  for (int e = e_lo + tid; e < e_hi; e += kThreads) {
+    const int qv = e / (HD / 4);
+    float M = -INFINITY;
+    for (int s2 = 0; s2 < NS; ++s2) M = fmaxf(M, rML[s2 * QR + qv].x);
+    const float Mu = M == -INFINITY ? 0.f : M;                      // a cluster no row can see
+    float L = 0.f;
+    float4 o = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int s2 = 0; s2 < NS; ++s2) {                               // in split order
+      const float2 ml = rML[s2 * QR + qv];
+      const float w = __expf(ml.x - Mu);
+      const float4 v = rAcc[s2 * share + (e - e_lo)];
+      L = fmaf(ml.y, w, L);
+      o.x = fmaf(w, v.x, o.x); o.y = fmaf(w, v.y, o.y);
+      o.z = fmaf(w, v.z, o.z); o.w = fmaf(w, v.w, o.w);
+    }
+    pacc[base + static_cast<size_t>(cr) * E4MAX + e] = o;
+    pml[base + static_cast<size_t>(cr) * E4MAX + e] = make_float2(M, L);
+  }
+  __threadfence();                                                  // the partials before the count
+  __syncthreads();
+  if (tid == 0) {
+    unsigned* cnt = static_cast<unsigned*>(a.part_cnt) + (static_cast<size_t>(g) * Hkv + kvh) * NS + rank;
+    *sLast = atomicInc(cnt, static_cast<unsigned>(R - 1)) == static_cast<unsigned>(R - 1) ? 1 : 0;
+  }
+  __syncthreads();
+  if (!*sLast) return;
+  __threadfence();                                                  // every cluster's partials are visible
+  for (int e = e_lo + tid; e < e_hi; e += kThreads) {
+    const int qv = e / (HD / 4), d4 = e % (HD / 4);
+    float M = -INFINITY;
+    for (int q = 0; q < R; ++q) M = fmaxf(M, __ldcg(&pml[base + static_cast<size_t>(q) * E4MAX + e]).x);
+    float L = 0.f;
+    float4 o = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int q = 0; q < R; ++q) {
+      const float2 ml = __ldcg(&pml[base + static_cast<size_t>(q) * E4MAX + e]);
+      const float4 v = __ldcg(&pacc[base + static_cast<size_t>(q) * E4MAX + e]);
+      const float w = ml.x == -INFINITY ? 0.f : __expf(ml.x - M);
+      L = fmaf(ml.y, w, L);
+      o.x = fmaf(w, v.x, o.x); o.y = fmaf(w, v.y, o.y);
+      o.z = fmaf(w, v.z, o.z); o.w = fmaf(w, v.w, o.w);
+    }
+    const float inv = 1.f / L;
+    const size_t rh = static_cast<size_t>(r0 + qv / G) * a.H + kvh * G + qv % G;
+    *reinterpret_cast<uint2*>(static_cast<bf16*>(a.out) + rh * HD + d4 * 4) =
+        make_uint2(pack_bf2(o.x * inv, o.y * inv), pack_bf2(o.z * inv, o.w * inv));
+  }
+}
+
 // NB: K/V tiles of the shared-memory layout (>= 2 when a.chunk > 64); ring: the split-merge
 // receive buffers lie over the K/V ring (n_splits > 1).
 template <int HD>
@@ -149,8 +211,11 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm<HD>) attn_kernel(const At
   __shared__ int sPmax[2];
   __shared__ int sRecv;
 
+  // x = context cluster r (of R) x rank in the cluster: split = blockIdx.x orders the context
+  // ranges, rank = the CTA's place in its cluster (its merge share)
   const int split = blockIdx.x, g = blockIdx.y, kvh = blockIdx.z;
-  const int NS = a.n_splits;
+  const int NS = a.n_splits, R = a.n_ctx_clusters > 1 ? a.n_ctx_clusters : 1;
+  const int rank = split % NS, cr = split / NS;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int g8 = lane >> 2, t4 = lane & 3;
   const int Hkv = a.kv.Hkv, G = a.H / Hkv;
@@ -179,7 +244,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm<HD>) attn_kernel(const At
   const int len = early ? a.pre_len[seq] : 0;
   int chunk = a.chunk;
   if (early) {
-    const int per = (len + a.pre_stable + a.pre_fresh + NS - 1) / NS;
+    const int per = (len + a.pre_stable + a.pre_fresh + NS * R - 1) / (NS * R);
     chunk = min(a.chunk, max(kTile, ((per + kTile - 1) / kTile) * kTile));
   }
   const int lo = split * chunk;
@@ -195,7 +260,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm<HD>) attn_kernel(const At
     fresh_hi = min(max(pre_hi, len + a.pre_stable + a.pre_fresh), row_end);
   }
   const int E4 = nqv * (HD / 4);                    // merge elements: (query vector, 4 dimensions)
-  const int e_lo = split * E4 / NS, e_hi = (split + 1) * E4 / NS;
+  const int e_lo = rank * E4 / NS, e_hi = (rank + 1) * E4 / NS;
   if (NS > 1 && tid == 0) {
     tc::mbar_init(rbar, 1);
     tc::mbar_expect_tx(rbar, static_cast<uint32_t>(NS * ((e_hi - e_lo) * 16 + nqv * 8)));
@@ -441,7 +506,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm<HD>) attn_kernel(const At
   }
   cluster_wait();                                   // every split's receive barrier is armed (and ring free)
   if (srow < nqv && squart == 0) {                  // (max, sum) of the query vector to every split
-    const uint32_t src = smem_u32(rML + split * QR + srow);
+    const uint32_t src = smem_u32(rML + rank * QR + srow);
     for (int s2 = 0; s2 < NS; ++s2)
       st_async_v2(dsmem_addr(src, static_cast<uint32_t>(s2)), dsmem_addr(rbar, static_cast<uint32_t>(s2)), m_run,
                   l_run);
@@ -458,7 +523,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm<HD>) attn_kernel(const At
         const int d = d0 + nt * 8 + 2 * t4;
         const int e = qv * (HD / 4) + (d >> 2);
         const int owner = ((e + 1) * NS - 1) / E4;
-        const uint32_t dst = smem_u32(rAcc + split * share + (e - owner * E4 / NS)) + static_cast<uint32_t>((d & 3) * 4);
+        const uint32_t dst = smem_u32(rAcc + rank * share + (e - owner * E4 / NS)) + static_cast<uint32_t>((d & 3) * 4);
         st_async_v2(dsmem_addr(dst, static_cast<uint32_t>(owner)), dsmem_addr(rbar, static_cast<uint32_t>(owner)),
                     acc[mt][nt][2 * half], acc[mt][nt][2 * half + 1]);
       }
@@ -473,6 +538,10 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm<HD>) attn_kernel(const At
   }
   __syncthreads();
   if (!sRecv) return;
+  if (R > 1) {
+    ctx_cluster_merge<HD>(a, rML, rAcc, QR, share, e_lo, e_hi, g, kvh, rank, cr, R, r0, G, &sRecv);
+    return;
+  }
   for (int e = e_lo + tid; e < e_hi; e += kThreads) {
     const int qv = e / (HD / 4), d4 = e % (HD / 4);
     // every split's values are loaded first (indices clamped, so no load waits behind a branch),
@@ -564,7 +633,8 @@ cudaError_t launch(const AttnArgs& a, cudaStream_t st) {
   // bound), the opt-in maximum otherwise. The merge buffers go over the ring only where that is
   // what makes it fit.
   const int max_nb = a.chunk > kTile ? std::min(kMaxBuf, a.chunk / kTile) : 1;
-  const long ctas = static_cast<long>(ns) * a.n_groups * a.kv.Hkv, sms = sm_count_cached();
+  const int R = a.n_ctx_clusters > 1 ? a.n_ctx_clusters : 1;
+  const long ctas = static_cast<long>(ns) * R * a.n_groups * a.kv.Hkv, sms = sm_count_cached();
   const int per_sm = static_cast<int>(std::min<long>(kCtasPerSm<HD>, (ctas + sms - 1) / sms));
   const size_t cap = per_sm <= 1 ? static_cast<size_t>(kMaxSmem) : smem_share(per_sm);
   int nb = std::min(2, max_nb), ring = 0;
@@ -580,8 +650,8 @@ cudaError_t launch(const AttnArgs& a, cudaStream_t st) {
     }
   const size_t smem = C::bytes(qr, a.chunk, ns, nb, ring);
   if (smem > static_cast<size_t>(kMaxSmem)) return cudaErrorInvalidValue;
-  return launch_pdl_cluster(attn_kernel<HD>, dim3(ns, a.n_groups, a.kv.Hkv), dim3(kThreads), smem, st, ns, a, nb,
-                            ring);
+  return launch_pdl_cluster(attn_kernel<HD>, dim3(ns * R, a.n_groups, a.kv.Hkv), dim3(kThreads), smem, st, ns, a,
+                            nb, ring);
 }
 
 }  // namespace
@@ -598,6 +668,7 @@ cudaError_t attention(const AttnArgs& a, cudaStream_t st) {
   if (a.n_splits < 1 || a.n_splits > kMaxSplits || a.chunk <= 0 || a.chunk % kTile != 0) return cudaErrorInvalidValue;
   if (a.kv.Hkv <= 0 || a.H % a.kv.Hkv != 0 || a.max_rows < 1 || a.max_rows * (a.H / a.kv.Hkv) > kMaxQV)
     return cudaErrorInvalidValue;
+  if (a.n_ctx_clusters > 1 && (a.n_splits < 2 || !a.part_acc || !a.part_ml || !a.part_cnt)) return cudaErrorInvalidValue;
   if (a.hd == 128) return launch<128>(a, st);
   if (a.hd == 64) return launch<64>(a, st);
   return cudaErrorInvalidValue;

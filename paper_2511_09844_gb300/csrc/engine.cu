@@ -14,6 +14,7 @@
 #include <string.h>
 
 #include <algorithm>
+#include <atomic>
 #include <string>
 #include <vector>
 
@@ -21,6 +22,7 @@
 #include "common.cuh"
 #include "kernels.h"
 #include "state.h"
+#include "tc.cuh"
 
 using namespace sd2;
 
@@ -107,11 +109,16 @@ struct sd2_ctx {
   bool use_chain = false;        // measured slower than the per-kernel path on GB300 (off by default)
   bool attn_in_o = false;        // decode attention inside the O projection: measured slower on GB300 (off by default)
   void *a = nullptr, *attn = nullptr, *h = nullptr, *g_bf = nullptr, *hml_in = nullptr;
+  // long-context attention: partials of the context clusters and the per-share arrival counters
+  void *attn_part_acc = nullptr, *attn_part_ml = nullptr, *attn_part_cnt = nullptr;
   int gemm_impl = 0;            // 0 tensor cores where the shape allows, 1 CUDA cores
   unsigned long long* samp_slot = nullptr;
   int* samp_counter = nullptr;
   AcceptScratch as{};
   int *tok_out = nullptr, *n_out = nullptr, *first = nullptr, *cu = nullptr;
+  // sd2_generate: the prompt on the device, the emitted tokens of a step, and their pinned host copy
+  int *gen_prompt = nullptr, *gen_first = nullptr, *gen_tok = nullptr, *gen_n = nullptr;
+  int* gen_host = nullptr;
   // step-shape plans
   Plan p_d1, p_dn, p_v;
   const int* logit_rows_d1 = nullptr;
@@ -123,6 +130,14 @@ struct sd2_ctx {
   bool stage_on = false;                  // stage markers inside the step (graph event nodes)
   bool stage_done = false;
   std::vector<cudaEvent_t> stage_ev;      // [k + 3]: before steer, after steer, after draft i, after verify
+  // in-graph GEMM timing: globaltimer stamps of every tensor-core GEMM launch of the step
+  bool gemm_timing = false;
+  bool gemm_timing_done = false;
+  unsigned long long* gstamp = nullptr;   // [kMaxStampedLaunches][3] (GemmArgs::stamp)
+  int gstamp_n = 0;                       // launches stamped by the step being enqueued
+  int cur_stage = -1;                     // 0 steering, 1..k drafter step i, k + 1 verify
+  std::vector<double> gstamp_bytes;
+  std::vector<int> gstamp_stage;
   std::vector<ProfRec> recs;
   std::vector<cudaEvent_t> ev_pool;
   std::vector<int> h_n;  // host copy of committed lengths while profiling
@@ -145,10 +160,23 @@ sd2_status fail(sd2_ctx* c, sd2_status s, const std::string& m) {
     if (e_ != cudaSuccess) return fail(c, SD2_ECUDA, std::string(#call) + ": " + cudaGetErrorString(e_)); \
   } while (0)
 
+// Test hook (sd2_debug_fail_alloc): the number of context allocations still to succeed before
+// one is made to fail; -1 when disarmed.
+std::atomic<int> g_fail_alloc_after{-1};
+
+bool injected_alloc_failure() {
+  int cur = g_fail_alloc_after.load();
+  while (cur >= 0 && !g_fail_alloc_after.compare_exchange_weak(cur, cur - 1)) {
+  }
+  return cur == 0;
+}
+
 template <typename T>
 sd2_status dalloc(sd2_ctx* c, T** p, size_t n) {
   void* v = nullptr;
   const size_t bytes = std::max<size_t>(n * sizeof(T), 256);
+  if (injected_alloc_failure())
+    return fail(c, SD2_ENOMEM, "cudaMalloc of " + std::to_string(bytes) + " bytes failed (injected by sd2_debug_fail_alloc)");
   if (cudaMalloc(&v, bytes) != cudaSuccess) {
     cudaGetLastError();
     return fail(c, SD2_ENOMEM, "cudaMalloc of " + std::to_string(bytes) + " bytes failed");
@@ -185,6 +213,9 @@ cudaError_t timed(sd2_ctx* c, int cls, double bytes, F fn) {
   c->recs.push_back(r);
   return e;
 }
+constexpr int kMaxCtxClusters = 4;   // context clusters of one long-context attention launch
+constexpr int kMaxCtxGroups = 4;     // attention row groups a launch with context clusters may have
+constexpr int kMaxStampedLaunches = 8192;   // GEMM launches of one step that in-graph timing can follow
 enum { PC_GEMM = 0, PC_ATTN = 1, PC_ACCEPT = 2, PC_SAMPLE = 3, PC_OTHER = 4, PC_VERIFY = 5, PC_DRAFT = 6, PC_STEER = 7,
        PC_N = 8 };
 
@@ -255,6 +286,24 @@ GemmArgs& tc(sd2_ctx* c, GemmArgs& g) {
   return g;
 }
 
+// One GEMM launch of the hot path: bracketed by events when profiling, and given a globaltimer
+// stamp slot when in-graph GEMM timing is on (bytes = its algorithmic bytes).
+sd2_status run_gemm(sd2_ctx* c, GemmArgs& g, double bytes) {
+  tc(c, g);
+  if (c->gemm_timing && c->gstamp && c->gstamp_n < kMaxStampedLaunches) {
+    g.stamp = c->gstamp + 3 * static_cast<size_t>(c->gstamp_n++);
+    c->gstamp_bytes.push_back(bytes);
+    c->gstamp_stage.push_back(c->cur_stage);
+  }
+  CK(timed(c, PC_GEMM, bytes, [&] { return gemm(g, c->st); }));
+  return SD2_OK;
+}
+#define RUN_GEMM(g, bytes)                        \
+  do {                                            \
+    sd2_status s_ = run_gemm(c, (g), (bytes));    \
+    if (s_ != SD2_OK) return s_;                  \
+  } while (0)
+
 // Steering bias entries per drafter layer: F_D for Eq. 2 (inside the MLP), d_D after the MLP.
 int bias_width(const sd2_ctx* c) { return c->cfg.steering_site ? c->D.c.d_model : c->D.c.d_ffn; }
 
@@ -288,7 +337,7 @@ sd2_status head(sd2_ctx* c, const Model& m, const Plan& p, const FwdOut& o, int 
       gl.norm_ssq_in = c->ssq; gl.norm_parts = final_parts; gl.norm_d = d; gl.norm_eps = mc.norm_eps;
       gl.ld_ssq = c->max_rows;
     }
-    CK(timed(c, PC_GEMM, gemm_bytes(o.n_logit_rows, mc.vocab, d, 4), [&] { return gemm(tc(c, gl), c->st); }));
+    RUN_GEMM(gl, gemm_bytes(o.n_logit_rows, mc.vocab, d, 4));
   }
   return SD2_OK;
 }
@@ -419,16 +468,16 @@ sd2_status forward(sd2_ctx* c, const Model& m, const Plan& p, const FwdOut& o) {
       c1.seg[0] = {static_cast<const char*>(c->w_c1x) + static_cast<size_t>(l) * dg * d * 2, dg}; c1.nseg = 1;
       c1.epi = EPI_SILU; c1.out_bf = c->cu_h; c1.ldh = dg;
       c1.bias = c->cg + static_cast<size_t>(l) * dg; c1.ld_bias = L * dg; c1.row_seq = p.seq;
-      CK(timed(c, PC_GEMM, gemm_bytes(M, dg, d, 2), [&] { return gemm(tc(c, c1), c->st); }));
+      RUN_GEMM(c1, gemm_bytes(M, dg, d, 2));
       GemmArgs c2{};
       c2.x = c->cu_h; c2.ldx = dg; c2.M = M; c2.K = dg;
       c2.seg[0] = {static_cast<const char*>(c->w_c2) + static_cast<size_t>(l) * F * dg * 2, F}; c2.nseg = 1;
       c2.epi = EPI_STORE; c2.out = c->rowbias; c2.ldo = F;
-      CK(timed(c, PC_GEMM, gemm_bytes(M, F, dg, 4), [&] { return gemm(tc(c, c2), c->st); }));
+      RUN_GEMM(c2, gemm_bytes(M, F, dg, 4));
     }
     GemmArgs g = qkv_args(l);
     if (fused) consume(g, parts);
-    CK(timed(c, PC_GEMM, gemm_bytes(M, m.qkv_width(), d, 4), [&] { return gemm(tc(c, g), c->st); }));
+    RUN_GEMM(g, gemm_bytes(M, m.qkv_width(), d, 4));
     // A decode step of one sequence may run its attention inside the O projection (gemm_tc.cu).
     GemmArgs go = o_args(l);
     if (fused) produce(go, m.W(l, SD2_W_MLP_NORM));
@@ -450,10 +499,24 @@ sd2_status forward(sd2_ctx* c, const Model& m, const Plan& p, const FwdOut& o) {
     at.grp_row0 = p.g_row0; at.grp_nrows = p.g_nrows; at.grp_seq = p.g_seq; at.n_groups = p.n_groups;
     at.M = M; at.H = H; at.hd = hd; at.n_splits = p.n_splits; at.chunk = p.chunk; at.max_rows = p.max_rows; at.out = c->attn;
     if (p.pre_len) {   // decode step: as many context splits as the GPU holds resident at once, no more
-      const int want = std::max(1, attention_ctas_per_sm(hd) * sm_count_cached() / std::max(1, p.n_groups * Hkv));
+      const long resident = static_cast<long>(attention_ctas_per_sm(hd)) * sm_count_cached();
+      const int want = std::max(1, static_cast<int>(resident / std::max(1, p.n_groups * Hkv)));
       if (want < at.n_splits) {
         at.n_splits = want;
         at.chunk = 64 * ((c->cfg.max_ctx + 64 * want - 1) / (64 * want));
+      } else if (at.n_splits >= 2 && p.n_groups <= kMaxCtxGroups) {
+        // long contexts: more clusters of splits along the context while the grid stays resident
+        // and every CTA keeps at least 4 tiles of 64 positions
+        int Rc = 1;
+        while (Rc < kMaxCtxClusters &&
+               static_cast<long>(at.n_splits) * (Rc + 1) * p.n_groups * Hkv <= resident &&
+               c->cfg.max_ctx >= 64 * 4 * at.n_splits * (Rc + 1))
+          ++Rc;
+        if (Rc > 1) {
+          at.n_ctx_clusters = Rc;
+          at.chunk = 64 * ((c->cfg.max_ctx + 64 * at.n_splits * Rc - 1) / (64 * at.n_splits * Rc));
+          at.part_acc = c->attn_part_acc; at.part_ml = c->attn_part_ml; at.part_cnt = c->attn_part_cnt;
+        }
       }
     }
     at.pre_len = p.pre_len; at.pre_stable = p.pre_stable; at.pre_fresh = p.pre_fresh; at.err = c->errw;
@@ -462,10 +525,10 @@ sd2_status forward(sd2_ctx* c, const Model& m, const Plan& p, const FwdOut& o) {
       for (int b = 0; b < c->B; ++b) kvb += 2.0 * 2.0 * Hkv * hd * (c->h_n[b] + 16);
     }
     if (in_o)
-      CK(timed(c, PC_GEMM, gemm_bytes(M, d, H * hd, 8) + kvb, [&] { return gemm(tc(c, go), c->st); }));
+      RUN_GEMM(go, gemm_bytes(M, d, H * hd, 8) + kvb);
     else {
       CK(timed(c, PC_ATTN, kvb, [&] { return attention(at, c->st); }));
-      CK(timed(c, PC_GEMM, gemm_bytes(M, d, H * hd, 8), [&] { return gemm(tc(c, go), c->st); }));
+      RUN_GEMM(go, gemm_bytes(M, d, H * hd, 8));
     }
     if (!fused)
       CK(timed(c, PC_OTHER, 0, [&] {
@@ -476,7 +539,7 @@ sd2_status forward(sd2_ctx* c, const Model& m, const Plan& p, const FwdOut& o) {
     if (c->cfg.steering_site == 2 && o.bias) {   // per-row biases of the conditional MLP (below)
       gu.bias = c->rowbias; gu.ld_bias = F; gu.row_seq = c->row_ident;
     }
-    CK(timed(c, PC_GEMM, gemm_bytes(M, 2 * F, d, 1), [&] { return gemm(tc(c, gu), c->st); }));
+    RUN_GEMM(gu, gemm_bytes(M, 2 * F, d, 1));
     GemmArgs gd = down_args(l);
     if (fused && l + 1 < L) {
       produce(gd, m.W(l + 1, SD2_W_ATTN_NORM));
@@ -487,7 +550,7 @@ sd2_status forward(sd2_ctx* c, const Model& m, const Plan& p, const FwdOut& o) {
       gd.tap = o.taps; gd.tap_row = o.tap_row; gd.tap_mask = tap_mask(L);
       parts = gemm_norm_parts(gd);
     }
-    CK(timed(c, PC_GEMM, gemm_bytes(M, d, F, 8), [&] { return gemm(tc(c, gd), c->st); }));
+    RUN_GEMM(gd, gemm_bytes(M, d, F, 8));
   }
   return head(c, m, p, o, fused && final_in_down ? parts : 0);
 }
@@ -502,7 +565,7 @@ sd2_status steer(sd2_ctx* c, const int* row_idx) {
   GemmArgs g{};
   g.x = c->hml_in; g.ldx = 3 * dv; g.M = B; g.K = 3 * dv;
   g.seg[0] = {c->w_hml, dg}; g.nseg = 1; g.epi = EPI_STORE; g.out = c->g_pre; g.ldo = dg;
-  CK(timed(c, PC_GEMM, gemm_bytes(B, dg, 3 * dv, 4), [&] { return gemm(tc(c, g), c->st); }));
+  RUN_GEMM(g, gemm_bytes(B, dg, 3 * dv, 4));
   CK(timed(c, PC_OTHER, 0, [&] {
     return layernorm(c->g_pre, c->ln_g, c->ln_b, c->cfg.steer_ln_eps, B, dg, c->g, c->g_bf, c->st);
   }));
@@ -511,11 +574,11 @@ sd2_status steer(sd2_ctx* c, const int* row_idx) {
   if (c->cfg.steering_site == 2) {        // the g half of the conditional bias MLP's first layer
     const int ncg = c->D.c.n_layers * dg;
     gs.seg[0] = {c->w_c1g, ncg}; gs.nseg = 1; gs.epi = EPI_STORE; gs.out = c->cg; gs.ldo = ncg;
-    CK(timed(c, PC_GEMM, gemm_bytes(B, ncg, dg, 4), [&] { return gemm(tc(c, gs), c->st); }));
+    RUN_GEMM(gs, gemm_bytes(B, ncg, dg, 4));
     return SD2_OK;
   }
   gs.seg[0] = {c->w_s, nb}; gs.nseg = 1; gs.epi = EPI_STORE; gs.out = c->bias; gs.ldo = nb;
-  CK(timed(c, PC_GEMM, gemm_bytes(B, nb, dg, 4), [&] { return gemm(tc(c, gs), c->st); }));
+  RUN_GEMM(gs, gemm_bytes(B, nb, dg, 4));
   return SD2_OK;
 }
 
@@ -531,15 +594,25 @@ sd2_status run_step(sd2_ctx* c) {
   auto mark = [&](int i) {
     if (c->stage_on) cudaEventRecordWithFlags(c->stage_ev[i], c->st, cudaEventRecordExternal);
   };
+  if (c->gemm_timing) {
+    // every stamp slot: entry and wait times at their maximum, exit time at zero
+    c->gstamp_n = 0;
+    c->gstamp_bytes.clear();
+    c->gstamp_stage.clear();
+    CK(cudaMemset2DAsync(c->gstamp, 24, 0xFF, 16, kMaxStampedLaunches, c->st));
+    CK(cudaMemset2DAsync(c->gstamp + 2, 24, 0, 8, kMaxStampedLaunches, c->st));
+  }
   mark(0);
   stage_begin();
   sd2_status s = SD2_OK;
+  c->cur_stage = 0;
   if (!c->cfg.no_steering && (s = steer(c, c->state + 2 * c->maxB)) != SD2_OK) return s;
   stage_end(PC_STEER, 2.0 * c->cfg.d_steer * 3 * c->V.c.d_model +
                           2.0 * c->cfg.d_steer * c->D.c.n_layers * static_cast<double>(c->D.c.d_ffn));
   mark(1);
   for (int i = 1; i <= k; ++i) {
     stage_begin();
+    c->cur_stage = i;
     const Plan& p = (i == 1) ? c->p_d1 : c->p_dn;
     CK(timed(c, PC_OTHER, 0, [&] {
       return plan_rows(i == 1 ? PLAN_DRAFT_FIRST : PLAN_DRAFT_NEXT, i, B, k, c->cfg.max_ctx, c->state, c->maxB,
@@ -564,6 +637,7 @@ sd2_status run_step(sd2_ctx* c) {
     mark(1 + i);
   }
   stage_begin();
+  c->cur_stage = k + 1;
   CK(timed(c, PC_OTHER, 0, [&] {
     return plan_rows(PLAN_VERIFY, 0, B, k, c->cfg.max_ctx, c->state, c->maxB, c->committed, c->xhat, c->row_tok,
                      c->row_pos, c->row_seq, c->row_valid, c->st);
@@ -583,6 +657,7 @@ sd2_status run_step(sd2_ctx* c) {
                                                  3.0 * c->V.c.d_model * c->V.c.d_ffn) +
                           2.0 * V * c->V.c.d_model);
   mark(k + 2);
+  c->cur_stage = -1;
   return SD2_OK;
 }
 
@@ -710,6 +785,16 @@ sd2_status sd2_init(const sd2_config* cfg, const sd2_weights* w, void* stream, s
     ALLOC(c->qkv, static_cast<size_t>(R) * qkvmax);
     ALLOC(c->q, static_cast<size_t>(R) * hmax);
     ALLOC(c->attn, static_cast<size_t>(R) * hmax * 2);
+    {
+      // [kMaxCtxGroups][Hkv][kMaxCtxClusters][64 * 128 / 4] float4 + float2 partials,
+      // [kMaxCtxGroups][Hkv][16] counters
+      const int hkv = std::max(cfg->verifier.n_kv_heads, cfg->drafter.n_kv_heads);
+      const size_t slots = static_cast<size_t>(kMaxCtxGroups) * hkv * kMaxCtxClusters * 64 * 32;
+      ALLOC(c->attn_part_acc, slots * 16);
+      ALLOC(c->attn_part_ml, slots * 8);
+      ALLOC(c->attn_part_cnt, static_cast<size_t>(kMaxCtxGroups) * hkv * 16 * 4);
+      CK(cudaMemset(c->attn_part_cnt, 0, static_cast<size_t>(kMaxCtxGroups) * hkv * 16 * 4));
+    }
     ALLOC(c->h, static_cast<size_t>(R) * fmax * 2);
     ALLOC(c->ssq, static_cast<size_t>(R) * (dmax / 128 + 1) * 8);
     if (cfg->steering_site == 2) {
@@ -741,6 +826,16 @@ sd2_status sd2_init(const sd2_config* cfg, const sd2_weights* w, void* stream, s
     ALLOC(c->n_out, maxB);
     ALLOC(c->first, maxB);
     ALLOC(c->cu, maxB + 1);
+    ALLOC(c->gen_prompt, cfg->max_prefill_tokens);
+    ALLOC(c->gen_first, maxB);
+    ALLOC(c->gen_tok, static_cast<size_t>(maxB) * (k + 1));
+    ALLOC(c->gen_n, maxB);
+    if (cudaHostAlloc(reinterpret_cast<void**>(&c->gen_host), sizeof(int) * static_cast<size_t>(maxB) * (k + 2),
+                      cudaHostAllocDefault) != cudaSuccess) {
+      cudaGetLastError();
+      c->gen_host = nullptr;
+      return fail(c, SD2_ENOMEM, "cudaHostAlloc of the pinned token staging buffer failed");
+    }
     CK(cudaMemset(c->samp_slot, 0, sizeof(unsigned long long) * maxB));
     CK(cudaMemset(c->samp_counter, 0, sizeof(int) * maxB));
     CK(cudaMemset(c->errw, 0, sizeof(unsigned)));
@@ -896,6 +991,7 @@ sd2_status sd2_step(sd2_ctx* c) {
     return s;
   }
   if (c->stage_on) c->stage_done = true;
+  if (c->gemm_timing) c->gemm_timing_done = true;
   c->phase = 2;
   return SD2_OK;
 }
@@ -917,6 +1013,46 @@ sd2_status sd2_accept(sd2_ctx* c, int32_t* d_tokens, int32_t* d_n) {
   return SD2_OK;
 }
 
+sd2_status sd2_generate(sd2_ctx* c, int32_t batch, const int32_t* h_tokens, const int32_t* h_cu_lens,
+                        const float* h_temperature, uint64_t seed, int32_t max_new, int32_t* h_out, int32_t* h_n_out) {
+  if (!c) return fail(nullptr, SD2_EINVAL, "null context");
+  if (!h_tokens || !h_cu_lens || !h_temperature || !h_out || !h_n_out) return fail(c, SD2_EINVAL, "null argument");
+  if (batch < 1 || batch > c->maxB) return fail(c, SD2_ECAPACITY, "batch exceeds max_batch");
+  if (max_new < 1) return fail(c, SD2_EINVAL, "max_new must be positive");
+  if (h_cu_lens[0] != 0 || h_cu_lens[batch] < batch) return fail(c, SD2_EINVAL, "bad h_cu_lens");
+  const int total = h_cu_lens[batch], k = c->cfg.k;
+  if (total > c->cfg.max_prefill_tokens) return fail(c, SD2_ECAPACITY, "prompt tokens exceed max_prefill_tokens");
+  CK(cudaMemcpyAsync(c->gen_prompt, h_tokens, sizeof(int) * static_cast<size_t>(total), cudaMemcpyHostToDevice, c->st));
+  sd2_status s = sd2_prefill(c, batch, c->gen_prompt, h_cu_lens, h_temperature, seed, c->gen_first);
+  if (s != SD2_OK) return s;
+  int* host = c->gen_host;
+  CK(cudaMemcpyAsync(host, c->gen_first, sizeof(int) * batch, cudaMemcpyDeviceToHost, c->st));
+  CK(cudaStreamSynchronize(c->st));
+  std::vector<char> stopped(batch, 0);
+  for (int b = 0; b < batch; ++b) {
+    h_out[static_cast<size_t>(b) * max_new] = host[b];
+    h_n_out[b] = 1;
+  }
+  for (;;) {
+    bool more = false;
+    for (int b = 0; b < batch; ++b) more |= !stopped[b] && h_n_out[b] < max_new;
+    if (!more) break;
+    if ((s = sd2_step(c)) != SD2_OK) return s;
+    if ((s = sd2_accept(c, c->gen_tok, c->gen_n)) != SD2_OK) return s;
+    CK(cudaMemcpyAsync(host, c->gen_tok, sizeof(int) * batch * (k + 1), cudaMemcpyDeviceToHost, c->st));
+    CK(cudaMemcpyAsync(host + static_cast<size_t>(batch) * (k + 1), c->gen_n, sizeof(int) * batch,
+                       cudaMemcpyDeviceToHost, c->st));
+    CK(cudaStreamSynchronize(c->st));
+    const int* hn = host + static_cast<size_t>(batch) * (k + 1);
+    for (int b = 0; b < batch; ++b) {
+      if (hn[b] <= 0) { stopped[b] = 1; continue; }      // capacity reached: the sequence has stopped
+      for (int t = 0; t < hn[b] && h_n_out[b] < max_new; ++t)
+        h_out[static_cast<size_t>(b) * max_new + h_n_out[b]++] = host[b * (k + 1) + t];
+    }
+  }
+  return SD2_OK;
+}
+
 sd2_status sd2_check(sd2_ctx* c) {
   if (!c) return fail(nullptr, SD2_EINVAL, "null context");
   unsigned w = 0;
@@ -926,6 +1062,18 @@ sd2_status sd2_check(sd2_ctx* c) {
   if (w & ERR_NONFINITE) return fail(c, SD2_ENUMERIC, "non-finite logits seen on the device");
   if (w & ERR_TIMEOUT) return fail(c, SD2_ETIMEOUT, "a device-side wait timed out");
   if (w & ERR_RANGE) return fail(c, SD2_ECAPACITY, "an attention row lay outside the positions planned for the step");
+  return SD2_OK;
+}
+
+sd2_status sd2_debug_fail_alloc(int32_t after) {
+  g_fail_alloc_after.store(after < 0 ? -1 : after);
+  return SD2_OK;
+}
+
+sd2_status sd2_debug_expire_wait(sd2_ctx* c, int64_t cycles) {
+  if (!c) return fail(nullptr, SD2_EINVAL, "null context");
+  if (cycles < 1 || cycles > sd2::tc::kWaitCycles) return fail(c, SD2_EINVAL, "cycles must be in [1, the kernels' wait budget]");
+  CK(expire_wait(c->errw, cycles, c->st));
   return SD2_OK;
 }
 
@@ -968,6 +1116,7 @@ sd2_status sd2_free(sd2_ctx* c) {
   for (auto e : c->stage_ev)
     if (e) cudaEventDestroy(e);
   if (c->cap_st) cudaStreamDestroy(c->cap_st);
+  if (c->gen_host) cudaFreeHost(c->gen_host);
   delete c;
   return SD2_OK;
 }
@@ -1023,6 +1172,30 @@ sd2_status sd2_stage_read(sd2_ctx* c, double* ms) {
   ms[1] = t;
   CK(cudaEventElapsedTime(&t, c->stage_ev[k + 1], c->stage_ev[k + 2]));
   ms[2] = t;
+  return SD2_OK;
+}
+
+sd2_status sd2_gemm_timing(sd2_ctx* c, int32_t enable) {
+  if (!c) return fail(nullptr, SD2_EINVAL, "null context");
+  const bool on = enable != 0;
+  if (on && !c->gstamp) ALLOC(c->gstamp, 3 * static_cast<size_t>(kMaxStampedLaunches));
+  if (on != c->gemm_timing) drop_graphs(c);
+  c->gemm_timing = on;
+  c->gemm_timing_done = false;
+  return SD2_OK;
+}
+
+sd2_status sd2_gemm_timing_read(sd2_ctx* c, int32_t cap, int32_t* n, uint64_t* stamps, double* bytes, int32_t* stage) {
+  if (!c || !n || !stamps || !bytes || !stage) return fail(c, SD2_EINVAL, "null argument");
+  if (!c->gemm_timing || !c->gemm_timing_done) return fail(c, SD2_ESTATE, "no step has run with GEMM timing on");
+  const int m = std::min(c->gstamp_n, std::max(0, cap));
+  *n = c->gstamp_n;
+  CK(cudaStreamSynchronize(c->st));
+  if (m > 0) CK(cudaMemcpy(stamps, c->gstamp, sizeof(uint64_t) * 3 * m, cudaMemcpyDeviceToHost));
+  for (int i = 0; i < m; ++i) {
+    bytes[i] = c->gstamp_bytes[i];
+    stage[i] = c->gstamp_stage[i];
+  }
   return SD2_OK;
 }
 

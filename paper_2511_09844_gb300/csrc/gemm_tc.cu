@@ -61,6 +61,7 @@ struct TcArgs {
   int sp;            // CTAs per tile (cluster size); 1 = whole tiles, persistent
   int tiles;
   unsigned* err;
+  unsigned long long* stamp;   // in-graph timing (GemmArgs::stamp), may be null
   // EPI_QKV
   float* q_out;
   bf16* kv_pool;
@@ -89,6 +90,12 @@ struct TcArgs {
 
 
 constexpr int kMaxNT = 256;  // token columns per tile
+
+__device__ __forceinline__ unsigned long long global_ns() {
+  unsigned long long t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
 constexpr int kXS = 17;   // padded row of the epilogue exchange buffer (128 rows x 16 columns)
 
 // ------------------------------------------------------------------------------ epilogue stores
@@ -486,6 +493,12 @@ __device__ __forceinline__ void splitk_epilogue(const TcArgs& a, const SplitK& s
     } else if (leader) {
       wait_bar_budget(sk.rbar, 0, kDrainCycles);   // let partials still in flight land before leaving
     }
+  } else if (leader) {
+    // This rank's accumulator never completed (a wait gave up), so it pushes nothing; the other
+    // ranks push their partials of its pairs right after their own accumulators, with no wait in
+    // between, and may still be doing so: let them land before the CTA (and its shared memory)
+    // goes away. Every rank reaches its pushes, or skips them, within the bounded waits above.
+    wait_bar_budget(sk.rbar, 0, kDrainCycles);
   }
 }
 
@@ -512,6 +525,7 @@ __global__ void __launch_bounds__(kThreads, 2) gemm_tc_kernel(const __grid_const
   uint32_t ncols = 32;
   while (ncols < static_cast<uint32_t>((sp == 1 ? 2 : 1) * NT)) ncols <<= 1;
   const int rank = sp > 1 ? static_cast<int>(cluster_rank()) : 0;
+  if (a.stamp && threadIdx.x == 0) atomicMin(&a.stamp[0], global_ns());
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
@@ -605,6 +619,7 @@ __global__ void __launch_bounds__(kThreads, 2) gemm_tc_kernel(const __grid_const
         load_a(j, ca);
       }
       pdl_wait();
+      if (a.stamp) atomicMin(&a.stamp[1], global_ns());
       for (uint32_t j = 0; j < pre; ++j, advance(cb)) load_b(j, cb);
       uint32_t j = pre;
       bool ok = true;
@@ -696,6 +711,7 @@ __global__ void __launch_bounds__(kThreads, 2) gemm_tc_kernel(const __grid_const
   __syncthreads();
   tc_fence_after();
   if (warp == 1) tmem_dealloc(tmem, ncols);
+  if (a.stamp && threadIdx.x == 0) atomicMax(&a.stamp[2], global_ns());
 }
 
 
@@ -1261,6 +1277,7 @@ cudaError_t gemm_tc(const GemmArgs& g, unsigned* err, cudaStream_t st) {
   a.epi = g.epi; a.out = g.out; a.ldo = g.ldo; a.out_bf = static_cast<bf16*>(g.out_bf); a.ldh = g.ldh;
   a.bias = g.bias; a.ld_bias = g.ld_bias; a.row_seq = g.row_seq;
   a.err = err;
+  a.stamp = g.stamp;
   a.q_out = g.q_out; a.kv_pool = static_cast<bf16*>(g.kv_pool); a.kv_table = g.kv_table;
   a.kv_bt_stride = g.kv_bt_stride; a.kv_n_blocks = g.kv_n_blocks; a.n_heads = g.n_heads;
   a.n_kv_heads = g.n_kv_heads; a.head_dim = g.head_dim; a.layer = g.layer; a.rope_cs = g.rope_cs;

@@ -85,6 +85,11 @@ struct GemmArgs {
   // shape allows, 1 = CUDA cores
   unsigned* err;
   int impl;
+  // In-graph timing (tensor-core path; may be null): three words per launch, set with atomics on
+  // %globaltimer (ns): [0] earliest CTA entry, [1] earliest return from the programmatic wait (the
+  // predecessor grid has completed), [2] latest CTA exit. The caller presets [0], [1] to ~0 and
+  // [2] to 0.
+  unsigned long long* stamp;
   // EPI_QKV
   float* q_out;
   void* kv_pool;
@@ -199,6 +204,14 @@ struct AttnArgs {
   const int* pre_len;
   int pre_stable, pre_fresh;
   unsigned* err;         // ERR_TIMEOUT (split merge), ERR_RANGE (a row outside the planned range); may be null
+  // Context clusters: R > 1 clusters of n_splits CTAs each share the context (R * n_splits splits of
+  // `chunk`); their partials meet in part_acc / part_ml ([n_groups][Hkv][R][64 * hd/4] float4 /
+  // float2) and the last owner of each share, counted in part_cnt ([n_groups][Hkv][n_splits],
+  // zero-initialised, self-resetting), writes the output. Needs n_splits >= 2.
+  int n_ctx_clusters = 1;
+  void* part_acc = nullptr;
+  void* part_ml = nullptr;
+  void* part_cnt = nullptr;
 };
 cudaError_t attention(const AttnArgs& a, cudaStream_t st);
 // Most context splits (= CTAs of one cluster) attention takes on this device: 16 where clusters of

@@ -13,6 +13,7 @@
 #include "common.cuh"
 #include "kernels.h"
 #include "state.h"
+#include "tc.cuh"
 
 namespace sd2 {
 namespace {
@@ -84,7 +85,27 @@ __global__ void prefill_init_kernel(int B, int max_ctx, const int* prompts, cons
   }
 }
 
+// One bounded mbarrier wait, in the form every wait of the library's kernels takes
+// (tc::wait_bar_limit), on a barrier that nothing arrives on: after `cycles` clock cycles the wait
+// gives up, latches ERR_TIMEOUT in *err and the kernel returns. Nothing is in flight when it does.
+__global__ void expire_wait_kernel(unsigned* err, long long cycles) {
+  __shared__ __align__(8) uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x == 0) {
+    tc::mbar_init(tc::smem_u32(&bar), 1);
+    abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) tc::wait_bar_limit(tc::smem_u32(&bar), 0, &abort_flag, err, cycles);
+}
+
 }  // namespace
+
+cudaError_t expire_wait(unsigned* err, long long cycles, cudaStream_t st) {
+  expire_wait_kernel<<<1, 32, 0, st>>>(err, cycles);
+  return cudaGetLastError();
+}
 
 cudaError_t plan_rows(int mode, int i, int B, int k, int max_ctx, const int* state, int maxB, const int* committed,
                       const int* xhat, int* tok, int* pos, int* seq, int* valid, cudaStream_t st) {

@@ -14,5 +14,8 @@ cudaError_t commit(int B, int k, int max_ctx, int* state, int maxB, int* committ
                    int* iter, cudaStream_t st);
 cudaError_t prefill_init(int B, int max_ctx, const int* prompts, const int* cu, const int* first, int* state, int maxB,
                          int* committed, int* first_out, cudaStream_t st);
+// One bounded device wait that nothing satisfies: gives up after `cycles` clock cycles and
+// latches ERR_TIMEOUT in *err (failure-detection test of the bounded waits).
+cudaError_t expire_wait(unsigned* err, long long cycles, cudaStream_t st);
 
 }  // namespace sd2

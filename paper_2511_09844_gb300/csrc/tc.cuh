@@ -109,20 +109,24 @@ __device__ __forceinline__ uint32_t idesc_bf16(int M, int N) {
 
 // Bounded wait on an mbarrier phase. Gives up when another role has aborted, or when the clock
 // budget runs out (then records the timeout and raises the abort flag itself).
-__device__ __forceinline__ bool wait_bar(uint32_t bar, uint32_t parity, volatile int* abort_flag, unsigned* err) {
+__device__ __forceinline__ bool wait_bar_limit(uint32_t bar, uint32_t parity, volatile int* abort_flag, unsigned* err,
+                                               long long limit) {
   if (mbar_try(bar, parity)) return true;
   const long long t0 = clock64();
   for (uint32_t it = 1;; ++it) {
     if (mbar_try(bar, parity)) return true;
     if ((it & 31) == 0) {
       if (*abort_flag) return false;
-      if (clock64() - t0 > kWaitCycles) {
+      if (clock64() - t0 > limit) {
         *abort_flag = 1;
         atomicOr(err, static_cast<unsigned>(ERR_TIMEOUT));
         return false;
       }
     }
   }
+}
+__device__ __forceinline__ bool wait_bar(uint32_t bar, uint32_t parity, volatile int* abort_flag, unsigned* err) {
+  return wait_bar_limit(bar, parity, abort_flag, err, kWaitCycles);
 }
 __device__ __forceinline__ bool wait_bar_budget(uint32_t bar, uint32_t parity, long long cycles) {
   const long long t0 = clock64();

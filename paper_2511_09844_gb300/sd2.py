@@ -28,7 +28,9 @@ EXPORTS = ["sd2_init", "sd2_prefill", "sd2_step", "sd2_accept", "sd2_check", "sd
            "sd2_set_graphs", "sd2_debug_buffer", "sd2_profile", "sd2_profile_read", "sd2_accept_workspace_bytes",
            "sd2_accept_logits", "sd2_steer_workspace_bytes", "sd2_steer", "sd2_swiglu_steered",
            "sd2_accept_logits_noalloc", "sd2_gemm", "sd2_set_gemm_impl", "sd2_stage_timing", "sd2_stage_read",
-           "sd2_set_drafter_chain", "sd2_attention", "sd2_set_fused_attention"]
+           "sd2_set_drafter_chain", "sd2_attention", "sd2_set_fused_attention",
+           "sd2_accept_logits_noalloc_check", "sd2_debug_fail_alloc", "sd2_debug_expire_wait",
+           "sd2_gemm_timing", "sd2_gemm_timing_read", "sd2_generate"]
 
 
 class LMConfig(ctypes.Structure):
@@ -98,6 +100,14 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
     lib.sd2_set_fused_attention.argtypes = [c_void_p, c_int32]
     lib.sd2_accept_logits_noalloc.argtypes = [c_void_p, c_void_p, c_int32, c_void_p, c_void_p, c_int32, c_int32,
                                               c_int32, c_uint64, c_uint32, c_void_p, c_void_p, c_void_p]
+    lib.sd2_accept_logits_noalloc_check.argtypes = [c_void_p]
+    lib.sd2_debug_fail_alloc.argtypes = [c_int32]
+    lib.sd2_gemm_timing.argtypes = [c_void_p, c_int32]
+    lib.sd2_generate.argtypes = [c_void_p, c_int32, POINTER(c_int32), POINTER(c_int32), POINTER(c_float), c_uint64,
+                                 c_int32, POINTER(c_int32), POINTER(c_int32)]
+    lib.sd2_gemm_timing_read.argtypes = [c_void_p, c_int32, POINTER(c_int32), POINTER(c_uint64), POINTER(c_double),
+                                         POINTER(c_int32)]
+    lib.sd2_debug_expire_wait.argtypes = [c_void_p, c_int64]
     for name in EXPORTS:
         if name not in ("sd2_last_error", "sd2_accept_workspace_bytes", "sd2_steer_workspace_bytes"):
             getattr(lib, name).restype = c_int32
@@ -207,6 +217,24 @@ class SD2Engine:
         self.n_out = torch.empty(self.batch, dtype=torch.int32, device="cuda")
         return first
 
+    def generate(self, prompts: Sequence[Sequence[int]], temps: Sequence[float], seed: int, max_new: int):
+        """A whole request through sd2_generate on host buffers: returns each sequence's new tokens."""
+        flat = [t for p in prompts for t in p]
+        cu = [0]
+        for p in prompts:
+            cu.append(cu[-1] + len(p))
+        B = len(prompts)
+        tok = (c_int32 * len(flat))(*flat)
+        cu_arr = (c_int32 * len(cu))(*cu)
+        t_arr = (c_float * B)(*[float(t) for t in temps])
+        out = (c_int32 * (B * max_new))()
+        n = (c_int32 * B)()
+        self._call(self.lib.sd2_generate(self.ctx, B, tok, cu_arr, t_arr, c_uint64(seed), max_new, out, n))
+        self.batch = B
+        self.tokens_out = torch.empty((B, self.k + 1), dtype=torch.int32, device="cuda")
+        self.n_out = torch.empty(B, dtype=torch.int32, device="cuda")
+        return [[out[b * max_new + t] for t in range(n[b])] for b in range(B)]
+
     def step(self):
         self._call(self.lib.sd2_step(self.ctx))
 
@@ -260,6 +288,18 @@ class SD2Engine:
         ms = (c_double * 3)()
         self._call(self.lib.sd2_stage_read(self.ctx, ms))
         return {"steer": ms[0], "draft": ms[1], "verify": ms[2]}
+
+    def gemm_timing(self, enable: bool):
+        """In-graph GEMM timing: globaltimer stamps of every tensor-core GEMM launch of a step."""
+        self._call(self.lib.sd2_gemm_timing(self.ctx, 1 if enable else 0))
+
+    def gemm_timing_read(self, cap: int = 8192):
+        """Launches of the last timed step in stream order: dicts with entry/wait/exit ns, bytes, stage."""
+        n = c_int32()
+        st, by, sg = (c_uint64 * (3 * cap))(), (c_double * cap)(), (c_int32 * cap)()
+        self._call(self.lib.sd2_gemm_timing_read(self.ctx, cap, ctypes.byref(n), st, by, sg))
+        return [{"entry": st[3 * i], "wait": st[3 * i + 1], "exit": st[3 * i + 2], "bytes": by[i], "stage": sg[i]}
+                for i in range(min(n.value, cap))]
 
     def close(self):
         if getattr(self, "ctx", None) is not None and self.ctx.value:

@@ -85,6 +85,18 @@ def test_long_context_verify_16k():
     assert rep.blocks == 1
 
 
+def test_long_context_two_ragged_sequences():
+    """Two sequences of 12000 and 16384 tokens (8B/1B one-layer slices, k = 2): at this context the
+    drafter's decode attention spreads each sequence over two clusters of context splits whose
+    partials meet in global scratch, and the two sequences split their own contexts differently."""
+    work = _one_layer(W.WORKLOADS["llama8b_1b"], k=2, batch=2, prompt_len=(12000, 16384))
+    vw, dw, st = _weights(work, 37)
+    V = work.verifier.vocab
+    prompts = W.make_prompts(V, 1, (12000, 12000), seed=23) + W.make_prompts(V, 1, (16384, 16384), seed=24)
+    rep = parity.run(work, vw, dw, st, prompts, [1.0, 0.0], seed=9, n_steps=2)
+    assert rep.blocks == 4
+
+
 def test_full_depth_decisions_bit_exact():
     """Full 32-layer / 16-layer models at the benchmark's shape: the oracle's draft samples and
     acceptance on the engine's logits equal the engine's tokens; committed state follows."""
