@@ -123,8 +123,27 @@ __global__ void __launch_bounds__(kThreads) gemm_simt_kernel(const GemmArgs a, i
 
 }  // namespace
 
+// Token rows above which the tensor-core QKV projection stores plain q/k/v and a separate kernel
+// rotates and appends them: the fused epilogue fetches each output's rotary factors and cache
+// block from global memory, and with this many token columns per tile those dependent loads
+// (several rounds per owner thread) cost more than one extra elementwise kernel.
+constexpr int kQkvFusedMaxRows = 64;
+
 cudaError_t gemm(const GemmArgs& a, cudaStream_t st) {
   if (a.attn_q) return a.impl != 1 && a.err && gemm_attn_supported(a) ? gemm_tc(a, a.err, st) : cudaErrorNotSupported;
+  if (a.impl != 1 && a.err && a.epi == EPI_QKV && a.M > kQkvFusedMaxRows) {
+    GemmArgs s = a;
+    s.epi = EPI_STORE;
+    if (gemm_tc_supported(s)) {
+      cudaError_t e = gemm_tc(s, a.err, st);
+      if (e != cudaSuccess) return e;
+      KVCache kv;
+      kv.pool = a.kv_pool; kv.table = a.kv_table; kv.bt_stride = a.kv_bt_stride; kv.n_blocks = a.kv_n_blocks;
+      kv.Hkv = a.n_kv_heads; kv.hd = a.head_dim;
+      return rope_append(a.out, a.rope_cs, a.M, a.n_heads, a.n_kv_heads, a.head_dim, a.row_seq, a.row_pos,
+                         a.row_valid, kv, a.layer, a.q_out, st);
+    }
+  }
   if (a.impl != 1 && a.err && gemm_tc_supported(a)) return gemm_tc(a, a.err, st);
   if (a.norm_out || a.norm_ssq_in) return cudaErrorNotSupported;  // the fused RMSNorm is tensor-core only
   if (a.epi != EPI_QKV) return gemm_simt(a, st);

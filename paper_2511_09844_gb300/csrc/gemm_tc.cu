@@ -1113,6 +1113,37 @@ int sm_count() {
 constexpr int kSmemBudget = 227 * 1024;
 constexpr int kSmemShared = 110 * 1024;
 
+// Clusters of `size` CTAs of gemm_tc_kernel with `smem` bytes of dynamic shared memory that the
+// device holds at once. Clusters must fit whole into a GPC, so this is less than
+// SMs x (CTAs per SM) / size: with one CTA per SM, 46 clusters of 3 (138 CTAs) or 15 of 7 fit on a
+// 152-SM GB300. Cached per (size, smem).
+int max_active_clusters(int size, int smem) {
+  static std::mutex mu;
+  static std::unordered_map<long long, int> cache;
+  const long long key = (static_cast<long long>(size) << 32) | static_cast<unsigned>(smem);
+  std::lock_guard<std::mutex> lock(mu);
+  auto it = cache.find(key);
+  if (it != cache.end()) return it->second;
+  int n = 0;
+  if (cudaFuncSetAttribute(gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024) == cudaSuccess) {
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = dim3(static_cast<unsigned>(size));
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = static_cast<size_t>(smem);
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = static_cast<unsigned>(size);
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    if (cudaOccupancyMaxActiveClusters(&n, gemm_tc_kernel, &cfg) != cudaSuccess) n = 0;
+  }
+  cudaGetLastError();
+  cache.emplace(key, n);
+  return n;
+}
+
 // Launch shape of a grid of `tiles` weight tiles x token tiles: split factor sp (CTAs per tile, one
 // cluster), ring stages, dynamic shared memory and grid. Two CTAs share an SM when the ring (at
 // least 3 stages) and the split-K receive buffer fit in half its shared memory: more weight bytes in
@@ -1148,6 +1179,9 @@ TcPlan plan_tc(int tiles, int NT, int KB) {
       pl.sp = sp;
       pl.stages = S;
       pl.smem = fixed_of(sp) + S * stage_bytes;
+      // every tile's cluster must be resident in the one wave (a cluster left over would run after
+      // the others and double the launch's time)
+      if (sp > 1 && max_active_clusters(sp, pl.smem) < tiles) continue;
       pl.grid = sp > 1 ? tiles * sp : std::min(tiles, occ * sms);
       const int active = std::min(pl.grid, occ * sms);
       if (active > best_active) {
