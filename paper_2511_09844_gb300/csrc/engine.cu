@@ -84,6 +84,8 @@ struct sd2_ctx {
   cudaStream_t st = nullptr, cap_st = nullptr;
   int B = 0, phase = 0, maxB = 0, max_rows = 0;
   unsigned long long seed = 0;
+  unsigned long long* seed_d = nullptr;   // the request's seed on the device, read by the captured step
+  std::vector<int> graph_key;             // batch, k and the step-shape tables the captured graphs were built on
   std::string err;
   std::vector<void*> allocs;
   // device state
@@ -627,7 +629,7 @@ sd2_status run_step(sd2_ctx* c) {
     s = chain_takes(c, p) ? forward_chain(c, c->D, p, o) : forward(c, c->D, p, o);
     if (s != SD2_OK) return s;
     CK(timed(c, PC_SAMPLE, 4.0 * B * V, [&] {
-      return sample_rows(o.logits, o.ld_logits, B, V, c->temp, c->seed, RNG_DRAFT, i, c->iter, 0, c->xhat + (i - 1), k,
+      return sample_rows(o.logits, o.ld_logits, B, V, c->temp, Seed{0, c->seed_d}, RNG_DRAFT, i, c->iter, 0, c->xhat + (i - 1), k,
                          nullptr, 0, c->samp_slot, c->samp_counter, c->errw, c->st);
     }));
     stage_end(PC_DRAFT, 2.0 * c->D.c.n_layers * (static_cast<double>(c->D.c.d_model) * c->D.qkv_width() +
@@ -664,7 +666,7 @@ sd2_status run_step(sd2_ctx* c) {
 sd2_status run_accept(sd2_ctx* c) {
   const int B = c->B, k = c->cfg.k, V = c->V.c.vocab;
   CK(timed(c, PC_ACCEPT, 4.0 * B * (2 * k + 1) * V, [&] {
-    return accept_blocks(c->logits_t, c->logits_d, SD2_DTYPE_F32, c->xhat, c->temp, B, k, V, c->seed, 0, c->iter,
+    return accept_blocks(c->logits_t, c->logits_d, SD2_DTYPE_F32, c->xhat, c->temp, B, k, V, Seed{0, c->seed_d}, 0, c->iter,
                          c->state + 3 * c->maxB, c->tok_out, c->n_out, c->as, c->errw, c->st);
   }));
   CK(timed(c, PC_OTHER, 0, [&] {
@@ -774,6 +776,7 @@ sd2_status sd2_init(const sd2_config* cfg, const sd2_weights* w, void* stream, s
     ALLOC(c->state, 4 * maxB);
     ALLOC(c->committed, static_cast<size_t>(maxB) * cfg->max_ctx);
     ALLOC(c->iter, 1);
+    ALLOC(c->seed_d, 1);
     ALLOC(c->xhat, static_cast<size_t>(maxB) * k);
     ALLOC(c->temp, maxB);
     ALLOC(c->errw, 1);
@@ -879,7 +882,6 @@ sd2_status sd2_prefill(sd2_ctx* c, int32_t batch, const int32_t* d_tokens, const
     maxlen = std::max(maxlen, len);
   }
   if (total > c->cfg.max_prefill_tokens) return fail(c, SD2_ECAPACITY, "prompt tokens exceed max_prefill_tokens");
-  drop_graphs(c);
   c->B = batch;
   c->seed = seed;
   c->phase = 0;
@@ -908,16 +910,29 @@ sd2_status sd2_prefill(sd2_ctx* c, int32_t batch, const int32_t* d_tokens, const
     add_groups(sr0, snr, ssq, b * (k + 1), k + 1, b, c->V.group_rows());
     lr1.push_back(2 * b + 1);
   }
-  const int o_pos = push(pos), o_seq = push(seq), o_valid = push(valid), o_lr = push(logit_rows), o_tr = push(tap_row);
-  const int o_vr0 = push(vr0), o_vnr = push(vnr), o_vsq = push(vsq);
-  const int o_dr0 = push(dr0), o_dnr = push(dnr), o_dsq = push(dsq);
+  // The step-shape tables come first: they depend on the batch and k alone, so a step graph captured
+  // after an earlier prefill of the same batch size reads the same addresses and stays valid.
   const int o_d1r0 = push(d1r0), o_d1nr = push(d1nr), o_d1sq = push(d1sq);
   const int o_dnr0 = push(dnr0), o_dnnr = push(dnnr), o_dnsq = push(dnsq);
   const int o_sr0 = push(sr0), o_snr = push(snr), o_ssq = push(ssq), o_lr1 = push(lr1);
+  std::vector<int> key = {batch, k};
+  key.insert(key.end(), st.begin(), st.end());
+  if (key != c->graph_key) {
+    drop_graphs(c);
+    c->graph_key = key;
+  }
+  const int o_pos = push(pos), o_seq = push(seq), o_valid = push(valid), o_lr = push(logit_rows), o_tr = push(tap_row);
+  const int o_vr0 = push(vr0), o_vnr = push(vnr), o_vsq = push(vsq);
+  const int o_dr0 = push(dr0), o_dnr = push(dnr), o_dsq = push(dsq);
   std::vector<int> cu(h_cu_lens, h_cu_lens + batch + 1);
   const int o_cu = push(cu);
-  if ((int)st.size() > c->statics_cap) return fail(c, SD2_ECAPACITY, "plan tables exceed their buffer");
+  if ((int)st.size() > c->statics_cap) {
+    drop_graphs(c);
+    c->graph_key.clear();
+    return fail(c, SD2_ECAPACITY, "plan tables exceed their buffer");
+  }
   CK(cudaMemcpyAsync(c->statics, st.data(), st.size() * sizeof(int), cudaMemcpyHostToDevice, c->st));
+  CK(cudaMemcpyAsync(c->seed_d, &seed, sizeof(seed), cudaMemcpyHostToDevice, c->st));
   std::vector<float> temps(h_temperature, h_temperature + batch);
   CK(cudaMemcpyAsync(c->temp, temps.data(), batch * sizeof(float), cudaMemcpyHostToDevice, c->st));
   CK(cudaMemsetAsync(c->iter, 0, sizeof(int), c->st));
@@ -958,7 +973,7 @@ sd2_status sd2_prefill(sd2_ctx* c, int32_t batch, const int32_t* d_tokens, const
   o.logit_rows = S + o_lr; o.n_logit_rows = batch; o.logits = c->logits_t; o.ld_logits = static_cast<long long>(k + 1) * V;
   sd2_status s = forward(c, c->V, pv, o);
   if (s != SD2_OK) return s;
-  CK(sample_rows(c->logits_t, static_cast<long long>(k + 1) * V, batch, V, c->temp, seed, RNG_RESAMPLE, 0, nullptr, 0,
+  CK(sample_rows(c->logits_t, static_cast<long long>(k + 1) * V, batch, V, c->temp, Seed{seed, nullptr}, RNG_RESAMPLE, 0, nullptr, 0,
                  c->first, 1, nullptr, 0, c->samp_slot, c->samp_counter, c->errw, c->st));
   CK(prefill_init(batch, c->cfg.max_ctx, d_tokens, S + o_cu, c->first, c->state, c->maxB, c->committed, d_first_token,
                   c->st));
@@ -1240,7 +1255,7 @@ sd2_status sd2_accept_logits(const void* d_target, const void* d_draft, int32_t 
   err = reinterpret_cast<unsigned*>(s.jmode + 2 * B);
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   CK(cudaMemsetAsync(err, 0, sizeof(unsigned), st));
-  CK(accept_blocks(d_target, d_draft, dtype, d_xhat, d_temperature, B, k, V, seed, step, nullptr, nullptr, d_tokens, d_n,
+  CK(accept_blocks(d_target, d_draft, dtype, d_xhat, d_temperature, B, k, V, Seed{seed, nullptr}, step, nullptr, nullptr, d_tokens, d_n,
                    s, err, st));
   return SD2_OK;
 }

@@ -269,20 +269,26 @@ struct AcceptScratch {
   int* jmode;                   // [B, 2] j and mode
 };
 size_t accept_scratch_bytes(int B, int k);
+// Philox key of the sampling kernels: `value`, or the word at `ptr` when ptr is set (so that a
+// captured step can take a new request's seed without being captured again).
+struct Seed {
+  unsigned long long value;
+  const unsigned long long* ptr;
+};
 AcceptScratch accept_scratch_carve(void* base, int B, int k);
 // Acceptance of B blocks. logits are f32 (dtype 0) or bf16 (1); target row stride ld_t
 // between consecutive rows of one sequence is V and sequence stride (k+1)V, likewise the draft
 // with kV. Writes tokens [B, k+1] and n [B]; n_live (optional) masks stopped sequences
 // (n_live[b] == 0 -> n[b] = 0). step_ptr (optional) overrides `step` from device memory.
 cudaError_t accept_blocks(const void* target, const void* draft, int dtype, const int* xhat, const float* temp,
-                          int B, int k, int V, unsigned long long seed, unsigned step, const int* step_ptr,
+                          int B, int k, int V, Seed seed, unsigned step, const int* step_ptr,
                           const int* live, int* tokens, int* n, const AcceptScratch& s, unsigned* err,
                           cudaStream_t st);
 // Token from one row per sequence (draft sample or bonus/first token): T = 0 -> argmax,
 // else the exponential race argmax_v (z_v/T - ln(-ln u_v)) with u from counter
 // (v>>2, purpose<<16 | i, b, step). Row of sequence b at logits + b*ld. The result goes to
 // out[b*ld_out] and, if out2, out2[b*ld_out2].
-cudaError_t sample_rows(const float* logits, long long ld, int B, int V, const float* temp, unsigned long long seed,
+cudaError_t sample_rows(const float* logits, long long ld, int B, int V, const float* temp, Seed seed,
                         int purpose, int i, const int* step_ptr, unsigned step, int* out, int ld_out, int* out2,
                         int ld_out2, unsigned long long* slot, int* counter, unsigned* err, cudaStream_t st);
 

@@ -141,7 +141,7 @@ sd2_status sd2_accept_logits_noalloc(const void* d_target, const void* d_draft, 
   // and counters reset inside accept_blocks before they are used.
   cudaError_t e = cudaMemsetAsync(err, 0, sizeof(unsigned), st);
   if (e == cudaSuccess)
-    e = sd2::accept_blocks(d_target, d_draft, dtype, d_xhat, d_temperature, B, k, V, seed, step, nullptr, nullptr,
+    e = sd2::accept_blocks(d_target, d_draft, dtype, d_xhat, d_temperature, B, k, V, sd2::Seed{seed, nullptr}, step, nullptr, nullptr,
                            d_tokens, d_n, sc, err, st);
   if (e != cudaSuccess) return fail(SD2_ECUDA, std::string("acceptance launch: ") + cudaGetErrorString(e));
   return SD2_OK;

@@ -123,15 +123,19 @@ __device__ __forceinline__ RowRef row_ref(int r, int B, int k, int V) {
 __device__ __forceinline__ unsigned step_value(const int* step_ptr, unsigned step) {
   return step_ptr ? static_cast<unsigned>(*step_ptr) : step;
 }
+__device__ __forceinline__ unsigned long long seed_value(const Seed& s) { return s.ptr ? *s.ptr : s.value; }
 
 // Pass 1: packed (max, argmax) of s = z/T (or z at T = 0) per row.
 template <typename T>
 __global__ void __launch_bounds__(kThreads) rowmax_kernel(const T* target, const T* draft, int B, int k, int V,
                                                           const float* temp, const int* stopped,
-                                                          unsigned long long* rowkey, unsigned* err, int span) {
+                                                          unsigned long long* rowkey, unsigned long long* rowsum,
+                                                          unsigned* err, int span) {
   pdl_trigger();
   pdl_wait();
   __shared__ unsigned long long red[32];
+  // the normaliser pass adds into rowsum; it runs after this grid has completed
+  if (blockIdx.y == 0 && threadIdx.x == 0) rowsum[blockIdx.x] = 0ull;
   const RowRef rr = row_ref(blockIdx.x, B, k, V);
   if (stopped && stopped[rr.b]) return;
   const float t = temp[rr.b];
@@ -235,7 +239,7 @@ __device__ __forceinline__ float prob(float z, float invT, RowDist d) {
 // Sequential decisions of one block per sequence (one thread per sequence).
 template <typename T>
 __global__ void decide_kernel(const T* target, const T* draft, const int* xhat, const float* temp, int B, int k, int V,
-                              unsigned long long seed, const int* step_ptr, unsigned step, const int* stopped,
+                              Seed seed_arg, const int* step_ptr, unsigned step, const int* stopped,
                               const unsigned long long* rowkey, const unsigned long long* rowsum, int* tokens, int* n,
                               AcceptScratch s) {
   pdl_trigger();
@@ -269,6 +273,7 @@ __global__ void decide_kernel(const T* target, const T* draft, const int* xhat, 
   }
   const float invT = inv_temp(t);
   const unsigned stp = step_value(step_ptr, step);
+  const unsigned long long seed = seed_value(seed_arg);
   const uint32_t k0 = static_cast<uint32_t>(seed), k1 = static_cast<uint32_t>(seed >> 32);
   int j = k;
   for (int i = 1; i <= k; ++i) {
@@ -290,7 +295,7 @@ __global__ void decide_kernel(const T* target, const T* draft, const int* xhat, 
 // Replacement token (residual race, with the log-form race as its fallback) or bonus token.
 template <typename T>
 __global__ void __launch_bounds__(kThreads) resample_kernel(const T* target, const T* draft, const float* temp, int B,
-                                                            int k, int V, unsigned long long seed, const int* step_ptr,
+                                                            int k, int V, Seed seed_arg, const int* step_ptr,
                                                             unsigned step, const unsigned long long* rowkey,
                                                             const unsigned long long* rowsum, int* tokens, int* n,
                                                             AcceptScratch s, int span) {
@@ -304,6 +309,7 @@ __global__ void __launch_bounds__(kThreads) resample_kernel(const T* target, con
   const int j = s.jmode[2 * b];
   const float invT = inv_temp(temp[b]);
   const unsigned stp = step_value(step_ptr, step);
+  const unsigned long long seed = seed_value(seed_arg);
   const uint32_t k0 = static_cast<uint32_t>(seed), k1 = static_cast<uint32_t>(seed >> 32);
   const int nt = B * (k + 1);
   const int rt = b * (k + 1) + j;
@@ -362,7 +368,7 @@ __global__ void __launch_bounds__(kThreads) resample_kernel(const T* target, con
 
 // One token per row: argmax (T = 0) or the log-form exponential race.
 __global__ void __launch_bounds__(kThreads) sample_kernel(const float* logits, long long ld, int V, const float* temp,
-                                                          unsigned long long seed, int purpose, int i,
+                                                          Seed seed_arg, int purpose, int i,
                                                           const int* step_ptr, unsigned step, int* out, int ld_out,
                                                           int* out2, int ld_out2, unsigned long long* slot,
                                                           int* counter, unsigned* err, int span) {
@@ -376,6 +382,7 @@ __global__ void __launch_bounds__(kThreads) sample_kernel(const float* logits, l
   const bool greedy = !(t > 0.f);
   const float invT = greedy ? 1.f : inv_temp(t);
   const unsigned stp = step_value(step_ptr, step);
+  const unsigned long long seed = seed_value(seed_arg);
   const uint32_t k0 = static_cast<uint32_t>(seed), k1 = static_cast<uint32_t>(seed >> 32);
   const int lo = blockIdx.y * span, hi = min(V, lo + span);
   unsigned long long best = 0;
@@ -420,14 +427,17 @@ __global__ void __launch_bounds__(kThreads) sample_kernel(const float* logits, l
 
 template <typename T>
 cudaError_t accept_typed(const T* target, const T* draft, const int* xhat, const float* temp, int B, int k, int V,
-                         unsigned long long seed, unsigned step, const int* step_ptr, const int* stopped, int* tokens,
+                         Seed seed, unsigned step, const int* step_ptr, const int* stopped, int* tokens,
                          int* n, const AcceptScratch& s, unsigned* err, cudaStream_t st) {
   const int R = B * (2 * k + 1);
   const int span = vocab_span(V, B, 4, kPerCta), S = (V + span - 1) / span;
   const int sspan = vocab_span(V, R, 8, kStatsPerCta), SS = (V + sspan - 1) / sspan;
-  cudaError_t e = cudaMemsetAsync(s.rowkey, 0, sizeof(unsigned long long) * 2 * R, st);  // rowkey + rowsum
+  // rowkey takes atomic maxima from every CTA of its row, so it is cleared before the first pass;
+  // rowsum (placed after the rowkey of the scratch's own batch size, which may exceed B) is cleared
+  // by the first pass itself
+  cudaError_t e = cudaMemsetAsync(s.rowkey, 0, sizeof(unsigned long long) * R, st);
   if (e != cudaSuccess) return e;
-  { const cudaError_t e_ = launch_pdl(rowmax_kernel<T>, dim3(dim3(R, SS)), dim3(kThreads), 0, st, target, draft, B, k, V, temp, stopped, s.rowkey, err, sspan); if (e_ != cudaSuccess) return e_; }
+  { const cudaError_t e_ = launch_pdl(rowmax_kernel<T>, dim3(dim3(R, SS)), dim3(kThreads), 0, st, target, draft, B, k, V, temp, stopped, s.rowkey, s.rowsum, err, sspan); if (e_ != cudaSuccess) return e_; }
   { const cudaError_t e_ = launch_pdl(rowsum_kernel<T>, dim3(dim3(R, SS)), dim3(kThreads), 0, st, target, draft, B, k, V, temp, stopped, s.rowkey, s.rowsum, sspan); if (e_ != cudaSuccess) return e_; }
   { const cudaError_t e_ = launch_pdl(decide_kernel<T>, dim3((B + 127) / 128), dim3(128), 0, st, target, draft, xhat, temp, B, k, V, seed, step_ptr, step, stopped,
                                                     s.rowkey, s.rowsum, tokens, n, s); if (e_ != cudaSuccess) return e_; }
@@ -456,7 +466,7 @@ AcceptScratch accept_scratch_carve(void* base, int B, int k) {
 }
 
 cudaError_t accept_blocks(const void* target, const void* draft, int dtype, const int* xhat, const float* temp, int B,
-                          int k, int V, unsigned long long seed, unsigned step, const int* step_ptr, const int* stopped,
+                          int k, int V, Seed seed, unsigned step, const int* step_ptr, const int* stopped,
                           int* tokens, int* n, const AcceptScratch& s, unsigned* err, cudaStream_t st) {
   if (B <= 0) return cudaSuccess;
   if (dtype == 1)
@@ -466,7 +476,7 @@ cudaError_t accept_blocks(const void* target, const void* draft, int dtype, cons
                              seed, step, step_ptr, stopped, tokens, n, s, err, st);
 }
 
-cudaError_t sample_rows(const float* logits, long long ld, int B, int V, const float* temp, unsigned long long seed,
+cudaError_t sample_rows(const float* logits, long long ld, int B, int V, const float* temp, Seed seed,
                         int purpose, int i, const int* step_ptr, unsigned step, int* out, int ld_out, int* out2,
                         int ld_out2, unsigned long long* slot, int* counter, unsigned* err, cudaStream_t st) {
   if (B <= 0) return cudaSuccess;

@@ -53,7 +53,8 @@ class ParityReport:
 
 
 def run(work, vw, dw, st, prompts, temps, seed, n_steps, max_ctx=None, graphs=True, tol=TOL,
-        check_taps=True, gemm_impl=0, steering=True, chain=False, fused_attention=False) -> ParityReport:
+        check_taps=True, gemm_impl=0, steering=True, chain=False, fused_attention=False,
+        max_batch=None) -> ParityReport:
     """Run prefill + n_steps iterations on the GPU and check each against the oracle.
 
     steering=False runs the engine's pretrained-drafter mode (no steering stage, no bias); the
@@ -62,7 +63,7 @@ def run(work, vw, dw, st, prompts, temps, seed, n_steps, max_ctx=None, graphs=Tr
     if max_ctx is None:
         max_ctx = max(len(p) for p in prompts) + n_steps * (k + 1) + k + 4
     dev = (to_device(vw), to_device(dw), to_device(st))
-    eng = sd2.SD2Engine(work, *dev, max_batch=B, max_ctx=max_ctx,
+    eng = sd2.SD2Engine(work, *dev, max_batch=B if max_batch is None else max_batch, max_ctx=max_ctx,
                         max_prefill_tokens=sum(len(p) for p in prompts), steering=steering)
     eng.set_graphs(graphs)
     eng.set_gemm_impl(gemm_impl)

@@ -51,6 +51,16 @@ def test_tiny_longest_draft_and_wider_batch():
     assert rep.blocks == 24
 
 
+def test_batch_below_context_capacity():
+    """A context built for 5 sequences serving 2: the per-row scratch of the acceptance pass is laid
+    out for the capacity, and every decision still matches the oracle."""
+    work = dataclasses.replace(parity.tiny_work(), k=4)
+    vw, dw, st = parity.tiny_weights(work, seed=12)
+    prompts = W.make_prompts(work.verifier.vocab, 2, (17, 38), seed=13)
+    rep = parity.run(work, vw, dw, st, prompts, [1.0, 0.7], seed=55, n_steps=6, max_batch=5)
+    assert rep.blocks == 12
+
+
 def test_high_acceptance_with_self_drafting():
     """Drafter = verifier with W_s = 0 at T = 0: every block is fully accepted (tau = k + 1)."""
     base = parity.tiny_work()
@@ -83,6 +93,51 @@ def test_graphs_and_direct_launches_agree():
         assert torch.equal(na, nb)
         for b in range(2):
             assert torch.equal(ta[b, :na[b]], tb[b, :nb[b]])
+
+
+def _step_loop(eng, prompts, temps, seed, max_new):
+    """One request by sd2_prefill and sd2_step/sd2_accept pairs, tokens gathered on the host."""
+    out = [[f] for f in eng.prefill(prompts, temps, seed=seed).cpu().tolist()]
+    while any(len(o) < max_new for o in out):
+        eng.step()
+        t, n = eng.accept()
+        t, n = t.cpu(), n.cpu()
+        assert int(n.min()) > 0
+        for b, o in enumerate(out):
+            o.extend(t[b, :n[b]].tolist())
+    return [o[:max_new] for o in out]
+
+
+def test_generate_and_graphs_across_requests():
+    """sd2_generate on host buffers equals the prefill/step/accept loop, and a context serving a
+    run of requests (same batch with other prompt lengths and seeds, then another batch size, then
+    back) gives every request the tokens a fresh context without graphs gives it."""
+    work = parity.tiny_work()
+    vw, dw, st = parity.tiny_weights(work, seed=6)
+    dev = [parity.to_device(x) for x in (vw, dw, st)]
+    V = work.verifier.vocab
+    requests = [
+        (W.make_prompts(V, 2, (30, 40), seed=20), [1.0, 0.0], 101, "generate"),
+        (W.make_prompts(V, 2, (12, 47), seed=21), [0.7, 1.0], 102, "loop"),
+        (W.make_prompts(V, 1, (25, 25), seed=22), [1.0], 103, "generate"),
+        (W.make_prompts(V, 2, (8, 33), seed=23), [1.0, 1.0], 104, "generate"),
+    ]
+    max_new = 24
+    eng = sd2.SD2Engine(work, *dev, max_batch=2, max_ctx=160, max_prefill_tokens=100)
+    served = []
+    for prompts, temps, seed, how in requests:
+        if how == "generate":
+            served.append(eng.generate(prompts, temps, seed=seed, max_new=max_new))
+        else:
+            served.append(_step_loop(eng, prompts, temps, seed, max_new))
+    eng.check()
+    eng.close()
+    for (prompts, temps, seed, _), got in zip(requests, served):
+        ref = sd2.SD2Engine(work, *dev, max_batch=2, max_ctx=160, max_prefill_tokens=100)
+        ref.set_graphs(False)
+        want = _step_loop(ref, prompts, temps, seed, max_new)
+        ref.close()
+        assert got == want
 
 
 @pytest.mark.parametrize("temp", [0.0, 1.0])
