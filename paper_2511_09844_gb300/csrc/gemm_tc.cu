@@ -1113,10 +1113,18 @@ int sm_count() {
 constexpr int kSmemBudget = 227 * 1024;
 constexpr int kSmemShared = 110 * 1024;
 
-// Clusters of `size` CTAs of gemm_tc_kernel with `smem` bytes of dynamic shared memory that the
-// device holds at once. Clusters must fit whole into a GPC, so this is less than
-// SMs x (CTAs per SM) / size: with one CTA per SM, 46 clusters of 3 (138 CTAs) or 15 of 7 fit on a
-// 152-SM GB300. Cached per (size, smem).
+// Stand-in for gemm_tc_kernel in residency queries: the same block size and launch bounds, no
+// tensor memory. The occupancy calculator reports one CTA per SM for gemm_tc_kernel at any shared
+// memory size (measured: 152 clusters of 1, 76 of 2, ... even at 60 KB), while the hardware places
+// two of its CTAs on an SM whenever their shared memory fits (per-CTA %smid traces of its launches);
+// for this kernel the calculator's answers match a measured first wave at every size. Never launched.
+__global__ void __launch_bounds__(kThreads, 2) residency_proxy_kernel() {}
+
+// Clusters of `size` CTAs with `smem` bytes of dynamic shared memory each that the device holds at
+// once. Clusters must fit whole into a GPC, so this is less than SMs x (CTAs per SM) / size: at two
+// CTAs per SM, 97 clusters of 3 or 36 of 8; at one, 46 of 3 or 15 of 7 on a 152-SM GB300. The
+// registers of gemm_tc_kernel must allow two CTAs per SM for the two-per-SM figures to hold; if they
+// do not, one CTA per SM is assumed. Cached per (size, smem).
 int max_active_clusters(int size, int smem) {
   static std::mutex mu;
   static std::unordered_map<long long, int> cache;
@@ -1124,12 +1132,19 @@ int max_active_clusters(int size, int smem) {
   std::lock_guard<std::mutex> lock(mu);
   auto it = cache.find(key);
   if (it != cache.end()) return it->second;
+  cudaFuncAttributes fa{};
+  // registers are allocated per warp in units of 256
+  const bool two_fit = cudaFuncGetAttributes(&fa, gemm_tc_kernel) == cudaSuccess &&
+                       2 * (kThreads / 32) * ((fa.numRegs * 32 + 255) / 256 * 256) <= 65536;
+  // one CTA per SM when the registers say so: pad the shared memory beyond half an SM
+  const int q_smem = (!two_fit && smem <= kSmemShared) ? kSmemShared + 4096 : smem;
   int n = 0;
-  if (cudaFuncSetAttribute(gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024) == cudaSuccess) {
+  if (cudaFuncSetAttribute(residency_proxy_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBudget) ==
+      cudaSuccess) {
     cudaLaunchConfig_t cfg{};
     cfg.gridDim = dim3(static_cast<unsigned>(size));
     cfg.blockDim = dim3(kThreads);
-    cfg.dynamicSmemBytes = static_cast<size_t>(smem);
+    cfg.dynamicSmemBytes = static_cast<size_t>(q_smem);
     cudaLaunchAttribute at[1];
     at[0].id = cudaLaunchAttributeClusterDimension;
     at[0].val.clusterDim.x = static_cast<unsigned>(size);
@@ -1137,7 +1152,7 @@ int max_active_clusters(int size, int smem) {
     at[0].val.clusterDim.z = 1;
     cfg.attrs = at;
     cfg.numAttrs = 1;
-    if (cudaOccupancyMaxActiveClusters(&n, gemm_tc_kernel, &cfg) != cudaSuccess) n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, residency_proxy_kernel, &cfg) != cudaSuccess) n = 0;
   }
   cudaGetLastError();
   cache.emplace(key, n);
