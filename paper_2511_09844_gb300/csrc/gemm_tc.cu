@@ -423,10 +423,11 @@ __device__ __forceinline__ void splitk_epilogue(const TcArgs& a, const SplitK& s
   const uint32_t dst = dsmem_addr(smem_u32(recv + slot), static_cast<uint32_t>(owner));
   const uint32_t dst_bar = dsmem_addr(sk.rbar, static_cast<uint32_t>(owner));
   if (a.norm_ssq_in) tile_rstd(a, tt, rs, tid);
+  cluster_wait();                          // every rank's receive barrier is armed (every thread of the
+                                           // cluster arrived at kernel start: taken while the MMAs run)
   if (leader) flags[4] = wait_bar(sk.tfull0, 0, abort_flag, a.err) ? 1 : 0;
   named_bar_epi();                         // the accumulator is complete (or the wait gave up); rs is set
   tc_fence_after();
-  cluster_wait();                          // every rank's receive barrier is armed
   if (flags[4] != 0) {
     const uint32_t tbase = sk.tmem + (static_cast<uint32_t>(q * 32) << 16);
     for (int ch = 0; ch * 16 < cols; ++ch) {
@@ -570,57 +571,68 @@ __global__ void __launch_bounds__(kThreads, 2) gemm_tc_kernel(const __grid_const
   pdl_trigger();                             // the next kernel may start its own prologue
   PairOps pf{};                              // split-K: operands of this thread's first output pair
   if (warp == 0) {
-    if (lane == 0) {
-      // Stage use j loads k-block (kb_lo + j % nkb) of the CTA's (j / nkb)-th tile: the weight
-      // half first, then the token half. Weights never depend on earlier kernels, so the first
-      // stages' weight tiles are requested before waiting for the predecessor grid. Cursors
-      // advance one k-block at a time (no divisions in the issue loop).
-      struct Cursor {
-        int tile, kb, wt, tt, seg, row0;
-      };
-      auto locate = [&](Cursor& c) {
-        c.wt = c.tile % a.n_wtiles;
-        c.tt = c.tile / a.n_wtiles;
-        c.seg = 0;
-        c.row0 = c.wt * kWRows;
-        if (!a.swiglu)
-          while (c.seg + 1 < a.nseg && c.row0 >= a.seg_rows[c.seg]) c.row0 -= a.seg_rows[c.seg++];
-      };
-      auto advance = [&](Cursor& c) {
-        if (++c.kb == kb_hi) { c.kb = kb_lo; c.tile += tile_step; if (c.tile < a.tiles) locate(c); }
-      };
-      int n_my_tiles = 0;
-      for (int t = first_tile; t < a.tiles; t += tile_step) ++n_my_tiles;
-      const uint32_t n_units = static_cast<uint32_t>(n_my_tiles * nkb);
-      const uint64_t wpol = l2_evict_first();
-      Cursor ca;
-      ca.tile = first_tile;
-      ca.kb = kb_lo;
-      if (ca.tile < a.tiles) locate(ca);
-      Cursor cb = ca;
-      auto load_a = [&](uint32_t j, const Cursor& c) {
-        const uint32_t s = j % S;
-        const uint32_t dst = smem_u32(smem + static_cast<size_t>(s) * stage_bytes);
-        if (a.swiglu) {
-          tma_load_2d_stream(dst, &a.mapA[0], c.kb * kBK, c.wt * 64, full0 + 8 * s, wpol);
-          tma_load_2d_stream(dst + a_bytes / 2, &a.mapA[1], c.kb * kBK, c.wt * 64, full0 + 8 * s, wpol);
-        } else {
-          tma_load_2d_stream(dst, &a.mapA[c.seg], c.kb * kBK, c.row0, full0 + 8 * s, wpol);
-        }
-      };
-      auto load_b = [&](uint32_t j, const Cursor& c) {
-        const uint32_t s = j % S;
-        const uint32_t dst = smem_u32(smem + static_cast<size_t>(s) * stage_bytes);
-        tma_load_2d(dst + a_bytes, &a.mapB, c.kb * kBK, c.tt * NT, full0 + 8 * s);
-      };
-      const uint32_t pre = n_units < static_cast<uint32_t>(S) ? n_units : static_cast<uint32_t>(S);
+    // Stage use j loads k-block (kb_lo + j % nkb) of the CTA's (j / nkb)-th tile: the weight half
+    // first, then the token half. Weights never depend on earlier kernels, so the first stages'
+    // weight tiles are requested before waiting for the predecessor grid. Cursors advance one
+    // k-block at a time (no divisions in the issue loop).
+    struct Cursor {
+      int tile, kb, wt, tt, seg, row0;
+    };
+    auto locate = [&](Cursor& c) {
+      c.wt = c.tile % a.n_wtiles;
+      c.tt = c.tile / a.n_wtiles;
+      c.seg = 0;
+      c.row0 = c.wt * kWRows;
+      if (!a.swiglu)
+        while (c.seg + 1 < a.nseg && c.row0 >= a.seg_rows[c.seg]) c.row0 -= a.seg_rows[c.seg++];
+    };
+    auto advance = [&](Cursor& c) {
+      if (++c.kb == kb_hi) { c.kb = kb_lo; c.tile += tile_step; if (c.tile < a.tiles) locate(c); }
+    };
+    int n_my_tiles = 0;
+    for (int t = first_tile; t < a.tiles; t += tile_step) ++n_my_tiles;
+    const uint32_t n_units = static_cast<uint32_t>(n_my_tiles * nkb);
+    const uint64_t wpol = l2_evict_first();
+    Cursor ca;
+    ca.tile = first_tile;
+    ca.kb = kb_lo;
+    if (ca.tile < a.tiles) locate(ca);
+    auto load_a = [&](uint32_t j, const Cursor& c) {
+      const uint32_t s = j % S;
+      const uint32_t dst = smem_u32(smem + static_cast<size_t>(s) * stage_bytes);
+      if (a.swiglu) {
+        tma_load_2d_stream(dst, &a.mapA[0], c.kb * kBK, c.wt * 64, full0 + 8 * s, wpol);
+        tma_load_2d_stream(dst + a_bytes / 2, &a.mapA[1], c.kb * kBK, c.wt * 64, full0 + 8 * s, wpol);
+      } else {
+        tma_load_2d_stream(dst, &a.mapA[c.seg], c.kb * kBK, c.row0, full0 + 8 * s, wpol);
+      }
+    };
+    auto load_b = [&](uint32_t j, const Cursor& c) {
+      const uint32_t s = j % S;
+      const uint32_t dst = smem_u32(smem + static_cast<size_t>(s) * stage_bytes);
+      tma_load_2d(dst + a_bytes, &a.mapB, c.kb * kBK, c.tt * NT, full0 + 8 * s);
+    };
+    const uint32_t pre = n_units < static_cast<uint32_t>(S) ? n_units : static_cast<uint32_t>(S);
+    if (lane == 0)
       for (uint32_t j = 0; j < pre; ++j, advance(ca)) {   // first use of each stage: no wait
         mbar_expect_tx(full0 + 8 * j, stage_bytes);
         load_a(j, ca);
       }
-      pdl_wait();
-      if (a.stamp) atomicMin(&a.stamp[1], global_ns());
-      for (uint32_t j = 0; j < pre; ++j, advance(cb)) load_b(j, cb);
+    __syncwarp();                            // the stages' expected bytes are set before any token load
+    pdl_wait();
+    if (lane == 0 && a.stamp) atomicMin(&a.stamp[1], global_ns());
+    // The token halves of the first stages, one lane each: one issue instead of `pre` in a row
+    // (each TMA issue takes a few hundred cycles).
+    if (lane < pre) {
+      Cursor cb;
+      cb.tile = first_tile + static_cast<int>(lane / static_cast<uint32_t>(nkb)) * tile_step;
+      cb.kb = kb_lo + static_cast<int>(lane % static_cast<uint32_t>(nkb));
+      locate(cb);
+      tma_load_2d(smem_u32(smem + static_cast<size_t>(lane) * stage_bytes) + a_bytes, &a.mapB, cb.kb * kBK,
+                  cb.tt * NT, full0 + 8 * lane);
+    }
+    __syncwarp();
+    if (lane == 0) {
       uint32_t j = pre;
       bool ok = true;
       for (; j < n_units; ++j, advance(ca)) {
@@ -638,7 +650,16 @@ __global__ void __launch_bounds__(kThreads, 2) gemm_tc_kernel(const __grid_const
   } else if (warp == 1) {
     if (lane == 0) {
       const uint32_t idesc = idesc_bf16(kWRows, NT);
-      uint32_t j = 0, segi = 0;
+      // stage s of use j = j mod S and its phase, advanced incrementally; a stage's descriptors are
+      // the ring base's plus the stage offset (the address field is addr >> 4, below 2^14)
+      const uint64_t desc0 = sw128_desc(smem_u32(smem));
+      const uint64_t dstage = stage_bytes >> 4, dB = a_bytes >> 4;
+      // With every stage used once (all of the CTA's k-blocks fit the ring) the producer never
+      // waits for a stage to drain: no per-stage release, and nothing for its abort path to count.
+      int n_my_tiles = 0;
+      for (int t = first_tile; t < a.tiles; t += tile_step) ++n_my_tiles;
+      const bool reuse = n_my_tiles * nkb > S;
+      uint32_t j = 0, segi = 0, s = 0, ph = 0;
       bool ok = true;
       for (int t = first_tile; t < a.tiles && ok; t += tile_step, ++segi) {
         const uint32_t acc = segi & 1;
@@ -646,16 +667,17 @@ __global__ void __launch_bounds__(kThreads, 2) gemm_tc_kernel(const __grid_const
         tc_fence_after();
         const uint32_t d = tmem + acc * NT;
         for (int i = 0; i < nkb; ++i, ++j) {
-          const uint32_t s = j % S;
-          if (!wait_bar(full0 + 8 * s, (j / S) & 1, abort_flag, a.err)) { ok = false; break; }
+          if (!wait_bar(full0 + 8 * s, ph, abort_flag, a.err)) { ok = false; break; }
           tc_fence_after();
-          const uint32_t abase = smem_u32(smem + static_cast<size_t>(s) * stage_bytes);
-          const uint64_t ad = sw128_desc(abase), bd = sw128_desc(abase + a_bytes);
+          const uint64_t ad = desc0 + s * dstage, bd = ad + dB;
 #pragma unroll
           for (int kk = 0; kk < kBK / 16; ++kk)
             mma_bf16(d, ad + 2 * kk, bd + 2 * kk, idesc, (i > 0 || kk > 0) ? 1u : 0u);
-          mma_commit(empty0 + 8 * s);
-          flags[3] = static_cast<int>(j + 1);
+          if (reuse) {
+            mma_commit(empty0 + 8 * s);
+            flags[3] = static_cast<int>(j + 1);
+          }
+          if (++s == static_cast<uint32_t>(S)) { s = 0; ph ^= 1u; }
         }
         if (!ok) break;
         mma_commit(tfull0 + 8 * acc);
