@@ -524,7 +524,9 @@ __global__ void __launch_bounds__(kThreads, 2) gemm_tc_kernel(const __grid_const
                  drain = tempty0 + 16, rbar = drain + 8;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   uint32_t ncols = 32;
-  while (ncols < static_cast<uint32_t>((sp == 1 ? 2 : 1) * NT)) ncols <<= 1;
+  // two accumulators (double buffering) only for a CTA that takes several whole tiles
+  const bool one_acc = sp > 1 || a.tiles <= static_cast<int>(gridDim.x);
+  while (ncols < static_cast<uint32_t>((one_acc ? 1 : 2) * NT)) ncols <<= 1;
   const int rank = sp > 1 ? static_cast<int>(cluster_rank()) : 0;
   if (a.stamp && threadIdx.x == 0) atomicMin(&a.stamp[0], global_ns());
 
@@ -1201,8 +1203,11 @@ TcPlan plan_tc(int tiles, int NT, int KB) {
   int best_active = 0;
   for (int occ = 2; occ >= 1; --occ) {
     const int budget = occ == 2 ? kSmemShared : kSmemBudget;
-    const int min_stages = occ == 2 ? 3 : 2;
-    if (occ == 2 && NT > 128) continue;                  // the accumulators would not fit twice in TMEM
+    // Wide token tiles (NT > 128) take two CTAs per SM only as one whole tile per CTA: a single
+    // accumulator (at most 256 TMEM columns, so two CTAs fit), and a two-stage ring is accepted.
+    const bool wide = NT > 128;
+    if (occ == 2 && wide && tiles > 2 * sms) continue;
+    const int min_stages = occ == 2 && !wide ? 3 : 2;
     int sp = 1;
     if (tiles < sms * occ) {                             // split-K tiles keep one NT-column accumulator
       sp = ((occ == 2 ? 3 * sms / 2 : sms) + tiles / 2) / tiles;
