@@ -61,6 +61,39 @@ def test_batch_below_context_capacity():
     assert rep.blocks == 12
 
 
+def test_single_draft_token():
+    """k = 1: one draft, two verify rows per sequence, at mixed temperatures."""
+    work = dataclasses.replace(parity.tiny_work(), k=1, batch=2)
+    vw, dw, st = parity.tiny_weights(work, seed=14)
+    prompts = W.make_prompts(work.verifier.vocab, 2, (21, 44), seed=15)
+    rep = parity.run(work, vw, dw, st, prompts, [1.0, 0.0], seed=61, n_steps=8)
+    assert rep.blocks == 16
+
+
+def test_prompts_at_block_and_tile_boundaries():
+    """Prompts of 1, 16, 64 and 65 tokens: a lone token, one full 16-position cache block, one full
+    64-position attention tile, and one position past it."""
+    work = dataclasses.replace(parity.tiny_work(), batch=4)
+    vw, dw, st = parity.tiny_weights(work, seed=16)
+    V = work.verifier.vocab
+    prompts = [p[:n] for p, n in zip(W.make_prompts(V, 4, (65, 65), seed=17), (1, 16, 64, 65))]
+    rep = parity.run(work, vw, dw, st, prompts, [1.0, 0.7, 0.0, 1.0], seed=62, n_steps=5)
+    assert rep.blocks == 20
+
+
+def test_long_context_many_tiles_grouped_heads():
+    """A 300-token prompt (five attention tiles) with 4 query heads per KV head on both models, and
+    a capacity far above the context (empty context splits)."""
+    base = parity.tiny_work()
+    vs = W.shrink(base.verifier, n_kv_heads=1)
+    ds = W.shrink(base.drafter, n_kv_heads=1, n_heads=2)
+    work = dataclasses.replace(base, verifier=vs, drafter=ds, batch=1)
+    vw, dw, st = parity.tiny_weights(work, seed=18)
+    prompts = W.make_prompts(vs.vocab, 1, (300, 300), seed=19)
+    rep = parity.run(work, vw, dw, st, prompts, [1.0], seed=63, n_steps=4, max_ctx=2048)
+    assert rep.blocks == 4
+
+
 def test_high_acceptance_with_self_drafting():
     """Drafter = verifier with W_s = 0 at T = 0: every block is fully accepted (tau = k + 1)."""
     base = parity.tiny_work()
