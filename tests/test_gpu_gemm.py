@@ -24,6 +24,8 @@ SHAPES = [
     (40, 512, 2048), (144, 256, 1024), (256, 128, 192), (300, 384, 512),
     (6, 128, 14336),      # one weight tile split across every CTA
     (2, 4096, 4096),      # the 8B O projection at drafter-step M
+    (144, 28672, 256),    # wide token tiles, 224 whole tiles: two CTAs per SM, one tile each
+    (256, 16384, 128),    # the widest token tile (256 columns), 128 whole tiles
 ]
 
 
@@ -85,7 +87,7 @@ def test_silu_bias_epilogue(impl, M, N, K):
 
 
 @pytest.mark.parametrize("impl", [1, 2])
-@pytest.mark.parametrize("M,F,K", [(6, 256, 512), (18, 192, 2048), (1, 64, 4864)])
+@pytest.mark.parametrize("M,F,K", [(6, 256, 512), (18, 192, 2048), (1, 64, 4864), (144, 14336, 512)])
 def test_steered_swiglu_epilogue(impl, M, F, K):
     g = torch.Generator().manual_seed(M + F)
     x = torch.randn(M, K, generator=g).to(torch.bfloat16)
