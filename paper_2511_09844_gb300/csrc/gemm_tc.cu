@@ -599,8 +599,7 @@ __global__ void __launch_bounds__(kThreads, 2) gemm_tc_kernel(const __grid_const
     ca.tile = first_tile;
     ca.kb = kb_lo;
     if (ca.tile < a.tiles) locate(ca);
-    auto load_a = [&](uint32_t j, const Cursor& c) {
-      const uint32_t s = j % S;
+    auto load_a = [&](uint32_t s, const Cursor& c) {   // into stage s
       const uint32_t dst = smem_u32(smem + static_cast<size_t>(s) * stage_bytes);
       if (a.swiglu) {
         tma_load_2d_stream(dst, &a.mapA[0], c.kb * kBK, c.wt * 64, full0 + 8 * s, wpol);
@@ -609,8 +608,7 @@ __global__ void __launch_bounds__(kThreads, 2) gemm_tc_kernel(const __grid_const
         tma_load_2d_stream(dst, &a.mapA[c.seg], c.kb * kBK, c.row0, full0 + 8 * s, wpol);
       }
     };
-    auto load_b = [&](uint32_t j, const Cursor& c) {
-      const uint32_t s = j % S;
+    auto load_b = [&](uint32_t s, const Cursor& c) {
       const uint32_t dst = smem_u32(smem + static_cast<size_t>(s) * stage_bytes);
       tma_load_2d(dst + a_bytes, &a.mapB, c.kb * kBK, c.tt * NT, full0 + 8 * s);
     };
@@ -636,13 +634,14 @@ __global__ void __launch_bounds__(kThreads, 2) gemm_tc_kernel(const __grid_const
     __syncwarp();
     if (lane == 0) {
       uint32_t j = pre;
+      uint32_t s = pre % static_cast<uint32_t>(S), ph = (pre / static_cast<uint32_t>(S)) & 1;   // stage of use j, its phase
       bool ok = true;
       for (; j < n_units; ++j, advance(ca)) {
-        const uint32_t s = j % S;
-        if (!wait_bar(empty0 + 8 * s, ((j / S) & 1) ^ 1, abort_flag, a.err)) { ok = false; break; }
+        if (!wait_bar(empty0 + 8 * s, ph ^ 1, abort_flag, a.err)) { ok = false; break; }
         mbar_expect_tx(full0 + 8 * s, stage_bytes);
-        load_a(j, ca);
-        load_b(j, ca);
+        load_a(s, ca);
+        load_b(s, ca);
+        if (++s == static_cast<uint32_t>(S)) { s = 0; ph ^= 1u; }
       }
       if (!ok) {  // let the loads already issued land before the CTA exits
         const uint32_t done = static_cast<uint32_t>(flags[3]);
