@@ -89,6 +89,15 @@ struct TcArgs {
 };
 
 
+// The kernel's arguments with the epilogue kind fixed at compile time: epi and swiglu hide the
+// base's run-time fields, so each instantiation of the kernel (one per epilogue) carries only its
+// own epilogue's code.
+template <int E>
+struct TcArgsE : TcArgs {
+  static constexpr int epi = E;
+  static constexpr int swiglu = E == EPI_SWIGLU ? 1 : 0;
+};
+
 constexpr int kMaxNT = 256;  // token columns per tile
 
 __device__ __forceinline__ unsigned long long global_ns() {
@@ -104,7 +113,8 @@ __device__ __forceinline__ float add_bias_of(const TcArgs& a, int n, int m) {
   return a.bias ? a.bias[static_cast<size_t>(a.row_seq ? a.row_seq[m] : 0) * a.ld_bias + n] : 0.f;
 }
 __device__ __forceinline__ float silu_f(float y) { return y / (1.f + __expf(-y)); }
-__device__ __forceinline__ void emit_plain(const TcArgs& a, int wt, int row, int m, float v) {
+template <class A>
+__device__ __forceinline__ void emit_plain(const A& a, int wt, int row, int m, float v) {
   const int n = wt * kWRows + row;
   if (a.epi == EPI_SILU) {
     a.out_bf[static_cast<size_t>(m) * a.ldh + n] = __float2bfloat16_rn(silu_f(v + add_bias_of(a, n, m)));
@@ -188,7 +198,8 @@ __device__ __forceinline__ void tile_rstd(const TcArgs& a, int tt, float* rs, in
 
 // Whole-tile epilogue: thread r holds weight row r for 16 token columns j0..j0+15; rows that
 // need another row (SwiGLU pairs, rotate-half partners) are exchanged through shared memory.
-__device__ __forceinline__ void finish_chunk(const TcArgs& a, int wt, int tt, int r, int j0, float (&v)[16],
+template <class A>
+__device__ __forceinline__ void finish_chunk(const A& a, int wt, int tt, int r, int j0, float (&v)[16],
                                              float* xbuf, const float* rs) {
   const int m0 = tt * a.NT + j0;
   if (a.norm_ssq_in)
@@ -248,14 +259,18 @@ __device__ __forceinline__ void finish_chunk(const TcArgs& a, int wt, int tt, in
 // Split-K pairs: the 128 rows of a tile as 64 pairs whose members one epilogue needs together.
 // SwiGLU: (gate f, up f) = rows (p, p + 64); QKV with hd = 128: rotate-half partners (i, i + 64);
 // QKV with hd = 64 (two heads per tile): (64h + i, 64h + i + 32); plain outputs: (p, p + 64).
-__device__ __forceinline__ bool pairs_of_32(const TcArgs& a) { return a.epi == EPI_QKV && a.head_dim == 64; }
-__device__ __forceinline__ int pair_of(const TcArgs& a, int row) {
+template <class A>
+__device__ __forceinline__ bool pairs_of_32(const A& a) { return a.epi == EPI_QKV && a.head_dim == 64; }
+template <class A>
+__device__ __forceinline__ int pair_of(const A& a, int row) {
   return pairs_of_32(a) ? (row >> 6) * 32 + (row & 31) : (row & 63);
 }
-__device__ __forceinline__ int member_of(const TcArgs& a, int row) {
+template <class A>
+__device__ __forceinline__ int member_of(const A& a, int row) {
   return pairs_of_32(a) ? ((row >> 5) & 1) : (row >> 6);
 }
-__device__ __forceinline__ int pair_row(const TcArgs& a, int p, int m) {
+template <class A>
+__device__ __forceinline__ int pair_row(const A& a, int p, int m) {
   return pairs_of_32(a) ? (p >> 5) * 64 + m * 32 + (p & 31) : p + 64 * m;
 }
 // Rank r of sp owns pairs [64 r / sp, 64 (r + 1) / sp); its receive buffer holds, per source
@@ -280,7 +295,8 @@ struct PairOps {
   float2 cs;
   int pos, blk;
 };
-__device__ __forceinline__ PairOps pair_ops(const TcArgs& a, int wt, int p, int m) {
+template <class A>
+__device__ __forceinline__ PairOps pair_ops(const A& a, int wt, int p, int m) {
   PairOps o{0.f, 0.f, 0.f, 0.f, 0.f, 0.f, make_float2(1.f, 0.f), 0, -1};
   if (a.swiglu) {
     if (a.bias) o.bias = a.bias[static_cast<size_t>(a.row_seq ? a.row_seq[m] : 0) * a.ld_bias + wt * 64 + p];
@@ -311,7 +327,8 @@ __device__ __forceinline__ PairOps pair_ops(const TcArgs& a, int wt, int p, int 
 }
 // Epilogue of one output pair from its split-K sums s0 (member 0) and s1 (member 1). Returns the
 // pair's contribution to the token's sum of squares when it produces a fused RMSNorm.
-__device__ __forceinline__ float pair_emit(const TcArgs& a, int wt, int p, int m, float s0, float s1, const PairOps& o) {
+template <class A>
+__device__ __forceinline__ float pair_emit(const A& a, int wt, int p, int m, float s0, float s1, const PairOps& o) {
   if (a.swiglu) {
     const float up = s1 + o.bias;
     a.out_bf[static_cast<size_t>(m) * a.ldh + wt * 64 + p] = __float2bfloat16_rn(up * (s0 / (1.f + __expf(-s0))));
@@ -367,7 +384,8 @@ struct SplitK {
   int rank, sp, npmax, NT, first_tile;
 };
 // The global operands of the first output this epilogue thread (tid 0..127) owns, fetched early.
-__device__ __forceinline__ PairOps first_pair_ops(const TcArgs& a, int rank, int sp, int NT, int first_tile, int tid) {
+template <class A>
+__device__ __forceinline__ PairOps first_pair_ops(const A& a, int rank, int sp, int NT, int first_tile, int tid) {
   const int wt = first_tile % a.n_wtiles, tt = first_tile / a.n_wtiles;
   const int cols = min(NT, a.M - tt * NT);
   const int p_lo = rank * 64 / sp, np = (rank + 1) * 64 / sp - p_lo;
@@ -407,7 +425,8 @@ __device__ __forceinline__ void sum_parts_any(const float* rv, int rstride, int 
 // (st.async onto the owner's receive barrier); the owner waits for its own pairs only, sums the
 // partials in rank order and runs the epilogue. Everything but the sums is prepared while the
 // MMAs run. pf: the operands of the thread's first owned output (first_pair_ops).
-__device__ __forceinline__ void splitk_epilogue(const TcArgs& a, const SplitK& sk, int warp, int lane, const PairOps& pf) {
+template <class A>
+__device__ __forceinline__ void splitk_epilogue(const A& a, const SplitK& sk, int warp, int lane, const PairOps& pf) {
   const int q = warp & 3, r = q * 32 + lane, tid = threadIdx.x - 64;
   const bool leader = (warp == 2 && lane == 0);
   const int sp = sk.sp, npmax = sk.npmax, NT = sk.NT, rank = sk.rank;
@@ -503,7 +522,8 @@ __device__ __forceinline__ void splitk_epilogue(const TcArgs& a, const SplitK& s
   }
 }
 
-__global__ void __launch_bounds__(kThreads, 2) gemm_tc_kernel(const __grid_constant__ TcArgs a) {
+template <class A>
+__global__ void __launch_bounds__(kThreads, 2) gemm_tc_kernel(const __grid_constant__ A a) {
   extern __shared__ unsigned char smem_raw[];
   unsigned char* smem =
       reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -1136,6 +1156,27 @@ int sm_count() {
 constexpr int kSmemBudget = 227 * 1024;
 constexpr int kSmemShared = 110 * 1024;
 
+// Registers a thread of the most demanding instantiation of gemm_tc_kernel uses (0 if unknown).
+int gemm_tc_max_regs() {
+  static const int regs = [] {
+    int r = 0;
+    auto take = [&](const void* f) {
+      cudaFuncAttributes fa{};
+      if (cudaFuncGetAttributes(&fa, f) == cudaSuccess) r = std::max(r, fa.numRegs);
+      else r = -1000;
+    };
+    take(reinterpret_cast<const void*>(gemm_tc_kernel<TcArgs>));
+    take(reinterpret_cast<const void*>(gemm_tc_kernel<TcArgsE<EPI_STORE>>));
+    take(reinterpret_cast<const void*>(gemm_tc_kernel<TcArgsE<EPI_ADD>>));
+    take(reinterpret_cast<const void*>(gemm_tc_kernel<TcArgsE<EPI_SWIGLU>>));
+    take(reinterpret_cast<const void*>(gemm_tc_kernel<TcArgsE<EPI_QKV>>));
+    take(reinterpret_cast<const void*>(gemm_tc_kernel<TcArgsE<EPI_SILU>>));
+    cudaGetLastError();
+    return r;
+  }();
+  return regs;
+}
+
 // Stand-in for gemm_tc_kernel in residency queries: the same block size and launch bounds, no
 // tensor memory. The occupancy calculator reports one CTA per SM for gemm_tc_kernel at any shared
 // memory size (measured: 152 clusters of 1, 76 of 2, ... even at 60 KB), while the hardware places
@@ -1155,10 +1196,9 @@ int max_active_clusters(int size, int smem) {
   std::lock_guard<std::mutex> lock(mu);
   auto it = cache.find(key);
   if (it != cache.end()) return it->second;
-  cudaFuncAttributes fa{};
   // registers are allocated per warp in units of 256
-  const bool two_fit = cudaFuncGetAttributes(&fa, gemm_tc_kernel) == cudaSuccess &&
-                       2 * (kThreads / 32) * ((fa.numRegs * 32 + 255) / 256 * 256) <= 65536;
+  const int regs = gemm_tc_max_regs();
+  const bool two_fit = regs > 0 && 2 * (kThreads / 32) * ((regs * 32 + 255) / 256 * 256) <= 65536;
   // one CTA per SM when the registers say so: pad the shared memory beyond half an SM
   const int q_smem = (!two_fit && smem <= kSmemShared) ? kSmemShared + 4096 : smem;
   int n = 0;
@@ -1331,6 +1371,20 @@ cudaError_t gemm_attn(const GemmArgs& g, unsigned* err, cudaStream_t st) {
                             a.sp, a);
 }
 
+namespace {
+// One launch of the instantiation for argument type A (its shared-memory opt-in set once).
+template <class A>
+cudaError_t launch_tc(const TcArgs& a, const TcPlan& pl, cudaStream_t st) {
+  static const cudaError_t configured =
+      cudaFuncSetAttribute(gemm_tc_kernel<A>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBudget);
+  if (configured != cudaSuccess) return configured;
+  A ae;
+  static_cast<TcArgs&>(ae) = a;
+  return launch_pdl_cluster(gemm_tc_kernel<A>, dim3(static_cast<unsigned>(pl.grid)), dim3(kThreads),
+                            static_cast<size_t>(pl.smem), st, pl.sp, ae);
+}
+}  // namespace
+
 cudaError_t gemm_tc(const GemmArgs& g, unsigned* err, cudaStream_t st) {
   if (g.attn_q) return gemm_attn(g, err, st);
   TcArgs a{};  // built on the host; passed by value as the kernel parameter
@@ -1366,16 +1420,19 @@ cudaError_t gemm_tc(const GemmArgs& g, unsigned* err, cudaStream_t st) {
   const int sp = pl.sp;
   a.sp = sp;
   a.stages = pl.stages;
-  const int smem = pl.smem;
-  static bool configured = false;
-  if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBudget);
-    if (e != cudaSuccess) return e;
-    configured = true;
+  // Narrow token tiles (up to 16 columns: batch-1 decode) share one kernel whatever the epilogue:
+  // their launches are short, and one body of code stays warm in the instruction caches across
+  // a layer's projections (per-epilogue kernels made the 1B drafter step 4% slower). Wider tiles,
+  // whose owner passes run many outputs per thread, take the kernel of their own epilogue.
+  if (a.NT <= 16) return launch_tc<TcArgs>(a, pl, st);
+  switch (a.epi) {
+    case EPI_STORE: return launch_tc<TcArgsE<EPI_STORE>>(a, pl, st);
+    case EPI_ADD: return launch_tc<TcArgsE<EPI_ADD>>(a, pl, st);
+    case EPI_SWIGLU: return launch_tc<TcArgsE<EPI_SWIGLU>>(a, pl, st);
+    case EPI_QKV: return launch_tc<TcArgsE<EPI_QKV>>(a, pl, st);
+    case EPI_SILU: return launch_tc<TcArgsE<EPI_SILU>>(a, pl, st);
+    default: return cudaErrorInvalidValue;
   }
-  const int grid = pl.grid;
-  return launch_pdl_cluster(gemm_tc_kernel, dim3(static_cast<unsigned>(grid)), dim3(kThreads),
-                            static_cast<size_t>(smem), st, sp, a);
 }
 
 }  // namespace sd2
