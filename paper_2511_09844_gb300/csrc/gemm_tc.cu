@@ -522,17 +522,20 @@ __device__ __forceinline__ void splitk_epilogue(const A& a, const SplitK& sk, in
   }
 }
 
-template <class A>
+// SPLIT: 1 = every launch of this instantiation splits K (sp > 1), 2 = whole tiles (sp == 1),
+// 0 = decided at run time.
+template <class A, int SPLIT>
 __global__ void __launch_bounds__(kThreads, 2) gemm_tc_kernel(const __grid_constant__ A a) {
   extern __shared__ unsigned char smem_raw[];
   unsigned char* smem =
       reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-  const int S = a.stages, NT = a.NT, sp = a.sp;
+  const int S = a.stages, NT = a.NT, sp = SPLIT == 2 ? 1 : a.sp;
+  const bool split = SPLIT == 1 ? true : (SPLIT == 2 ? false : sp > 1);
   const uint32_t a_bytes = kWRows * kBK * 2;
   const uint32_t b_bytes = static_cast<uint32_t>(NT) * kBK * 2;
   const uint32_t stage_bytes = a_bytes + b_bytes;
   const int npmax = pairs_max(sp);
-  const uint32_t recv_bytes = sp > 1 ? static_cast<uint32_t>(sp * npmax * 2 * NT * 4) : 0u;
+  const uint32_t recv_bytes = split ? static_cast<uint32_t>(sp * npmax * 2 * NT * 4) : 0u;
   float* recv = reinterpret_cast<float*>(smem + static_cast<size_t>(S) * stage_bytes);  // split-K partials in
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + static_cast<size_t>(S) * stage_bytes + recv_bytes);
   // bars: full[S], empty[S], tfull[2], tempty[2], drain, recv (split-K partials of this rank's pairs)
@@ -545,9 +548,9 @@ __global__ void __launch_bounds__(kThreads, 2) gemm_tc_kernel(const __grid_const
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   uint32_t ncols = 32;
   // two accumulators (double buffering) only for a CTA that takes several whole tiles
-  const bool one_acc = sp > 1 || a.tiles <= static_cast<int>(gridDim.x);
+  const bool one_acc = split || a.tiles <= static_cast<int>(gridDim.x);
   while (ncols < static_cast<uint32_t>((one_acc ? 1 : 2) * NT)) ncols <<= 1;
-  const int rank = sp > 1 ? static_cast<int>(cluster_rank()) : 0;
+  const int rank = split ? static_cast<int>(cluster_rank()) : 0;
   if (a.stamp && threadIdx.x == 0) atomicMin(&a.stamp[0], global_ns());
 
   if (threadIdx.x == 0) {
@@ -560,7 +563,7 @@ __global__ void __launch_bounds__(kThreads, 2) gemm_tc_kernel(const __grid_const
     mbar_init(tempty0, 4);
     mbar_init(tempty0 + 8, 4);
     mbar_init(drain, 1);
-    if (sp > 1) {
+    if (split) {
       // Split-K: every rank pushes its partial of each row to the rank owning the row's pair;
       // the owner's receive barrier completes when all sp partials of its pairs have landed:
       // sp x (2 rows x its pairs) x 64 bytes per 16 token columns.
@@ -579,14 +582,14 @@ __global__ void __launch_bounds__(kThreads, 2) gemm_tc_kernel(const __grid_const
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  if (sp > 1) cluster_arrive_relaxed();      // waited for before the first push into another rank
+  if (split) cluster_arrive_relaxed();      // waited for before the first push into another rank
   const uint32_t tmem = static_cast<uint32_t>(flags[1]);
   volatile int* abort_flag = flags;
 
   // This CTA's segments: sp > 1 -> one K-slice of tile blockIdx.x / sp; sp == 1 -> whole tiles
   // blockIdx.x, blockIdx.x + gridDim.x, ...
-  const int first_tile = sp > 1 ? static_cast<int>(blockIdx.x) / sp : static_cast<int>(blockIdx.x);
-  const int tile_step = sp > 1 ? a.tiles : static_cast<int>(gridDim.x);
+  const int first_tile = split ? static_cast<int>(blockIdx.x) / sp : static_cast<int>(blockIdx.x);
+  const int tile_step = split ? a.tiles : static_cast<int>(gridDim.x);
   const int kb_lo = rank * a.KB / sp, kb_hi = (rank + 1) * a.KB / sp;
   const int nkb = kb_hi - kb_lo;
 
@@ -706,7 +709,7 @@ __global__ void __launch_bounds__(kThreads, 2) gemm_tc_kernel(const __grid_const
       mma_commit(drain);                      // all MMAs issued by this thread have completed
       wait_bar_budget(drain, 0, kDrainCycles);
     }
-  } else if (sp > 1) {
+  } else if (split) {
     // Split-K epilogue of the CTA's single tile. Everything but the sums (this thread's
     // destination in the owner's receive buffer, the operands of its first owned output, the
     // RMSNorm scales) is prepared while the MMAs run.
@@ -746,7 +749,7 @@ __global__ void __launch_bounds__(kThreads, 2) gemm_tc_kernel(const __grid_const
     }
   }
 
-  if (sp > 1 && warp < 2) {                  // the producer and MMA warps take their half of the cluster barrier
+  if (split && warp < 2) {                  // the producer and MMA warps take their half of the cluster barrier
     __syncwarp();
     cluster_wait();
   }
@@ -1165,12 +1168,13 @@ int gemm_tc_max_regs() {
       if (cudaFuncGetAttributes(&fa, f) == cudaSuccess) r = std::max(r, fa.numRegs);
       else r = -1000;
     };
-    take(reinterpret_cast<const void*>(gemm_tc_kernel<TcArgs>));
-    take(reinterpret_cast<const void*>(gemm_tc_kernel<TcArgsE<EPI_STORE>>));
-    take(reinterpret_cast<const void*>(gemm_tc_kernel<TcArgsE<EPI_ADD>>));
-    take(reinterpret_cast<const void*>(gemm_tc_kernel<TcArgsE<EPI_SWIGLU>>));
-    take(reinterpret_cast<const void*>(gemm_tc_kernel<TcArgsE<EPI_QKV>>));
-    take(reinterpret_cast<const void*>(gemm_tc_kernel<TcArgsE<EPI_SILU>>));
+    take(reinterpret_cast<const void*>(gemm_tc_kernel<TcArgs, 1>));
+    take(reinterpret_cast<const void*>(gemm_tc_kernel<TcArgs, 2>));
+    take(reinterpret_cast<const void*>(gemm_tc_kernel<TcArgsE<EPI_STORE>, 0>));
+    take(reinterpret_cast<const void*>(gemm_tc_kernel<TcArgsE<EPI_ADD>, 0>));
+    take(reinterpret_cast<const void*>(gemm_tc_kernel<TcArgsE<EPI_SWIGLU>, 0>));
+    take(reinterpret_cast<const void*>(gemm_tc_kernel<TcArgsE<EPI_QKV>, 0>));
+    take(reinterpret_cast<const void*>(gemm_tc_kernel<TcArgsE<EPI_SILU>, 0>));
     cudaGetLastError();
     return r;
   }();
@@ -1373,14 +1377,14 @@ cudaError_t gemm_attn(const GemmArgs& g, unsigned* err, cudaStream_t st) {
 
 namespace {
 // One launch of the instantiation for argument type A (its shared-memory opt-in set once).
-template <class A>
+template <class A, int SPLIT>
 cudaError_t launch_tc(const TcArgs& a, const TcPlan& pl, cudaStream_t st) {
   static const cudaError_t configured =
-      cudaFuncSetAttribute(gemm_tc_kernel<A>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBudget);
+      cudaFuncSetAttribute(gemm_tc_kernel<A, SPLIT>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBudget);
   if (configured != cudaSuccess) return configured;
   A ae;
   static_cast<TcArgs&>(ae) = a;
-  return launch_pdl_cluster(gemm_tc_kernel<A>, dim3(static_cast<unsigned>(pl.grid)), dim3(kThreads),
+  return launch_pdl_cluster(gemm_tc_kernel<A, SPLIT>, dim3(static_cast<unsigned>(pl.grid)), dim3(kThreads),
                             static_cast<size_t>(pl.smem), st, pl.sp, ae);
 }
 }  // namespace
@@ -1424,13 +1428,13 @@ cudaError_t gemm_tc(const GemmArgs& g, unsigned* err, cudaStream_t st) {
   // their launches are short, and one body of code stays warm in the instruction caches across
   // a layer's projections (per-epilogue kernels made the 1B drafter step 4% slower). Wider tiles,
   // whose owner passes run many outputs per thread, take the kernel of their own epilogue.
-  if (a.NT <= 16) return launch_tc<TcArgs>(a, pl, st);
+  if (a.NT <= 16) return sp > 1 ? launch_tc<TcArgs, 1>(a, pl, st) : launch_tc<TcArgs, 2>(a, pl, st);
   switch (a.epi) {
-    case EPI_STORE: return launch_tc<TcArgsE<EPI_STORE>>(a, pl, st);
-    case EPI_ADD: return launch_tc<TcArgsE<EPI_ADD>>(a, pl, st);
-    case EPI_SWIGLU: return launch_tc<TcArgsE<EPI_SWIGLU>>(a, pl, st);
-    case EPI_QKV: return launch_tc<TcArgsE<EPI_QKV>>(a, pl, st);
-    case EPI_SILU: return launch_tc<TcArgsE<EPI_SILU>>(a, pl, st);
+    case EPI_STORE: return launch_tc<TcArgsE<EPI_STORE>, 0>(a, pl, st);
+    case EPI_ADD: return launch_tc<TcArgsE<EPI_ADD>, 0>(a, pl, st);
+    case EPI_SWIGLU: return launch_tc<TcArgsE<EPI_SWIGLU>, 0>(a, pl, st);
+    case EPI_QKV: return launch_tc<TcArgsE<EPI_QKV>, 0>(a, pl, st);
+    case EPI_SILU: return launch_tc<TcArgsE<EPI_SILU>, 0>(a, pl, st);
     default: return cudaErrorInvalidValue;
   }
 }
