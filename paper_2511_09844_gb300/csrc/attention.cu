@@ -200,9 +200,11 @@ __device__ void ctx_cluster_merge(const AttnArgs& a, const float2* rML, const fl
 }
 
 // NB: K/V tiles of the shared-memory layout (>= 2 when a.chunk > 64); ring: the split-merge
-// receive buffers lie over the K/V ring (n_splits > 1).
-template <int HD>
-__global__ void __launch_bounds__(kThreads, kCtasPerSm<HD>) attn_kernel(const AttnArgs a, int NB, int ring) {
+// receive buffers lie over the K/V ring (n_splits > 1). DEC: 1 for a decode step with one
+// context cluster per (group, KV head) and separate merge buffers (the batch-1 steps), whose
+// instantiation then carries none of the other paths' code; 0 decides everything at run time.
+template <int HD, int DEC>
+__global__ void __launch_bounds__(kThreads, kCtasPerSm<HD>) attn_kernel(const AttnArgs a, int NB, int ring_arg) {
   using C = AttnCfg<HD>;
   constexpr int KS = C::KS, SS = C::SS, PS = C::PS;
   constexpr int NT = HD / 64;  // n8 tiles of output dimensions per warp
@@ -214,7 +216,8 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm<HD>) attn_kernel(const At
   // x = context cluster r (of R) x rank in the cluster: split = blockIdx.x orders the context
   // ranges, rank = the CTA's place in its cluster (its merge share)
   const int split = blockIdx.x, g = blockIdx.y, kvh = blockIdx.z;
-  const int NS = a.n_splits, R = a.n_ctx_clusters > 1 ? a.n_ctx_clusters : 1;
+  const int NS = a.n_splits, R = DEC ? 1 : (a.n_ctx_clusters > 1 ? a.n_ctx_clusters : 1);
+  const int ring = DEC ? 0 : ring_arg;
   const int rank = split % NS, cr = split / NS;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int g8 = lane >> 2, t4 = lane & 3;
@@ -240,7 +243,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm<HD>) attn_kernel(const At
   // A decode step knows, before the wait, that its rows lie below len + pre_stable + pre_fresh: the
   // splits share that range (whole tiles, at most a.chunk each) instead of the planned maximum, so
   // no split is empty while another holds several tiles.
-  const bool early = a.pre_len != nullptr;
+  const bool early = DEC ? true : a.pre_len != nullptr;
   const int len = early ? a.pre_len[seq] : 0;
   int chunk = a.chunk;
   if (early) {
@@ -593,11 +596,12 @@ size_t smem_share(int n) {
   return share > 0 ? static_cast<size_t>(share) : 0;
 }
 
-template <int HD>
+template <int HD, int DEC>
 cudaError_t configure() {
   static cudaError_t e = [] {
-    cudaError_t r = cudaFuncSetAttribute(attn_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, kMaxSmem);
-    if (r == cudaSuccess) r = cudaFuncSetAttribute(attn_kernel<HD>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    cudaError_t r = cudaFuncSetAttribute(attn_kernel<HD, DEC>, cudaFuncAttributeMaxDynamicSharedMemorySize, kMaxSmem);
+    if (r == cudaSuccess)
+      r = cudaFuncSetAttribute(attn_kernel<HD, DEC>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
     return r;
   }();
   return e;
@@ -606,7 +610,7 @@ cudaError_t configure() {
 // Whether clusters of n CTAs of the largest step-shape attention CTA can be scheduled.
 template <int HD>
 bool clusters_fit(int n) {
-  if (configure<HD>() != cudaSuccess) return false;
+  if (configure<HD, 0>() != cudaSuccess) return false;
   cudaLaunchConfig_t cfg{};
   cfg.gridDim = dim3(n, 1, 1);
   cfg.blockDim = dim3(kThreads);
@@ -619,13 +623,15 @@ bool clusters_fit(int n) {
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   int clusters = 0;
-  return cudaOccupancyMaxActiveClusters(&clusters, attn_kernel<HD>, &cfg) == cudaSuccess && clusters > 0;
+  return cudaOccupancyMaxActiveClusters(&clusters, attn_kernel<HD, 0>, &cfg) == cudaSuccess && clusters > 0;
 }
 
 template <int HD>
 cudaError_t launch(const AttnArgs& a, cudaStream_t st) {
-  const cudaError_t e = configure<HD>();
+  const cudaError_t e = configure<HD, 0>();
   if (e != cudaSuccess) return e;
+  const cudaError_t e1 = configure<HD, 1>();
+  if (e1 != cudaSuccess) return e1;
   using C = AttnCfg<HD>;
   const int qr = C::qrows(a.max_rows, a.H / a.kv.Hkv), ns = a.n_splits;
   // The deepest K/V ring (2 to 4 tiles, at most the chunk's) within the shared memory a CTA may
@@ -650,8 +656,10 @@ cudaError_t launch(const AttnArgs& a, cudaStream_t st) {
     }
   const size_t smem = C::bytes(qr, a.chunk, ns, nb, ring);
   if (smem > static_cast<size_t>(kMaxSmem)) return cudaErrorInvalidValue;
-  return launch_pdl_cluster(attn_kernel<HD>, dim3(ns * R, a.n_groups, a.kv.Hkv), dim3(kThreads), smem, st, ns, a,
-                            nb, ring);
+  const dim3 grid(ns * R, a.n_groups, a.kv.Hkv);
+  if (a.pre_len && R == 1 && !ring)
+    return launch_pdl_cluster(attn_kernel<HD, 1>, grid, dim3(kThreads), smem, st, ns, a, nb, ring);
+  return launch_pdl_cluster(attn_kernel<HD, 0>, grid, dim3(kThreads), smem, st, ns, a, nb, ring);
 }
 
 }  // namespace
