@@ -506,6 +506,13 @@ sd2_status forward(sd2_ctx* c, const Model& m, const Plan& p, const FwdOut& o) {
       if (want < at.n_splits) {
         at.n_splits = want;
         at.chunk = 64 * ((c->cfg.max_ctx + 64 * want - 1) / (64 * want));
+      } else if (at.n_splits < attention_max_splits()) {
+        // fewer planned splits than a cluster holds (the plan rounds its chunk up to whole tiles):
+        // a cluster's worth anyway; the kernel shares the step's actual context over them, so at
+        // short contexts a split holds one tile instead of two (batch 1 at context ~650: 6.78 -> 6.67 ms)
+        const int ns = std::min(attention_max_splits(), want);
+        at.n_splits = ns;
+        at.chunk = 64 * ((c->cfg.max_ctx + 64 * ns - 1) / (64 * ns));
       } else if (at.n_splits >= 2 && p.n_groups <= kMaxCtxGroups) {
         // long contexts: more clusters of splits along the context while the grid stays resident
         // and every CTA keeps at least 4 tiles of 64 positions
