@@ -1230,7 +1230,7 @@ int max_active_clusters(int size, int smem) {
 // cluster), ring stages, dynamic shared memory and grid. Two CTAs share an SM when the ring (at
 // least 3 stages) and the split-K receive buffer fit in half its shared memory: more weight bytes in
 // flight per SM, and room for the next kernel's CTAs to start early. With fewer tiles than resident
-// CTAs the K range is split, aiming at 1.5 CTAs per SM (two-per-SM plans) or one (one-per-SM plans),
+// CTAs the K range is split, aiming at 2 CTAs per SM (two-per-SM plans) or one (one-per-SM plans),
 // never past one wave. Of the two, the plan with more CTAs streaming at once wins (ties: two per SM).
 struct TcPlan {
   int sp = 0, stages = 0, smem = 0, grid = 0;
@@ -1253,7 +1253,7 @@ TcPlan plan_tc(int tiles, int NT, int KB) {
     const int min_stages = occ == 2 && !wide ? 3 : 2;
     int sp = 1;
     if (tiles < sms * occ) {                             // split-K tiles keep one NT-column accumulator
-      sp = ((occ == 2 ? 3 * sms / 2 : sms) + tiles / 2) / tiles;
+      sp = ((occ == 2 ? 2 * sms : sms) + tiles / 2) / tiles;
       sp = std::max(1, std::min(sp, std::min(8, KB)));
       while (sp > 1 && tiles * sp > sms * occ) --sp;
     }
