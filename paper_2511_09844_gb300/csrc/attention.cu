@@ -28,6 +28,10 @@
 #include <limits.h>
 #include <math.h>
 
+#include <array>
+#include <mutex>
+#include <vector>
+
 #include "common.cuh"
 #include "kernels.h"
 #include "tc.cuh"
@@ -626,40 +630,98 @@ bool clusters_fit(int n) {
   return cudaOccupancyMaxActiveClusters(&clusters, attn_kernel<HD, 0>, &cfg) == cudaSuccess && clusters > 0;
 }
 
+// The launch's K/V ring and shared memory: the deepest ring (2 to 4 tiles, at most the chunk's)
+// within the shared memory a CTA may take, its share of the SM when the grid needs several CTAs
+// per SM resident (up to the register bound), the opt-in maximum otherwise. The merge buffers go
+// over the ring only where that is what makes it fit.
+struct Shape {
+  int nb, ring;
+  size_t smem;
+  bool dec;      // the decode instantiation (one context cluster, separate merge buffers)
+};
+
+template <int HD>
+Shape shape_of(const AttnArgs& a) {
+  using C = AttnCfg<HD>;
+  const int qr = C::qrows(a.max_rows, a.H / a.kv.Hkv), ns = a.n_splits;
+  const int max_nb = a.chunk > kTile ? std::min(kMaxBuf, a.chunk / kTile) : 1;
+  const int R = a.n_ctx_clusters > 1 ? a.n_ctx_clusters : 1;
+  const long ctas = static_cast<long>(ns) * R * a.n_groups * a.kv.Hkv, sms = sm_count_cached();
+  const int per_sm = static_cast<int>(std::min<long>(kCtasPerSm<HD>, (ctas + sms - 1) / sms));
+  const size_t cap = per_sm <= 1 ? static_cast<size_t>(kMaxSmem) : smem_share(per_sm);
+  Shape sh{std::min(2, max_nb), 0, 0, false};
+  bool found = false;
+  for (int n = max_nb; n >= std::min(2, max_nb) && !found; --n)
+    for (int r = 0; r <= 1 && !found; ++r) {
+      if (r && (ns == 1 || C::merge_bytes(qr, ns) > static_cast<size_t>(n) * C::KV_TILE)) continue;
+      if (C::bytes(qr, a.chunk, ns, n, r) <= cap) {
+        sh.nb = n;
+        sh.ring = r;
+        found = true;
+      }
+    }
+  sh.smem = C::bytes(qr, a.chunk, ns, sh.nb, sh.ring);
+  sh.dec = a.pre_len && R == 1 && !sh.ring;
+  return sh;
+}
+
 template <int HD>
 cudaError_t launch(const AttnArgs& a, cudaStream_t st) {
   const cudaError_t e = configure<HD, 0>();
   if (e != cudaSuccess) return e;
   const cudaError_t e1 = configure<HD, 1>();
   if (e1 != cudaSuccess) return e1;
-  using C = AttnCfg<HD>;
-  const int qr = C::qrows(a.max_rows, a.H / a.kv.Hkv), ns = a.n_splits;
-  // The deepest K/V ring (2 to 4 tiles, at most the chunk's) within the shared memory a CTA may
-  // take: its share of the SM when the grid needs several CTAs per SM resident (up to the register
-  // bound), the opt-in maximum otherwise. The merge buffers go over the ring only where that is
-  // what makes it fit.
-  const int max_nb = a.chunk > kTile ? std::min(kMaxBuf, a.chunk / kTile) : 1;
-  const int R = a.n_ctx_clusters > 1 ? a.n_ctx_clusters : 1;
-  const long ctas = static_cast<long>(ns) * R * a.n_groups * a.kv.Hkv, sms = sm_count_cached();
-  const int per_sm = static_cast<int>(std::min<long>(kCtasPerSm<HD>, (ctas + sms - 1) / sms));
-  const size_t cap = per_sm <= 1 ? static_cast<size_t>(kMaxSmem) : smem_share(per_sm);
-  int nb = std::min(2, max_nb), ring = 0;
-  bool found = false;
-  for (int n = max_nb; n >= std::min(2, max_nb) && !found; --n)
-    for (int r = 0; r <= 1 && !found; ++r) {
-      if (r && (ns == 1 || C::merge_bytes(qr, ns) > static_cast<size_t>(n) * C::KV_TILE)) continue;
-      if (C::bytes(qr, a.chunk, ns, n, r) <= cap) {
-        nb = n;
-        ring = r;
-        found = true;
-      }
-    }
-  const size_t smem = C::bytes(qr, a.chunk, ns, nb, ring);
-  if (smem > static_cast<size_t>(kMaxSmem)) return cudaErrorInvalidValue;
+  const Shape sh = shape_of<HD>(a);
+  if (sh.smem > static_cast<size_t>(kMaxSmem)) return cudaErrorInvalidValue;
+  const int ns = a.n_splits, R = a.n_ctx_clusters > 1 ? a.n_ctx_clusters : 1;
   const dim3 grid(ns * R, a.n_groups, a.kv.Hkv);
-  if (a.pre_len && R == 1 && !ring)
-    return launch_pdl_cluster(attn_kernel<HD, 1>, grid, dim3(kThreads), smem, st, ns, a, nb, ring);
-  return launch_pdl_cluster(attn_kernel<HD, 0>, grid, dim3(kThreads), smem, st, ns, a, nb, ring);
+  if (sh.dec)
+    return launch_pdl_cluster(attn_kernel<HD, 1>, grid, dim3(kThreads), sh.smem, st, ns, a, sh.nb, sh.ring);
+  return launch_pdl_cluster(attn_kernel<HD, 0>, grid, dim3(kThreads), sh.smem, st, ns, a, sh.nb, sh.ring);
+}
+
+// Clusters of this shape the device holds at once (cudaOccupancyMaxActiveClusters, remembered per
+// instantiation, cluster size and shared memory: the answer depends on how clusters pack into the
+// GPCs, which a per-SM count does not see).
+template <int HD>
+int max_clusters(const Shape& sh, int ns) {
+  static std::mutex mu;
+  static std::vector<std::array<long, 3>> seen;   // (dec * 32 + ns, smem, clusters)
+  const long key = (sh.dec ? 32 : 0) + ns;
+  {
+    std::lock_guard<std::mutex> lk(mu);
+    for (const auto& v : seen)
+      if (v[0] == key && v[1] == static_cast<long>(sh.smem)) return static_cast<int>(v[2]);
+  }
+  if (configure<HD, 0>() != cudaSuccess || configure<HD, 1>() != cudaSuccess) return 0;
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3(ns, 1, 1);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = sh.smem;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = static_cast<unsigned>(ns);
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  int n = 0;
+  const cudaError_t e = sh.dec ? cudaOccupancyMaxActiveClusters(&n, attn_kernel<HD, 1>, &cfg)
+                               : cudaOccupancyMaxActiveClusters(&n, attn_kernel<HD, 0>, &cfg);
+  if (e != cudaSuccess) {
+    cudaGetLastError();
+    n = 0;
+  }
+  std::lock_guard<std::mutex> lk(mu);
+  seen.push_back({key, static_cast<long>(sh.smem), static_cast<long>(n)});
+  return n;
+}
+
+template <int HD>
+int clusters_max(const AttnArgs& a) {
+  const Shape sh = shape_of<HD>(a);
+  if (sh.smem > static_cast<size_t>(kMaxSmem)) return 0;
+  return max_clusters<HD>(sh, a.n_splits);
 }
 
 }  // namespace
@@ -669,6 +731,13 @@ int attention_ctas_per_sm(int hd) { return hd == 64 ? kCtasPerSm<64> : kCtasPerS
 int attention_max_splits() {
   static const int n = (clusters_fit<128>(kMaxSplits) && clusters_fit<64>(kMaxSplits)) ? kMaxSplits : 8;
   return n;
+}
+
+int attention_max_clusters(const AttnArgs& a) {
+  if (a.n_splits < 1 || a.n_splits > kMaxSplits || a.chunk <= 0 || a.kv.Hkv <= 0 || a.H % a.kv.Hkv != 0) return 0;
+  if (a.hd == 128) return clusters_max<128>(a);
+  if (a.hd == 64) return clusters_max<64>(a);
+  return 0;
 }
 
 cudaError_t attention(const AttnArgs& a, cudaStream_t st) {

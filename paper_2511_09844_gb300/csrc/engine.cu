@@ -503,29 +503,52 @@ sd2_status forward(sd2_ctx* c, const Model& m, const Plan& p, const FwdOut& o) {
     if (p.pre_len) {   // decode step: as many context splits as the GPU holds resident at once, no more
       const long resident = static_cast<long>(attention_ctas_per_sm(hd)) * sm_count_cached();
       const int want = std::max(1, static_cast<int>(resident / std::max(1, p.n_groups * Hkv)));
+      const int max_ctx = c->cfg.max_ctx;
+      auto chunk_for = [max_ctx](int ns, int R) { return 64 * ((max_ctx + 64 * ns * R - 1) / (64 * ns * R)); };
+      at.pre_len = p.pre_len;
       if (want < at.n_splits) {
         at.n_splits = want;
-        at.chunk = 64 * ((c->cfg.max_ctx + 64 * want - 1) / (64 * want));
+        at.chunk = chunk_for(want, 1);
       } else if (at.n_splits < attention_max_splits()) {
         // fewer planned splits than a cluster holds (the plan rounds its chunk up to whole tiles):
         // a cluster's worth anyway; the kernel shares the step's actual context over them, so at
         // short contexts a split holds one tile instead of two (batch 1 at context ~650: 6.78 -> 6.67 ms)
         const int ns = std::min(attention_max_splits(), want);
         at.n_splits = ns;
-        at.chunk = 64 * ((c->cfg.max_ctx + 64 * ns - 1) / (64 * ns));
+        at.chunk = chunk_for(ns, 1);
       } else if (at.n_splits >= 2 && p.n_groups <= kMaxCtxGroups) {
-        // long contexts: more clusters of splits along the context while the grid stays resident
-        // and every CTA keeps at least 4 tiles of 64 positions
-        int Rc = 1;
-        while (Rc < kMaxCtxClusters &&
-               static_cast<long>(at.n_splits) * (Rc + 1) * p.n_groups * Hkv <= resident &&
-               c->cfg.max_ctx >= 64 * 4 * at.n_splits * (Rc + 1))
-          ++Rc;
-        if (Rc > 1) {
-          at.n_ctx_clusters = Rc;
-          at.chunk = 64 * ((c->cfg.max_ctx + 64 * at.n_splits * Rc - 1) / (64 * at.n_splits * Rc));
+        // long contexts: R clusters of 8 splits share the context, R as large as keeps every CTA at
+        // 4 or more tiles of 64 positions, the clusters within what the occupancy calculator says
+        // the device holds at once and the CTAs within 3/4 of the per-SM count. Measured on the
+        // 16K-context step, where the calculator allows 36 clusters of 8 at two CTAs per SM: the
+        // 8B verify's 32 clusters (256 CTAs, the per-SM count's 304 nearly full) still ran partly in
+        // a second wave, 24 did not (4.25 -> 3.84 ms); the 1B drafter's 32 (of 608) did not (step
+        // 1.02 -> 0.93 ms); clusters of 16 lost to clusters of 8 at every CTA count.
+        const int ns = std::min(at.n_splits, 8);
+        int best_R = 0;
+        for (int Rc = 1; Rc <= kMaxCtxClusters; ++Rc) {
+          const long per_head = static_cast<long>(ns) * Rc;
+          if (4 * per_head * p.n_groups * Hkv > 3 * resident || max_ctx < 64 * 4 * per_head) break;
+          AttnArgs t = at;
+          t.n_splits = ns; t.n_ctx_clusters = Rc; t.chunk = chunk_for(ns, Rc);
+          t.part_acc = c->attn_part_acc; t.part_ml = c->attn_part_ml; t.part_cnt = c->attn_part_cnt;
+          // (not monotone in R: more CTAs per SM take less shared memory each)
+          if (static_cast<long>(Rc) * p.n_groups * Hkv > attention_max_clusters(t)) continue;
+          best_R = Rc;
+        }
+        if (best_R >= 2 && ns * best_R > at.n_splits) {   // else the planned single cluster
+          at.n_splits = ns;
+          at.n_ctx_clusters = best_R;
+          at.chunk = chunk_for(ns, best_R);
           at.part_acc = c->attn_part_acc; at.part_ml = c->attn_part_ml; at.part_cnt = c->attn_part_cnt;
         }
+      }
+      // a single cluster per (group, KV head) whose clusters cannot all be resident at once would
+      // run in two waves: fewer splits instead
+      while (at.n_ctx_clusters == 1 && at.n_splits > 1 &&
+             static_cast<long>(p.n_groups) * Hkv > attention_max_clusters(at)) {
+        --at.n_splits;
+        at.chunk = chunk_for(at.n_splits, 1);
       }
     }
     at.pre_len = p.pre_len; at.pre_stable = p.pre_stable; at.pre_fresh = p.pre_fresh; at.err = c->errw;

@@ -219,6 +219,10 @@ cudaError_t attention(const AttnArgs& a, cudaStream_t st);
 int attention_max_splits();
 // CTAs of one attention launch an SM can hold at once for head dim hd (4 for 64, 2 for 128).
 int attention_ctas_per_sm(int hd);
+// Clusters of the launch `a` describes (n_splits CTAs each, with the shared memory attention()
+// would give them) that the device holds at once: the occupancy calculator's count, which sees how
+// clusters pack into the GPCs where the per-SM count above does not. 0 for shapes attention() rejects.
+int attention_max_clusters(const AttnArgs& a);
 
 // ---------------------------------------------------------------- persistent layer chain
 // Every decoder layer of one forward pass over at most 16 token rows in one cooperative launch
