@@ -93,7 +93,6 @@ struct AttnCfg {
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }
-__device__ __forceinline__ uint32_t ld_u32(const bf16* p) { return *reinterpret_cast<const uint32_t*>(p); }
 __device__ __forceinline__ uint32_t pack_bf2(float x, float y) {
   const __nv_bfloat162 h = __floats2bfloat162_rn(x, y);
   return *reinterpret_cast<const uint32_t*>(&h);
@@ -127,6 +126,12 @@ __device__ __forceinline__ void mma_bf16(float (&d)[4], uint32_t a0, uint32_t a1
       "{%0,%1,%2,%3};"
       : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
       : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr)
+               : "memory");
 }
 __device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
   asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
@@ -381,11 +386,9 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm<HD>) attn_kernel(const At
       const int n0 = warp * 8;
       uint32_t kb[HD / 16][2];
 #pragma unroll
-      for (int kk = 0; kk < HD / 16; ++kk) {
-        const bf16* p = sK + (n0 + g8) * KS + kk * 16 + 2 * t4;
-        kb[kk][0] = ld_u32(p);
-        kb[kk][1] = ld_u32(p + 8);
-      }
+      for (int kk = 0; kk < HD / 16; kk += 2)
+        ldsm_x4(smem_u32(sK + (n0 + (lane & 7)) * KS + kk * 16 + (lane >> 3) * 8), kb[kk][0], kb[kk][1],
+                kb[kk + 1][0], kb[kk + 1][1]);
       const int pc = t0 + n0 + 2 * t4;
 #pragma unroll
       for (int mt = 0; mt < 4; ++mt) {
@@ -393,8 +396,9 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm<HD>) attn_kernel(const At
           float c[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
           for (int kk = 0; kk < HD / 16; ++kk) {
-            const bf16* qa = sQ + (mt * 16 + g8) * KS + kk * 16 + 2 * t4;
-            mma_bf16(c, ld_u32(qa), ld_u32(qa + 8 * KS), ld_u32(qa + 8), ld_u32(qa + 8 * KS + 8), kb[kk][0], kb[kk][1]);
+            uint32_t a0, a1, a2, a3;
+            ldsm_x4(smem_u32(sQ + (mt * 16 + (lane & 15)) * KS + kk * 16 + (lane >> 4) * 8), a0, a1, a2, a3);
+            mma_bf16(c, a0, a1, a2, a3, kb[kk][0], kb[kk][1]);
           }
           const int qv = mt * 16 + g8;
           const int pa = sPos[qv], pb = sPos[qv + 8];
@@ -470,8 +474,8 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm<HD>) attn_kernel(const At
           }
 #pragma unroll
           for (int kk = 0; kk < kTile / 16; ++kk) {
-            const bf16* pa = sP + (mt * 16 + g8) * PS + kk * 16 + 2 * t4;
-            const uint32_t a0 = ld_u32(pa), a1 = ld_u32(pa + 8 * PS), a2 = ld_u32(pa + 8), a3 = ld_u32(pa + 8 * PS + 8);
+            uint32_t a0, a1, a2, a3;
+            ldsm_x4(smem_u32(sP + (mt * 16 + (lane & 15)) * PS + kk * 16 + (lane >> 4) * 8), a0, a1, a2, a3);
 #pragma unroll
             for (int nt = 0; nt < NT; ++nt) mma_bf16(acc[mt][nt], a0, a1, a2, a3, vb[kk][nt][0], vb[kk][nt][1]);
           }
