@@ -9,6 +9,11 @@ namespace {
 
 constexpr int kNormThreads = 256;
 
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  const __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<const uint32_t*>(&h);
+}
+
 __device__ __forceinline__ float row_inv_rms(const float* xr, int d, float eps, float* red) {
   float ss = 0.f;
   for (int j = threadIdx.x * 4; j < d; j += blockDim.x * 4) {
@@ -107,14 +112,18 @@ __global__ void __launch_bounds__(kNormThreads) rmsnorm_kernel(const float* x, c
   }
 }
 
-// One CTA per row; thread t handles rotation pairs (head, i) with i < hd/2 over all q, k, v heads.
-__global__ void rope_append_kernel(const float* qkv, const float* cs, int H, int Hkv, int hd, const int* row_seq,
-                                   const int* row_pos, const int* row_valid, KVCache kv, int layer, float* q) {
+// One CTA per row; a work item is 4 consecutive rotation pairs (head, i .. i+3), i < hd/2, over all
+// q, k, v heads. The pointers do not alias, and each thread issues the loads of all its items (4 per
+// round) before any store, so a row costs about one round trip to L2 instead of one per item.
+__global__ void rope_append_kernel(const float* __restrict__ qkv, const float* __restrict__ cs, int H, int Hkv,
+                                   int hd, const int* __restrict__ row_seq, const int* __restrict__ row_pos,
+                                   const int* __restrict__ row_valid, KVCache kv, int layer, float* __restrict__ q) {
   pdl_trigger();
   pdl_wait();
+  constexpr int kPer = 4;
   const int m = blockIdx.x;
-  const int half = hd / 2;
-  const int nh = H + 2 * Hkv;
+  const int half = hd / 2, quads = half / 4;
+  const int nh = H + 2 * Hkv, items = nh * quads;
   const int pos = row_pos[m];
   const bool valid = row_valid ? row_valid[m] != 0 : true;
   const float* src = qkv + static_cast<size_t>(m) * nh * hd;
@@ -125,25 +134,46 @@ __global__ void rope_append_kernel(const float* qkv, const float* cs, int H, int
     const int blk = kv.table[static_cast<size_t>(row_seq[m]) * kv.bt_stride + (pos >> 4)];
     blk_base = (static_cast<size_t>(layer) * kv.n_blocks + blk) * 2 * Hkv * 16 * hd + (pos & 15) * hd;
   }
-  for (int idx = threadIdx.x; idx < nh * half; idx += blockDim.x) {
-    const int h = idx / half, i = idx % half;
-    const float x1 = src[h * hd + i], x2 = src[h * hd + i + half];
-    if (h < H + Hkv) {
-      const float cv = c[2 * i], sv = c[2 * i + 1];
-      const float r1 = x1 * cv - x2 * sv, r2 = x2 * cv + x1 * sv;
-      if (h < H) {
-        float* qo = q + (static_cast<size_t>(m) * H + h) * hd;
-        qo[i] = r1;
-        qo[i + half] = r2;
-      } else if (valid) {
-        bf16* ko = pool + blk_base + static_cast<size_t>(h - H) * 16 * hd;
-        ko[i] = __float2bfloat16_rn(r1);
-        ko[i + half] = __float2bfloat16_rn(r2);
+  for (int base = threadIdx.x; base < items; base += blockDim.x * kPer) {
+    float4 x1[kPer], x2[kPer], c0[kPer], c1[kPer];
+#pragma unroll
+    for (int u = 0; u < kPer; ++u) {
+      const int idx = base + u * blockDim.x;
+      if (idx < items) {
+        const int h = idx / quads, i = (idx % quads) * 4;
+        x1[u] = *reinterpret_cast<const float4*>(src + h * hd + i);
+        x2[u] = *reinterpret_cast<const float4*>(src + h * hd + i + half);
+        if (h < H + Hkv) {
+          c0[u] = *reinterpret_cast<const float4*>(c + 2 * i);       // cos i, sin i, cos i+1, sin i+1
+          c1[u] = *reinterpret_cast<const float4*>(c + 2 * i + 4);   // cos i+2, sin i+2, cos i+3, sin i+3
+        }
       }
-    } else if (valid) {
-      bf16* vo = pool + blk_base + static_cast<size_t>(Hkv) * 16 * hd + static_cast<size_t>(h - H - Hkv) * 16 * hd;
-      vo[i] = __float2bfloat16_rn(x1);
-      vo[i + half] = __float2bfloat16_rn(x2);
+    }
+#pragma unroll
+    for (int u = 0; u < kPer; ++u) {
+      const int idx = base + u * blockDim.x;
+      if (idx >= items) break;
+      const int h = idx / quads, i = (idx % quads) * 4;
+      const float4 a = x1[u], b = x2[u];
+      if (h < H + Hkv) {
+        const float4 r1 = make_float4(a.x * c0[u].x - b.x * c0[u].y, a.y * c0[u].z - b.y * c0[u].w,
+                                      a.z * c1[u].x - b.z * c1[u].y, a.w * c1[u].z - b.w * c1[u].w);
+        const float4 r2 = make_float4(b.x * c0[u].x + a.x * c0[u].y, b.y * c0[u].z + a.y * c0[u].w,
+                                      b.z * c1[u].x + a.z * c1[u].y, b.w * c1[u].z + a.w * c1[u].w);
+        if (h < H) {
+          float* qo = q + (static_cast<size_t>(m) * H + h) * hd;
+          *reinterpret_cast<float4*>(qo + i) = r1;
+          *reinterpret_cast<float4*>(qo + i + half) = r2;
+        } else if (valid) {
+          bf16* ko = pool + blk_base + static_cast<size_t>(h - H) * 16 * hd;
+          *reinterpret_cast<uint2*>(ko + i) = make_uint2(pack_bf16x2(r1.x, r1.y), pack_bf16x2(r1.z, r1.w));
+          *reinterpret_cast<uint2*>(ko + i + half) = make_uint2(pack_bf16x2(r2.x, r2.y), pack_bf16x2(r2.z, r2.w));
+        }
+      } else if (valid) {
+        bf16* vo = pool + blk_base + static_cast<size_t>(Hkv) * 16 * hd + static_cast<size_t>(h - H - Hkv) * 16 * hd;
+        *reinterpret_cast<uint2*>(vo + i) = make_uint2(pack_bf16x2(a.x, a.y), pack_bf16x2(a.z, a.w));
+        *reinterpret_cast<uint2*>(vo + i + half) = make_uint2(pack_bf16x2(b.x, b.y), pack_bf16x2(b.z, b.w));
+      }
     }
   }
 }
