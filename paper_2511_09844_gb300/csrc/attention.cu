@@ -46,6 +46,7 @@ constexpr int kMaxQV = 64;              // query vectors per CTA
 constexpr int kMaxSplits = 16;          // context splits = CTAs of one cluster (16: non-portable size)
 constexpr int kMaxSmem = 200 * 1024;   // dynamic shared memory opt-in (static arrays come on top)
 constexpr int kMaxBuf = 4;             // K/V tiles of the ring
+constexpr int kFlatMaxSplits = 32;     // slots one row group takes in flat mode
 // Resident CTAs per SM the register budget allows: hd = 64 fits 64 registers a thread, so four
 // CTAs; hd = 128 keeps two.
 template <int HD>
@@ -224,11 +225,58 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm<HD>) attn_kernel(const At
 
   // x = context cluster r (of R) x rank in the cluster: split = blockIdx.x orders the context
   // ranges, rank = the CTA's place in its cluster (its merge share)
-  const int split = blockIdx.x, g = blockIdx.y, kvh = blockIdx.z;
+  int split = blockIdx.x, g = blockIdx.y;
+  const int kvh = blockIdx.z;
   const int NS = a.n_splits, R = DEC ? 1 : (a.n_ctx_clusters > 1 ? a.n_ctx_clusters : 1);
   const int ring = DEC ? 0 : ring_arg;
-  const int rank = split % NS, cr = split / NS;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  // Flat mode: slot blockIdx.x of this KV head -> (group g, split of Rf). Group j takes
+  // ceil(tiles_j / t) slots, tiles_j its visible length in 64-position tiles and t the smallest
+  // count for which all groups fit the slots, so no slot holds more than t tiles; slots past the
+  // last group have nothing to do. Every CTA derives the same map from the pre-step lengths.
+  int Rf = 1, slot0 = 0;
+  if (!DEC && a.flat > 0) {
+    __shared__ int sMap[3];
+    if (warp == 0) {
+      const int ng = a.n_groups, W = a.flat;
+      auto tiles_of = [&](int j) {
+        const int L = a.pre_len[a.grp_seq[j]] + a.pre_stable + a.pre_fresh;
+        return max(1, (L + kTile - 1) / kTile);
+      };
+      const int t0 = lane < ng ? tiles_of(lane) : 0, t1 = lane + 32 < ng ? tiles_of(lane + 32) : 0;
+      const int T = __reduce_add_sync(0xffffffffu, t0 + t1);
+      const int tmax = __reduce_max_sync(0xffffffffu, max(t0, t1));
+      // at most kFlatMaxSplits slots a group (the merge stages their weights in shared memory)
+      int t_lo = max(max(1, (T + W - 1) / W), (tmax + kFlatMaxSplits - 1) / kFlatMaxSplits), t_hi = max(t_lo, tmax);
+      while (t_lo < t_hi) {                          // warp-uniform bisection
+        const int t = (t_lo + t_hi) >> 1;
+        const int need = __reduce_add_sync(0xffffffffu, (t0 + t - 1) / t + (t1 + t - 1) / t);
+        if (need <= W) t_hi = t; else t_lo = t + 1;
+      }
+      const int n0 = (t0 + t_lo - 1) / t_lo, n1 = (t1 + t_lo - 1) / t_lo;
+      int p0 = n0, p1 = n1;                          // inclusive prefix sums over groups 0..31, 32..63
+#pragma unroll
+      for (int off = 1; off < 32; off <<= 1) {
+        const int v0 = __shfl_up_sync(0xffffffffu, p0, off), v1 = __shfl_up_sync(0xffffffffu, p1, off);
+        if (lane >= off) { p0 += v0; p1 += v1; }
+      }
+      p1 += __shfl_sync(0xffffffffu, p0, 31);
+      const int sl = blockIdx.x;
+      const bool in0 = lane < ng && sl >= p0 - n0 && sl < p0;
+      const bool in1 = lane + 32 < ng && sl >= p1 - n1 && sl < p1;
+      if (lane == 0) sMap[0] = -1;
+      __syncwarp();
+      if (in0) { sMap[0] = lane; sMap[1] = p0 - n0; sMap[2] = n0; }
+      if (in1) { sMap[0] = lane + 32; sMap[1] = p1 - n1; sMap[2] = n1; }
+    }
+    __syncthreads();
+    g = sMap[0];
+    if (g < 0) return;                               // a slot past the last group
+    slot0 = sMap[1];
+    Rf = sMap[2];
+    split = blockIdx.x - slot0;
+  }
+  const int rank = split % NS, cr = split / NS;
   const int g8 = lane >> 2, t4 = lane & 3;
   const int Hkv = a.kv.Hkv, G = a.H / Hkv;
   const int QR = C::qrows(a.max_rows, G);
@@ -256,7 +304,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm<HD>) attn_kernel(const At
   const int len = early ? a.pre_len[seq] : 0;
   int chunk = a.chunk;
   if (early) {
-    const int per = (len + a.pre_stable + a.pre_fresh + NS * R - 1) / (NS * R);
+    const int per = (len + a.pre_stable + a.pre_fresh + NS * R * Rf - 1) / (NS * R * Rf);
     chunk = min(a.chunk, max(kTile, ((per + kTile - 1) / kTile) * kTile));
   }
   const int lo = split * chunk;
@@ -487,8 +535,91 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm<HD>) attn_kernel(const At
 
   const int d0 = warp * 8 * NT;
   if (NS == 1) {
-    if (srow < nmt * 16 && squart == 0) sL[srow] = l_run;
+    float* sMx = sCorr + kMaxQV;                    // the row data's max slot
+    if (srow < nmt * 16 && squart == 0) {
+      sL[srow] = l_run;
+      sMx[srow] = m_run;
+    }
     __syncthreads();
+    if (Rf > 1) {
+      // Flat mode merge: this split's unnormalised accumulators and (max, sum) per query vector go
+      // to its slot; it counts itself in (self-resetting), and the group's last split combines the
+      // Rf slots in split order: out = sum_s acc_s e^{m_s - M} / sum_s l_s e^{m_s - M}.
+      const size_t sl = static_cast<size_t>(kvh) * a.flat + blockIdx.x;
+      float* pacc = static_cast<float*>(a.flat_acc) + sl * (kMaxQV * HD);
+      float2* pml = static_cast<float2*>(a.flat_ml);
+#pragma unroll
+      for (int mt = 0; mt < 4; ++mt) {
+        if (mt >= nmt) break;
+#pragma unroll
+        for (int half = 0; half < 2; ++half) {
+          const int qv = mt * 16 + g8 + 8 * half;
+          if (qv >= nqv) continue;
+#pragma unroll
+          for (int nt = 0; nt < NT; ++nt)
+            *reinterpret_cast<float2*>(pacc + qv * HD + d0 + nt * 8 + 2 * t4) =
+                make_float2(acc[mt][nt][2 * half], acc[mt][nt][2 * half + 1]);
+        }
+      }
+      if (tid < nqv) pml[sl * kMaxQV + tid] = make_float2(sMx[tid], sL[tid]);
+      __threadfence();                              // the partial before the count
+      __syncthreads();
+      if (tid == 0) {
+        unsigned* cnt = a.flat_cnt + static_cast<size_t>(g) * Hkv + kvh;
+        sRecv = atomicInc(cnt, static_cast<unsigned>(Rf - 1)) == static_cast<unsigned>(Rf - 1) ? 1 : 0;
+      }
+      __syncthreads();
+      if (!sRecv) return;
+      __threadfence();                              // every split's partial is visible
+      const size_t s0 = static_cast<size_t>(kvh) * a.flat + slot0;
+      const float* acc0 = static_cast<const float*>(a.flat_acc) + s0 * (kMaxQV * HD);
+      // weights w[q][qv] = e^{m_q - M} / sum_q l_q e^{m_q - M} in shared memory (over the K/V ring,
+      // whose copies have all landed): the (max, sum) pairs staged in parallel, then one thread per
+      // query vector
+      float* sW = reinterpret_cast<float*>(sKV);                     // [kFlatMaxSplits][kMaxQV]
+      float2* sML = reinterpret_cast<float2*>(sKV + kFlatMaxSplits * kMaxQV * 4);
+      for (int i = tid; i < Rf * nqv; i += kThreads) {
+        const int q = i / nqv, qv = i % nqv;
+        sML[q * kMaxQV + qv] = __ldcg(&pml[(s0 + q) * kMaxQV + qv]);
+      }
+      __syncthreads();
+      if (tid < nqv) {
+        float M = -INFINITY;
+        for (int q = 0; q < Rf; ++q) M = fmaxf(M, sML[q * kMaxQV + tid].x);
+        float L = 0.f;
+        for (int q = 0; q < Rf; ++q) {                               // in split order
+          const float2 ml = sML[q * kMaxQV + tid];
+          const float w = ml.x == -INFINITY ? 0.f : __expf(ml.x - M);
+          sW[q * kMaxQV + tid] = w;
+          L = fmaf(ml.y, w, L);
+        }
+        const float inv = 1.f / L;
+        for (int q = 0; q < Rf; ++q) sW[q * kMaxQV + tid] *= inv;
+      }
+      __syncthreads();
+      for (int e = tid; e < nqv * (HD / 4); e += kThreads) {
+        const int qv = e / (HD / 4), d4 = e % (HD / 4);
+        const float4* src = reinterpret_cast<const float4*>(acc0 + qv * HD) + d4;
+        float4 o = make_float4(0.f, 0.f, 0.f, 0.f);
+        for (int q0 = 0; q0 < Rf; q0 += 8) {                        // 8 slots' loads in flight
+          float4 v[8];
+#pragma unroll
+          for (int u = 0; u < 8; ++u)
+            if (q0 + u < Rf) v[u] = __ldcg(src + static_cast<size_t>(q0 + u) * (kMaxQV * HD / 4));
+#pragma unroll
+          for (int u = 0; u < 8; ++u)
+            if (q0 + u < Rf) {
+              const float w = sW[(q0 + u) * kMaxQV + qv];
+              o.x = fmaf(w, v[u].x, o.x); o.y = fmaf(w, v[u].y, o.y);
+              o.z = fmaf(w, v[u].z, o.z); o.w = fmaf(w, v[u].w, o.w);
+            }
+        }
+        const size_t rh = static_cast<size_t>(r0 + qv / G) * a.H + kvh * G + qv % G;
+        *reinterpret_cast<uint2*>(static_cast<bf16*>(a.out) + rh * HD + d4 * 4) =
+            make_uint2(pack_bf2(o.x, o.y), pack_bf2(o.z, o.w));
+      }
+      return;
+    }
 #pragma unroll
     for (int mt = 0; mt < 4; ++mt) {
       if (mt >= nmt) break;
@@ -650,7 +781,8 @@ Shape shape_of(const AttnArgs& a) {
   const int qr = C::qrows(a.max_rows, a.H / a.kv.Hkv), ns = a.n_splits;
   const int max_nb = a.chunk > kTile ? std::min(kMaxBuf, a.chunk / kTile) : 1;
   const int R = a.n_ctx_clusters > 1 ? a.n_ctx_clusters : 1;
-  const long ctas = static_cast<long>(ns) * R * a.n_groups * a.kv.Hkv, sms = sm_count_cached();
+  const long ctas = a.flat > 0 ? static_cast<long>(a.flat) * a.kv.Hkv : static_cast<long>(ns) * R * a.n_groups * a.kv.Hkv;
+  const long sms = sm_count_cached();
   const int per_sm = static_cast<int>(std::min<long>(kCtasPerSm<HD>, (ctas + sms - 1) / sms));
   const size_t cap = per_sm <= 1 ? static_cast<size_t>(kMaxSmem) : smem_share(per_sm);
   Shape sh{std::min(2, max_nb), 0, 0, false};
@@ -665,7 +797,7 @@ Shape shape_of(const AttnArgs& a) {
       }
     }
   sh.smem = C::bytes(qr, a.chunk, ns, sh.nb, sh.ring);
-  sh.dec = a.pre_len && R == 1 && !sh.ring;
+  sh.dec = a.pre_len && R == 1 && !sh.ring && a.flat <= 0;
   return sh;
 }
 
@@ -678,7 +810,7 @@ cudaError_t launch(const AttnArgs& a, cudaStream_t st) {
   const Shape sh = shape_of<HD>(a);
   if (sh.smem > static_cast<size_t>(kMaxSmem)) return cudaErrorInvalidValue;
   const int ns = a.n_splits, R = a.n_ctx_clusters > 1 ? a.n_ctx_clusters : 1;
-  const dim3 grid(ns * R, a.n_groups, a.kv.Hkv);
+  const dim3 grid = a.flat > 0 ? dim3(a.flat, 1, a.kv.Hkv) : dim3(ns * R, a.n_groups, a.kv.Hkv);
   if (sh.dec)
     return launch_pdl_cluster(attn_kernel<HD, 1>, grid, dim3(kThreads), sh.smem, st, ns, a, sh.nb, sh.ring);
   return launch_pdl_cluster(attn_kernel<HD, 0>, grid, dim3(kThreads), sh.smem, st, ns, a, sh.nb, sh.ring);
@@ -750,6 +882,10 @@ cudaError_t attention(const AttnArgs& a, cudaStream_t st) {
   if (a.kv.Hkv <= 0 || a.H % a.kv.Hkv != 0 || a.max_rows < 1 || a.max_rows * (a.H / a.kv.Hkv) > kMaxQV)
     return cudaErrorInvalidValue;
   if (a.n_ctx_clusters > 1 && (a.n_splits < 2 || !a.part_acc || !a.part_ml || !a.part_cnt)) return cudaErrorInvalidValue;
+  if (a.flat > 0 && (!a.pre_len || a.n_splits != 1 || a.n_ctx_clusters > 1 || a.n_groups > a.flat || a.n_groups > 64 ||
+                     a.chunk < 2 * kTile ||   // a ring of two tiles holds the merge's weights
+                     !a.flat_acc || !a.flat_ml || !a.flat_cnt))
+    return cudaErrorInvalidValue;
   if (a.hd == 128) return launch<128>(a, st);
   if (a.hd == 64) return launch<64>(a, st);
   return cudaErrorInvalidValue;

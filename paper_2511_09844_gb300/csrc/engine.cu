@@ -113,6 +113,8 @@ struct sd2_ctx {
   void *a = nullptr, *attn = nullptr, *h = nullptr, *g_bf = nullptr, *hml_in = nullptr;
   // long-context attention: partials of the context clusters and the per-share arrival counters
   void *attn_part_acc = nullptr, *attn_part_ml = nullptr, *attn_part_cnt = nullptr;
+  void *attn_flat_acc = nullptr, *attn_flat_ml = nullptr;   // flat-mode attention partials
+  unsigned* attn_flat_cnt = nullptr;
   int gemm_impl = 0;            // 0 tensor cores where the shape allows, 1 CUDA cores
   unsigned long long* samp_slot = nullptr;
   int* samp_counter = nullptr;
@@ -216,6 +218,14 @@ cudaError_t timed(sd2_ctx* c, int cls, double bytes, F fn) {
   return e;
 }
 constexpr int kMaxCtxClusters = 4;   // context clusters of one long-context attention launch
+constexpr int kMaxFlatGroups = 64;   // row groups of one flat-mode attention launch
+// Fewest row groups, and rows per group, for flat mode. Balancing pays where the tile loop
+// dominates: the batch-16 verify (9 rows a group, 128-1280 positions) went from 5.95 to 5.73 ms,
+// while its drafter steps (1-2 rows a group) went from 0.939 to 0.961 ms and 4 sequences of equal
+// length (the Qwen pair) gained nothing, the merge through global memory costing more than the
+// cluster's.
+constexpr int kMinFlatGroups = 8;
+constexpr int kMinFlatRows = 4;
 constexpr int kMaxCtxGroups = 4;     // attention row groups a launch with context clusters may have
 constexpr int kMaxStampedLaunches = 8192;   // GEMM launches of one step that in-graph timing can follow
 enum { PC_GEMM = 0, PC_ATTN = 1, PC_ACCEPT = 2, PC_SAMPLE = 3, PC_OTHER = 4, PC_VERIFY = 5, PC_DRAFT = 6, PC_STEER = 7,
@@ -506,7 +516,16 @@ sd2_status forward(sd2_ctx* c, const Model& m, const Plan& p, const FwdOut& o) {
       const int max_ctx = c->cfg.max_ctx;
       auto chunk_for = [max_ctx](int ns, int R) { return 64 * ((max_ctx + 64 * ns * R - 1) / (64 * ns * R)); };
       at.pre_len = p.pre_len;
-      if (want < at.n_splits) {
+      const int W = static_cast<int>(resident / Hkv);
+      if (p.n_groups >= kMinFlatGroups && p.n_groups <= kMaxFlatGroups && p.max_rows >= kMinFlatRows &&
+          W >= p.n_groups && max_ctx > 64) {
+        // many row groups (sequences of ragged lengths) of several rows each: flat mode, every
+        // resident CTA a slot, the slots shared out on the device by the sequences' lengths
+        at.n_splits = 1;
+        at.flat = W;
+        at.chunk = 64 * ((max_ctx + 63) / 64);
+        at.flat_acc = c->attn_flat_acc; at.flat_ml = c->attn_flat_ml; at.flat_cnt = c->attn_flat_cnt;
+      } else if (want < at.n_splits) {
         at.n_splits = want;
         at.chunk = chunk_for(want, 1);
       } else if (at.n_splits < attention_max_splits()) {
@@ -827,6 +846,18 @@ sd2_status sd2_init(const sd2_config* cfg, const sd2_weights* w, void* stream, s
       ALLOC(c->attn_part_ml, slots * 8);
       ALLOC(c->attn_part_cnt, static_cast<size_t>(kMaxCtxGroups) * hkv * 16 * 4);
       CK(cudaMemset(c->attn_part_cnt, 0, static_cast<size_t>(kMaxCtxGroups) * hkv * 16 * 4));
+      // flat-mode attention: a slot per resident CTA of either model ([Hkv][W][64][hd] f32 and
+      // [Hkv][W][64] float2, W * Hkv <= the resident CTAs), counters [kMaxFlatGroups][Hkv]
+      size_t acc_b = 0, ml_b = 0;
+      for (const sd2_lm_config* mc : {&cfg->verifier, &cfg->drafter}) {
+        const size_t ctas = static_cast<size_t>(attention_ctas_per_sm(mc->head_dim)) * sm_count_cached();
+        acc_b = std::max(acc_b, ctas * 64 * mc->head_dim * 4);
+        ml_b = std::max(ml_b, ctas * 64 * 8);
+      }
+      ALLOC(c->attn_flat_acc, acc_b);
+      ALLOC(c->attn_flat_ml, ml_b);
+      ALLOC(c->attn_flat_cnt, static_cast<size_t>(kMaxFlatGroups) * hkv);
+      CK(cudaMemset(c->attn_flat_cnt, 0, static_cast<size_t>(kMaxFlatGroups) * hkv * sizeof(unsigned)));
     }
     ALLOC(c->h, static_cast<size_t>(R) * fmax * 2);
     ALLOC(c->ssq, static_cast<size_t>(R) * (dmax / 128 + 1) * 8);

@@ -212,6 +212,16 @@ struct AttnArgs {
   void* part_acc = nullptr;
   void* part_ml = nullptr;
   void* part_cnt = nullptr;
+  // Flat mode (decode steps of several row groups, ragged lengths): `flat` > 0 CTAs ("slots") per KV
+  // head, one-CTA clusters, shared out over the groups on the device from their pre-step lengths so
+  // that no slot holds more tiles than needed; a group's splits meet in flat_acc ([Hkv][flat][64][hd]
+  // f32, unnormalised) and flat_ml ([Hkv][flat][64] float2: max, sum), counted in flat_cnt
+  // ([n_groups][Hkv], zero-initialised, self-resetting); the last split of a group writes its output.
+  // Needs pre_len, n_splits == 1, n_ctx_clusters == 1, n_groups <= flat and n_groups <= 64.
+  int flat = 0;
+  void* flat_acc = nullptr;
+  void* flat_ml = nullptr;
+  unsigned* flat_cnt = nullptr;
 };
 cudaError_t attention(const AttnArgs& a, cudaStream_t st);
 // Most context splits (= CTAs of one cluster) attention takes on this device: 16 where clusters of
