@@ -25,6 +25,9 @@
 // goes through global memory and no cluster barrier is held while the partials travel. Where
 // two CTAs per SM fit only that way, the receive buffers lie over the K/V ring: each split then
 // arrives on the cluster barrier after its last tile, so no partial lands in a ring still read.
+// Long contexts add clusters along the context whose owners meet through global partials; decode
+// steps over many ragged sequences run in flat mode (one-CTA clusters shared out by length on the
+// device, global partials, the last split of a sequence merging).
 #include <limits.h>
 #include <math.h>
 

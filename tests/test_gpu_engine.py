@@ -51,6 +51,22 @@ def test_tiny_longest_draft_and_wider_batch():
     assert rep.blocks == 24
 
 
+def test_flat_attention_ragged_batch():
+    """Eight sequences, one of 2100 tokens among seven of 9-40: the verify steps' attention runs in
+    flat mode (every resident CTA a slot, shared out on the device by length). The long sequence's
+    33 tiles spread over 17 slots (the per-sequence cap of 32 raises the tiles per slot to 2), each
+    short one takes one slot, most slots have nothing to do; every decision matches the oracle."""
+    work = dataclasses.replace(parity.tiny_work(), batch=8)
+    vw, dw, st = parity.tiny_weights(work, seed=31)
+    V = work.verifier.vocab
+    long_prompt = W.make_prompts(V, 1, (2100, 2100), seed=32)[0]
+    short = W.make_prompts(V, 7, (9, 40), seed=33)
+    prompts = [short[0], short[1], long_prompt, *short[2:]]
+    temps = [1.0, 0.0, 1.0, 0.7, 1.0, 0.0, 1.0, 0.5]
+    rep = parity.run(work, vw, dw, st, prompts, temps, seed=93, n_steps=3)
+    assert rep.blocks == 24
+
+
 def test_batch_below_context_capacity():
     """A context built for 5 sequences serving 2: the per-row scratch of the acceptance pass is laid
     out for the capacity, and every decision still matches the oracle."""
