@@ -291,6 +291,27 @@ sd2_status sd2_attention(const float* d_q, int32_t M, int32_t H, int32_t Hkv, in
                          const int32_t* d_pre_len, int32_t pre_stable, int32_t pre_fresh, void* d_out,
                          uint32_t* d_err, void* stream);
 
+/* Bytes of device workspace sd2_attention_flat needs for `slots` CTAs per KV head. */
+size_t sd2_attention_flat_workspace_bytes(int32_t Hkv, int32_t slots, int32_t hd);
+
+/* The same attention laid out as the engine runs decode steps over many sequences of ragged lengths
+ * (flat mode): `slots` CTAs per KV head are shared out over the groups on the device, each group
+ * taking ceil(t_g / t) of them (t_g its visible length d_pre_len[s] + pre_stable + pre_fresh in tiles
+ * of 64 positions, t the smallest tile count per CTA for which all groups fit, at most 32 CTAs a
+ * group); the splits of a group merge through the workspace and the group's last split writes its
+ * output. Same arguments as sd2_attention except: d_pre_len is required; 1 <= n_groups <= 64 and
+ * n_groups <= slots; max_ctx (> 64) bounds every visible length; d_work is
+ * sd2_attention_flat_workspace_bytes(Hkv, slots, hd) bytes of device memory, 16-byte aligned, zeroed
+ * by the caller before its first use and left zeroed by every call that completes (its counters reset
+ * themselves), used by one call at a time. Errors: SD2_EINVAL for a bad shape or a null pointer; the
+ * d_err bits as in sd2_attention. No device memory is allocated. */
+sd2_status sd2_attention_flat(const float* d_q, int32_t M, int32_t H, int32_t Hkv, int32_t hd, const void* d_pool,
+                              int32_t n_blocks, const int32_t* d_table, int32_t bt_stride, int32_t layer,
+                              const int32_t* d_row_pos, const int32_t* d_grp_row0, const int32_t* d_grp_nrows,
+                              const int32_t* d_grp_seq, int32_t n_groups, int32_t max_rows, int32_t slots,
+                              int32_t max_ctx, const int32_t* d_pre_len, int32_t pre_stable, int32_t pre_fresh,
+                              void* d_work, void* d_out, uint32_t* d_err, void* stream);
+
 /* Choose the GEMM of a context: 0 tensor cores where the shape allows (default), 1 CUDA cores.
  * Drops captured graphs. */
 sd2_status sd2_set_gemm_impl(sd2_ctx* ctx, int32_t impl);

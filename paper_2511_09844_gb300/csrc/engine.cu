@@ -1423,6 +1423,49 @@ sd2_status sd2_attention(const float* d_q, int32_t M, int32_t H, int32_t Hkv, in
   return SD2_OK;
 }
 
+// flat-mode workspace: partial accumulators [Hkv][slots][64][hd] f32, (max, sum) [Hkv][slots][64]
+// float2, counters [64][Hkv]
+size_t sd2_attention_flat_workspace_bytes(int32_t Hkv, int32_t slots, int32_t hd) {
+  if (Hkv < 1 || slots < 1 || hd < 1) return 0;
+  const size_t n = static_cast<size_t>(Hkv) * slots * 64;
+  return n * hd * 4 + n * 8 + static_cast<size_t>(64) * Hkv * 4;
+}
+
+sd2_status sd2_attention_flat(const float* d_q, int32_t M, int32_t H, int32_t Hkv, int32_t hd, const void* d_pool,
+                              int32_t n_blocks, const int32_t* d_table, int32_t bt_stride, int32_t layer,
+                              const int32_t* d_row_pos, const int32_t* d_grp_row0, const int32_t* d_grp_nrows,
+                              const int32_t* d_grp_seq, int32_t n_groups, int32_t max_rows, int32_t slots,
+                              int32_t max_ctx, const int32_t* d_pre_len, int32_t pre_stable, int32_t pre_fresh,
+                              void* d_work, void* d_out, uint32_t* d_err, void* stream) {
+  sd2_ctx* c = nullptr;
+  if (!d_q || !d_pool || !d_table || !d_row_pos || !d_grp_row0 || !d_grp_nrows || !d_grp_seq || !d_out ||
+      !d_pre_len || !d_work)
+    return fail(nullptr, SD2_EINVAL, "null input, output, pre-step lengths or workspace");
+  if (reinterpret_cast<uintptr_t>(d_work) % 16) return fail(nullptr, SD2_EINVAL, "workspace must be 16-byte aligned");
+  if (M < 1 || Hkv < 1 || H < Hkv || H % Hkv || (hd != 64 && hd != 128) || n_blocks < 1 || bt_stride < 1 ||
+      layer < 0 || max_rows < 1 || max_rows * (H / Hkv) > 64)
+    return fail(nullptr, SD2_EINVAL, "bad attention shape (hd 64 or 128, max_rows x H/Hkv <= 64)");
+  if (n_groups < 1 || n_groups > 64 || slots < n_groups || max_ctx <= 64 || pre_fresh < 0)
+    return fail(nullptr, SD2_EINVAL, "flat mode needs 1 <= n_groups <= 64, n_groups <= slots, max_ctx > 64");
+  AttnArgs at{};
+  at.q = d_q;
+  at.kv.pool = const_cast<void*>(d_pool); at.kv.table = d_table; at.kv.bt_stride = bt_stride;
+  at.kv.n_blocks = n_blocks; at.kv.Hkv = Hkv; at.kv.hd = hd;
+  at.layer = layer; at.row_pos = d_row_pos;
+  at.grp_row0 = d_grp_row0; at.grp_nrows = d_grp_nrows; at.grp_seq = d_grp_seq; at.n_groups = n_groups;
+  at.M = M; at.H = H; at.hd = hd; at.n_splits = 1; at.chunk = 64 * ((max_ctx + 63) / 64); at.max_rows = max_rows;
+  at.out = d_out;
+  at.pre_len = d_pre_len; at.pre_stable = pre_stable; at.pre_fresh = pre_fresh; at.err = d_err;
+  const size_t n = static_cast<size_t>(Hkv) * slots * 64;
+  unsigned char* w = static_cast<unsigned char*>(d_work);
+  at.flat = slots;
+  at.flat_acc = w;
+  at.flat_ml = w + n * hd * 4;
+  at.flat_cnt = reinterpret_cast<unsigned*>(w + n * hd * 4 + n * 8);
+  CK(attention(at, static_cast<cudaStream_t>(stream)));
+  return SD2_OK;
+}
+
 sd2_status sd2_swiglu_steered(const float* d_gate, const float* d_up, const float* d_bias, const int32_t* d_seq,
                               int32_t M, int32_t F, void* d_h, void* stream) {
   sd2_ctx* c = nullptr;

@@ -30,7 +30,8 @@ EXPORTS = ["sd2_init", "sd2_prefill", "sd2_step", "sd2_accept", "sd2_check", "sd
            "sd2_accept_logits_noalloc", "sd2_gemm", "sd2_set_gemm_impl", "sd2_stage_timing", "sd2_stage_read",
            "sd2_set_drafter_chain", "sd2_attention", "sd2_set_fused_attention",
            "sd2_accept_logits_noalloc_check", "sd2_debug_fail_alloc", "sd2_debug_expire_wait",
-           "sd2_gemm_timing", "sd2_gemm_timing_read", "sd2_generate"]
+           "sd2_gemm_timing", "sd2_gemm_timing_read", "sd2_generate", "sd2_attention_flat_workspace_bytes",
+           "sd2_attention_flat"]
 
 
 class LMConfig(ctypes.Structure):
@@ -96,6 +97,12 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
     lib.sd2_attention.argtypes = [c_void_p, c_int32, c_int32, c_int32, c_int32, c_void_p, c_int32, c_void_p, c_int32,
                                   c_int32, c_void_p, c_void_p, c_void_p, c_void_p, c_int32, c_int32, c_int32, c_int32,
                                   c_void_p, c_int32, c_int32, c_void_p, c_void_p, c_void_p]
+    lib.sd2_attention_flat_workspace_bytes.argtypes = [c_int32, c_int32, c_int32]
+    lib.sd2_attention_flat_workspace_bytes.restype = c_size_t
+    lib.sd2_attention_flat.argtypes = [c_void_p, c_int32, c_int32, c_int32, c_int32, c_void_p, c_int32, c_void_p,
+                                       c_int32, c_int32, c_void_p, c_void_p, c_void_p, c_void_p, c_int32, c_int32,
+                                       c_int32, c_int32, c_void_p, c_int32, c_int32, c_void_p, c_void_p, c_void_p,
+                                       c_void_p]
     lib.sd2_set_drafter_chain.argtypes = [c_void_p, c_int32]
     lib.sd2_set_fused_attention.argtypes = [c_void_p, c_int32]
     lib.sd2_accept_logits_noalloc.argtypes = [c_void_p, c_void_p, c_int32, c_void_p, c_void_p, c_int32, c_int32,
@@ -109,7 +116,8 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
                                          POINTER(c_int32)]
     lib.sd2_debug_expire_wait.argtypes = [c_void_p, c_int64]
     for name in EXPORTS:
-        if name not in ("sd2_last_error", "sd2_accept_workspace_bytes", "sd2_steer_workspace_bytes"):
+        if name not in ("sd2_last_error", "sd2_accept_workspace_bytes", "sd2_steer_workspace_bytes",
+                        "sd2_attention_flat_workspace_bytes"):
             getattr(lib, name).restype = c_int32
     _LIB = lib
     return lib
@@ -370,6 +378,28 @@ def attention(q: torch.Tensor, pool: torch.Tensor, table: torch.Tensor, layer: i
                                   _ptr(row_pos), _ptr(grp_row0), _ptr(grp_nrows), _ptr(grp_seq), grp_row0.numel(),
                                   max_rows, n_splits, chunk, _ptr(pre_len), pre_stable, pre_fresh, _ptr(out),
                                   _ptr(err), _stream(stream)))
+    return out
+
+
+def attention_flat(q: torch.Tensor, pool: torch.Tensor, table: torch.Tensor, layer: int, row_pos: torch.Tensor,
+                   grp_row0: torch.Tensor, grp_nrows: torch.Tensor, grp_seq: torch.Tensor, max_rows: int,
+                   slots: int, max_ctx: int, pre_len: torch.Tensor, pre_stable: int = 0, pre_fresh: int = 0,
+                   workspace: Optional[torch.Tensor] = None, err: Optional[torch.Tensor] = None,
+                   stream=None) -> torch.Tensor:
+    """Standalone flat-mode attention (sd2_attention_flat): `slots` CTAs per KV head shared out over
+    the groups by length; arguments as attention(), plus the workspace (zeroed uint8, allocated here
+    when not given). Returns bf16 [M, H * hd]."""
+    lib = load_library()
+    M, H, hd = q.shape
+    Hkv, n_blocks = pool.shape[3], pool.shape[1]
+    if workspace is None:
+        workspace = torch.zeros(lib.sd2_attention_flat_workspace_bytes(Hkv, slots, hd), dtype=torch.uint8,
+                                device=q.device)
+    out = torch.empty((M, H * hd), dtype=torch.bfloat16, device=q.device)
+    _check(lib, lib.sd2_attention_flat(_ptr(q), M, H, Hkv, hd, _ptr(pool), n_blocks, _ptr(table), table.shape[1],
+                                       layer, _ptr(row_pos), _ptr(grp_row0), _ptr(grp_nrows), _ptr(grp_seq),
+                                       grp_row0.numel(), max_rows, slots, max_ctx, _ptr(pre_len), pre_stable,
+                                       pre_fresh, _ptr(workspace), _ptr(out), _ptr(err), _stream(stream)))
     return out
 
 

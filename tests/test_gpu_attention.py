@@ -181,3 +181,54 @@ def test_many_sequences_four_ctas_per_sm():
     out, err = _run(c, 4, 320)
     assert err == 0
     _check(out, ref)
+
+
+def _run_flat(c, slots, max_ctx, pre_len, pre_stable, pre_fresh, workspace=None):
+    dev = {k: v.cuda() for k, v in c.items() if isinstance(v, torch.Tensor)}
+    err = torch.zeros(1, dtype=torch.int32, device="cuda")
+    out = sd2.attention_flat(dev["q"].float().contiguous(), dev["pool"], dev["table"], c["layer"], dev["row_pos"],
+                             dev["grp_row0"], dev["grp_nrows"], dev["grp_seq"], int(c["grp_nrows"].max()), slots,
+                             max_ctx, torch.tensor(pre_len, dtype=torch.int32, device="cuda"), pre_stable=pre_stable,
+                             pre_fresh=pre_fresh, workspace=workspace, err=err)
+    torch.cuda.synchronize()
+    return out.float().cpu(), int(err.item())
+
+
+def test_flat_mode_sixty_four_ragged_sequences():
+    """Flat mode (sd2_attention_flat) with the most groups a launch takes, 64 drafter-shaped groups of
+    ragged lengths: groups 32..63 take the slot map's second lane half; most of the 150 slots a KV
+    head has are idle. A second call on the same workspace checks that its counters reset."""
+    lens = [30 + (97 * i) % 301 for i in range(64)]
+    k1 = 2
+    c = _case(9, seq_lens=lens, rows_per_group=[k1] * 64, H=8, Hkv=2, hd=64)
+    ref = _reference(c)
+    pre_len = [L - k1 for L in lens]
+    ws = torch.zeros(sd2.load_library().sd2_attention_flat_workspace_bytes(2, 150, 64), dtype=torch.uint8,
+                     device="cuda")
+    for _ in range(2):
+        out, err = _run_flat(c, 150, max(lens) + 8, pre_len, 0, k1, workspace=ws)
+        assert err == 0
+        _check(out, ref)
+
+
+@pytest.mark.parametrize("slots", [100, 3])
+def test_flat_mode_long_sequence_over_many_slots(slots):
+    """Verify-shaped groups (6 rows x 4 heads, hd 128), one sequence of 2100 positions among two
+    short ones. With 100 slots the per-group cap of 32 slots sets the tiles per slot (2: the long
+    sequence over 17 slots); with 3 slots every group takes one."""
+    lens = [2100, 70, 150]
+    k1 = 6
+    c = _case(10, seq_lens=lens, rows_per_group=[k1] * 3, H=8, Hkv=2, hd=128)
+    ref = _reference(c)
+    pre_len = [L - k1 + 1 for L in lens]      # verifier convention: rows at n-1 .. n-1+k
+    out, err = _run_flat(c, slots, max(lens) + 8, pre_len, -1, k1 + 1)
+    assert err == 0
+    _check(out, ref)
+
+
+def test_flat_mode_bad_arguments_are_rejected_on_the_host():
+    c = _case(11, seq_lens=[100, 90], rows_per_group=[2, 2], H=32, Hkv=8, hd=128)
+    with pytest.raises(sd2.SD2Error):
+        _run_flat(c, 1, 120, [98, 88], 0, 2)       # fewer slots than groups
+    with pytest.raises(sd2.SD2Error):
+        _run_flat(c, 8, 64, [98, 88], 0, 2)        # a context bound of one tile
