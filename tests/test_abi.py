@@ -117,3 +117,21 @@ def test_standalone_entry_points_check_arguments_on_the_host(lib):
     assert err_is(attn(hd=96), b"bad attention shape")
     assert err_is(attn(H=30), b"bad attention shape")       # H not a multiple of Hkv
     assert err_is(attn(max_rows=17), b"bad attention shape")  # 17 rows x 4 heads > 64 query vectors
+
+    # flat-mode attention: workspace size, then the host's rejections
+    assert L.sd2_attention_flat_workspace_bytes(0, 38, 128) == 0
+    assert L.sd2_attention_flat_workspace_bytes(8, 38, 128) == 8 * 38 * 64 * (128 * 4 + 8) + 64 * 8 * 4
+
+    def flat(q=P, H=32, Hkv=8, hd=128, n_groups=2, max_rows=6, slots=38, max_ctx=1024, pre_len=P, work=P):
+        return L.sd2_attention_flat(q, 12, H, Hkv, hd, P, 64, P, 8, 0, P, P, P, P, n_groups, max_rows, slots,
+                                    max_ctx, pre_len, 0, 6, work, P, None, None)
+    assert err_is(flat(q=None), b"null")
+    assert err_is(flat(pre_len=None), b"null")
+    assert err_is(flat(work=None), b"null")
+    assert err_is(flat(work=U), b"16-byte")
+    assert err_is(flat(hd=96), b"bad attention shape")
+    assert err_is(flat(max_rows=17), b"bad attention shape")
+    assert err_is(flat(n_groups=0), b"flat mode")
+    assert err_is(flat(n_groups=65, slots=100), b"flat mode")
+    assert err_is(flat(n_groups=3, slots=2), b"flat mode")
+    assert err_is(flat(max_ctx=64), b"flat mode")
